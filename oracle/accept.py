@@ -1,0 +1,107 @@
+"""Oracle: target/draft softmax, acceptance and residual resampling (float64).
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).
+
+Sec. 3.3 "Verification as Auto Correction", strategy (C), applied to every
+drafted position independently:
+  * q_k is the draft distribution, p_k the backbone's distribution;
+  * the draft token is t_hat = argmax_v q_k(v);
+  * t_hat is accepted with probability alpha = min(p_k(t_hat) / q_k(t_hat), 1);
+  * on rejection the token is drawn from the residual distribution
+    [p_k - q_k]_+ / sum_v' [p_k - q_k]_+.
+Sec. 4 / App. "Configuration": temperature 1.0.
+
+Readings (the paper states the distributions, not the mechanism):
+  * p = softmax(l_p / T), q = softmax(l_q / T);
+  * argmax ties go to the lowest vocabulary index; the argmax is taken on the
+    raw logits (T > 0 keeps the order);
+  * the ratio is evaluated in log space; if q(t_hat) is 0 the draft is
+    accepted;
+  * accept iff u_acc < alpha with u_acc uniform on [0, 1) (probability alpha);
+  * the residual draw is the inverse CDF in ascending vocabulary order with
+    one uniform u_res: the smallest v with sum_{v' <= v} w_v' > u_res * Z,
+    w = [p - q]_+, Z = sum w; if rounding runs past the end the last v with
+    w_v > 0 is taken; if Z == 0 the draw is made from p instead.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+NEAR_TIE = 1e-4  # decisions within this distance of a threshold are reported, not compared
+
+
+def softmax(logits: np.ndarray, temperature: float = 1.0):
+    """Row softmax in float64.  Returns (probabilities, log-sum-exp of l/T)."""
+    x = np.asarray(logits, dtype=np.float64) / float(temperature)
+    m = x.max(axis=-1, keepdims=True)
+    e = np.exp(x - m)
+    s = e.sum(axis=-1, keepdims=True)
+    return e / s, (m + np.log(s))[..., 0]
+
+
+def draft_token(drf_logits: np.ndarray) -> np.ndarray:
+    """argmax_v q(v) per row, lowest index on ties (np.argmax returns the first)."""
+    return np.argmax(np.asarray(drf_logits), axis=-1).astype(np.int64)
+
+
+def inverse_cdf(w: np.ndarray, u: float):
+    """Smallest index v with cumsum(w)[v] > u * sum(w); see module readings.
+
+    Returns (v, margin) where margin = distance of u*Z to the nearest CDF
+    boundary of the chosen bin, relative to Z (for the near-tie report)."""
+    c = np.cumsum(w)
+    Z = c[-1]
+    target = u * Z
+    idx = np.nonzero(c > target)[0]
+    if idx.size:
+        v = int(idx[0])
+    else:
+        v = int(np.nonzero(w > 0)[0][-1])
+    lo = c[v - 1] if v > 0 else 0.0
+    margin = min(abs(target - lo), abs(c[v] - target)) / Z
+    return v, margin
+
+
+def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.0):
+    """Strategy (C) on every row.
+
+    tgt_logits, drf_logits: [rows, V]; uniforms: [rows, 2] = (u_acc, u_res);
+    draft_tok: [rows] or None (then t_hat = argmax q).
+    Returns a dict of per-row arrays: out_tok, accepted, t_hat, ratio, alpha,
+    lse_p, lse_q, resampled_from_p (Z == 0 fallback), tie_accept (|alpha -
+    u_acc| < NEAR_TIE), tie_resample (u_res * Z within NEAR_TIE * Z of a CDF
+    boundary of the chosen bin).
+    """
+    lp = np.asarray(tgt_logits, dtype=np.float64)
+    lq = np.asarray(drf_logits, dtype=np.float64)
+    u = np.asarray(uniforms, dtype=np.float64)
+    rows = lp.shape[0]
+    p, lse_p = softmax(lp, temperature)
+    q, lse_q = softmax(lq, temperature)
+    t = draft_token(lq) if draft_tok is None else np.asarray(draft_tok, dtype=np.int64)
+    out = dict(out_tok=np.zeros(rows, np.int64), accepted=np.zeros(rows, bool),
+               t_hat=t.copy(), ratio=np.zeros(rows), alpha=np.zeros(rows),
+               lse_p=lse_p, lse_q=lse_q, resampled_from_p=np.zeros(rows, bool),
+               tie_accept=np.zeros(rows, bool), tie_resample=np.zeros(rows, bool))
+    for r in range(rows):
+        tr = int(t[r])
+        log_ratio = (lp[r, tr] / temperature - lse_p[r]) - (lq[r, tr] / temperature - lse_q[r])
+        ratio = np.exp(log_ratio)
+        alpha = min(ratio, 1.0)
+        out["ratio"][r] = ratio
+        out["alpha"][r] = alpha
+        out["tie_accept"][r] = abs(alpha - u[r, 0]) < NEAR_TIE
+        if u[r, 0] < alpha:
+            out["accepted"][r] = True
+            out["out_tok"][r] = tr
+            continue
+        w = np.maximum(p[r] - q[r], 0.0)
+        if w.sum() > 0.0:
+            v, margin = inverse_cdf(w, u[r, 1])
+        else:
+            v, margin = inverse_cdf(p[r], u[r, 1])
+            out["resampled_from_p"][r] = True
+        out["out_tok"][r] = v
+        out["tie_resample"][r] = margin < NEAR_TIE
+    return out
+
