@@ -1,0 +1,382 @@
+"""Throughput of the SSD verification pass on GB300.
+
+One bench step = one whole verification pass (frontier, frontier attention,
+acceptance with residual resampling, counts) over one batch of synthetic
+input, through the C ABI of libssd.  The default workload is the 24x24
+(LlamaGen-XL-like) sweep: 25 cache lengths 120 -> 696 (one grid row apart),
+each an independent batch-1 verification problem with its own seed, issued
+together as one ragged batch of 25 sequences per ssd_verify_step call.
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle
+(the float64 restatement of the method) on the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "verify steps/s & accepted tokens/s per GB300; attention+accept HBM GB/s vs ~8 TB/s"
+UNIT = "sequence verify steps/s"  # one unit = one sequence's whole verification pass
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ssd", choices=["ssd", "reference"])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 5])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="approximate budget of the CPU-oracle sample")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- workloads
+def workload(cfg: int, rank: int, set_index: int = 0):
+    """Host arrays of one input set; rank and set_index pick the seeds."""
+    base = 1000 * rank + 100 * set_index
+    if cfg == 1:
+        return synth.config1(seed=base)
+    if cfg == 2:
+        return synth.config2(seed0=base)
+    if cfg == 3:
+        return synth.config3(seed=3 + base)
+    if cfg == 5:
+        return synth.config5(seed=5 + base)
+    raise ValueError(cfg)
+
+
+WORKLOAD_NAMES = {
+    1: "16x16 grid, prefix 32, cache 192, 8x64 heads, V=4096, batch 1",
+    2: "24x24 sweep: cache 120->696 step 24 (25 batch-1 problems as one ragged batch), "
+       "prefix 120, 16x128 MHA, V=16384",
+    3: "16 x 32x32 grids, prefix 64, cache U[64,1088], GQA 32/8x128, V=16384, Zipf draft",
+    5: "8 x 64x64 grids, prefix 256, first replay step (cache = prefix), 32x128 MHA, V=65536",
+}
+
+
+def algorithmic_bytes(c, n_drafts):
+    """Bytes one verification pass must move: every K/V row of the visible
+    keys once per KV head, Q and O of each draft, both logit rows of each
+    draft, and the per-row / per-sequence outputs."""
+    n = np.asarray(n_drafts, dtype=np.int64)
+    L = c.cache_len.astype(np.int64) + n
+    kv = int((L * c.Hkv * c.d * 2 * 2).sum())
+    qo = int((n * c.Hq * c.d * 2 * 2).sum())
+    attn = kv + qo + int(n.sum()) * c.Hq * 4  # + lse
+    acc = int(n.sum()) * (2 * c.V * 4 + 4 + 1 + 4)
+    return attn, acc
+
+
+# ------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out = self.proc.communicate(timeout=5)[0]
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out = self.proc.communicate()[0]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d.get("hbm_gbs", 6800.0), "measured"
+    return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_pass(c):
+    """One verification pass of the CPU oracle over every sequence of c."""
+    from oracle import step as ostep
+    q = synth.bf16_bits_to_f32(c.q).astype(np.float64)
+    k = synth.bf16_bits_to_f32(c.k).astype(np.float64)
+    v = synth.bf16_bits_to_f32(c.v).astype(np.float64)
+    ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
+                         q, k, v, c.Hq, c.Hkv)
+    r = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max,
+                          c.tgt_logits, c.drf_logits, c.uniforms)
+    return r
+
+
+def sub_case(c, seqs):
+    """The sequences `seqs` of c as a Case of their own (views, no copies of logits rows)."""
+    import copy
+    s = copy.copy(c)
+    seqs = np.asarray(seqs)
+    s.B = len(seqs)
+    s.cache_len = c.cache_len[seqs]
+    s.q, s.k, s.v = c.q[seqs], c.k[seqs], c.v[seqs]
+    rows = (seqs[:, None] * c.D_max + np.arange(c.D_max)[None]).reshape(-1)
+    s.tgt_logits, s.drf_logits, s.uniforms = c.tgt_logits[rows], c.drf_logits[rows], c.uniforms[rows]
+    return s
+
+
+def cpu_oracle_rate(c, budget_s):
+    """Verify steps/s of the oracle on a bounded sample of the workload: whole
+    sequences of the batch, one after another, until the budget is spent."""
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
+    t0 = time.perf_counter()
+    done = 0
+    for b in range(c.B):
+        oracle_pass(sub_case(c, [b]))
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    rate = done / el  # sequence verification passes per second
+    cores = int(threads) if threads else (os.cpu_count() or 1)
+    return {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{done} of the {c.B} sequences of one step ({el:.1f} s); "
+                      f"float64 NumPy, BLAS threads up to {cores}"}
+
+
+# -------------------------------------------------------------------- main
+def main():
+    a = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if a.impl == "reference":
+        if rank != 0:
+            return 0
+        c = workload(a.config, 0)
+        cpu = cpu_oracle_rate(c, a.cpu_seconds)
+        line = {"impl": "reference", "metric": METRIC, "value": cpu["value"], "unit": UNIT,
+                "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
+                "ms_per_step": 1000.0 * c.B / cpu["value"], "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": WORKLOAD_NAMES[a.config]},
+                "cpu_baseline": cpu,
+                "e2e": {"value": cpu["value"], "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
+
+    import torch
+    if not torch.cuda.is_available():
+        print(json.dumps({"error": "no CUDA device"}))
+        return 1
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+
+    from paper_2606_20543_gb300 import build
+    build.build()
+    import paper_2606_20543_gb300 as ssd
+    from paper_2606_20543_gb300.step import VerifyStep
+
+    # two input sets alternate so that consecutive steps never reuse L2
+    cases = [workload(a.config, rank, s) for s in range(2)]
+    c = cases[0]
+    steps_obj = []
+    for cs in cases:
+        st = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max,
+                        c.V, k_v=c.k_v, device=dev)
+        st.upload(cache_len=cs.cache_len, q=cs.q, k=cs.k, v=cs.v, tgt_logits=cs.tgt_logits,
+                  drf_logits=cs.drf_logits)
+        steps_obj.append(st)
+    stream = torch.cuda.current_stream(dev)
+    seed = 1234 + rank
+
+    def run(i):
+        st = steps_obj[i & 1]
+        st.set_rng(seed, i)
+        st.run(stream)
+
+    for i in range(a.warmup):
+        run(i)
+    torch.cuda.synchronize(dev)
+    n_drafts = [st.n_drafts.cpu().numpy() for st in steps_obj]
+    launches = ssd.ssd_verify_step_launches(steps_obj[0].args)
+    attn_bytes, acc_bytes = algorithmic_bytes(c, n_drafts[0])
+
+    # ---------------- timed region: K verification passes
+    clocks = ClockSampler(dev.index or 0)
+    clocks.start()
+    time.sleep(0.2)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(a.steps):
+        run(a.warmup + i)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / a.steps
+    value = world * a.steps * c.B / (ms / 1000.0)
+
+    accepted_tok = []
+    for st in steps_obj:
+        accepted_tok.append(int(st.accepted_count.sum().item()))
+    acc_tok_per_step = float(np.mean(accepted_tok))
+    committed = float(np.mean([(st.next_cache_len - st.cache_len).sum().item() for st in steps_obj]))
+
+    # ---------------- per-kernel durations: the same K passes issued per
+    # entry point, CUDA events around each kernel on the launching stream
+    st = steps_obj[0]
+    g = st.g
+    nd, pos = st.n_drafts, st.draft_pos
+    wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    kk = min(a.steps, 200)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(kk)]
+    for i in range(kk):
+        s = steps_obj[i & 1]
+        s.set_rng(seed, i)
+        ssd.ssd_frontier(g, c.B, s.cache_len, c.D_max, nd, pos, s.status, stream)
+        ev[i][0].record(stream)
+        ssd.ssd_verify_attention(g, c.B, c.Hq, c.Hkv, c.d, s.cache_len, nd, pos, c.D_max, c.L_max,
+                                 s.q, s.k, s.v, 0.0, s.o, None, ws, wsb, s.status, stream)
+        ev[i][1].record(stream)
+        ssd.ssd_accept(c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0, s.rng, s.out_tok,
+                       s.accepted, s.ratio, None, s.status, stream)
+        ev[i][2].record(stream)
+    torch.cuda.synchronize(dev)
+    attn_ms = statistics.mean(ev[i][0].elapsed_time(ev[i][1]) for i in range(kk))
+    acc_ms = statistics.mean(ev[i][1].elapsed_time(ev[i][2]) for i in range(kk))
+    hbm_peak, peak_kind = measured_peaks()
+    # the standalone ssd_accept call processes every row of the padded batch
+    acc_bytes_all = c.B * c.D_max * (2 * c.V * 4 + 4 + 1 + 4)
+    kern = {"attention": (attn_bytes, attn_ms), "accept": (acc_bytes_all, acc_ms)}
+    dom = max(kern, key=lambda k: kern[k][1])
+    dom_bytes, dom_ms = kern[dom]
+    achieved = dom_bytes / (dom_ms / 1000.0) / 1e9
+    status = int(max(s.status.item() for s in steps_obj))
+
+    # ---------------- end to end: host buffers, copies inside the timed region
+    host = {}
+    for name in ("cache_len", "q", "k", "v", "tgt", "drf"):
+        t = getattr(st, name)
+        host[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        host[name].copy_(t)
+    outs = {n: torch.empty(getattr(st, n).shape, dtype=getattr(st, n).dtype, pin_memory=True)
+            for n in ("out_tok", "accepted", "accepted_count", "next_cache_len")}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in outs.values())
+    ke = max(3, min(a.steps, 50))
+    torch.cuda.synchronize(dev)
+    f0 = torch.cuda.Event(enable_timing=True)
+    f1 = torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for i in range(ke):
+        for name, t in host.items():
+            getattr(st, name).copy_(t, non_blocking=True)
+        st.set_rng(seed, i)
+        st.run(stream)
+        for name, t in outs.items():
+            t.copy_(getattr(st, name), non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = f0.elapsed_time(f1) / ke
+    e2e_value = world * c.B * 1000.0 / e2e_ms
+
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return 0
+
+    cpu = None
+    if not a.no_cpu_baseline:
+        cpu = cpu_oracle_rate(cases[0], a.cpu_seconds)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
+        "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16 attention / f32 acceptance",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAMES[a.config], "sequences_per_step": c.B,
+                   "drafts_per_step": int(n_drafts[0].sum()), "vocab": c.V,
+                   "heads": f"{c.Hq}/{c.Hkv}x{c.d}",
+                   "l2": "two input sets alternate; each step streams "
+                         f"{(attn_bytes + acc_bytes) / 1e6:.0f} MB > 129 MB L2",
+                   "parallelism": f"replicas x{world}"},
+        "accepted_tokens_per_s": world * acc_tok_per_step * a.steps / (ms / 1000.0),
+        "committed_tokens_per_step": committed,
+        "hbm_gbs_per_step": (attn_bytes + acc_bytes) / (ms_per_step / 1000.0) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
+                     "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": None,
+                     "peak_kind": peak_kind,
+                     "kernels": {k: {"bytes": b, "ms": m, "gbs": b / (m / 1000.0) / 1e9}
+                                 for k, (b, m) in kern.items()}},
+        "clocks": clk,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": ke},
+        "gpu_launches": launches * a.steps,
+        "device_status": status,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

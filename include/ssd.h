@@ -1,0 +1,246 @@
+/*
+ * ssd.h — C ABI of libssd: the verification pass of Spatially Speculative
+ * Decoding (SSD) on one GB300 (sm_103a).
+ *
+ * One verification step (Sec. 3.3, "Verification as Auto Correction") takes
+ * the drafted frontier of every sequence (the remainder of the current grid
+ * row, drafted by the horizontal heads, plus the row(s) directly below it,
+ * drafted column-parallel by the vertical heads), scores it against the KV
+ * cache under the spatial dependency mask, and accepts each draft with
+ * probability min(p/q, 1) or replaces it by a draw from [p - q]_+.
+ *
+ * Conventions for every entry point:
+ *  - Pointers marked "dev" are device pointers on the current CUDA device;
+ *    "host" pointers are read during the call and not kept.  The caller owns
+ *    every buffer; the library allocates nothing on these paths.  Workspace,
+ *    where needed, is sized by the matching *_workspace() query and passed in.
+ *  - All work is enqueued asynchronously on `stream` (NULL = the legacy
+ *    default stream).  Nothing synchronises.
+ *  - Host-side checks (null pointers, unsupported shapes, too little
+ *    workspace) return a status synchronously and enqueue nothing.
+ *    SSD_ERR_CUDA reports a failed launch (cudaGetLastError).
+ *  - Device-side checks (a cache length outside [prefix, prefix + H*W], a
+ *    draft position outside the grid, a draft token outside [0, V), a grid
+ *    barrier that gave up waiting) record the FIRST error code in the device
+ *    int32 `*status` with an atomic compare-and-swap from SSD_OK.  The library
+ *    never clears `*status`; the caller zeroes it and reads it after a sync.
+ *  - Row-major layouts, innermost index last.  bf16 buffers hold IEEE
+ *    bfloat16 bit patterns (2 bytes per element).
+ *  - Draft slot j of sequence b is row b*D_max + j of every per-draft array;
+ *    slots j >= n_drafts[b] are padding: they are neither read nor used, and
+ *    their per-row outputs are set to out_tok = -1, accepted = 0, ratio = 0.
+ */
+#ifndef SSD_H
+#define SSD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; declared here so callers need no CUDA header. */
+typedef struct CUstream_st* ssd_stream_t;
+
+typedef enum {
+  SSD_OK = 0,
+  SSD_ERR_INVALID_ARG = 1,   /* null pointer, negative size, bad enum       */
+  SSD_ERR_SHAPE = 2,         /* sizes inconsistent with each other          */
+  SSD_ERR_UNSUPPORTED = 3,   /* a valid shape this build has no kernel for  */
+  SSD_ERR_CUDA = 4,          /* a CUDA call or launch failed                */
+  SSD_ERR_TIMEOUT = 5,       /* device: a bounded grid-barrier wait expired */
+  SSD_ERR_DEVICE_BOUNDS = 6, /* device: a position / token / length out of range */
+  SSD_ERR_WORKSPACE = 7      /* workspace pointer null or too small         */
+} ssd_status;
+
+/* The image-token grid of Sec. 3.1 after its text prefix (Eq. 1).
+ * Grid token (y, x) sits at flat sequence position
+ *     prefix_len + y * row_stride + x.
+ * row_stride is W, or W + 1 for backbones that close each row with an
+ * end-of-line token.  k_v is the number of grid rows drafted below the
+ * current one (vertical heads, Sec. 3.3); the frontier rule of
+ * ssd_frontier() needs row_stride == W. */
+typedef struct {
+  int32_t grid_h;     /* H: grid rows                                     */
+  int32_t grid_w;     /* W: grid columns                                  */
+  int32_t row_stride; /* W or W + 1                                       */
+  int32_t prefix_len; /* text-prefix tokens before grid token (0, 0)      */
+  int32_t k_v;        /* rows drafted below the current row, >= 1         */
+} ssd_grid;
+
+/* Per-draft uniforms (u_acc, u_res).  If `uniforms` (dev, float32
+ * [rows][2]) is non-NULL it is used as given.  Otherwise row r draws them
+ * from Philox4x32-10 (Salmon et al., SC'11) with counter
+ * (r, offset_lo, offset_hi, 0) and key (seed_lo, seed_hi):
+ * u_acc = (x0 >> 8) * 2^-24, u_res = (x1 >> 8) * 2^-24. */
+typedef struct {
+  uint64_t seed;
+  uint64_t offset;
+  const float* uniforms;
+} ssd_rng;
+
+/* ABI version of this header (increment on any signature change). */
+#define SSD_ABI_VERSION 1
+int32_t ssd_abi_version(void);
+
+/* Human-readable name of a status code (static string). */
+const char* ssd_status_string(ssd_status s);
+
+/* ---------------------------------------------------------------------------
+ * a1. Frontier (Sec. 3.3: horizontal heads complete the current row, the
+ * vertical heads draft the k_v rows below it; Sec. 3.1 raster order).
+ * For each sequence b, with n_c = cache_len[b] - prefix_len committed grid
+ * tokens and the first uncommitted token at (y0, c) = (n_c / W, n_c % W):
+ *     n_drafts[b] = (W - c) + k_v * W, clipped at the grid's last row,
+ *     draft_pos[b][j] = n_c + j (grid index y * W + x), j < n_drafts[b];
+ * padding slots get -1.
+ *   cache_len  dev int32 [B]
+ *   n_drafts   dev int32 [B]             (out)
+ *   draft_pos  dev int32 [B][D_max]      (out); D_max >= (k_v + 1) * W
+ * Device errors: cache_len outside [prefix, prefix + H*W] -> DEVICE_BOUNDS
+ * (that sequence gets n_drafts = 0).
+ * ------------------------------------------------------------------------- */
+ssd_status ssd_frontier(const ssd_grid* grid, int32_t B, const int32_t* cache_len,
+                        int32_t D_max, int32_t* n_drafts, int32_t* draft_pos,
+                        int32_t* status, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * a2. Frontier attention (Sec. 3.3 "Verification as Auto Correction": the
+ * drafted block passes through the backbone in parallel; App. "Deviation
+ * from AR": each draft's context may hold other drafts).
+ * For draft j of sequence b and query head h (KV head g = h / (Hq / Hkv)):
+ *     O[b][j][h] = softmax_s(scale * Q[b][j][h] . K[b][g][s] + M(s, j)) V[b][g][s]
+ * over key slots s < cache_len[b] + n_drafts[b].  Slots [0, cache_len) are
+ * the committed cache (flat position s); slot cache_len + j' holds draft
+ * j''s own key/value (flat position of draft_pos[b][j']).  M = 0 iff
+ * pos(key) <= pos(query), else -inf.  scale = 0 selects 1/sqrt(d).
+ *   q          dev bf16 [B][D_max][Hq][d]
+ *   k, v       dev bf16 [B][Hkv][L_max][d]; cache_len + n_drafts <= L_max
+ *   cache_len, n_drafts  dev int32 [B]
+ *   draft_pos  dev int32 [B][D_max]  grid index y * W + x
+ *   o          dev bf16 [B][D_max][Hq][d]   (out; padding slots untouched)
+ *   lse        dev float32 [B][Hq][D_max] or NULL: log-sum-exp of the
+ *              scaled scores (natural log)
+ *   workspace  dev, >= ssd_verify_attention_workspace(...) bytes (split-KV
+ *              partials and the schedule); may be NULL if that is 0.
+ * Supported: d in {64, 128}; Hq % Hkv == 0; 1 <= D_max <= 128;
+ * D_max * (Hq / Hkv) <= 512.  Device errors: a draft position outside the
+ * grid or a key count above L_max -> DEVICE_BOUNDS (rows left untouched).
+ * ------------------------------------------------------------------------- */
+size_t ssd_verify_attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                                      int32_t D_max, int32_t L_max);
+ssd_status ssd_verify_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int32_t Hkv,
+                                int32_t d, const int32_t* cache_len, const int32_t* n_drafts,
+                                const int32_t* draft_pos, int32_t D_max, int32_t L_max,
+                                const void* q, const void* k, const void* v, float scale,
+                                void* o, float* lse, void* workspace, size_t workspace_bytes,
+                                int32_t* status, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * a3-a5. Acceptance (Sec. 3.3 strategy (C); temperature of App.
+ * "Configuration").  For every row r < rows:
+ *     p = softmax(tgt[r] / T), q = softmax(drf[r] / T)
+ *     t = draft_tok[r], or argmax_v drf[r][v] (lowest index on ties) if NULL
+ *     ratio = p(t) / q(t) (evaluated in log space)
+ *     accept iff u_acc < min(ratio, 1)
+ *     on reject: out = smallest v with sum_{v' <= v} [p - q]_+ > u_res * Z,
+ *                Z = sum_v [p - q]_+ (if Z == 0: the same draw from p)
+ *   tgt_logits, drf_logits  dev float32, row r at + r * ld, V entries;
+ *                           16-byte aligned, ld % 4 == 0, V % 4 == 0
+ *   draft_tok  dev int32 [rows] or NULL
+ *   out_tok    dev int32 [rows] (out); accepted dev uint8 [rows] (out)
+ *   ratio      dev float32 [rows] or NULL (out)
+ *   lse        dev float32 [rows][2] or NULL (out): log-sum-exp of tgt/T and
+ *              of drf/T
+ * Device errors: draft_tok outside [0, V) -> DEVICE_BOUNDS (row gets
+ * out_tok = -1, accepted = 0).
+ * ------------------------------------------------------------------------- */
+ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
+                      int64_t ld, const int32_t* draft_tok, float temperature, const ssd_rng* rng,
+                      int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
+                      int32_t* status, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * a6. Fused lm_head + acceptance (Sec. 3.3, after Eq. 2: tokens are decoded
+ * through the base model's GenHead).  Logits l_p = H_t W_t and l_q = H_d W_d
+ * are formed on chip (tcgen05, fp32 accumulation) and fed to the rule of
+ * ssd_accept() without being written to memory.
+ *   h_tgt, h_drf  dev bf16 [rows][K] (already normalised hidden states)
+ *   w_tgt, w_drf  dev bf16 [K][V]   (may alias each other)
+ *   other arguments as ssd_accept(); lse may be NULL.
+ *   workspace     dev, >= ssd_lmhead_accept_workspace(rows, V) bytes
+ * Supported: 1 <= rows <= 256, K % 64 == 0, V % 128 == 0, V / 128 no more
+ * than the co-resident CTAs of the device.  The kernel's CTAs meet at two
+ * bounded grid barriers; a barrier that waits too long records
+ * SSD_ERR_TIMEOUT and the kernel returns without writing its outputs.
+ * ------------------------------------------------------------------------- */
+size_t ssd_lmhead_accept_workspace(int32_t rows, int32_t V);
+ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_tgt,
+                             const void* h_drf, const void* w_tgt, const void* w_drf,
+                             const int32_t* draft_tok, float temperature, const ssd_rng* rng,
+                             int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
+                             void* workspace, size_t workspace_bytes, int32_t* status,
+                             ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * a1-a7. One whole verification step: frontier (a1), frontier attention
+ * (a2), acceptance from logits (a3-a5) or from hidden states through the
+ * fused lm_head (a6), and the counts that advance the cache (a7):
+ *     accepted_count[b]  = drafts of b accepted
+ *     accepted_prefix[b] = leading drafts of b (raster order) accepted
+ *     next_cache_len[b]  = cache_len[b] + min(accepted_prefix[b] + 1, n_d)
+ *                          (the first rejected draft carries its resampled
+ *                          token; an empty frontier leaves cache_len as is)
+ * Acceptance rows are b*D_max + j; the Philox counter row is the same index.
+ * Logits path: tgt_logits/drf_logits non-NULL ([B*D_max] rows of ld floats).
+ * Fused path:  logits NULL and h_tgt, h_drf, w_tgt, w_drf non-NULL (hidden
+ *              = K of ssd_lmhead_accept).
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  ssd_grid grid;
+  int32_t B, Hq, Hkv, d, D_max, L_max, V;
+  const int32_t* cache_len;   /* dev int32 [B]                         */
+  const void* q;              /* dev bf16 [B][D_max][Hq][d]            */
+  const void* k;              /* dev bf16 [B][Hkv][L_max][d]           */
+  const void* v;              /* dev bf16 [B][Hkv][L_max][d]           */
+  float scale;                /* 0 -> 1/sqrt(d)                        */
+  const float* tgt_logits;    /* dev float32 [B*D_max][ld] or NULL     */
+  const float* drf_logits;    /* dev float32 [B*D_max][ld] or NULL     */
+  int64_t ld;
+  const void* h_tgt;          /* dev bf16 [B*D_max][hidden] or NULL    */
+  const void* h_drf;
+  const void* w_tgt;          /* dev bf16 [hidden][V] or NULL          */
+  const void* w_drf;
+  int32_t hidden;
+  const int32_t* draft_tok;   /* dev int32 [B*D_max] or NULL (argmax q)*/
+  float temperature;
+  ssd_rng rng;
+} ssd_verify_args;
+
+typedef struct {
+  int32_t* n_drafts;          /* dev int32 [B]                          */
+  int32_t* draft_pos;         /* dev int32 [B][D_max]                   */
+  void* o;                    /* dev bf16 [B][D_max][Hq][d]             */
+  float* lse;                 /* dev float32 [B][Hq][D_max] or NULL     */
+  int32_t* out_tok;           /* dev int32 [B*D_max]                    */
+  uint8_t* accepted;          /* dev uint8 [B*D_max]                    */
+  float* ratio;               /* dev float32 [B*D_max] or NULL          */
+  int32_t* accepted_count;    /* dev int32 [B]                          */
+  int32_t* accepted_prefix;   /* dev int32 [B]                          */
+  int32_t* next_cache_len;    /* dev int32 [B]                          */
+  int32_t* status;            /* dev int32 [1]                          */
+} ssd_verify_out;
+
+size_t ssd_verify_step_workspace(const ssd_verify_args* args);
+/* Number of kernels one ssd_verify_step() with these arguments launches
+ * (host query, no GPU work); -1 if the arguments would be rejected. */
+int32_t ssd_verify_step_launches(const ssd_verify_args* args);
+ssd_status ssd_verify_step(const ssd_verify_args* args, const ssd_verify_out* out,
+                           void* workspace, size_t workspace_bytes, ssd_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SSD_H */

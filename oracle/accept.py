@@ -27,7 +27,8 @@ from __future__ import annotations
 
 import numpy as np
 
-NEAR_TIE = 1e-4  # decisions within this distance of a threshold are reported, not compared
+NEAR_TIE = 1e-4      # |alpha - u_acc| below this: the accept decision is a near-tie
+NEAR_TIE_CDF = 1e-6  # u_res * Z within this fraction of Z of a CDF boundary: resample near-tie
 
 
 def softmax(logits: np.ndarray, temperature: float = 1.0):
@@ -68,9 +69,10 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
     tgt_logits, drf_logits: [rows, V]; uniforms: [rows, 2] = (u_acc, u_res);
     draft_tok: [rows] or None (then t_hat = argmax q).
     Returns a dict of per-row arrays: out_tok, accepted, t_hat, ratio, alpha,
-    lse_p, lse_q, resampled_from_p (Z == 0 fallback), tie_accept (|alpha -
-    u_acc| < NEAR_TIE), tie_resample (u_res * Z within NEAR_TIE * Z of a CDF
-    boundary of the chosen bin).
+    lse_p, lse_q, resampled_from_p (Z == 0 fallback), accept_margin = |alpha -
+    u_acc|, tie_accept (accept_margin < NEAR_TIE), cdf_margin (distance of
+    u_res * Z to the nearest boundary of the chosen bin, over Z), tie_resample
+    (cdf_margin < NEAR_TIE_CDF).
     """
     lp = np.asarray(tgt_logits, dtype=np.float64)
     lq = np.asarray(drf_logits, dtype=np.float64)
@@ -82,7 +84,8 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
     out = dict(out_tok=np.zeros(rows, np.int64), accepted=np.zeros(rows, bool),
                t_hat=t.copy(), ratio=np.zeros(rows), alpha=np.zeros(rows),
                lse_p=lse_p, lse_q=lse_q, resampled_from_p=np.zeros(rows, bool),
-               tie_accept=np.zeros(rows, bool), tie_resample=np.zeros(rows, bool))
+               tie_accept=np.zeros(rows, bool), tie_resample=np.zeros(rows, bool),
+               accept_margin=np.zeros(rows), cdf_margin=np.full(rows, np.inf))
     for r in range(rows):
         tr = int(t[r])
         log_ratio = (lp[r, tr] / temperature - lse_p[r]) - (lq[r, tr] / temperature - lse_q[r])
@@ -90,6 +93,7 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
         alpha = min(ratio, 1.0)
         out["ratio"][r] = ratio
         out["alpha"][r] = alpha
+        out["accept_margin"][r] = abs(alpha - u[r, 0])
         out["tie_accept"][r] = abs(alpha - u[r, 0]) < NEAR_TIE
         if u[r, 0] < alpha:
             out["accepted"][r] = True
@@ -102,6 +106,7 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
             v, margin = inverse_cdf(p[r], u[r, 1])
             out["resampled_from_p"][r] = True
         out["out_tok"][r] = v
-        out["tie_resample"][r] = margin < NEAR_TIE
+        out["cdf_margin"][r] = margin
+        out["tie_resample"][r] = margin < NEAR_TIE_CDF
     return out
 

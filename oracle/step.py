@@ -101,6 +101,7 @@ def replay(grid_h, grid_w, prefix_len, k_v, B, D_max, step_inputs, max_steps=100
                          accepted_count=r["accepted_count"].copy(),
                          accepted_prefix=r["accepted_prefix"].copy(),
                          next_cache_len=r["next_cache_len"].copy(),
-                         ties=int(np.sum(dec["tie_accept"])) + int(np.sum(dec["tie_resample"]))))
+                         accept_ties=int(np.sum(dec["tie_accept"])),
+                         resample_ties=int(np.sum(dec["tie_resample"]))))
         cache_len = r["next_cache_len"].copy()
     return hist, grid_tok, cache_len

@@ -1,0 +1,197 @@
+"""Python binding of libssd, the GB300 (sm_103a) verification pass of
+Spatially Speculative Decoding.
+
+Argument marshalling only: every function here forwards to the entry point
+of the same name in ``include/ssd.h``; every step of the pass runs in the
+library's CUDA kernels.  Device buffers are torch CUDA tensors (PyTorch is
+used for device memory and streams only).  There is no CPU path: if the
+library has not been built, importing a function raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libssd.so")
+
+SSD_OK = 0
+STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "SSD_ERR_UNSUPPORTED",
+                4: "SSD_ERR_CUDA", 5: "SSD_ERR_TIMEOUT", 6: "SSD_ERR_DEVICE_BOUNDS",
+                7: "SSD_ERR_WORKSPACE"}
+
+EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
+            "ssd_verify_attention", "ssd_accept", "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
+            "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
+
+
+class SsdError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} returned {STATUS_NAMES.get(code, code)}")
+        self.code = code
+
+
+class Grid(ctypes.Structure):
+    _fields_ = [("grid_h", ctypes.c_int32), ("grid_w", ctypes.c_int32),
+                ("row_stride", ctypes.c_int32), ("prefix_len", ctypes.c_int32),
+                ("k_v", ctypes.c_int32)]
+
+
+class Rng(ctypes.Structure):
+    _fields_ = [("seed", ctypes.c_uint64), ("offset", ctypes.c_uint64),
+                ("uniforms", ctypes.c_void_p)]
+
+
+class VerifyArgs(ctypes.Structure):
+    _fields_ = [("grid", Grid),
+                ("B", ctypes.c_int32), ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32),
+                ("d", ctypes.c_int32), ("D_max", ctypes.c_int32), ("L_max", ctypes.c_int32),
+                ("V", ctypes.c_int32),
+                ("cache_len", ctypes.c_void_p), ("q", ctypes.c_void_p), ("k", ctypes.c_void_p),
+                ("v", ctypes.c_void_p), ("scale", ctypes.c_float),
+                ("tgt_logits", ctypes.c_void_p), ("drf_logits", ctypes.c_void_p),
+                ("ld", ctypes.c_int64),
+                ("h_tgt", ctypes.c_void_p), ("h_drf", ctypes.c_void_p),
+                ("w_tgt", ctypes.c_void_p), ("w_drf", ctypes.c_void_p),
+                ("hidden", ctypes.c_int32),
+                ("draft_tok", ctypes.c_void_p), ("temperature", ctypes.c_float),
+                ("rng", Rng)]
+
+
+class VerifyOut(ctypes.Structure):
+    _fields_ = [("n_drafts", ctypes.c_void_p), ("draft_pos", ctypes.c_void_p),
+                ("o", ctypes.c_void_p), ("lse", ctypes.c_void_p),
+                ("out_tok", ctypes.c_void_p), ("accepted", ctypes.c_void_p),
+                ("ratio", ctypes.c_void_p), ("accepted_count", ctypes.c_void_p),
+                ("accepted_prefix", ctypes.c_void_p), ("next_cache_len", ctypes.c_void_p),
+                ("status", ctypes.c_void_p)]
+
+
+_LIB: Optional[ctypes.CDLL] = None
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libssd.so (built by ``paper_2606_20543_gb300.build``); raise if absent."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"libssd.so not built ({path} missing): run "
+                           "`python -m paper_2606_20543_gb300.build` (needs nvcc)")
+    lib = ctypes.CDLL(path)
+    P, I32, I64, F, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    sig = {
+        "ssd_abi_version": (I32, []),
+        "ssd_status_string": (ctypes.c_char_p, [I32]),
+        "ssd_frontier": (I32, [ctypes.POINTER(Grid), I32, P, I32, P, P, P, P]),
+        "ssd_verify_attention_workspace": (SZ, [I32, I32, I32, I32, I32, I32]),
+        "ssd_verify_attention": (I32, [ctypes.POINTER(Grid), I32, I32, I32, I32, P, P, P, I32, I32,
+                                       P, P, P, F, P, P, P, SZ, P, P]),
+        "ssd_accept": (I32, [I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P, P, P, P]),
+        "ssd_lmhead_accept_workspace": (SZ, [I32, I32]),
+        "ssd_lmhead_accept": (I32, [I32, I32, I32, P, P, P, P, P, F, ctypes.POINTER(Rng), P, P, P,
+                                    P, P, SZ, P, P]),
+        "ssd_verify_step_workspace": (SZ, [ctypes.POINTER(VerifyArgs)]),
+        "ssd_verify_step_launches": (I32, [ctypes.POINTER(VerifyArgs)]),
+        "ssd_verify_step": (I32, [ctypes.POINTER(VerifyArgs), ctypes.POINTER(VerifyOut), P, SZ, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _LIB = lib
+    return lib
+
+
+def _ptr(t) -> Optional[int]:
+    """Device address of a torch tensor (None stays None)."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("libssd takes device (CUDA) tensors")
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+def _check(fn: str, code: int) -> None:
+    if code != SSD_OK:
+        raise SsdError(fn, code)
+
+
+def grid(grid_h: int, grid_w: int, prefix_len: int, row_stride: Optional[int] = None,
+         k_v: int = 1) -> Grid:
+    return Grid(grid_h, grid_w, grid_w if row_stride is None else row_stride, prefix_len, k_v)
+
+
+def rng(seed: int = 0, offset: int = 0, uniforms=None) -> Rng:
+    return Rng(seed, offset, _ptr(uniforms))
+
+
+def ssd_abi_version() -> int:
+    return load().ssd_abi_version()
+
+
+def ssd_status_string(code: int) -> str:
+    return load().ssd_status_string(code).decode()
+
+
+def ssd_frontier(g: Grid, B: int, cache_len, D_max: int, n_drafts, draft_pos, status,
+                 stream=None) -> None:
+    _check("ssd_frontier", load().ssd_frontier(ctypes.byref(g), B, _ptr(cache_len), D_max,
+                                               _ptr(n_drafts), _ptr(draft_pos), _ptr(status),
+                                               _stream(stream)))
+
+
+def ssd_verify_attention_workspace(B, Hq, Hkv, d, D_max, L_max) -> int:
+    return load().ssd_verify_attention_workspace(B, Hq, Hkv, d, D_max, L_max)
+
+
+def ssd_verify_attention(g: Grid, B, Hq, Hkv, d, cache_len, n_drafts, draft_pos, D_max, L_max,
+                         q, k, v, scale, o, lse, workspace, workspace_bytes, status,
+                         stream=None) -> None:
+    _check("ssd_verify_attention", load().ssd_verify_attention(
+        ctypes.byref(g), B, Hq, Hkv, d, _ptr(cache_len), _ptr(n_drafts), _ptr(draft_pos), D_max,
+        L_max, _ptr(q), _ptr(k), _ptr(v), scale, _ptr(o), _ptr(lse), _ptr(workspace),
+        workspace_bytes, _ptr(status), _stream(stream)))
+
+
+def ssd_accept(rows, V, tgt_logits, drf_logits, ld, draft_tok, temperature, r: Rng, out_tok,
+               accepted, ratio, lse, status, stream=None) -> None:
+    _check("ssd_accept", load().ssd_accept(
+        rows, V, _ptr(tgt_logits), _ptr(drf_logits), ld, _ptr(draft_tok), temperature,
+        ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
+        _stream(stream)))
+
+
+def ssd_lmhead_accept_workspace(rows, V) -> int:
+    return load().ssd_lmhead_accept_workspace(rows, V)
+
+
+def ssd_lmhead_accept(rows, V, K, h_tgt, h_drf, w_tgt, w_drf, draft_tok, temperature, r: Rng,
+                      out_tok, accepted, ratio, lse, workspace, workspace_bytes, status,
+                      stream=None) -> None:
+    _check("ssd_lmhead_accept", load().ssd_lmhead_accept(
+        rows, V, K, _ptr(h_tgt), _ptr(h_drf), _ptr(w_tgt), _ptr(w_drf), _ptr(draft_tok),
+        temperature, ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse),
+        _ptr(workspace), workspace_bytes, _ptr(status), _stream(stream)))
+
+
+def ssd_verify_step_workspace(args: VerifyArgs) -> int:
+    return load().ssd_verify_step_workspace(ctypes.byref(args))
+
+
+def ssd_verify_step_launches(args: VerifyArgs) -> int:
+    return load().ssd_verify_step_launches(ctypes.byref(args))
+
+
+def ssd_verify_step(args: VerifyArgs, out: VerifyOut, workspace, workspace_bytes,
+                    stream=None) -> None:
+    _check("ssd_verify_step", load().ssd_verify_step(
+        ctypes.byref(args), ctypes.byref(out), _ptr(workspace), workspace_bytes, _stream(stream)))

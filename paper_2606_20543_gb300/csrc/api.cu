@@ -1,0 +1,332 @@
+// api.cu — the extern "C" entry points of libssd declared in include/ssd.h:
+// host-side argument checks, workspace carving, and kernel launches on the
+// caller's stream.  No allocation, no synchronisation.
+#include <math.h>
+
+#include "kernels.cuh"
+
+using namespace ssd;
+
+namespace {
+
+ssd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SSD_OK : SSD_ERR_CUDA; }
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+ssd_status check_grid(const ssd_grid* g) {
+  if (g == nullptr) return SSD_ERR_INVALID_ARG;
+  if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 1) return SSD_ERR_SHAPE;
+  if (g->row_stride != g->grid_w && g->row_stride != g->grid_w + 1) return SSD_ERR_SHAPE;
+  if ((int64_t)g->grid_h * g->row_stride + g->prefix_len > INT32_MAX / 2) return SSD_ERR_SHAPE;
+  return SSD_OK;
+}
+
+ssd_status check_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                           int32_t D_max, int32_t L_max) {
+  ssd_status s = check_grid(grid);
+  if (s != SSD_OK) return s;
+  if (B < 0 || Hq <= 0 || Hkv <= 0 || D_max <= 0 || L_max <= 0) return SSD_ERR_SHAPE;
+  if (Hq % Hkv != 0) return SSD_ERR_SHAPE;
+  if (d != 64 && d != 128) return SSD_ERR_UNSUPPORTED;
+  if (D_max > 128 || (int64_t)D_max * (Hq / Hkv) > 512) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)B * Hkv > 65535) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)B * Hkv * L_max >= (int64_t)1 << 31) return SSD_ERR_UNSUPPORTED;
+  return SSD_OK;
+}
+
+ssd_status check_accept_common(int32_t rows, int32_t V, float temperature, const ssd_rng* rng,
+                               const int32_t* out_tok, const uint8_t* accepted,
+                               const int32_t* status) {
+  if (rows < 0 || V <= 0) return SSD_ERR_SHAPE;
+  if (rng == nullptr || out_tok == nullptr || accepted == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !isfinite(temperature)) return SSD_ERR_INVALID_ARG;
+  if (rng->uniforms != nullptr && (reinterpret_cast<uintptr_t>(rng->uniforms) & 7u) != 0)
+    return SSD_ERR_INVALID_ARG;  // read as float2
+  return SSD_OK;
+}
+
+ssd_status check_logits(int32_t rows, int32_t V, const float* tgt, const float* drf, int64_t ld) {
+  if (rows == 0) return SSD_OK;
+  if (tgt == nullptr || drf == nullptr) return SSD_ERR_INVALID_ARG;
+  if (V % 4 != 0 || ld % 4 != 0 || ld < V) return SSD_ERR_SHAPE;
+  if (!aligned16(tgt) || !aligned16(drf)) return SSD_ERR_INVALID_ARG;
+  if (!accept_supported(V)) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)rows * 8 > INT32_MAX) return SSD_ERR_UNSUPPORTED;
+  return SSD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t ssd_abi_version(void) { return SSD_ABI_VERSION; }
+
+const char* ssd_status_string(ssd_status s) {
+  switch (s) {
+    case SSD_OK: return "SSD_OK";
+    case SSD_ERR_INVALID_ARG: return "SSD_ERR_INVALID_ARG";
+    case SSD_ERR_SHAPE: return "SSD_ERR_SHAPE";
+    case SSD_ERR_UNSUPPORTED: return "SSD_ERR_UNSUPPORTED";
+    case SSD_ERR_CUDA: return "SSD_ERR_CUDA";
+    case SSD_ERR_TIMEOUT: return "SSD_ERR_TIMEOUT";
+    case SSD_ERR_DEVICE_BOUNDS: return "SSD_ERR_DEVICE_BOUNDS";
+    case SSD_ERR_WORKSPACE: return "SSD_ERR_WORKSPACE";
+  }
+  return "SSD_ERR_UNKNOWN";
+}
+
+ssd_status ssd_frontier(const ssd_grid* grid, int32_t B, const int32_t* cache_len, int32_t D_max,
+                        int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
+                        ssd_stream_t stream) {
+  ssd_status s = check_grid(grid);
+  if (s != SSD_OK) return s;
+  if (grid->row_stride != grid->grid_w) return SSD_ERR_UNSUPPORTED;
+  if (B < 0 || D_max <= 0) return SSD_ERR_SHAPE;
+  if ((int64_t)(grid->k_v + 1) * grid->grid_w > D_max) return SSD_ERR_SHAPE;
+  if (B == 0) return SSD_OK;
+  if (cache_len == nullptr || n_drafts == nullptr || draft_pos == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  return from_cuda(launch_frontier(*grid, B, cache_len, D_max, n_drafts, draft_pos, status,
+                                   (cudaStream_t)stream));
+}
+
+size_t ssd_verify_attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                                      int32_t D_max, int32_t L_max) {
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || D_max <= 0 || L_max <= 0) return 0;
+  return attention_workspace(B, Hq, Hkv, d, D_max, L_max);
+}
+
+ssd_status ssd_verify_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int32_t Hkv,
+                                int32_t d, const int32_t* cache_len, const int32_t* n_drafts,
+                                const int32_t* draft_pos, int32_t D_max, int32_t L_max,
+                                const void* q, const void* k, const void* v, float scale,
+                                void* o, float* lse, void* workspace, size_t workspace_bytes,
+                                int32_t* status, ssd_stream_t stream) {
+  ssd_status s = check_attention(grid, B, Hq, Hkv, d, D_max, L_max);
+  if (s != SSD_OK) return s;
+  if (B == 0) return SSD_OK;
+  if (cache_len == nullptr || n_drafts == nullptr || draft_pos == nullptr || q == nullptr ||
+      k == nullptr || v == nullptr || o == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(q) || !aligned16(o)) return SSD_ERR_INVALID_ARG;
+  if (!(scale >= 0.f) || !isfinite(scale)) return SSD_ERR_INVALID_ARG;
+  const size_t need = attention_workspace(B, Hq, Hkv, d, D_max, L_max);
+  if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
+  AttnArgs a;
+  a.grid = *grid;
+  a.B = B;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.d = d;
+  a.D_max = D_max;
+  a.L_max = L_max;
+  a.cache_len = cache_len;
+  a.n_drafts = n_drafts;
+  a.draft_pos = draft_pos;
+  a.q = q;
+  a.k = k;
+  a.v = v;
+  a.scale = scale;
+  a.o = o;
+  a.lse = lse;
+  a.status = status;
+  return from_cuda(launch_attention(a, workspace, workspace_bytes, (cudaStream_t)stream));
+}
+
+ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
+                      int64_t ld, const int32_t* draft_tok, float temperature, const ssd_rng* rng,
+                      int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
+                      int32_t* status, ssd_stream_t stream) {
+  ssd_status s = check_accept_common(rows, V, temperature, rng, out_tok, accepted, status);
+  if (s != SSD_OK) return s;
+  s = check_logits(rows, V, tgt_logits, drf_logits, ld);
+  if (s != SSD_OK) return s;
+  if (rows == 0) return SSD_OK;
+  AcceptArgs a;
+  a.rows = rows;
+  a.V = V;
+  a.tgt = tgt_logits;
+  a.drf = drf_logits;
+  a.ld = ld;
+  a.draft_tok = draft_tok;
+  a.temperature = temperature;
+  a.rng = *rng;
+  a.out_tok = out_tok;
+  a.accepted = accepted;
+  a.ratio = ratio;
+  a.lse = lse;
+  a.status = status;
+  a.n_drafts = nullptr;
+  a.D_max = 1;
+  return from_cuda(launch_accept(a, (cudaStream_t)stream));
+}
+
+size_t ssd_lmhead_accept_workspace(int32_t rows, int32_t V) {
+  if (rows <= 0 || V <= 0) return 0;
+  return lmhead_workspace(rows, V);
+}
+
+ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_tgt,
+                             const void* h_drf, const void* w_tgt, const void* w_drf,
+                             const int32_t* draft_tok, float temperature, const ssd_rng* rng,
+                             int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
+                             void* workspace, size_t workspace_bytes, int32_t* status,
+                             ssd_stream_t stream) {
+  ssd_status s = check_accept_common(rows, V, temperature, rng, out_tok, accepted, status);
+  if (s != SSD_OK) return s;
+  if (rows == 0) return SSD_OK;
+  s = lmhead_check(rows, V, K);
+  if (s != SSD_OK) return s;
+  if (h_tgt == nullptr || h_drf == nullptr || w_tgt == nullptr || w_drf == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  if (!aligned16(h_tgt) || !aligned16(h_drf) || !aligned16(w_tgt) || !aligned16(w_drf))
+    return SSD_ERR_INVALID_ARG;
+  if (workspace == nullptr || workspace_bytes < lmhead_workspace(rows, V)) return SSD_ERR_WORKSPACE;
+  LmHeadArgs a;
+  a.rows = rows;
+  a.V = V;
+  a.K = K;
+  a.h_tgt = h_tgt;
+  a.h_drf = h_drf;
+  a.w_tgt = w_tgt;
+  a.w_drf = w_drf;
+  a.draft_tok = draft_tok;
+  a.temperature = temperature;
+  a.rng = *rng;
+  a.out_tok = out_tok;
+  a.accepted = accepted;
+  a.ratio = ratio;
+  a.lse = lse;
+  a.status = status;
+  a.n_drafts = nullptr;
+  a.D_max = 1;
+  return from_cuda(launch_lmhead(a, workspace, workspace_bytes, (cudaStream_t)stream));
+}
+
+size_t ssd_verify_step_workspace(const ssd_verify_args* x) {
+  if (x == nullptr || x->B <= 0) return 0;
+  size_t bytes = align256(ssd_verify_attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max,
+                                                         x->L_max));
+  if (x->tgt_logits == nullptr && x->w_tgt != nullptr)
+    bytes += align256(ssd_lmhead_accept_workspace(x->B * x->D_max, x->V));
+  return bytes;
+}
+
+int32_t ssd_verify_step_launches(const ssd_verify_args* x) {
+  if (x == nullptr) return -1;
+  if (check_attention(&x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max) != SSD_OK) return -1;
+  if (x->B == 0) return 0;
+  // frontier + attention (+ split combine) + acceptance + counts
+  return 3 + attention_launches(x->B, x->Hq, x->Hkv, x->D_max, x->L_max);
+}
+
+ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, void* workspace,
+                           size_t workspace_bytes, ssd_stream_t stream_) {
+  if (x == nullptr || y == nullptr) return SSD_ERR_INVALID_ARG;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  ssd_status s = check_attention(&x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max);
+  if (s != SSD_OK) return s;
+  if (x->grid.row_stride != x->grid.grid_w) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)(x->grid.k_v + 1) * x->grid.grid_w > x->D_max) return SSD_ERR_SHAPE;
+  if (x->B == 0) return SSD_OK;
+  if (x->cache_len == nullptr || x->q == nullptr || x->k == nullptr || x->v == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  if (y->n_drafts == nullptr || y->draft_pos == nullptr || y->o == nullptr ||
+      y->out_tok == nullptr || y->accepted == nullptr || y->accepted_count == nullptr ||
+      y->accepted_prefix == nullptr || y->next_cache_len == nullptr || y->status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  const int32_t rows = x->B * x->D_max;
+  s = check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
+  if (s != SSD_OK) return s;
+  const bool fused = (x->tgt_logits == nullptr);
+  if (fused) {
+    if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
+      return SSD_ERR_INVALID_ARG;
+    s = lmhead_check(rows, x->V, x->hidden);
+    if (s != SSD_OK) return s;
+  } else {
+    s = check_logits(rows, x->V, x->tgt_logits, x->drf_logits, x->ld);
+    if (s != SSD_OK) return s;
+  }
+  if (!(x->scale >= 0.f) || !isfinite(x->scale)) return SSD_ERR_INVALID_ARG;
+  const size_t need = ssd_verify_step_workspace(x);
+  if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
+  unsigned char* ws = static_cast<unsigned char*>(workspace);
+  const size_t attn_ws = align256(attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max));
+
+  // a1: frontier
+  cudaError_t e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts, y->draft_pos,
+                                  y->status, stream);
+  if (e != cudaSuccess) return SSD_ERR_CUDA;
+  // a2: attention of the drafted block
+  AttnArgs a;
+  a.grid = x->grid;
+  a.B = x->B;
+  a.Hq = x->Hq;
+  a.Hkv = x->Hkv;
+  a.d = x->d;
+  a.D_max = x->D_max;
+  a.L_max = x->L_max;
+  a.cache_len = x->cache_len;
+  a.n_drafts = y->n_drafts;
+  a.draft_pos = y->draft_pos;
+  a.q = x->q;
+  a.k = x->k;
+  a.v = x->v;
+  a.scale = x->scale;
+  a.o = y->o;
+  a.lse = y->lse;
+  a.status = y->status;
+  e = launch_attention(a, ws, attn_ws, stream);
+  if (e != cudaSuccess) return SSD_ERR_CUDA;
+  // a3-a6: acceptance
+  if (fused) {
+    LmHeadArgs h;
+    h.rows = rows;
+    h.V = x->V;
+    h.K = x->hidden;
+    h.h_tgt = x->h_tgt;
+    h.h_drf = x->h_drf;
+    h.w_tgt = x->w_tgt;
+    h.w_drf = x->w_drf;
+    h.draft_tok = x->draft_tok;
+    h.temperature = x->temperature;
+    h.rng = x->rng;
+    h.out_tok = y->out_tok;
+    h.accepted = y->accepted;
+    h.ratio = y->ratio;
+    h.lse = nullptr;
+    h.status = y->status;
+    h.n_drafts = y->n_drafts;
+    h.D_max = x->D_max;
+    e = launch_lmhead(h, ws + attn_ws, workspace_bytes - attn_ws, stream);
+  } else {
+    AcceptArgs c;
+    c.rows = rows;
+    c.V = x->V;
+    c.tgt = x->tgt_logits;
+    c.drf = x->drf_logits;
+    c.ld = x->ld;
+    c.draft_tok = x->draft_tok;
+    c.temperature = x->temperature;
+    c.rng = x->rng;
+    c.out_tok = y->out_tok;
+    c.accepted = y->accepted;
+    c.ratio = y->ratio;
+    c.lse = nullptr;
+    c.status = y->status;
+    c.n_drafts = y->n_drafts;
+    c.D_max = x->D_max;
+    e = launch_accept(c, stream);
+  }
+  if (e != cudaSuccess) return SSD_ERR_CUDA;
+  // a7: counts and the next cache length
+  e = launch_counts(x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted, y->accepted_count,
+                    y->accepted_prefix, y->next_cache_len, stream);
+  return from_cuda(e);
+}
+
+}  // extern "C"

@@ -1,0 +1,502 @@
+// attention.cu — frontier attention (step a2): every draft query of a
+// sequence attends to the committed KV cache plus the drafted block's own
+// keys under the spatial dependency mask (Sec. 3.3 "Verification as Auto
+// Correction": the drafted block passes through the backbone in parallel;
+// App. "Deviation from AR": a draft's context may hold other drafts).
+//
+//   O[b][j][h] = softmax_s(scale * Q[b][j][h] . K[b][g][s] + M(s, j)) V[b][g][s]
+//   M(s, j) = 0 iff pos(s) <= pos(j), pos(s) = s for cache slots s < cache_len,
+//   pos(cache_len + j') = prefix + y' * row_stride + x' of draft j'.
+//
+// Design (GB300): one CTA per (KV split, sequence b, KV head g, query tile).
+// All draft queries of the KV group (drafts x the Hq/Hkv query heads sharing
+// g) sit in the CTA's warps, 16 query rows per warp, so each K/V tile is
+// read from HBM once per KV head.  K/V tiles of 64 keys are staged by TMA
+// (2D tensor maps, 128-byte swizzle, evict-first L2 policy) through a
+// 3-stage mbarrier ring; QK^T and PV run on the tensor cores (bf16 inputs,
+// fp32 accumulation), the mask predicate is evaluated in registers only on
+// tiles that reach the drafted block, and the softmax is the online
+// (running max / running sum) form with quad shuffles.  Long caches are split
+// over CTAs; a combine kernel merges the splits by their log-sum-exp.
+#include "kernels.cuh"
+
+namespace ssd {
+
+namespace {
+
+constexpr int KT = 64;        // keys per tile
+constexpr int kStages = 3;
+constexpr int kMaxWarps = 8;  // 128 query rows per CTA
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Byte offset of 16-byte chunk `ch` of row `row` inside a [rows x 128 B]
+// TMA box written with CU_TENSOR_MAP_SWIZZLE_128B (1024-byte aligned base).
+__device__ __forceinline__ uint32_t swz(int row, int ch) {
+  return (uint32_t)(row * 128 + ((ch ^ (row & 7)) << 4));
+}
+
+struct AttnLaunch {
+  int32_t splits;        // KV splits (host-chosen)
+  int32_t kps;           // keys per split, multiple of KT
+  int32_t nwarps;        // warps per CTA (16 query rows each)
+  float* part_o;         // [B][Hq][D_max][splits][d] fp32 (splits > 1)
+  float* part_lse;       // [B][Hq][D_max][splits]
+  int32_t* seq_ok;       // [B] 1 if the sequence's inputs were in range
+};
+
+// Validity of one sequence's frontier; identical in every CTA of b.
+__device__ __forceinline__ bool load_draft_positions(const AttnArgs& a, int32_t b, int32_t nd,
+                                                     int32_t* kflat, int32_t* bad) {
+  const int32_t HW = a.grid.grid_h * a.grid.grid_w;
+  for (int32_t j = threadIdx.x; j < nd; j += blockDim.x) {
+    const int32_t gidx = a.draft_pos[(int64_t)b * a.D_max + j];
+    if (gidx < 0 || gidx >= HW) {
+      *bad = 1;
+      kflat[j] = 0;
+    } else {
+      const int32_t y = gidx / a.grid.grid_w, x = gidx - y * a.grid.grid_w;
+      kflat[j] = a.grid.prefix_len + y * a.grid.row_stride + x;
+    }
+  }
+  __syncthreads();
+  return *bad == 0;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kMaxWarps * 32, 1)
+frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                     AttnArgs a, AttnLaunch L) {
+  constexpr int NSUB = D / 64;                 // 128-byte column boxes per row
+  constexpr int TILE_BYTES = KT * D * 2;       // one K (or V) tile
+  constexpr int KSTEPS = D / 16;               // k16 steps of QK^T
+  constexpr int NT_O = D / 8;                  // n8 tiles of O
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  // 1024-byte alignment for the swizzle atoms
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* sK = smem;                                  // [stages][TILE]
+  unsigned char* sV = smem + kStages * TILE_BYTES;           // [stages][TILE]
+  uint64_t* full = reinterpret_cast<uint64_t*>(sV + kStages * TILE_BYTES);
+  int32_t* kflat = reinterpret_cast<int32_t*>(full + kStages);  // [128]
+  int32_t* bad = kflat + 128;
+
+  const int32_t split = blockIdx.x;
+  const int32_t bg = blockIdx.y;
+  const int32_t b = bg / a.Hkv, g = bg - b * a.Hkv;
+  const int32_t G = a.Hq / a.Hkv;
+  const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  const int32_t cache = a.cache_len[b];
+  const int32_t nd = a.n_drafts[b];
+  const int32_t Lk = cache + nd;
+  if (tid == 0) *bad = (nd < 0 || nd > a.D_max || cache < 0 || Lk > a.L_max) ? 1 : 0;
+  __syncthreads();
+  const bool seq_valid = (*bad == 0) && load_draft_positions(a, b, nd, kflat, bad);
+  if (split == 0 && g == 0 && blockIdx.z == 0 && tid == 0) {
+    L.seq_ok[b] = seq_valid ? 1 : 0;
+    if (!seq_valid) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+  }
+  if (!seq_valid || nd == 0) return;
+
+  const int32_t rows_total = nd * G;
+  const int32_t row0 = blockIdx.z * (L.nwarps * 16);
+  if (row0 >= rows_total) return;
+  const int32_t k_lo = split * L.kps;
+  if (k_lo >= Lk) return;
+  const int32_t k_hi = min(Lk, k_lo + L.kps);
+  const int32_t ntiles = (k_hi - k_lo + KT - 1) / KT;
+  const int32_t n_active = (Lk + L.kps - 1) / L.kps;  // splits holding keys of b
+
+  // ---- rows of this warp: r = row0 + warp * 16 + {lane/4, lane/4 + 8}
+  const int32_t wrow = row0 + warp * 16;
+  const bool warp_active = wrow < rows_total;
+  int32_t qpos[2];
+  int32_t rr[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    rr[i] = wrow + (lane >> 2) + 8 * i;
+    qpos[i] = (rr[i] < rows_total) ? kflat[rr[i] / G] : 0x7fffffff;
+  }
+  // first key index whose visibility is not implied (cache slots below every
+  // query position of this CTA are visible to all of its rows)
+  int32_t minq = 0x7fffffff;
+  for (int32_t r = row0; r < min(rows_total, row0 + L.nwarps * 16); ++r)
+    minq = min(minq, kflat[r / G]);
+  const int32_t mask_from = min(cache, minq + 1);
+
+  // ---- Q fragments (A operand of QK^T), straight from global memory
+  uint32_t qf[KSTEPS][4];
+  {
+    const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(a.q);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int32_t r = rr[i];
+      const bool live = r < rows_total;
+      const int32_t j = live ? r / G : 0, h = g * G + (live ? r % G : 0);
+      const uint32_t* src =
+          reinterpret_cast<const uint32_t*>(qb + (((int64_t)b * a.D_max + j) * a.Hq + h) * D);
+#pragma unroll
+      for (int ks = 0; ks < KSTEPS; ++ks) {
+        const int col = ks * 16 + (lane & 3) * 2;
+        qf[ks][i] = live ? src[col / 2] : 0u;
+        qf[ks][2 + i] = live ? src[(col + 8) / 2] : 0u;
+      }
+    }
+  }
+
+  // ---- TMA producer: one thread fills the ring
+  const uint64_t policy = policy_evict_first();
+  const int32_t kvrow0 = (b * a.Hkv + g) * a.L_max;  // row of slot 0 in the 2D view
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+    fence_barrier_init();
+    prefetch_tensormap(&tmK);
+    prefetch_tensormap(&tmV);
+  }
+  __syncthreads();
+  auto issue = [&](int t) {
+    const int s = t % kStages;
+    mbar_arrive_expect_tx(&full[s], 2 * TILE_BYTES);
+    const int32_t row = kvrow0 + k_lo + t * KT;
+#pragma unroll
+    for (int c = 0; c < NSUB; ++c) {
+      tma_load_2d(sK + s * TILE_BYTES + c * (KT * 128), &tmK, c * 64, row, &full[s], policy);
+      tma_load_2d(sV + s * TILE_BYTES + c * (KT * 128), &tmV, c * 64, row, &full[s], policy);
+    }
+  };
+  if (tid == 0) {
+    for (int t = 0; t < min(kStages - 1, ntiles); ++t) issue(t);
+  }
+
+  const float c2 = (a.scale != 0.f ? a.scale : rsqrtf((float)D)) * kLog2e;
+  float o[NT_O][4];
+#pragma unroll
+  for (int n = 0; n < NT_O; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY};
+  float l_run[2] = {0.f, 0.f};
+  bool ok = true;
+
+  for (int t = 0; t < ntiles; ++t) {
+    if (tid == 0 && t + kStages - 1 < ntiles) issue(t + kStages - 1);
+    const int s = t % kStages;
+    if (!mbar_wait(&full[s], (t / kStages) & 1, a.status)) ok = false;
+    if (warp_active && ok) {
+      const uint32_t kbase = smem_u32(sK + s * TILE_BYTES);
+      const uint32_t vbase = smem_u32(sV + s * TILE_BYTES);
+      // ---- S = Q K^T for 16 rows x 64 keys
+      float sc[8][4];
+#pragma unroll
+      for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < KSTEPS; ++ks) {
+        const int sub = ks >> 2, cb = (ks & 3) * 2;
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {  // pairs of n8 tiles: keys np*16 .. +15
+          const int mi = lane >> 3;
+          const int key = np * 16 + (lane & 7) + ((mi >> 1) << 3);
+          const int ch = cb + (mi & 1);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(kbase + sub * (KT * 128) + swz(key, ch), b0, b1, b2, b3);
+          mma_bf16(sc[2 * np], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], b0, b1);
+          mma_bf16(sc[2 * np + 1], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], b2, b3);
+        }
+      }
+      // ---- mask: keys past this split / the sequence, and the spatial predicate
+      const int32_t tile0 = k_lo + t * KT;
+      if (tile0 + KT > k_hi || tile0 + KT > mask_from) {
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int32_t key = tile0 + n * 8 + (lane & 3) * 2 + (e & 1);
+            const int32_t kp = key < cache ? key : (key < Lk ? kflat[key - cache] : 0x7fffffff);
+            const bool vis = key < k_hi && kp <= qpos[e >> 1];
+            if (!vis) sc[n][e] = -INFINITY;
+          }
+        }
+      }
+      // ---- online softmax (rows lane/4 and lane/4 + 8; quads share a row)
+      float alpha[2];
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        float mx = -INFINITY;
+#pragma unroll
+        for (int n = 0; n < 8; ++n) mx = fmaxf(mx, fmaxf(sc[n][2 * i], sc[n][2 * i + 1]));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const float m_new = fmaxf(m_run[i], mx);
+        const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+        alpha[i] = exp2f((m_run[i] - m_use) * c2);  // 0 when nothing was accumulated
+        m_run[i] = m_new;
+        const float moff = m_use * c2;
+        float rs = 0.f;
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+          sc[n][2 * i] = exp2f(fmaf(sc[n][2 * i], c2, -moff));
+          sc[n][2 * i + 1] = exp2f(fmaf(sc[n][2 * i + 1], c2, -moff));
+          rs += sc[n][2 * i] + sc[n][2 * i + 1];
+        }
+        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+        l_run[i] = l_run[i] * alpha[i] + rs;
+      }
+#pragma unroll
+      for (int n = 0; n < NT_O; ++n) {
+        o[n][0] *= alpha[0];
+        o[n][1] *= alpha[0];
+        o[n][2] *= alpha[1];
+        o[n][3] *= alpha[1];
+      }
+      // ---- O += P V (P re-packed from the S accumulators as A fragments)
+#pragma unroll
+      for (int kk = 0; kk < KT / 16; ++kk) {
+        const uint32_t a0 = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
+        const uint32_t a1 = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
+        const uint32_t a2 = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+        const uint32_t a3 = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+        for (int np = 0; np < NT_O / 2; ++np) {  // pairs of n8 tiles: d cols np*16 .. +15
+          const int mi = lane >> 3;
+          const int key = kk * 16 + (lane & 7) + ((mi & 1) << 3);
+          const int dc = np * 16 + ((mi >> 1) << 3);  // first d column of the 8x8 block
+          const int sub = dc >> 6, ch = (dc & 63) >> 3;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(vbase + sub * (KT * 128) + swz(key, ch), b0, b1, b2, b3);
+          mma_bf16(o[2 * np], a0, a1, a2, a3, b0, b1);
+          mma_bf16(o[2 * np + 1], a0, a1, a2, a3, b2, b3);
+        }
+      }
+    }
+    // stage s is free for the producer; a timed-out wait anywhere stops every thread
+    if (!__syncthreads_and(ok)) { ok = false; break; }
+  }
+  if (!ok || !warp_active) return;
+
+  // ---- epilogue: normalise, write O (bf16) or the split partial (fp32)
+  const bool direct = (n_active == 1);
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int32_t r = rr[i];
+    if (r >= rows_total) continue;
+    const int32_t j = r / G, h = g * G + r % G;
+    const float inv_l = l_run[i] > 0.f ? 1.0f / l_run[i] : 0.f;
+    const float lse = (l_run[i] > 0.f) ? (m_run[i] * (c2 / kLog2e) + logf(l_run[i])) : -INFINITY;
+    if (direct) {
+      __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.o) +
+                          (((int64_t)b * a.D_max + j) * a.Hq + h) * D;
+#pragma unroll
+      for (int n = 0; n < NT_O; ++n) {
+        const int col = n * 8 + (lane & 3) * 2;
+        *reinterpret_cast<uint32_t*>(ob + col) =
+            pack_bf16x2(o[n][2 * i] * inv_l, o[n][2 * i + 1] * inv_l);
+      }
+      if (a.lse != nullptr && (lane & 3) == 0)
+        a.lse[((int64_t)b * a.Hq + h) * a.D_max + j] = lse;
+    } else {
+      const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + j) * L.splits + split;
+      float* po = L.part_o + prow * D;
+#pragma unroll
+      for (int n = 0; n < NT_O; ++n) {
+        const int col = n * 8 + (lane & 3) * 2;
+        *reinterpret_cast<float2*>(po + col) = make_float2(o[n][2 * i] * inv_l, o[n][2 * i + 1] * inv_l);
+      }
+      if ((lane & 3) == 0) L.part_lse[prow] = lse;
+    }
+  }
+}
+
+// One warp per (b, j, h) row: merge the active splits by log-sum-exp.
+template <int D>
+__global__ void attn_combine_kernel(AttnArgs a, AttnLaunch L) {
+  const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int32_t lane = threadIdx.x & 31;
+  const int64_t total = (int64_t)a.B * a.D_max * a.Hq;
+  if (gw >= total) return;
+  const int32_t h = (int32_t)(gw % a.Hq);
+  const int32_t j = (int32_t)((gw / a.Hq) % a.D_max);
+  const int32_t b = (int32_t)(gw / ((int64_t)a.Hq * a.D_max));
+  if (!L.seq_ok[b]) return;
+  const int32_t nd = a.n_drafts[b];
+  if (j >= nd) return;
+  const int32_t Lk = a.cache_len[b] + nd;
+  const int32_t n_active = (Lk + L.kps - 1) / L.kps;
+  if (n_active <= 1) return;  // written directly by the attention kernel
+  const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + j) * L.splits;
+  float mx = -INFINITY;
+  for (int s = 0; s < n_active; ++s) mx = fmaxf(mx, L.part_lse[prow + s]);
+  constexpr int PER = D / 32;
+  float acc[PER];
+#pragma unroll
+  for (int k = 0; k < PER; ++k) acc[k] = 0.f;
+  float wsum = 0.f;
+  for (int s = 0; s < n_active; ++s) {
+    const float ls = L.part_lse[prow + s];
+    const float w = (ls == -INFINITY) ? 0.f : expf(ls - mx);
+    wsum += w;
+    const float* po = L.part_o + (prow + s) * D + lane * PER;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) acc[k] += w * po[k];
+  }
+  const float inv = 1.0f / wsum;
+  __nv_bfloat16* ob =
+      reinterpret_cast<__nv_bfloat16*>(a.o) + (((int64_t)b * a.D_max + j) * a.Hq + h) * D + lane * PER;
+#pragma unroll
+  for (int k = 0; k < PER; k += 2)
+    *reinterpret_cast<uint32_t*>(ob + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
+  if (a.lse != nullptr && lane == 0) a.lse[((int64_t)b * a.Hq + h) * a.D_max + j] = mx + logf(wsum);
+}
+
+// ------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2D view [rows, d] of a bf16 [B][Hkv][L_max][d] tensor, box [KT rows x 64 cols].
+bool make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int32_t d) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  cuuint32_t box[2] = {64, KT};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Plan {
+  int32_t nwarps, mtiles, splits, kps;
+};
+
+Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
+  Plan p;
+  const int32_t G = Hq / Hkv;
+  const int32_t rows = D_max * G;
+  p.nwarps = min(kMaxWarps, (rows + 15) / 16);
+  p.mtiles = (rows + p.nwarps * 16 - 1) / (p.nwarps * 16);
+  const int64_t base = (int64_t)B * Hkv * p.mtiles;
+  const int32_t target = 2 * device_sm_count();
+  const int32_t max_splits = max(1, (L_max + 2 * KT - 1) / (2 * KT));  // >= 2 tiles per split
+  int32_t splits = (int32_t)((target + base - 1) / base);
+  splits = max(1, min(splits, max_splits));
+  int32_t kps = (L_max + splits - 1) / splits;
+  kps = ((kps + KT - 1) / KT) * KT;
+  p.splits = (L_max + kps - 1) / kps;
+  p.kps = kps;
+  return p;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+}  // namespace
+
+int device_sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  return n;
+}
+
+size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
+                           int32_t L_max) {
+  const Plan p = make_plan(B, Hq, Hkv, D_max, L_max);
+  size_t bytes = align256((size_t)B * sizeof(int32_t));
+  if (p.splits > 1) {
+    const size_t prow = (size_t)B * Hq * D_max * p.splits;
+    bytes += align256(prow * d * sizeof(float)) + align256(prow * sizeof(float));
+  }
+  return bytes;
+}
+
+int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
+  if (B == 0) return 0;
+  return make_plan(B, Hq, Hkv, D_max, L_max).splits > 1 ? 2 : 1;
+}
+
+cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (a.B == 0) return cudaSuccess;
+  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.D_max, a.L_max);
+  AttnLaunch L;
+  L.splits = p.splits;
+  L.kps = p.kps;
+  L.nwarps = p.nwarps;
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  L.seq_ok = reinterpret_cast<int32_t*>(w);
+  w += align256((size_t)a.B * sizeof(int32_t));
+  L.part_o = nullptr;
+  L.part_lse = nullptr;
+  if (p.splits > 1) {
+    const size_t prow = (size_t)a.B * a.Hq * a.D_max * p.splits;
+    L.part_o = reinterpret_cast<float*>(w);
+    w += align256(prow * a.d * sizeof(float));
+    L.part_lse = reinterpret_cast<float*>(w);
+  }
+  CUtensorMap tmK, tmV;
+  const int64_t rows = (int64_t)a.B * a.Hkv * a.L_max;
+  if (!make_kv_map(&tmK, a.k, rows, a.d) || !make_kv_map(&tmV, a.v, rows, a.d))
+    return cudaErrorInvalidValue;
+  const dim3 grid(p.splits, a.B * a.Hkv, p.mtiles);
+  const dim3 block(p.nwarps * 32);
+  cudaError_t e;
+  if (a.d == 128) {
+    const size_t smem = 1024 + kStages * 2 * (KT * 128 * 2) + kStages * 8 + 129 * 4;
+    e = cudaFuncSetAttribute(frontier_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    frontier_attn_kernel<128><<<grid, block, smem, stream>>>(tmK, tmV, a, L);
+  } else {
+    const size_t smem = 1024 + kStages * 2 * (KT * 64 * 2) + kStages * 8 + 129 * 4;
+    e = cudaFuncSetAttribute(frontier_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    frontier_attn_kernel<64><<<grid, block, smem, stream>>>(tmK, tmV, a, L);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess || p.splits == 1) return e;
+  const int64_t rows_c = (int64_t)a.B * a.D_max * a.Hq;
+  const int wpb = 8;
+  const unsigned blocks = (unsigned)((rows_c + wpb - 1) / wpb);
+  if (a.d == 128)
+    attn_combine_kernel<128><<<blocks, wpb * 32, 0, stream>>>(a, L);
+  else
+    attn_combine_kernel<64><<<blocks, wpb * 32, 0, stream>>>(a, L);
+  return cudaGetLastError();
+}
+
+}  // namespace ssd

@@ -1,0 +1,100 @@
+// frontier.cu — the drafted frontier (step a1) and the accepted counts /
+// next cache length (step a7) of one verification step.
+//
+// Frontier (Sec. 3.3): the horizontal heads complete the current grid row,
+// the vertical heads draft the k_v rows below it in one column-parallel step.
+// With n_c committed grid tokens and the first uncommitted one at
+// (y0, c) = (n_c / W, n_c % W), the frontier is the next
+// (W - c) + k_v * W raster positions, clipped at the last grid row.
+//
+// Counts (Sec. 3.3 and Sec. 4 "SSD Configuration", one verification round):
+// the drafts up to and including the first rejected one are committed, the
+// rejected one carrying its resampled token.
+#include "kernels.cuh"
+
+namespace ssd {
+
+__device__ __forceinline__ int32_t frontier_size(const ssd_grid& g, int32_t n_c) {
+  const int32_t y0 = n_c / g.grid_w;
+  const int32_t c = n_c - y0 * g.grid_w;
+  if (y0 >= g.grid_h) return 0;
+  const int32_t rows_below = min(g.k_v, g.grid_h - 1 - y0);
+  return (g.grid_w - c) + rows_below * g.grid_w;
+}
+
+// One block per sequence.  Writes n_drafts[b] and draft_pos[b][0..D_max).
+__global__ void frontier_kernel(ssd_grid g, const int32_t* __restrict__ cache_len, int32_t D_max,
+                                int32_t* __restrict__ n_drafts, int32_t* __restrict__ draft_pos,
+                                int32_t* status) {
+  const int32_t b = blockIdx.x;
+  const int32_t n_c = cache_len[b] - g.prefix_len;
+  int32_t n = 0;
+  if (n_c < 0 || n_c > g.grid_h * g.grid_w) {
+    if (threadIdx.x == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
+  } else {
+    n = frontier_size(g, n_c);
+    if (n > D_max) {  // host checks D_max >= (k_v + 1) * W; keep the guard
+      if (threadIdx.x == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
+      n = 0;
+    }
+  }
+  if (threadIdx.x == 0) n_drafts[b] = n;
+  for (int32_t j = threadIdx.x; j < D_max; j += blockDim.x)
+    draft_pos[(int64_t)b * D_max + j] = (j < n) ? (n_c + j) : -1;
+}
+
+// One warp per sequence: accepted count, leading accepted run, next length.
+__global__ void counts_kernel(int32_t B, int32_t D_max, const int32_t* __restrict__ cache_len,
+                              const int32_t* __restrict__ n_drafts,
+                              const uint8_t* __restrict__ accepted,
+                              int32_t* __restrict__ accepted_count,
+                              int32_t* __restrict__ accepted_prefix,
+                              int32_t* __restrict__ next_cache_len) {
+  const int32_t b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int32_t lane = threadIdx.x & 31;
+  if (b >= B) return;
+  const int32_t n = n_drafts[b];
+  int32_t count = 0, prefix = 0;
+  bool run = true;  // still inside the leading accepted run
+  for (int32_t j0 = 0; j0 < n; j0 += 32) {
+    const int32_t j = j0 + lane;
+    const bool a = (j < n) && accepted[(int64_t)b * D_max + j] != 0;
+    const uint32_t acc_mask = __ballot_sync(0xffffffffu, a);
+    count += __popc(acc_mask);
+    if (run) {
+      const uint32_t valid = (n - j0 >= 32) ? 0xffffffffu : ((1u << (n - j0)) - 1u);
+      const uint32_t rejected = valid & ~acc_mask;
+      if (rejected) {
+        prefix += __ffs(rejected) - 1;
+        run = false;
+      } else {
+        prefix += __popc(valid);
+      }
+    }
+  }
+  if (lane == 0) {
+    accepted_count[b] = count;
+    accepted_prefix[b] = prefix;
+    next_cache_len[b] = cache_len[b] + (n > 0 ? min(prefix + 1, n) : 0);
+  }
+}
+
+cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
+                            int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
+                            cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  frontier_kernel<<<B, 128, 0, stream>>>(g, cache_len, D_max, n_drafts, draft_pos, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_counts(int32_t B, int32_t D_max, const int32_t* cache_len,
+                          const int32_t* n_drafts, const uint8_t* accepted, int32_t* accepted_count,
+                          int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  const int warps = 4;
+  counts_kernel<<<(B + warps - 1) / warps, warps * 32, 0, stream>>>(
+      B, D_max, cache_len, n_drafts, accepted, accepted_count, accepted_prefix, next_cache_len);
+  return cudaGetLastError();
+}
+
+}  // namespace ssd

@@ -1,0 +1,81 @@
+// kernels.cuh — internal launch interface between the C ABI (api.cu) and the
+// kernels.  Not installed; callers use include/ssd.h.
+#pragma once
+
+#include "common.cuh"
+
+namespace ssd {
+
+// ---- frontier.cu
+cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
+                            int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
+                            cudaStream_t stream);
+cudaError_t launch_counts(int32_t B, int32_t D_max, const int32_t* cache_len,
+                          const int32_t* n_drafts, const uint8_t* accepted, int32_t* accepted_count,
+                          int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream);
+
+// ---- accept.cu
+struct AcceptArgs {
+  int32_t rows, V;
+  const float* tgt;
+  const float* drf;
+  int64_t ld;
+  const int32_t* draft_tok;  // nullable
+  float temperature;
+  ssd_rng rng;
+  int32_t* out_tok;
+  uint8_t* accepted;
+  float* ratio;              // nullable
+  float* lse;                // nullable
+  int32_t* status;
+  const int32_t* n_drafts;   // nullable: row r valid iff r % D_max < n_drafts[r / D_max]
+  int32_t D_max;
+};
+bool accept_supported(int32_t V);
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);
+
+// ---- attention.cu
+struct AttnArgs {
+  ssd_grid grid;
+  int32_t B, Hq, Hkv, d, D_max, L_max;
+  const int32_t* cache_len;
+  const int32_t* n_drafts;
+  const int32_t* draft_pos;
+  const void* q;
+  const void* k;
+  const void* v;
+  float scale;
+  void* o;
+  float* lse;  // nullable
+  int32_t* status;
+};
+size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
+                           int32_t L_max);
+cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
+int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
+
+// ---- lmhead.cu
+struct LmHeadArgs {
+  int32_t rows, V, K;
+  const void* h_tgt;
+  const void* h_drf;
+  const void* w_tgt;
+  const void* w_drf;
+  const int32_t* draft_tok;
+  float temperature;
+  ssd_rng rng;
+  int32_t* out_tok;
+  uint8_t* accepted;
+  float* ratio;
+  float* lse;
+  int32_t* status;
+  const int32_t* n_drafts;  // nullable, as AcceptArgs
+  int32_t D_max;
+};
+size_t lmhead_workspace(int32_t rows, int32_t V);
+ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K);
+cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+int device_sm_count();
+
+}  // namespace ssd

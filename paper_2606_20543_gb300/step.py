@@ -1,0 +1,160 @@
+"""Device buffers for one verification problem shape and the calls that run
+it through ``ssd_verify_step`` — the public API a caller uses end to end.
+
+Marshalling only: host arrays (numpy or torch, pinned or not) are copied to
+preallocated device tensors, the C-ABI entry point runs every step of the
+pass, and results are copied back on request.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import (Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid, ssd_verify_step,
+               ssd_verify_step_workspace)
+
+
+def _dev(shape, dtype, device):
+    return torch.empty(shape, dtype=dtype, device=device)
+
+
+def _as_torch(x, dtype):
+    if isinstance(x, torch.Tensor):
+        return x
+    x = np.ascontiguousarray(x)
+    if dtype == torch.bfloat16:
+        return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
+    return torch.from_numpy(x)
+
+
+class VerifyStep:
+    """Preallocated inputs, outputs and workspace for ssd_verify_step.
+
+    Shapes follow include/ssd.h: q [B, D_max, Hq, d], k/v [B, Hkv, L_max, d]
+    (bf16), logits [B*D_max, V] (float32) or hidden [B*D_max, hidden] with
+    lm_head weights [hidden, V] (bf16)."""
+
+    def __init__(self, grid_h, grid_w, prefix_len, B, Hq, Hkv, d, D_max, L_max, V,
+                 hidden=0, k_v=1, row_stride=None, device="cuda", scale=0.0, temperature=1.0):
+        self.g: Grid = make_grid(grid_h, grid_w, prefix_len, row_stride, k_v)
+        self.B, self.Hq, self.Hkv, self.d = B, Hq, Hkv, d
+        self.D_max, self.L_max, self.V, self.hidden = D_max, L_max, V, hidden
+        self.device = device
+        self.scale, self.temperature = scale, temperature
+        rows = B * D_max
+        self.rows = rows
+        dv = device
+        self.cache_len = _dev((B,), torch.int32, dv)
+        self.q = _dev((B, D_max, Hq, d), torch.bfloat16, dv)
+        self.k = _dev((B, Hkv, L_max, d), torch.bfloat16, dv)
+        self.v = _dev((B, Hkv, L_max, d), torch.bfloat16, dv)
+        if hidden:
+            self.tgt = self.drf = None
+            self.h_tgt = _dev((rows, hidden), torch.bfloat16, dv)
+            self.h_drf = _dev((rows, hidden), torch.bfloat16, dv)
+            self.w_tgt = _dev((hidden, V), torch.bfloat16, dv)
+            self.w_drf = _dev((hidden, V), torch.bfloat16, dv)
+        else:
+            self.tgt = _dev((rows, V), torch.float32, dv)
+            self.drf = _dev((rows, V), torch.float32, dv)
+            self.h_tgt = self.h_drf = self.w_tgt = self.w_drf = None
+        self.uniforms = None
+        self.draft_tok = None
+        # outputs
+        self.n_drafts = _dev((B,), torch.int32, dv)
+        self.draft_pos = _dev((B, D_max), torch.int32, dv)
+        self.o = torch.zeros((B, D_max, Hq, d), dtype=torch.bfloat16, device=dv)
+        self.lse = _dev((B, Hq, D_max), torch.float32, dv)
+        self.out_tok = _dev((rows,), torch.int32, dv)
+        self.accepted = _dev((rows,), torch.uint8, dv)
+        self.ratio = _dev((rows,), torch.float32, dv)
+        self.accepted_count = _dev((B,), torch.int32, dv)
+        self.accepted_prefix = _dev((B,), torch.int32, dv)
+        self.next_cache_len = _dev((B,), torch.int32, dv)
+        self.status = torch.zeros((1,), dtype=torch.int32, device=dv)
+        self.rng = Rng(0, 0, None)
+        self.args = self._args()
+        self.ws_bytes = ssd_verify_step_workspace(self.args)
+        self.workspace = _dev((max(self.ws_bytes, 256),), torch.uint8, dv)
+        self.out = self._out()
+
+    # ------------------------------------------------------------------ args
+    def _args(self) -> VerifyArgs:
+        a = VerifyArgs()
+        a.grid = self.g
+        a.B, a.Hq, a.Hkv, a.d = self.B, self.Hq, self.Hkv, self.d
+        a.D_max, a.L_max, a.V = self.D_max, self.L_max, self.V
+        a.cache_len = self.cache_len.data_ptr()
+        a.q, a.k, a.v = self.q.data_ptr(), self.k.data_ptr(), self.v.data_ptr()
+        a.scale = self.scale
+        if self.hidden:
+            a.tgt_logits = a.drf_logits = None
+            a.ld = 0
+            a.h_tgt, a.h_drf = self.h_tgt.data_ptr(), self.h_drf.data_ptr()
+            a.w_tgt, a.w_drf = self.w_tgt.data_ptr(), self.w_drf.data_ptr()
+            a.hidden = self.hidden
+        else:
+            a.tgt_logits, a.drf_logits = self.tgt.data_ptr(), self.drf.data_ptr()
+            a.ld = self.V
+            a.h_tgt = a.h_drf = a.w_tgt = a.w_drf = None
+            a.hidden = 0
+        a.draft_tok = None if self.draft_tok is None else self.draft_tok.data_ptr()
+        a.temperature = self.temperature
+        a.rng = self.rng
+        return a
+
+    def _out(self) -> VerifyOut:
+        y = VerifyOut()
+        y.n_drafts, y.draft_pos = self.n_drafts.data_ptr(), self.draft_pos.data_ptr()
+        y.o, y.lse = self.o.data_ptr(), self.lse.data_ptr()
+        y.out_tok, y.accepted = self.out_tok.data_ptr(), self.accepted.data_ptr()
+        y.ratio = self.ratio.data_ptr()
+        y.accepted_count = self.accepted_count.data_ptr()
+        y.accepted_prefix = self.accepted_prefix.data_ptr()
+        y.next_cache_len = self.next_cache_len.data_ptr()
+        y.status = self.status.data_ptr()
+        return y
+
+    # ----------------------------------------------------------------- inputs
+    def upload(self, cache_len=None, q=None, k=None, v=None, tgt_logits=None, drf_logits=None,
+               h_tgt=None, h_drf=None, w_tgt=None, w_drf=None, uniforms=None, draft_tok=None,
+               non_blocking=False):
+        """Copy host arrays into the device buffers (bf16 given as uint16 bits
+        or torch.bfloat16).  Arguments left None keep their current contents."""
+        pairs = [(cache_len, self.cache_len, torch.int32), (q, self.q, torch.bfloat16),
+                 (k, self.k, torch.bfloat16), (v, self.v, torch.bfloat16),
+                 (tgt_logits, self.tgt, torch.float32), (drf_logits, self.drf, torch.float32),
+                 (h_tgt, self.h_tgt, torch.bfloat16), (h_drf, self.h_drf, torch.bfloat16),
+                 (w_tgt, self.w_tgt, torch.bfloat16), (w_drf, self.w_drf, torch.bfloat16)]
+        for src, dst, dt in pairs:
+            if src is not None:
+                dst.copy_(_as_torch(src, dt).reshape(dst.shape), non_blocking=non_blocking)
+        if uniforms is not None:
+            if self.uniforms is None:
+                self.uniforms = _dev((self.rows, 2), torch.float32, self.device)
+            self.uniforms.copy_(_as_torch(uniforms, torch.float32).reshape(self.rows, 2),
+                                non_blocking=non_blocking)
+            self.rng.uniforms = self.uniforms.data_ptr()
+        if draft_tok is not None:
+            self.draft_tok = _dev((self.rows,), torch.int32, self.device)
+            self.draft_tok.copy_(_as_torch(draft_tok, torch.int32).reshape(-1))
+            self.args = self._args()
+        self.args.rng = self.rng
+
+    def set_rng(self, seed: int, offset: int, use_uniforms: bool = False):
+        self.rng.seed, self.rng.offset = seed, offset
+        if not use_uniforms:
+            self.rng.uniforms = None
+        self.args.rng = self.rng
+
+    # -------------------------------------------------------------------- run
+    def run(self, stream=None) -> None:
+        ssd_verify_step(self.args, self.out, self.workspace, self.ws_bytes, stream)
+
+    def results(self) -> dict:
+        names = ["n_drafts", "draft_pos", "out_tok", "accepted", "ratio", "accepted_count",
+                 "accepted_prefix", "next_cache_len", "status"]
+        r = {n: getattr(self, n).cpu().numpy() for n in names}
+        r["o"] = self.o.float().cpu().numpy()
+        r["lse"] = self.lse.cpu().numpy()
+        return r

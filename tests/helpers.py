@@ -1,0 +1,45 @@
+"""Shared helpers of the GPU parity tests: upload a synth.Case, run the CUDA
+path through the C ABI, compare with the oracle."""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+
+ATTN_TOL = 2e-2     # normwise max relative error per (b, h), bf16 inputs
+PROB_TOL = 1e-5     # relative error of ratio / log-sum-exp, fp32 logits path
+
+
+def bf16_to_f64(bits):
+    return synth.bf16_bits_to_f32(bits).astype(np.float64)
+
+
+def attention_error(o_gpu, o_ref):
+    """max |gpu - ref| / max |ref| over one (b, h) block."""
+    den = np.abs(o_ref).max()
+    return np.abs(o_gpu - o_ref).max() / max(den, 1e-6)
+
+
+def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what=""):
+    """Bit-exact comparison of accept flags and tokens, except near-tie rows.
+
+    dec: oracle accept_rows() dict for the compared rows; out_tok/accepted:
+    the GPU's values for the same rows.  Returns the number of excused rows."""
+    tie = dec["tie_accept"] | dec["tie_resample"]
+    acc_g = accepted.astype(bool)
+    ok_acc = (acc_g == dec["accepted"]) | tie
+    ok_tok = (out_tok == dec["out_tok"]) | tie
+    bad = np.nonzero(~(ok_acc & ok_tok))[0]
+    assert bad.size == 0, (f"{what}: {bad.size} rows differ, first {bad[:5]}: gpu tok "
+                           f"{out_tok[bad[:5]]} acc {acc_g[bad[:5]]}, oracle tok "
+                           f"{dec['out_tok'][bad[:5]]} acc {dec['accepted'][bad[:5]]}")
+    if ratio is not None:
+        ref = dec["ratio"]
+        fin = np.isfinite(ref) & (ref < 1e30)
+        rel = np.abs(ratio[fin] - ref[fin]) / np.maximum(np.abs(ref[fin]), 1e-30)
+        assert rel.max(initial=0) < PROB_TOL, f"{what}: ratio rel err {rel.max()}"
+    if lse is not None:
+        for k, key in enumerate(("lse_p", "lse_q")):
+            rel = np.abs(lse[:, k] - dec[key]) / np.abs(dec[key])
+            assert rel.max(initial=0) < PROB_TOL, f"{what}: {key} rel err {rel.max()}"
+    return int(tie.sum())

@@ -1,0 +1,86 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/ssd.h declares; host-side argument checks return their codes without
+touching a GPU."""
+import ctypes
+import os
+import re
+import shutil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "ssd.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2606_20543_gb300 import build
+    build.build()
+    import paper_2606_20543_gb300 as ssd
+    return ssd
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ssd_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("ssd_verify_attention", "ssd_accept", "ssd_verify_step", "ssd_frontier",
+                     "ssd_lmhead_accept"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = ctypes.CDLL(lib.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(so, name), name
+    assert set(declared_functions()) == set(lib.EXPORTED)
+
+
+def test_abi_version_and_status_strings(lib):
+    assert lib.ssd_abi_version() == 1
+    for code, name in lib.STATUS_NAMES.items():
+        assert lib.ssd_status_string(code) == name
+
+
+def test_host_side_validation(lib):
+    so = lib.load()
+    g = lib.grid(16, 16, 32)
+    r = lib.rng(0, 0)
+    P = ctypes.c_void_p
+    fake = P(0x1000)  # never dereferenced: every call below fails its checks first
+    # bad head_dim / group / D_max
+    assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 8, 96, fake, fake, fake, 32, 288, fake,
+                                   fake, fake, 0.0, fake, None, fake, 1 << 20, fake, None) == 3
+    assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 3, 64, fake, fake, fake, 32, 288, fake,
+                                   fake, fake, 0.0, fake, None, fake, 1 << 20, fake, None) == 2
+    assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 8, 64, fake, fake, fake, 200, 288, fake,
+                                   fake, fake, 0.0, fake, None, fake, 1 << 20, fake, None) == 3
+    # null pointers
+    assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 8, 64, None, fake, fake, 32, 288, fake,
+                                   fake, fake, 0.0, fake, None, fake, 1 << 20, fake, None) == 1
+    # accept: vocabulary not a multiple of 4, bad temperature, null rng
+    assert so.ssd_accept(4, 4098, fake, fake, 4100, None, 1.0, ctypes.byref(r), fake, fake, None,
+                         None, fake, None) == 2
+    assert so.ssd_accept(4, 4096, fake, fake, 4096, None, 0.0, ctypes.byref(r), fake, fake, None,
+                         None, fake, None) == 1
+    assert so.ssd_accept(4, 4096, fake, fake, 4096, None, 1.0, None, fake, fake, None, None, fake,
+                         None) == 1
+    # misaligned logits
+    assert so.ssd_accept(4, 4096, P(0x1004), fake, 4096, None, 1.0, ctypes.byref(r), fake, fake,
+                         None, None, fake, None) == 1
+    # zero rows is a no-op
+    assert so.ssd_accept(0, 4096, None, None, 4096, None, 1.0, ctypes.byref(r), fake, fake, None,
+                         None, fake, None) == 0
+    # frontier: D_max too small for (k_v + 1) * W, end-of-line stride unsupported
+    assert so.ssd_frontier(ctypes.byref(g), 1, fake, 31, fake, fake, fake, None) == 2
+    g2 = lib.grid(16, 16, 32, row_stride=17)
+    assert so.ssd_frontier(ctypes.byref(g2), 1, fake, 32, fake, fake, fake, None) == 3
+    # workspace too small
+    assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 8, 64, fake, fake, fake, 32, 288, fake,
+                                   fake, fake, 0.0, fake, None, None, 0, fake, None) == 7

@@ -1,0 +1,139 @@
+"""GPU parity of the acceptance kernel (steps a3-a5) against the oracle:
+decisions and tokens bit-exact except counted near-ties, ratio and
+log-sum-exp within 1e-5 relative."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import accept as oacc
+from tests.helpers import compare_decisions
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ssd():
+    import paper_2606_20543_gb300 as m
+    from paper_2606_20543_gb300 import build
+    build.build()
+    m.load()
+    return m
+
+
+def run_accept(ssd, tgt, drf, uniforms=None, seed=0, offset=0, draft_tok=None, T=1.0, ld=None):
+    rows, V = tgt.shape
+    ld = V if ld is None else ld
+    dev = "cuda"
+    tg = torch.zeros((rows, ld), dtype=torch.float32, device=dev)
+    dg = torch.zeros((rows, ld), dtype=torch.float32, device=dev)
+    tg[:, :V] = torch.from_numpy(np.ascontiguousarray(tgt))
+    dg[:, :V] = torch.from_numpy(np.ascontiguousarray(drf))
+    u = None if uniforms is None else torch.from_numpy(uniforms).to(dev)
+    dt = None if draft_tok is None else torch.from_numpy(draft_tok.astype(np.int32)).to(dev)
+    out_tok = torch.full((rows,), -7, dtype=torch.int32, device=dev)
+    acc = torch.full((rows,), 7, dtype=torch.uint8, device=dev)
+    ratio = torch.zeros((rows,), dtype=torch.float32, device=dev)
+    lse = torch.zeros((rows, 2), dtype=torch.float32, device=dev)
+    status = torch.zeros((1,), dtype=torch.int32, device=dev)
+    ssd.ssd_accept(rows, V, tg, dg, ld, dt, T, ssd.rng(seed, offset, u), out_tok, acc, ratio, lse,
+                   status)
+    torch.cuda.synchronize()
+    return (out_tok.cpu().numpy(), acc.cpu().numpy(), ratio.cpu().numpy(), lse.cpu().numpy(),
+            int(status.item()))
+
+
+@pytest.mark.parametrize("V,rows,logits,seed", [
+    (4096, 64, "normal", 0),      # one CTA per row
+    (16384, 48, "normal", 1),     # cluster of 4
+    (16384, 40, "zipf", 2),       # skewed draft vs perturbed target
+    (4100, 30, "normal", 3),      # ragged: 2 CTAs, uneven slices
+    (65536, 8, "zipf", 4),        # cluster of 8
+    (12, 16, "normal", 5),        # tiny vocabulary
+])
+def test_accept_matches_oracle(ssd, V, rows, logits, seed):
+    rng = np.random.default_rng(seed)
+    if logits == "normal":
+        tgt, drf = synth._logits_normal(rng, rows, V)
+    else:
+        tgt, drf = synth._logits_zipf(rng, rows, V)
+    u = synth.philox_uniforms(seed, 11, rows)
+    tok, acc, ratio, lse, st = run_accept(ssd, tgt, drf, u)
+    assert st == 0
+    dec = oacc.accept_rows(tgt, drf, u)
+    ties = compare_decisions(dec, tok, acc, ratio, lse, what=f"V={V}")
+    assert ties <= max(2, rows // 10)
+
+
+def test_device_philox_matches_generator(ssd):
+    """uniforms=NULL draws Philox4x32-10 on the device; it must reproduce the
+    generator's stream bit for bit, so both runs decide identically."""
+    rng = np.random.default_rng(7)
+    rows, V = 512, 4096
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    a = run_accept(ssd, tgt, drf, synth.philox_uniforms(1234567890123, 99, rows))
+    b = run_accept(ssd, tgt, drf, None, seed=1234567890123, offset=99)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+    # and the decisions really depend on the uniforms
+    c = run_accept(ssd, tgt, drf, None, seed=1234567890123, offset=100)
+    assert not np.array_equal(a[0], c[0])
+
+
+def test_given_draft_token_and_temperature(ssd):
+    rng = np.random.default_rng(8)
+    rows, V = 64, 8192
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    dt = rng.integers(0, V, rows).astype(np.int64)
+    u = synth.philox_uniforms(5, 0, rows)
+    for T in (1.0, 0.7):
+        tok, acc, ratio, lse, st = run_accept(ssd, tgt, drf, u, draft_tok=dt, T=T)
+        assert st == 0
+        dec = oacc.accept_rows(tgt, drf, u, draft_tok=dt, temperature=T)
+        compare_decisions(dec, tok, acc, ratio, lse, what=f"T={T}")
+
+
+def test_identical_distributions_all_accepted(ssd):
+    rng = np.random.default_rng(9)
+    rows, V = 64, 16384
+    l = (rng.standard_normal((rows, V)) * 2).astype(np.float32)
+    u = synth.philox_uniforms(3, 0, rows)
+    u[:, 0] = 1 - 2**-24
+    tok, acc, ratio, _, st = run_accept(ssd, l, l.copy(), u)
+    assert st == 0 and acc.all()
+    assert np.array_equal(tok, np.argmax(l, 1))
+    assert np.all(ratio == 1.0)
+
+
+def test_resampled_tokens_are_valid(ssd):
+    rng = np.random.default_rng(10)
+    rows, V = 256, 16384
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    u = synth.philox_uniforms(4, 0, rows)
+    tok, acc, _, _, st = run_accept(ssd, tgt, drf, u)
+    p = np.exp(tgt - tgt.max(1, keepdims=True)); p /= p.sum(1, keepdims=True)
+    q = np.exp(drf - drf.max(1, keepdims=True)); q /= q.sum(1, keepdims=True)
+    rej = np.nonzero(acc == 0)[0]
+    assert rej.size > 0
+    t_hat = np.argmax(drf, 1)
+    assert np.all(tok[rej] != t_hat[rej])
+    assert np.all(p[rej, tok[rej]] > q[rej, tok[rej]])
+
+
+def test_padded_leading_dimension(ssd):
+    rng = np.random.default_rng(11)
+    rows, V = 32, 4096
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    u = synth.philox_uniforms(6, 0, rows)
+    a = run_accept(ssd, tgt, drf, u, ld=V + 12)
+    dec = oacc.accept_rows(tgt, drf, u)
+    compare_decisions(dec, a[0], a[1], a[2], a[3], what="ld")
+
+
+def test_out_of_range_draft_token_sets_status(ssd):
+    rng = np.random.default_rng(12)
+    tgt, drf = synth._logits_normal(rng, 4, 4096)
+    dt = np.array([1, 4096, 3, -1])
+    tok, acc, _, _, st = run_accept(ssd, tgt, drf, synth.philox_uniforms(0, 0, 4), draft_tok=dt)
+    assert st == 6
+    assert tok[1] == -1 and tok[3] == -1 and acc[1] == 0 and acc[3] == 0
+    assert tok[0] >= 0 and tok[2] >= 0

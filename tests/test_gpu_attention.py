@@ -1,0 +1,114 @@
+"""GPU parity of frontier attention (step a2) against the oracle: normwise
+max relative error 2e-2 per (sequence, head) for bf16 inputs, log-sum-exp
+within 2e-2 absolute."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import step as ostep
+from tests.helpers import ATTN_TOL, attention_error, bf16_to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ssd():
+    import paper_2606_20543_gb300 as m
+    from paper_2606_20543_gb300 import build
+    build.build()
+    m.load()
+    return m
+
+
+def _bf(x):
+    return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def run_attention(ssd, c, scale=0.0):
+    dev = "cuda"
+    g = ssd.grid(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v)
+    cl = torch.from_numpy(c.cache_len.astype(np.int32)).to(dev)
+    nd = torch.empty(c.B, dtype=torch.int32, device=dev)
+    pos = torch.empty((c.B, c.D_max), dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ssd.ssd_frontier(g, c.B, cl, c.D_max, nd, pos, status)
+    q, k, v = _bf(c.q), _bf(c.k), _bf(c.v)
+    o = torch.zeros((c.B, c.D_max, c.Hq, c.d), dtype=torch.bfloat16, device=dev)
+    lse = torch.zeros((c.B, c.Hq, c.D_max), dtype=torch.float32, device=dev)
+    wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    ssd.ssd_verify_attention(g, c.B, c.Hq, c.Hkv, c.d, cl, nd, pos, c.D_max, c.L_max, q, k, v,
+                             scale, o, lse, ws, wsb, status)
+    torch.cuda.synchronize()
+    return (o.float().cpu().numpy(), lse.cpu().numpy(), nd.cpu().numpy(), int(status.item()))
+
+
+def check_case(ssd, c, seqs=None, scale=0.0):
+    o, lse, nd, st = run_attention(ssd, c, scale)
+    assert st == 0
+    q, k, v = bf16_to_f64(c.q), bf16_to_f64(c.k), bf16_to_f64(c.v)
+    ref = ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
+                               q, k, v, c.Hq, c.Hkv, scale if scale else None, seqs)
+    worst = 0.0
+    for b, (o_ref, lse_ref) in ref.items():
+        n = o_ref.shape[0]
+        assert nd[b] == n
+        for h in range(c.Hq):
+            if n == 0:
+                continue
+            e = attention_error(o[b, :n, h], o_ref[:, h])
+            worst = max(worst, e)
+            assert e < ATTN_TOL, f"b={b} h={h} err={e}"
+            assert np.abs(lse[b, h, :n] - lse_ref[h]).max() < 2e-2
+    return worst
+
+
+def test_config1_shape(ssd):
+    check_case(ssd, synth.config1(cache_len=192))
+    check_case(ssd, synth.config1(cache_len=112))
+
+
+def test_config2_sweep_points(ssd):
+    # first, middle, last-with-drafts and empty-frontier points of the sweep
+    c = synth.config2(points=[120, 144, 408, 672, 696], with_logits=False)
+    check_case(ssd, c)
+
+
+def test_gqa_ragged_batch(ssd):
+    # config-3 shapes (GQA 32/8 x 128) on a smaller ragged batch
+    rng = np.random.default_rng(5)
+    cl = rng.integers(64, 1088 + 1, size=5).astype(np.int32)
+    cl[0] = 64          # empty cache beyond the prefix, drafts start at row 0
+    cl[1] = 64 + 1024   # complete grid: no drafts
+    cl[2] = 64 + 31     # one draft left on the row plus the next row
+    c = synth.make_case("gqa", grid_h=32, grid_w=32, prefix_len=64, cache_len=cl, Hq=32, Hkv=8,
+                        d=128, V=64, seed=5, with_logits=False)
+    check_case(ssd, c)
+
+
+def test_head_dim_64_and_custom_scale(ssd):
+    c = synth.make_case("d64", grid_h=12, grid_w=12, prefix_len=7, cache_len=[7, 50, 100, 151],
+                        Hq=6, Hkv=2, d=64, V=64, seed=6, with_logits=False)
+    check_case(ssd, c)
+    check_case(ssd, c, scale=0.05)
+
+
+def test_long_cache_many_splits(ssd):
+    # a long cache on one sequence: the key range is split over CTAs and merged
+    c = synth.make_case("long", grid_h=64, grid_w=64, prefix_len=256, cache_len=[256 + 64 * 40 + 9],
+                        Hq=4, Hkv=4, d=128, V=64, seed=7, with_logits=False)
+    check_case(ssd, c)
+
+
+def test_k_v_two_rows(ssd):
+    c = synth.make_case("kv2", grid_h=10, grid_w=10, prefix_len=5, cache_len=[5, 38, 85],
+                        Hq=8, Hkv=8, d=128, V=64, seed=8, k_v=2, with_logits=False)
+    check_case(ssd, c)
+
+
+def test_bad_cache_length_sets_status(ssd):
+    c = synth.config1(cache_len=192)
+    c.cache_len = np.array([10], np.int32)  # below the prefix
+    o, lse, nd, st = run_attention(ssd, c)
+    assert st == 6 and nd[0] == 0

@@ -1,0 +1,133 @@
+"""GPU parity of the whole verification step (steps a1-a5, a7) through
+ssd_verify_step against the oracle: frontier and counts bit-exact,
+attention within 2e-2, decisions bit-exact except counted near-ties."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import step as ostep
+from oracle import frontier as ofr
+from tests.helpers import ATTN_TOL, attention_error, bf16_to_f64, compare_decisions
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ssd():
+    import paper_2606_20543_gb300 as m
+    from paper_2606_20543_gb300 import build
+    build.build()
+    m.load()
+    return m
+
+
+def make_step(c):
+    from paper_2606_20543_gb300.step import VerifyStep
+    s = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V,
+                   k_v=c.k_v)
+    s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=c.tgt_logits,
+             drf_logits=c.drf_logits, uniforms=c.uniforms)
+    return s
+
+
+def check_step(c, res, attention_seqs=None):
+    ref = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max,
+                            c.tgt_logits, c.drf_logits, c.uniforms)
+    assert res["status"][0] == 0
+    assert np.array_equal(res["n_drafts"], ref["n_drafts"])
+    assert np.array_equal(res["draft_pos"], ref["draft_pos"])
+    rows = ref["decisions"]["rows"]
+    ties = 0
+    if rows.size:
+        ties = compare_decisions(ref["decisions"], res["out_tok"][rows], res["accepted"][rows],
+                                 res["ratio"][rows], what=c.name)
+    # padding rows
+    pad = np.setdiff1d(np.arange(c.B * c.D_max), rows)
+    assert np.all(res["out_tok"][pad] == -1) and np.all(res["accepted"][pad] == 0)
+    if ties == 0:
+        assert np.array_equal(res["accepted_count"], ref["accepted_count"])
+        assert np.array_equal(res["accepted_prefix"], ref["accepted_prefix"])
+        assert np.array_equal(res["next_cache_len"], ref["next_cache_len"])
+    att = ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
+                               bf16_to_f64(c.q), bf16_to_f64(c.k), bf16_to_f64(c.v), c.Hq, c.Hkv,
+                               None, attention_seqs)
+    for b, (o_ref, _) in att.items():
+        n = o_ref.shape[0]
+        for h in range(c.Hq):
+            if n:
+                assert attention_error(res["o"][b, :n, h], o_ref[:, h]) < ATTN_TOL
+    return ties
+
+
+def test_step_config1(ssd):
+    for cl in (192, 112):
+        c = synth.config1(cache_len=cl)
+        s = make_step(c)
+        s.run()
+        torch.cuda.synchronize()
+        check_step(c, s.results())
+
+
+def test_step_config2_sweep_subset(ssd):
+    c = synth.config2(points=[120, 312, 648, 672, 696])
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    check_step(c, s.results())
+
+
+def test_step_config3_shape(ssd):
+    # config-3 shapes with fewer sequences (full size is in test_gpu_fullsize)
+    c = synth.config3(B=4)
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    check_step(c, s.results())
+
+
+def test_frontier_all_cache_lengths(ssd):
+    """Every cache length of a 24x24 grid, k_v = 1 and 2, bit-exact."""
+    dev = "cuda"
+    for k_v in (1, 2):
+        H = W = 24
+        P = 120
+        cls = np.arange(P, P + H * W + 1, dtype=np.int32)
+        D_max = (k_v + 1) * W
+        g = ssd.grid(H, W, P, k_v=k_v)
+        nd = torch.empty(len(cls), dtype=torch.int32, device=dev)
+        pos = torch.empty((len(cls), D_max), dtype=torch.int32, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        ssd.ssd_frontier(g, len(cls), torch.from_numpy(cls).to(dev), D_max, nd, pos, st)
+        torch.cuda.synchronize()
+        nd, pos = nd.cpu().numpy(), pos.cpu().numpy()
+        assert st.item() == 0
+        for i, cl in enumerate(cls):
+            gidx = ofr.grid_index(ofr.frontier(H, W, P, int(cl), k_v), W)
+            assert nd[i] == len(gidx)
+            assert np.array_equal(pos[i, :nd[i]], gidx)
+            assert np.all(pos[i, nd[i]:] == -1)
+
+
+def test_counts_all_accept_and_all_reject(ssd):
+    c = synth.config1(cache_len=192)
+    # identical logits: every draft accepted, the whole frontier committed
+    c.tgt_logits = c.drf_logits.copy()
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    r = s.results()
+    assert r["accepted_count"][0] == 32 and r["accepted_prefix"][0] == 32
+    assert r["next_cache_len"][0] == 192 + 32
+    # disjoint supports: every draft rejected, one correction token committed
+    lp = np.full_like(c.drf_logits, -40.0)
+    lq = np.full_like(c.drf_logits, -40.0)
+    lp[:, :2048] = 0.0
+    lq[:, 2048:] = 0.0
+    s.upload(tgt_logits=lp, drf_logits=lq)
+    s.run()
+    torch.cuda.synchronize()
+    r = s.results()
+    assert r["accepted_count"][0] == 0 and r["accepted_prefix"][0] == 0
+    assert r["next_cache_len"][0] == 193
+    assert np.all(r["out_tok"][:32] < 2048)
