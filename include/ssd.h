@@ -138,6 +138,39 @@ ssd_status ssd_verify_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int
                                 int32_t* status, ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Frontier attention without a caller-provided workspace.  The paper has no
+ * counterpart: this is a deployment convenience of this library.
+ * Some callers cannot allocate device memory at all, for example a plugin
+ * inside an inference server whose host process has reserved all device
+ * memory for its own pool, or a real-time decode loop that may not call
+ * cudaMalloc because that call can synchronise the device and stall other
+ * streams.  This entry point computes exactly what ssd_verify_attention()
+ * computes (same arguments, minus the workspace), using instead a scratch
+ * array of SSD_NOALLOC_SCRATCH_BYTES that the library holds in device memory
+ * (a static __device__ array: every GPU that loads the library keeps it until
+ * the process exits).  It allocates nothing and calls no allocating routine.
+ *  - Limit: problems whose workspace (ssd_verify_attention_workspace()) is
+ *    larger than SSD_NOALLOC_SCRATCH_BYTES are rejected with
+ *    SSD_ERR_WORKSPACE before anything is enqueued.
+ *  - Set-up: the first call on each device looks up the device address of the
+ *    scratch array (cudaGetSymbolAddress, with that device current), which
+ *    may load the library's device code; make that first call before any
+ *    stream capture.  A failed look-up returns SSD_ERR_CUDA.
+ *  - Sharing: every call on a device uses the same scratch array and leaves
+ *    its contents behind.  Nothing in it needs to start at zero: each call
+ *    writes every scratch word it later reads.  Calls that overlap on the
+ *    GPU (other streams, other host threads) race on the array and must be
+ *    serialised by the caller.
+ * ------------------------------------------------------------------------- */
+#define SSD_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
+ssd_status ssd_verify_attention_noalloc(const ssd_grid* grid, int32_t B, int32_t Hq, int32_t Hkv,
+                                        int32_t d, const int32_t* cache_len,
+                                        const int32_t* n_drafts, const int32_t* draft_pos,
+                                        int32_t D_max, int32_t L_max, const void* q, const void* k,
+                                        const void* v, float scale, void* o, float* lse,
+                                        int32_t* status, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * a3-a5. Acceptance (Sec. 3.3 strategy (C); temperature of App.
  * "Configuration").  For every row r < rows:
  *     p = softmax(tgt[r] / T), q = softmax(drf[r] / T)

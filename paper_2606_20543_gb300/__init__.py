@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
                 7: "SSD_ERR_WORKSPACE"}
 
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
-            "ssd_verify_attention", "ssd_accept", "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
+            "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
             "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
 
 
@@ -88,6 +88,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_verify_attention_workspace": (SZ, [I32, I32, I32, I32, I32, I32]),
         "ssd_verify_attention": (I32, [ctypes.POINTER(Grid), I32, I32, I32, I32, P, P, P, I32, I32,
                                        P, P, P, F, P, P, P, SZ, P, P]),
+        "ssd_verify_attention_noalloc": (I32, [ctypes.POINTER(Grid), I32, I32, I32, I32, P, P, P,
+                                               I32, I32, P, P, P, F, P, P, P, P]),
         "ssd_accept": (I32, [I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P, P, P, P]),
         "ssd_lmhead_accept_workspace": (SZ, [I32, I32]),
         "ssd_lmhead_accept": (I32, [I32, I32, I32, P, P, P, P, P, F, ctypes.POINTER(Rng), P, P, P,
@@ -160,6 +162,18 @@ def ssd_verify_attention(g: Grid, B, Hq, Hkv, d, cache_len, n_drafts, draft_pos,
         ctypes.byref(g), B, Hq, Hkv, d, _ptr(cache_len), _ptr(n_drafts), _ptr(draft_pos), D_max,
         L_max, _ptr(q), _ptr(k), _ptr(v), scale, _ptr(o), _ptr(lse), _ptr(workspace),
         workspace_bytes, _ptr(status), _stream(stream)))
+
+
+def ssd_verify_attention_noalloc(g: Grid, B, Hq, Hkv, d, cache_len, n_drafts, draft_pos, D_max,
+                                 L_max, q, k, v, scale, o, lse, status, stream=None) -> None:
+    """ssd_verify_attention() for callers that cannot allocate device memory:
+    the library's own static device scratch replaces the workspace (limit
+    SSD_NOALLOC_SCRATCH_BYTES = 64 MiB; calls that overlap on the GPU race on
+    that scratch and must be serialised by the caller)."""
+    _check("ssd_verify_attention_noalloc", load().ssd_verify_attention_noalloc(
+        ctypes.byref(g), B, Hq, Hkv, d, _ptr(cache_len), _ptr(n_drafts), _ptr(draft_pos), D_max,
+        L_max, _ptr(q), _ptr(k), _ptr(v), scale, _ptr(o), _ptr(lse), _ptr(status),
+        _stream(stream)))
 
 
 def ssd_accept(rows, V, tgt_logits, drf_logits, ld, draft_tok, temperature, r: Rng, out_tok,

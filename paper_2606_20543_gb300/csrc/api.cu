@@ -136,6 +136,45 @@ ssd_status ssd_verify_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int
   return from_cuda(launch_attention(a, workspace, workspace_bytes, (cudaStream_t)stream));
 }
 
+ssd_status ssd_verify_attention_noalloc(const ssd_grid* grid, int32_t B, int32_t Hq, int32_t Hkv,
+                                        int32_t d, const int32_t* cache_len,
+                                        const int32_t* n_drafts, const int32_t* draft_pos,
+                                        int32_t D_max, int32_t L_max, const void* q, const void* k,
+                                        const void* v, float scale, void* o, float* lse,
+                                        int32_t* status, ssd_stream_t stream) {
+  ssd_status s = check_attention(grid, B, Hq, Hkv, d, D_max, L_max);
+  if (s != SSD_OK) return s;
+  if (B == 0) return SSD_OK;
+  if (cache_len == nullptr || n_drafts == nullptr || draft_pos == nullptr || q == nullptr ||
+      k == nullptr || v == nullptr || o == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(q) || !aligned16(o)) return SSD_ERR_INVALID_ARG;
+  if (!(scale >= 0.f) || !isfinite(scale)) return SSD_ERR_INVALID_ARG;
+  if (attention_workspace(B, Hq, Hkv, d, D_max, L_max) > SSD_NOALLOC_SCRATCH_BYTES)
+    return SSD_ERR_WORKSPACE;
+  AttnArgs a;
+  a.grid = *grid;
+  a.B = B;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.d = d;
+  a.D_max = D_max;
+  a.L_max = L_max;
+  a.cache_len = cache_len;
+  a.n_drafts = n_drafts;
+  a.draft_pos = draft_pos;
+  a.q = q;
+  a.k = k;
+  a.v = v;
+  a.scale = scale;
+  a.o = o;
+  a.lse = lse;
+  a.status = status;
+  const cudaError_t e = launch_attention_noalloc(a, (cudaStream_t)stream);
+  if (e == cudaErrorMemoryAllocation) return SSD_ERR_WORKSPACE;
+  return from_cuda(e);
+}
+
 ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
                       int64_t ld, const int32_t* draft_tok, float temperature, const ssd_rng* rng,
                       int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,

@@ -18,6 +18,8 @@
 // tiles that reach the drafted block, and the softmax is the online
 // (running max / running sum) form with quad shuffles.  Long caches are split
 // over CTAs; a combine kernel merges the splits by their log-sum-exp.
+#include <mutex>
+
 #include "kernels.cuh"
 
 namespace ssd {
@@ -497,6 +499,44 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
   else
     attn_combine_kernel<64><<<blocks, wpb * 32, 0, stream>>>(a, L);
   return cudaGetLastError();
+}
+
+// ------------------------------------------------- no-allocation variant
+// Scratch of ssd_verify_attention_noalloc(): it stands in for the caller's
+// workspace (per-sequence flags and split-KV partials).  Host code must not
+// pass `g_noalloc_scratch` itself to a kernel: on the host that name is a
+// stand-in, not a device address.  The device address is looked up once per
+// device below.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[SSD_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (set-up on the
+// first call per device, with that device current).  nullptr on failure.
+void* noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    g_scratch_ptr[dev] = p;
+  }
+  return g_scratch_ptr[dev];
+}
+
+}  // namespace
+
+cudaError_t launch_attention_noalloc(const AttnArgs& a, cudaStream_t stream) {
+  const size_t need = attention_workspace(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max);
+  if (need > SSD_NOALLOC_SCRATCH_BYTES) return cudaErrorMemoryAllocation;
+  void* ws = noalloc_scratch();
+  if (ws == nullptr) return cudaErrorInvalidDevice;
+  return launch_attention(a, ws, SSD_NOALLOC_SCRATCH_BYTES, stream);
 }
 
 }  // namespace ssd

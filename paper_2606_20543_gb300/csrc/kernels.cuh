@@ -53,6 +53,10 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
                            int32_t L_max);
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
 int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
+// Same as launch_attention with the library's static device scratch as the
+// workspace (ssd_verify_attention_noalloc); cudaErrorMemoryAllocation if the
+// problem needs more than SSD_NOALLOC_SCRATCH_BYTES.
+cudaError_t launch_attention_noalloc(const AttnArgs& a, cudaStream_t stream);
 
 // ---- lmhead.cu
 struct LmHeadArgs {
