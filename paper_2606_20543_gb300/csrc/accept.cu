@@ -4,20 +4,18 @@
 //   accept t with probability min(p(t) / q(t), 1); otherwise draw from
 //   [p - q]_+ / sum [p - q]_+ (inverse CDF in vocabulary order, one uniform).
 //
-// Design (GB300): one thread-block cluster per row.  CTA c of the cluster
-// owns the vocabulary slice [c * S, c * S + S) and pulls its slice of both
-// logit rows into shared memory with two bulk TMA copies, so every logit is
-// read from HBM exactly once.  Per-CTA max / sum-exp / argmax partials are
-// exchanged through distributed shared memory; every CTA combines them in
-// rank order (identical results everywhere), takes the decision, and on a
-// rejection computes its slice's residual mass from the resident slice.  A
-// second exchange of the per-CTA masses locates the CTA holding the CDF
-// crossing, which scans its slice (warp segments in vocabulary order).
-#include <cooperative_groups.h>
-
+// Design (GB300): one CTA of 256 threads per row, no shared-memory copy of
+// the row (so many rows stream at once).  Pass A reads both logit rows from
+// HBM once with 16-byte loads, four per row per thread in flight, and keeps
+// online (max, sum of 2^x) statistics and the first argmax in registers; one
+// block reduction in a fixed order gives the log-sum-exps and the draft
+// token, and thread 0 takes the decision.  Only rejected rows run pass B: the
+// rows are re-read from L2 (they were read microseconds earlier; these loads
+// mark the lines evict-first), the residual weights are formed with MUFU
+// exp2, and the mass of every 128-entry chunk goes to shared memory in
+// vocabulary order.  Warp 0 scans the chunk masses, finds the chunk holding
+// u_res * Z, and re-walks that chunk to pick the token.
 #include "kernels.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace ssd {
 
@@ -25,79 +23,103 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kMaxCluster = 8;
-constexpr int kSliceTarget = 4096;     // elements per CTA when the cluster has room
-constexpr int kSliceMax = 16384;       // 128 KB of shared memory for both rows
+constexpr int kUnroll = 4;             // float4 loads per row per thread in flight
+constexpr int kMaxV = 1 << 20;         // chunk-mass table: V / 128 floats of shared memory
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-struct Partial {
-  float max_p, sum_p;  // over this slice, sum of exp2((x - max) * c)
-  float max_q, sum_q;
-  float xq_t, xp_t;    // logits at the slice's candidate draft token
-  int32_t t;           // candidate draft token (argmax q of the slice, or the given one), -1 if none
-  float z;             // residual mass of the slice
-};
+// 2^x on the MUFU unit (results below 2^-126 flush to zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
-struct Shared {
-  Partial part;                 // this CTA's partial (read by the cluster)
-  float red_f[kWarps * 4];
-  int32_t red_i[kWarps];
-  float warp_mass[kWarps];
-  uint64_t bar;
-  // decision broadcast
-  float c_p, c_q;               // log2-domain normalisers: max * c + log2(sum)
-  int32_t t;
-  int32_t accept;
-  float u_res;
-};
+// Streaming 16-byte loads: the first read of a row keeps it in L2 for the
+// residual pass; the residual pass marks its lines evict-first (last use).
+__device__ __forceinline__ float4 ld_keep(const float4* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ float4 ld_last(const float4* p, uint64_t pol) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p), "l"(pol));
+  return v;
+}
 
 __device__ __forceinline__ bool better_arg(float v, int32_t i, float bv, int32_t bi) {
   return v > bv || (v == bv && (uint32_t)i < (uint32_t)bi);
 }
 
-// Residual weight of one entry: [p - q]_+ (or p itself for the Z == 0 draw).
-__device__ __forceinline__ float weight(float xp, float xq, float c, float c_p, float c_q,
-                                        bool from_p) {
-  const float pv = exp2f(fmaf(xp, c, -c_p));
-  if (from_p) return pv;
-  const float qv = exp2f(fmaf(xq, c, -c_q));
-  return fmaxf(pv - qv, 0.0f);
+// Online (max, sum of exp2((x - max) * c)) over 4 more entries.
+__device__ __forceinline__ void online4(float& m, float& s, const float4& x, float c) {
+  const float mx = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
+  if (mx > m) {
+    s *= ex2((m - mx) * c);  // m == -inf: s is 0 and stays 0
+    m = mx;
+  }
+  if (m != -INFINITY) {
+    const float mc = m * c;
+    s += (ex2(fmaf(x.x, c, -mc)) + ex2(fmaf(x.y, c, -mc))) +
+         (ex2(fmaf(x.z, c, -mc)) + ex2(fmaf(x.w, c, -mc)));
+  }
 }
 
-// Mass of warp `w`'s segment of the slice, iterations of 128 entries
-// (lane l holds entries 4l..4l+3 of the iteration), summed in a fixed order.
-__device__ __forceinline__ float4 weights4(const float* sp, const float* sq, int32_t e, int32_t n,
-                                           float c, float c_p, float c_q, bool from_p) {
-  float4 w = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (e < n) {  // n % 4 == 0, so a vector is either fully inside or outside
-    const float4 xp = *reinterpret_cast<const float4*>(sp + e);
-    const float4 xq = *reinterpret_cast<const float4*>(sq + e);
-    w.x = weight(xp.x, xq.x, c, c_p, c_q, from_p);
-    w.y = weight(xp.y, xq.y, c, c_p, c_q, from_p);
-    w.z = weight(xp.z, xq.z, c, c_p, c_q, from_p);
-    w.w = weight(xp.w, xq.w, c, c_p, c_q, from_p);
+// Merge two (max, sum) pairs.
+__device__ __forceinline__ void merge(float& m, float& s, float m2, float s2, float c) {
+  const float mn = fmaxf(m, m2);
+  if (mn == -INFINITY) return;
+  s = s * ex2((m - mn) * c) + s2 * ex2((m2 - mn) * c);
+  m = mn;
+}
+
+// Residual weights of 4 entries: [p - q]_+ with p = 2^(x_p c - Cp), q = 2^(x_q c - Cq),
+// or p itself for the draw from p.
+__device__ __forceinline__ float4 weights4(const float4& xp, const float4& xq, float c, float Cp,
+                                           float Cq, bool from_p) {
+  float4 w;
+  if (from_p) {
+    w.x = ex2(fmaf(xp.x, c, -Cp));
+    w.y = ex2(fmaf(xp.y, c, -Cp));
+    w.z = ex2(fmaf(xp.z, c, -Cp));
+    w.w = ex2(fmaf(xp.w, c, -Cp));
+  } else {
+    w.x = fmaxf(ex2(fmaf(xp.x, c, -Cp)) - ex2(fmaf(xq.x, c, -Cq)), 0.f);
+    w.y = fmaxf(ex2(fmaf(xp.y, c, -Cp)) - ex2(fmaf(xq.y, c, -Cq)), 0.f);
+    w.z = fmaxf(ex2(fmaf(xp.z, c, -Cp)) - ex2(fmaf(xq.z, c, -Cq)), 0.f);
+    w.w = fmaxf(ex2(fmaf(xp.w, c, -Cp)) - ex2(fmaf(xq.w, c, -Cq)), 0.f);
   }
   return w;
 }
 
-__global__ void __launch_bounds__(kThreads)
-accept_kernel(AcceptArgs a, int32_t slice, int32_t csize) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  float* sp = reinterpret_cast<float*>(smem_raw);
-  float* sq = sp + slice;
-  Shared& sh = *reinterpret_cast<Shared*>(sq + slice);
+struct Shared {
+  float red[kWarps][4];
+  int32_t red_i[kWarps];
+  float Cp, Cq;      // log2-domain normalisers: max * c + log2(sum)
+  int32_t accept;    // 1 accepted, 0 rejected, 2 no valid draft token
+  float u_res;
+};
 
+// One CTA per row.  Pass A streams both logit rows once from HBM and keeps
+// online statistics; pass B (rejected rows only) re-reads them from L2,
+// computes the residual weights and the mass of every 128-entry chunk (warp w
+// of iteration k owns entries [(8k + w) * 128, +128), so chunks are in
+// vocabulary order); warp 0 then scans the chunk masses and re-walks the
+// chunk holding the CDF crossing.
+__global__ void __launch_bounds__(kThreads, 4) accept_kernel(AcceptArgs a) {
+  extern __shared__ float chunk_mass[];  // [V / 128] (rounded up to whole iterations)
+  __shared__ Shared sh;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t r = blockIdx.x / csize;
-  const int32_t rank = blockIdx.x % csize;
-  const bool lead = (rank == 0) && (tid == 0);
+  const int64_t r = blockIdx.x;
 
   // ---- rows outside the frontier (padding slots of a verification step)
   if (a.n_drafts != nullptr) {
     const int32_t b = (int32_t)(r / a.D_max), j = (int32_t)(r % a.D_max);
     if (j >= a.n_drafts[b]) {
-      if (lead) {
+      if (tid == 0) {
         a.out_tok[r] = -1;
         a.accepted[r] = 0;
         if (a.ratio) a.ratio[r] = 0.f;
@@ -110,7 +132,7 @@ accept_kernel(AcceptArgs a, int32_t slice, int32_t csize) {
   if (a.draft_tok != nullptr) {
     given_t = a.draft_tok[r];
     if (given_t < 0 || given_t >= a.V) {
-      if (lead) {
+      if (tid == 0) {
         record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         a.out_tok[r] = -1;
         a.accepted[r] = 0;
@@ -120,321 +142,233 @@ accept_kernel(AcceptArgs a, int32_t slice, int32_t csize) {
     }
   }
 
-  const int32_t v0 = rank * slice;
-  const int32_t n = min(slice, a.V - v0);  // > 0 by construction, multiple of 4
-
-  // ---- stage the slice of both rows in shared memory (one HBM read)
-  if (tid == 0) {
-    mbar_init(&sh.bar, 1);
-    fence_barrier_init();
-  }
-  __syncthreads();
-  if (tid == 0) {
-    const uint32_t bytes = (uint32_t)n * 4u;
-    mbar_arrive_expect_tx(&sh.bar, 2u * bytes);
-    bulk_g2s(sp, a.tgt + r * a.ld + v0, bytes, &sh.bar);
-    bulk_g2s(sq, a.drf + r * a.ld + v0, bytes, &sh.bar);
-  }
-  const bool ok = mbar_wait(&sh.bar, 0, a.status);
-
-  cg::cluster_group cluster = cg::this_cluster();
+  const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
+  const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
+  const int32_t nv = a.V >> 2;
   const float c = kLog2e / a.temperature;
 
-  // ---- pass 1: max of both rows, argmax of the draft row
-  float mp = -INFINITY, mq = -INFINITY;
+  // ---- pass A: online max / sum-exp of both rows, first argmax of the draft row
+  float mp = -INFINITY, sp = 0.f, mq = -INFINITY, sq = 0.f;
   int32_t iq = 0x7fffffff;
-  const int32_t nv = n >> 2;
-  if (ok) {
-    for (int32_t i = tid; i < nv; i += kThreads) {
-      const float4 xp = reinterpret_cast<const float4*>(sp)[i];
-      const float4 xq = reinterpret_cast<const float4*>(sq)[i];
-      mp = fmaxf(mp, fmaxf(fmaxf(xp.x, xp.y), fmaxf(xp.z, xp.w)));
-      const int32_t e = v0 + 4 * i;
-      if (better_arg(xq.x, e, mq, iq)) { mq = xq.x; iq = e; }
-      if (better_arg(xq.y, e + 1, mq, iq)) { mq = xq.y; iq = e + 1; }
-      if (better_arg(xq.z, e + 2, mq, iq)) { mq = xq.z; iq = e + 2; }
-      if (better_arg(xq.w, e + 3, mq, iq)) { mq = xq.w; iq = e + 3; }
+  for (int32_t base = tid; base < nv; base += kThreads * kUnroll) {
+    float4 xp[kUnroll], xq[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int32_t i = base + u * kThreads;
+      if (i < nv) {
+        xp[u] = ld_keep(tp + i);
+        xq[u] = ld_keep(dp + i);
+      } else {
+        xp[u] = xq[u] = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      online4(mp, sp, xp[u], c);
+      // draft row: entries visited in ascending order, strict '>' keeps the first max
+      const float4 x = xq[u];
+      const float mx = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
+      if (mx > mq) {
+        const int32_t e = 4 * (base + u * kThreads);
+        iq = e + (x.x == mx ? 0 : x.y == mx ? 1 : x.z == mx ? 2 : 3);
+      }
+      online4(mq, sq, x, c);
     }
   }
+  // block reduction (fixed order: xor tree in warps, then warps 0..7)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    mp = fmaxf(mp, __shfl_xor_sync(0xffffffffu, mp, o));
-    const float oq = __shfl_xor_sync(0xffffffffu, mq, o);
+    merge(mp, sp, __shfl_xor_sync(0xffffffffu, mp, o), __shfl_xor_sync(0xffffffffu, sp, o), c);
+    const float om = __shfl_xor_sync(0xffffffffu, mq, o);
+    const float os = __shfl_xor_sync(0xffffffffu, sq, o);
     const int32_t oi = __shfl_xor_sync(0xffffffffu, iq, o);
-    if (better_arg(oq, oi, mq, iq)) { mq = oq; iq = oi; }
+    const bool take = better_arg(om, oi, mq, iq);
+    merge(mq, sq, om, os, c);
+    if (take) iq = oi;
   }
   if (lane == 0) {
-    sh.red_f[warp] = mp;
-    sh.red_f[kWarps + warp] = mq;
+    sh.red[warp][0] = mp;
+    sh.red[warp][1] = sp;
+    sh.red[warp][2] = mq;
+    sh.red[warp][3] = sq;
     sh.red_i[warp] = iq;
   }
   __syncthreads();
-  mp = sh.red_f[0];
-  mq = sh.red_f[kWarps];
-  iq = sh.red_i[0];
-  for (int w = 1; w < kWarps; ++w) {
-    mp = fmaxf(mp, sh.red_f[w]);
-    if (better_arg(sh.red_f[kWarps + w], sh.red_i[w], mq, iq)) {
-      mq = sh.red_f[kWarps + w];
-      iq = sh.red_i[w];
-    }
-  }
-  __syncthreads();
-
-  // ---- pass 2: sum of exp relative to the slice maxima
-  float s_p = 0.f, s_q = 0.f;
-  if (ok) {
-    const float mpc = mp * c, mqc = mq * c;
-    for (int32_t i = tid; i < nv; i += kThreads) {
-      const float4 xp = reinterpret_cast<const float4*>(sp)[i];
-      const float4 xq = reinterpret_cast<const float4*>(sq)[i];
-      s_p += exp2f(fmaf(xp.x, c, -mpc)) + exp2f(fmaf(xp.y, c, -mpc)) +
-             exp2f(fmaf(xp.z, c, -mpc)) + exp2f(fmaf(xp.w, c, -mpc));
-      s_q += exp2f(fmaf(xq.x, c, -mqc)) + exp2f(fmaf(xq.y, c, -mqc)) +
-             exp2f(fmaf(xq.z, c, -mqc)) + exp2f(fmaf(xq.w, c, -mqc));
-    }
-  }
-  s_p = warp_sum(s_p);
-  s_q = warp_sum(s_q);
-  if (lane == 0) {
-    sh.red_f[2 * kWarps + warp] = s_p;
-    sh.red_f[3 * kWarps + warp] = s_q;
-  }
-  __syncthreads();
   if (tid == 0) {
-    float tp = 0.f, tq = 0.f;
-    for (int w = 0; w < kWarps; ++w) {
-      tp += sh.red_f[2 * kWarps + w];
-      tq += sh.red_f[3 * kWarps + w];
+    float Mp = sh.red[0][0], Sp = sh.red[0][1], Mq = sh.red[0][2], Sq = sh.red[0][3];
+    int32_t t = sh.red_i[0];
+    for (int w = 1; w < kWarps; ++w) {
+      merge(Mp, Sp, sh.red[w][0], sh.red[w][1], c);
+      const bool take = better_arg(sh.red[w][2], sh.red_i[w], Mq, t);
+      merge(Mq, Sq, sh.red[w][2], sh.red[w][3], c);
+      if (take) t = sh.red_i[w];
     }
-    Partial& P = sh.part;
-    P.max_p = mp;
-    P.sum_p = tp;
-    P.max_q = mq;
-    P.sum_q = tq;
-    if (given_t >= 0) {
-      const bool mine = given_t >= v0 && given_t < v0 + n;
-      P.t = mine ? given_t : -1;
-      P.xp_t = mine ? sp[given_t - v0] : 0.f;
-      P.xq_t = mine ? sq[given_t - v0] : 0.f;
-    } else if (ok && iq >= v0 && iq < v0 + n) {
-      P.t = iq;
-      P.xq_t = mq;
-      P.xp_t = sp[iq - v0];
-    } else {  // no finite candidate in this slice (NaN logits or a failed copy)
-      P.t = -1;
-      P.xq_t = -INFINITY;
-      P.xp_t = 0.f;
-    }
-    P.z = 0.f;
-  }
-  if (csize > 1) cluster.sync(); else __syncthreads();
-
-  // ---- combine the cluster's partials in rank order, decide (thread 0)
-  if (tid == 0) {
-    float Mp = -INFINITY, Mq = -INFINITY;
-    for (int k = 0; k < csize; ++k) {
-      const Partial* P = cluster.map_shared_rank(&sh.part, k);
-      Mp = fmaxf(Mp, P->max_p);
-      Mq = fmaxf(Mq, P->max_q);
-    }
-    float Sp = 0.f, Sq = 0.f, xp_t = 0.f, xq_t = -INFINITY;
-    int32_t t = given_t >= 0 ? given_t : 0x7fffffff;
-    for (int k = 0; k < csize; ++k) {
-      const Partial* P = cluster.map_shared_rank(&sh.part, k);
-      Sp += P->sum_p * exp2f((P->max_p - Mp) * c);
-      Sq += P->sum_q * exp2f((P->max_q - Mq) * c);
-      if (given_t >= 0) {
-        if (P->t == given_t) { xp_t = P->xp_t; xq_t = P->xq_t; }
-      } else if (better_arg(P->xq_t, P->t, xq_t, t)) {
-        t = P->t;
-        xq_t = P->xq_t;
-        xp_t = P->xp_t;
-      }
-    }
-    const bool valid_t = (t >= 0 && t < a.V);
-    if (!valid_t) {
-      record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
-      t = -1;
-    }
-    const float l2p = (xp_t - Mp) * c - log2f(Sp);
-    const float l2q = (xq_t - Mq) * c - log2f(Sq);
-    const float ratio = exp2f(l2p - l2q);
+    if (given_t >= 0) t = given_t;
+    const bool valid_t = t >= 0 && t < a.V;
+    float ratio = 0.f;
+    bool acc = false;
     const float2 u = row_uniforms(a.rng, r);
-    const bool acc = valid_t && u.x < fminf(ratio, 1.0f);
-    sh.t = t;
-    sh.accept = acc ? 1 : (valid_t ? 0 : 2);  // 2: no valid draft token, skip the draw
-    sh.c_p = Mp * c + log2f(Sp);
-    sh.c_q = Mq * c + log2f(Sq);
+    if (valid_t) {
+      const float xp_t = a.tgt[r * a.ld + t];  // L2-resident after pass A
+      const float xq_t = a.drf[r * a.ld + t];
+      const float l2p = (xp_t - Mp) * c - log2f(Sp);
+      const float l2q = (xq_t - Mq) * c - log2f(Sq);
+      ratio = exp2f(l2p - l2q);
+      acc = u.x < fminf(ratio, 1.0f);
+    } else {
+      record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
+    }
+    sh.accept = acc ? 1 : (valid_t ? 0 : 2);
     sh.u_res = u.y;
-    if (rank == 0) {
-      a.accepted[r] = acc ? 1 : 0;
-      if (acc || !valid_t) a.out_tok[r] = t;
-      if (a.ratio) a.ratio[r] = ratio;
-      if (a.lse) {
-        a.lse[2 * r] = Mp / a.temperature + log2f(Sp) * kLn2;
-        a.lse[2 * r + 1] = Mq / a.temperature + log2f(Sq) * kLn2;
-      }
+    sh.Cp = Mp * c + log2f(Sp);
+    sh.Cq = Mq * c + log2f(Sq);
+    a.accepted[r] = acc ? 1 : 0;
+    if (acc) a.out_tok[r] = t;
+    else if (!valid_t) a.out_tok[r] = -1;
+    if (a.ratio) a.ratio[r] = ratio;
+    if (a.lse) {
+      a.lse[2 * r] = Mp / a.temperature + log2f(Sp) * kLn2;
+      a.lse[2 * r + 1] = Mq / a.temperature + log2f(Sq) * kLn2;
     }
   }
   __syncthreads();
+  if (sh.accept != 0) return;
 
-  if (sh.accept == 0) {
-    // ---- residual draw: [p - q]_+ (or p when that mass is zero)
-    const float c_p = sh.c_p, c_q = sh.c_q;
-    const int32_t wseg = ((n + kWarps * 128 - 1) / (kWarps * 128)) * 128;  // per-warp entries
-    const int32_t w_begin = warp * wseg;
-    const int32_t iters = wseg / 128;
-    for (int pass = 0; pass < 2; ++pass) {
-      const bool from_p = (pass == 1);
-      // R1: per-warp masses, fixed summation order (lane sums -> warp tree -> iterations)
-      float mass = 0.f;
-      if (ok) {
-        for (int32_t it = 0; it < iters; ++it) {
-          const float4 w = weights4(sp, sq, w_begin + it * 128 + 4 * lane, n, c, c_p, c_q, from_p);
-          mass += warp_sum((w.x + w.y) + (w.z + w.w));
+  // ---- pass B: residual draw from [p - q]_+ (or from p when that mass is zero)
+  const float Cp = sh.Cp, Cq = sh.Cq;
+  const uint64_t pol = policy_evict_first();
+  const int32_t iters = (nv + kThreads - 1) / kThreads;  // 1024 entries per iteration
+  const int32_t nchunks = iters * kWarps;
+  for (int pass = 0; pass < 2; ++pass) {
+    const bool from_p = (pass == 1);
+    for (int32_t k0 = 0; k0 < iters; k0 += kUnroll) {
+      float4 xp[kUnroll], xq[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int32_t i = (k0 + u) * kThreads + tid;
+        if (k0 + u < iters && i < nv) {
+          xp[u] = ld_last(tp + i, pol);
+          xq[u] = from_p ? xp[u] : ld_last(dp + i, pol);
+        } else {
+          xp[u] = xq[u] = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
         }
       }
-      if (lane == 0) sh.warp_mass[warp] = mass;
-      __syncthreads();
-      if (tid == 0) {
-        float z = 0.f;
-        for (int w = 0; w < kWarps; ++w) z += sh.warp_mass[w];
-        sh.part.z = z;
-      }
-      if (csize > 1) cluster.sync(); else __syncthreads();
-      // every thread reads the cluster's masses in rank order
-      float Z = 0.f;
-      for (int k = 0; k < csize; ++k) Z += cluster.map_shared_rank(&sh.part, k)->z;
-      if (!(Z > 0.f) && !from_p) {
-        if (csize > 1) cluster.sync(); else __syncthreads();  // everyone has read z
-        continue;  // zero residual mass: draw from p instead
-      }
-      const float target = sh.u_res * Z;
-      // locate the CTA holding the crossing
-      int32_t cstar = -1, clast = -1;
-      float tc = 0.f, cum = 0.f;
-      for (int k = 0; k < csize; ++k) {
-        const float zk = cluster.map_shared_rank(&sh.part, k)->z;
-        if (zk > 0.f) {
-          clast = k;
-          if (cstar < 0 && cum + zk > target) { cstar = k; tc = target - cum; }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        if (k0 + u < iters) {
+          const float4 w = weights4(xp[u], xq[u], c, Cp, Cq, from_p);
+          const float m = warp_sum((w.x + w.y) + (w.z + w.w));
+          if (lane == 0) chunk_mass[(k0 + u) * kWarps + warp] = m;
         }
-        cum += zk;
       }
-      if (clast < 0) {  // no positive mass anywhere (non-finite logits)
-        if (rank == 0 && tid == 0) {
+    }
+    __syncthreads();
+    if (warp == 0) {
+      // chunk masses in vocabulary order: lane l owns chunks [l*per, (l+1)*per)
+      const int32_t per = (nchunks + 31) / 32;
+      float ls = 0.f;
+      for (int32_t q = 0; q < per; ++q) {
+        const int32_t ch = lane * per + q;
+        ls += (ch < nchunks) ? chunk_mass[ch] : 0.f;
+      }
+      float incl = ls;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const float Z = __shfl_sync(0xffffffffu, incl, 31);
+      if (!(Z > 0.f)) {
+        if (from_p && lane == 0) {  // no positive mass at all (non-finite logits)
           a.out_tok[r] = -1;
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
-        break;
-      }
-      if (cstar < 0) { cstar = clast; tc = INFINITY; }  // rounding ran past the end
-      if (rank == cstar && ok) {
-        // locate the warp segment
-        int32_t wstar = -1, wlast = -1;
-        float tw = 0.f, cw = 0.f;
-        for (int w = 0; w < kWarps; ++w) {
-          const float mw = sh.warp_mass[w];
-          if (mw > 0.f) {
-            wlast = w;
-            if (wstar < 0 && cw + mw > tc) { wstar = w; tw = tc - cw; }
-          }
-          cw += mw;
-        }
-        if (wstar < 0) { wstar = wlast; tw = INFINITY; }
-        if (warp == wstar) {
-          // re-walk the segment with the same arithmetic as R1
-          float run = 0.f;
-          int32_t found = -1, last_pos = -1;
-          for (int32_t it = 0; it < iters && found < 0; ++it) {
-            const int32_t e = w_begin + it * 128 + 4 * lane;
-            const float4 w = weights4(sp, sq, e, n, c, c_p, c_q, from_p);
-            const float lsum = (w.x + w.y) + (w.z + w.w);
-            const float isum = warp_sum(lsum);
-            // last entry with positive weight so far (fallback)
-            int32_t lp = -1;
-            if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
-            else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
-            const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
-            if (hasp) last_pos = __shfl_sync(0xffffffffu, lp, 31 - __clz(hasp));
-            if (isum > 0.f && run + isum > tw) {
-              const float t3 = tw - run;
-              // inclusive scan of lane sums in lane order
-              float incl = lsum;
-#pragma unroll
-              for (int o = 1; o < 32; o <<= 1) {
-                const float y = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += y;
-              }
-              const float excl = incl - lsum;
-              const uint32_t cross = __ballot_sync(0xffffffffu, lsum > 0.f && incl > t3);
-              int32_t lstar = cross ? (__ffs(cross) - 1) : (31 - __clz(hasp));
-              int32_t pick = -1;
-              if (lane == lstar) {
-                const float t4 = t3 - excl;
-                float cc = 0.f;
-                const float ws[4] = {w.x, w.y, w.z, w.w};
-                for (int k = 0; k < 4 && pick < 0; ++k) {
-                  cc += ws[k];
-                  if (ws[k] > 0.f && cc > t4) pick = e + k;
-                }
-                if (pick < 0) pick = lp;  // last positive entry of this lane
-              }
-              found = __shfl_sync(0xffffffffu, pick, lstar);
+      } else {
+        const float target = sh.u_res * Z;
+        // lane holding the crossing (else the last lane with mass)
+        const uint32_t pos = __ballot_sync(0xffffffffu, ls > 0.f);
+        const uint32_t cross = __ballot_sync(0xffffffffu, ls > 0.f && incl > target);
+        const int32_t ls_star = cross ? (__ffs(cross) - 1) : (31 - __clz(pos));
+        float t1 = __shfl_sync(0xffffffffu, incl - ls, ls_star);
+        t1 = cross ? target - t1 : INFINITY;
+        // chunk inside that lane's range (same order as its sum)
+        int32_t chs = -1, chlast = -1;
+        float tch = INFINITY;
+        if (lane == ls_star) {
+          float cum = 0.f;
+          for (int32_t q = 0; q < per; ++q) {
+            const int32_t ch = lane * per + q;
+            const float m = (ch < nchunks) ? chunk_mass[ch] : 0.f;
+            if (m > 0.f) {
+              chlast = ch;
+              if (chs < 0 && cum + m > t1) { chs = ch; tch = t1 - cum; }
             }
-            run += isum;
+            cum += m;
           }
-          if (found < 0) found = last_pos;
-          if (lane == 0) a.out_tok[r] = v0 + found;
+          if (chs < 0) { chs = chlast; tch = INFINITY; }
+        }
+        chs = __shfl_sync(0xffffffffu, chs, ls_star);
+        tch = __shfl_sync(0xffffffffu, tch, ls_star);
+        // re-walk chunk chs = 8k + w: entries 4 * (k * 256 + w * 32 + lane) + 0..3
+        const int32_t kk = chs / kWarps, ww = chs % kWarps;
+        const int32_t i = kk * kThreads + ww * 32 + lane;
+        float4 xp = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY), xq = xp;
+        if (i < nv) {
+          xp = ld_keep(tp + i);
+          xq = from_p ? xp : ld_keep(dp + i);
+        }
+        const float4 w = weights4(xp, xq, c, Cp, Cq, from_p);
+        const float lsum = (w.x + w.y) + (w.z + w.w);
+        float li = lsum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const float y = __shfl_up_sync(0xffffffffu, li, o);
+          if (lane >= o) li += y;
+        }
+        const int32_t e = 4 * i;
+        int32_t lp = -1;  // last entry of this lane with positive weight
+        if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
+        else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
+        const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
+        const uint32_t lcross = __ballot_sync(0xffffffffu, lsum > 0.f && li > tch);
+        const int32_t lstar = lcross ? (__ffs(lcross) - 1) : (hasp ? 31 - __clz(hasp) : 0);
+        if (lane == lstar) {
+          const float t4 = tch - (li - lsum);
+          const float ws[4] = {w.x, w.y, w.z, w.w};
+          float cc = 0.f;
+          int32_t pick = -1;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            cc += ws[k];
+            if (pick < 0 && ws[k] > 0.f && cc > t4) pick = e + k;
+          }
+          if (pick < 0) pick = lp;
+          a.out_tok[r] = pick;
         }
       }
-      break;
+      if (lane == 0) sh.accept = (Z > 0.f) ? 3 : 0;  // 3: drawn
     }
+    __syncthreads();
+    if (sh.accept == 3 || from_p) break;
   }
-  // keep this CTA's shared memory alive until every peer finished reading it
-  if (csize > 1) cluster.sync();
-}
-
-int pick_cluster(int32_t V, int32_t* slice_out) {
-  int cs = (V + kSliceTarget - 1) / kSliceTarget;
-  if (cs > kMaxCluster) cs = kMaxCluster;
-  if (cs < 1) cs = 1;
-  int32_t slice = (V + cs - 1) / cs;
-  slice = (slice + 3) & ~3;
-  *slice_out = slice;
-  return cs;
 }
 
 }  // namespace
 
-bool accept_supported(int32_t V) {
-  int32_t slice;
-  pick_cluster(V, &slice);
-  return slice <= kSliceMax;
-}
+bool accept_supported(int32_t V) { return V <= kMaxV; }
 
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
   if (a.rows == 0) return cudaSuccess;
-  int32_t slice;
-  const int cs = pick_cluster(a.V, &slice);
-  const size_t smem = (size_t)slice * 8 + sizeof(Shared) + 16;
-  cudaError_t e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
-  if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)((int64_t)a.rows * cs), 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = cs;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, accept_kernel, a, slice, (int32_t)cs);
+  const int32_t nv = a.V / 4;
+  const int32_t iters = (nv + kThreads - 1) / kThreads;
+  const size_t smem = (size_t)iters * kWarps * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  accept_kernel<<<(unsigned)a.rows, kThreads, smem, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace ssd

@@ -113,23 +113,52 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   const int32_t cache = a.cache_len[b];
   const int32_t nd = a.n_drafts[b];
   const int32_t Lk = cache + nd;
-  if (tid == 0) *bad = (nd < 0 || nd > a.D_max || cache < 0 || Lk > a.L_max) ? 1 : 0;
+  const bool shape_ok = !(nd < 0 || nd > a.D_max || cache < 0 || Lk > a.L_max);
+  const int32_t rows_total = shape_ok ? nd * G : 0;
+  const int32_t row0 = blockIdx.z * (L.nwarps * 16);
+  const int32_t k_lo = split * L.kps;
+  const int32_t k_hi = min(Lk, k_lo + L.kps);
+  // CTAs with keys and query rows of a well-formed sequence start streaming
+  // K/V right away, before the dependent loads of the draft positions and Q
+  const bool has_work = shape_ok && nd > 0 && row0 < rows_total && k_lo < Lk;
+  const int32_t ntiles = has_work ? (k_hi - k_lo + KT - 1) / KT : 0;
+  const int32_t n_active = (Lk + L.kps - 1) / L.kps;  // splits holding keys of b
+
+  const uint64_t policy = policy_evict_first();
+  const int32_t kvrow0 = (b * a.Hkv + g) * a.L_max;  // row of slot 0 in the 2D view
+  if (tid == 0 && has_work) {
+    for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+    fence_barrier_init();
+  }
   __syncthreads();
-  const bool seq_valid = (*bad == 0) && load_draft_positions(a, b, nd, kflat, bad);
+  auto issue = [&](int t) {
+    const int s = t % kStages;
+    mbar_arrive_expect_tx(&full[s], 2 * TILE_BYTES);
+    const int32_t row = kvrow0 + k_lo + t * KT;
+#pragma unroll
+    for (int c = 0; c < NSUB; ++c) {
+      tma_load_2d(sK + s * TILE_BYTES + c * (KT * 128), &tmK, c * 64, row, &full[s], policy);
+      tma_load_2d(sV + s * TILE_BYTES + c * (KT * 128), &tmV, c * 64, row, &full[s], policy);
+    }
+  };
+  const int32_t n_pre = min(kStages - 1, ntiles);
+  if (tid == 0) {
+    for (int t = 0; t < n_pre; ++t) issue(t);
+  }
+
+  // ---- draft positions (validity is identical in every CTA of b)
+  if (tid == 0) *bad = shape_ok ? 0 : 1;
+  __syncthreads();
+  const bool seq_valid = shape_ok && load_draft_positions(a, b, nd, kflat, bad);
   if (split == 0 && g == 0 && blockIdx.z == 0 && tid == 0) {
     L.seq_ok[b] = seq_valid ? 1 : 0;
     if (!seq_valid) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
   }
-  if (!seq_valid || nd == 0) return;
-
-  const int32_t rows_total = nd * G;
-  const int32_t row0 = blockIdx.z * (L.nwarps * 16);
-  if (row0 >= rows_total) return;
-  const int32_t k_lo = split * L.kps;
-  if (k_lo >= Lk) return;
-  const int32_t k_hi = min(Lk, k_lo + L.kps);
-  const int32_t ntiles = (k_hi - k_lo + KT - 1) / KT;
-  const int32_t n_active = (Lk + L.kps - 1) / L.kps;  // splits holding keys of b
+  if (!seq_valid || !has_work) {
+    // never leave with copies in flight into this CTA's shared memory
+    for (int t = 0; t < n_pre; ++t) mbar_wait(&full[t % kStages], 0, a.status);
+    return;
+  }
 
   // ---- rows of this warp: r = row0 + warp * 16 + {lane/4, lane/4 + 8}
   const int32_t wrow = row0 + warp * 16;
@@ -166,30 +195,6 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
         qf[ks][2 + i] = live ? src[(col + 8) / 2] : 0u;
       }
     }
-  }
-
-  // ---- TMA producer: one thread fills the ring
-  const uint64_t policy = policy_evict_first();
-  const int32_t kvrow0 = (b * a.Hkv + g) * a.L_max;  // row of slot 0 in the 2D view
-  if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
-    fence_barrier_init();
-    prefetch_tensormap(&tmK);
-    prefetch_tensormap(&tmV);
-  }
-  __syncthreads();
-  auto issue = [&](int t) {
-    const int s = t % kStages;
-    mbar_arrive_expect_tx(&full[s], 2 * TILE_BYTES);
-    const int32_t row = kvrow0 + k_lo + t * KT;
-#pragma unroll
-    for (int c = 0; c < NSUB; ++c) {
-      tma_load_2d(sK + s * TILE_BYTES + c * (KT * 128), &tmK, c * 64, row, &full[s], policy);
-      tma_load_2d(sV + s * TILE_BYTES + c * (KT * 128), &tmV, c * 64, row, &full[s], policy);
-    }
-  };
-  if (tid == 0) {
-    for (int t = 0; t < min(kStages - 1, ntiles); ++t) issue(t);
   }
 
   const float c2 = (a.scale != 0.f ? a.scale : rsqrtf((float)D)) * kLog2e;
