@@ -1,15 +1,665 @@
-// lmhead.cu — fused lm_head + acceptance (step a6).  Placeholder until the
-// tcgen05 kernel lands: every call reports SSD_ERR_UNSUPPORTED.
+// lmhead.cu — fused lm_head + acceptance (step a6).  Sec. 3.3, after Eq. 2:
+// draft tokens are decoded through the base model's GenHead, a linear map
+// from the (normalised) hidden state to vocabulary logits.  Verification
+// needs it for the target hidden states H_t and the draft hidden states H_d:
+//   l_p = H_t W_t,  l_q = H_d W_d   ([rows x K] x [K x V])
+// followed by strategy (C) of Sec. 3.3 on every row (accept with probability
+// min(p/q, 1), otherwise draw from [p - q]_+), exactly as accept.cu, but
+// with the logits never written to memory.
+//
+// Design (GB300, tcgen05 + TMEM):
+//  * one CTA per tile of 128 vocabulary entries; draft rows on the MMA's M
+//    dimension (TMEM lanes, padded to 128 per row tile), vocabulary on N, so
+//    each epilogue thread owns one row's 128 logits of the tile;
+//  * A = hidden states (K-major), B = weights (MN-major: the vocabulary is
+//    contiguous in W[K][V]); both staged by TMA with the 128-byte swizzle
+//    through a 3-stage mbarrier ring, one thread producing, one thread
+//    issuing tcgen05.mma (bf16 x bf16 -> fp32) into two TMEM accumulators
+//    (target, draft), tcgen05.commit releasing each stage;
+//  * epilogue: tcgen05.ld of each row's tile, per-tile softmax partials to a
+//    small workspace, a bounded grid barrier (the launch is cooperative, so
+//    every CTA is resident), a warp-parallel combine of the partials in a
+//    fixed order (identical in every CTA), the decision, per-tile residual
+//    masses, a second barrier, and the CTA holding the CDF crossing scans
+//    its row tile sequentially.  Logits stay in TMEM throughout.
 #include "kernels.cuh"
 
 namespace ssd {
 
-size_t lmhead_workspace(int32_t rows, int32_t V) { return 256; }
+namespace {
 
-ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K) { return SSD_ERR_UNSUPPORTED; }
+constexpr int kBM = 128;        // rows per MMA tile (TMEM lanes)
+constexpr int kBN = 128;        // vocabulary entries per CTA
+constexpr int kBK = 64;         // K per stage: one 128-byte swizzle atom of bf16
+constexpr int kMMAK = 16;       // K per tcgen05.mma (kind::f16)
+constexpr int kThreadsL = 128;  // 4 warps = 128 TMEM lanes
+constexpr int kMaxRowTiles = 2; // rows <= 256
+constexpr float kLog2eL = 1.4426950408889634f;
+constexpr float kLn2L = 0.6931471805599453f;
+
+constexpr int kTileA = kBM * kBK * 2;   // 16 KB: [128 rows x 64 K] bf16
+constexpr int kTileB = kBK * kBN * 2;   // 16 KB: [64 K x 128 vocab] bf16 (two 64-wide boxes)
+
+struct LmPartial {  // one row, one vocabulary tile (32 bytes)
+  float max_p, sum_p, max_q, sum_q;
+  float xq_c, xp_c;  // logits at the tile's candidate (argmax of q, or the given token)
+  int32_t cand;      // candidate index, -1 if none
+  float pad;
+};
+
+// ---------------------------------------------------------------- tcgen05
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem], bf16 inputs, fp32 accumulation.
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on `bar` once every MMA this thread issued so far has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor (tcgen05): start address, leading and
+// stride byte offsets (16-byte units), descriptor version 1, 128-byte swizzle.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 D, bf16 A and B, A K-major,
+// B MN-major, N = 128, M = 128.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
+                            ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ bool better(float v, int32_t i, float bv, int32_t bi) {
+  return v > bv || (v == bv && (uint32_t)i < (uint32_t)bi);
+}
+
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c) {
+  const float mn = fmaxf(m, m2);
+  if (mn == -INFINITY) return;
+  s = s * ex2f((m - mn) * c) + s2 * ex2f((m2 - mn) * c);
+  m = mn;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const unsigned int* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Bounded grid barrier over `ncta` co-resident CTAs (cooperative launch).
+// Returns false in every thread if this CTA gave up waiting.
+__device__ bool grid_barrier(unsigned int* ctr, unsigned int target, int32_t* status,
+                             int32_t* flag) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(ctr, 1u);
+    bool ok = false;
+    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+      if (ld_acquire(ctr) >= target) { ok = true; break; }
+      if (i > 256) __nanosleep(64);
+    }
+    if (!ok) record_status(status, SSD_ERR_TIMEOUT);
+    __threadfence();
+    *flag = ok ? 1 : 0;
+  }
+  __syncthreads();
+  return *flag != 0;
+}
+
+struct LmSmemRow {  // per-row results of the decision, broadcast inside the CTA
+  float Cp, Cq;     // log2-domain normalisers max * c + log2(sum)
+  float u_res;
+  int32_t state;    // 0 skip (padding / accepted / invalid), 1 rejected: draw
+  int32_t cstar;    // CTA holding the crossing for this row, -1 none
+  float tc;         // remaining target inside that CTA's tile (INF: last positive)
+  int32_t from_p;   // 1: zero residual mass, draw from p
+  int32_t pad;
+};
+
+struct LmLaunch {
+  int32_t ncta, mt, stages;
+  LmPartial* part;      // [rows][ncta]
+  float* mass;          // [rows][ncta]
+  unsigned int* barrier;
+};
+
+__global__ void __launch_bounds__(kThreadsL, 1)
+lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_constant__ CUtensorMap tmHd,
+                     const __grid_constant__ CUtensorMap tmWt, const __grid_constant__ CUtensorMap tmWd,
+                     LmHeadArgs a, LmLaunch L) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int mt = L.mt, S = L.stages;
+  const int stage_bytes = 2 * mt * kTileA + 2 * kTileB;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * stage_bytes);
+  uint64_t* empty = full + S;
+  uint64_t* done = empty + S;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  int32_t* flag = reinterpret_cast<int32_t*>(tmem_slot + 1);
+  int32_t* fail = flag + 1;
+  LmSmemRow* rowinfo = reinterpret_cast<LmSmemRow*>(fail + 2);  // [mt * 128]
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int cta = blockIdx.x;
+  const int32_t v0 = cta * kBN;
+  const int32_t nkb = a.K / kBK;
+  const uint32_t ncols = (uint32_t)(mt * 2 * kBN);  // target + draft accumulators per row tile
+
+  // ---- set-up: barriers, TMEM
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    *fail = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, ncols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // ---- main loop: warp 0 lane 0 produces, warp 1 lane 0 issues the MMAs
+  if (warp == 0 && lane == 0) {
+    const uint64_t pol = policy_evict_first();     // weights: read once
+    const uint64_t pol_h = policy_evict_last();    // hidden states: read by every CTA
+    const uint32_t bytes = (uint32_t)stage_bytes;
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % S;
+      if (kb >= S && !mbar_wait(&empty[s], ((kb / S) - 1) & 1, a.status)) { *fail = 1; break; }
+      unsigned char* st = smem + s * stage_bytes;
+      mbar_arrive_expect_tx(&full[s], bytes);
+      for (int m = 0; m < mt; ++m) {
+        tma_load_2d(st + m * kTileA, &tmHt, kb * kBK, m * kBM, &full[s], pol_h);
+        tma_load_2d(st + (mt + m) * kTileA, &tmHd, kb * kBK, m * kBM, &full[s], pol_h);
+      }
+      unsigned char* bt = st + 2 * mt * kTileA;
+      unsigned char* bd = bt + kTileB;
+      tma_load_2d(bt, &tmWt, v0, kb * kBK, &full[s], pol);
+      tma_load_2d(bt + kTileB / 2, &tmWt, v0 + 64, kb * kBK, &full[s], pol);
+      tma_load_2d(bd, &tmWd, v0, kb * kBK, &full[s], pol);
+      tma_load_2d(bd + kTileB / 2, &tmWd, v0 + 64, kb * kBK, &full[s], pol);
+    }
+  } else if (warp == 1 && lane == 0) {
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % S;
+      if (!mbar_wait(&full[s], (kb / S) & 1, a.status)) { *fail = 1; break; }
+      tc_fence_after();
+      const uint32_t st = smem_u32(smem + s * stage_bytes);
+      const uint32_t bt = st + 2 * mt * kTileA, bd = bt + kTileB;
+#pragma unroll
+      for (int kk = 0; kk < kBK / kMMAK; ++kk) {
+        // B (MN-major): 64-wide vocabulary atoms 8 KB apart (LBO), 8-row K groups
+        // 1 KB apart (SBO); one MMA's K = 16 rows = 2 KB further per step.
+        const uint64_t db_t = smem_desc(bt + kk * 2048, 8192, 1024);
+        const uint64_t db_d = smem_desc(bd + kk * 2048, 8192, 1024);
+        for (int m = 0; m < mt; ++m) {
+          // A (K-major): 8-row groups 1 KB apart (SBO); K = 16 is 32 bytes along the row.
+          const uint64_t da_t = smem_desc(st + m * kTileA + kk * 32, 16, 1024);
+          const uint64_t da_d = smem_desc(st + (mt + m) * kTileA + kk * 32, 16, 1024);
+          const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
+          mma_bf16(tmem + m * 2 * kBN, da_t, db_t, kIdesc, acc);
+          mma_bf16(tmem + m * 2 * kBN + kBN, da_d, db_d, kIdesc, acc);
+        }
+      }
+      mma_commit(&empty[s]);
+    }
+    mma_commit(done);
+  }
+  // every thread waits for the accumulators
+  const bool mma_ok = mbar_wait(done, 0, a.status);
+  tc_fence_after();
+  bool ok = __syncthreads_and(mma_ok) != 0;
+  ok = ok && (*fail == 0);
+
+  const float c = kLog2eL / a.temperature;
+  const int32_t rows = a.rows;
+  // TMEM lane quarter of this warp: lanes 32*warp .. +31 (row tile m, row m*128 + tid)
+  const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+
+  // ---- epilogue 1: per-tile softmax partials of every row
+  for (int m = 0; m < mt && ok; ++m) {
+    const int32_t row = m * kBM + tid;
+    const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
+    float mp = -INFINITY, sp = 0.f, mq = -INFINITY, sq = 0.f;
+    float xq_c = -INFINITY, xp_c = 0.f;
+    int32_t cand = -1;
+    const int32_t given = (a.draft_tok != nullptr && row < rows) ? a.draft_tok[row] : -1;
+    float v[32], w[32];
+#pragma unroll 1
+    for (int ch = 0; ch < kBN / 32; ++ch) {
+      tmem_ld32(tp + ch * 32, v);
+      tmem_ld32(tq + ch * 32, w);
+      float cmp = -INFINITY, cmq = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        cmp = fmaxf(cmp, v[i]);
+        cmq = fmaxf(cmq, w[i]);
+      }
+      if (given < 0 && cmq > xq_c) {  // first maximum of q (ascending scan)
+#pragma unroll
+        for (int i = 31; i >= 0; --i)
+          if (w[i] == cmq) { cand = v0 + ch * 32 + i; xp_c = v[i]; }
+        xq_c = cmq;
+      }
+      if (given >= v0 + ch * 32 && given < v0 + ch * 32 + 32) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (given == v0 + ch * 32 + i) { cand = given; xp_c = v[i]; xq_c = w[i]; }
+      }
+      float lp = 0.f, lq = 0.f;
+      const float cmpc = cmp * c, cmqc = cmq * c;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        lp += ex2f(fmaf(v[i], c, -cmpc));
+        lq += ex2f(fmaf(w[i], c, -cmqc));
+      }
+      merge_ms(mp, sp, cmp, lp, c);
+      merge_ms(mq, sq, cmq, lq, c);
+    }
+    if (row < rows) {
+      LmPartial P;
+      P.max_p = mp;
+      P.sum_p = sp;
+      P.max_q = mq;
+      P.sum_q = sq;
+      P.xq_c = cand >= 0 ? xq_c : -INFINITY;
+      P.xp_c = xp_c;
+      P.cand = cand;
+      P.pad = 0.f;
+      reinterpret_cast<float4*>(L.part + (int64_t)row * L.ncta + cta)[0] =
+          make_float4(P.max_p, P.sum_p, P.max_q, P.sum_q);
+      reinterpret_cast<float4*>(L.part + (int64_t)row * L.ncta + cta)[1] =
+          make_float4(P.xq_c, P.xp_c, __int_as_float(P.cand), 0.f);
+    }
+  }
+  ok = grid_barrier(L.barrier, (unsigned)L.ncta, a.status, flag) && ok;
+
+  // ---- epilogue 2: combine the partials of each row (warp per row, lanes over
+  // tiles in a fixed order), decide, and on rejection prepare the draw
+  for (int m = 0; m < mt && ok; ++m) {
+    for (int rl = warp; rl < kBM; rl += kThreadsL / 32) {
+      const int32_t row = m * kBM + rl;
+      LmSmemRow& ri = rowinfo[m * kBM + rl];
+      if (row >= rows) {
+        if (lane == 0) ri.state = 0;
+        continue;
+      }
+      bool pad = false;
+      if (a.n_drafts != nullptr) {
+        const int32_t b = row / a.D_max, j = row - b * a.D_max;
+        pad = j >= a.n_drafts[b];
+      }
+      if (pad) {
+        if (lane == 0) {
+          ri.state = 0;
+          if (cta == 0) {
+            a.out_tok[row] = -1;
+            a.accepted[row] = 0;
+            if (a.ratio) a.ratio[row] = 0.f;
+            if (a.lse) { a.lse[2 * row] = 0.f; a.lse[2 * row + 1] = 0.f; }
+          }
+        }
+        continue;
+      }
+      float Mp = -INFINITY, Sp = 0.f, Mq = -INFINITY, Sq = 0.f, xq = -INFINITY, xp = 0.f;
+      int32_t t = 0x7fffffff;
+      for (int k = lane; k < L.ncta; k += 32) {
+        const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
+        const float4 p1 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[1];
+        merge_ms(Mp, Sp, p0.x, p0.y, c);
+        merge_ms(Mq, Sq, p0.z, p0.w, c);
+        const int32_t ck = __float_as_int(p1.z);
+        if (ck >= 0 && better(p1.x, ck, xq, t)) { xq = p1.x; xp = p1.y; t = ck; }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        merge_ms(Mp, Sp, __shfl_xor_sync(0xffffffffu, Mp, o), __shfl_xor_sync(0xffffffffu, Sp, o), c);
+        merge_ms(Mq, Sq, __shfl_xor_sync(0xffffffffu, Mq, o), __shfl_xor_sync(0xffffffffu, Sq, o), c);
+        const float oq = __shfl_xor_sync(0xffffffffu, xq, o);
+        const float op = __shfl_xor_sync(0xffffffffu, xp, o);
+        const int32_t ot = __shfl_xor_sync(0xffffffffu, t, o);
+        if (better(oq, ot, xq, t)) { xq = oq; xp = op; t = ot; }
+      }
+      if (lane == 0) {
+        const int32_t given = a.draft_tok != nullptr ? a.draft_tok[row] : -1;
+        const bool valid_t = (t >= 0 && t < a.V) && (given < 0 || t == given);
+        float ratio = 0.f;
+        bool acc = false;
+        const float2 u = row_uniforms(a.rng, row);
+        if (valid_t) {
+          const float l2p = (xp - Mp) * c - log2f(Sp);
+          const float l2q = (xq - Mq) * c - log2f(Sq);
+          ratio = exp2f(l2p - l2q);
+          acc = u.x < fminf(ratio, 1.0f);
+        }
+        ri.Cp = Mp * c + log2f(Sp);
+        ri.Cq = Mq * c + log2f(Sq);
+        ri.u_res = u.y;
+        ri.state = (valid_t && !acc) ? 1 : 0;
+        ri.from_p = 0;
+        ri.cstar = -1;
+        if (cta == 0) {
+          if (!valid_t) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+          a.accepted[row] = acc ? 1 : 0;
+          if (acc) a.out_tok[row] = t;
+          else if (!valid_t) a.out_tok[row] = -1;
+          if (a.ratio) a.ratio[row] = ratio;
+          if (a.lse) {
+            a.lse[2 * row] = Mp / a.temperature + log2f(Sp) * kLn2L;
+            a.lse[2 * row + 1] = Mq / a.temperature + log2f(Sq) * kLn2L;
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- epilogue 3: residual mass of this tile for every rejected row
+  // (sequential over the tile in vocabulary order)
+  for (int m = 0; m < mt && ok; ++m) {
+    const int32_t row = m * kBM + tid;
+    const LmSmemRow& ri = rowinfo[m * kBM + tid];
+    const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
+    float mass = 0.f;
+    float v[32], w[32];
+    // every lane of the warp takes part in tcgen05.ld; rows that do not draw
+    // simply discard the values
+    const bool draw = row < rows && ri.state == 1;
+#pragma unroll 1
+    for (int ch = 0; ch < kBN / 32; ++ch) {
+      tmem_ld32(tp + ch * 32, v);
+      tmem_ld32(tq + ch * 32, w);
+      if (draw) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          mass += fmaxf(ex2f(fmaf(v[i], c, -ri.Cp)) - ex2f(fmaf(w[i], c, -ri.Cq)), 0.f);
+      }
+    }
+    if (draw) L.mass[(int64_t)row * L.ncta + cta] = mass;
+  }
+  ok = grid_barrier(L.barrier, 2u * (unsigned)L.ncta, a.status, flag) && ok;
+
+  // ---- epilogue 4: locate the tile holding u_res * Z (warp per row, lanes over
+  // tiles in order; the same arithmetic in every CTA)
+  for (int m = 0; m < mt && ok; ++m) {
+    for (int rl = warp; rl < kBM; rl += kThreadsL / 32) {
+      LmSmemRow& ri = rowinfo[m * kBM + rl];
+      if (ri.state != 1) continue;
+      const int32_t row = m * kBM + rl;
+      const int32_t per = (L.ncta + 31) / 32;
+      for (int fp = 0; fp < 2; ++fp) {
+        // lane l owns tiles [l*per, (l+1)*per); fp = 1: masses of p itself
+        float ls = 0.f;
+        for (int q = 0; q < per; ++q) {
+          const int k = lane * per + q;
+          if (k < L.ncta) {
+            if (fp == 0) {
+              ls += L.mass[(int64_t)row * L.ncta + k];
+            } else {
+              const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
+              ls += p0.y * ex2f(p0.x * c - ri.Cp);
+            }
+          }
+        }
+        float incl = ls;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const float y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const float Z = __shfl_sync(0xffffffffu, incl, 31);
+        if (!(Z > 0.f)) {
+          if (fp == 1 && lane == 0 && cta == 0) {
+            a.out_tok[row] = -1;
+            record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+          }
+          continue;  // zero residual mass: try p
+        }
+        const float target = ri.u_res * Z;
+        const uint32_t pos = __ballot_sync(0xffffffffu, ls > 0.f);
+        const uint32_t cross = __ballot_sync(0xffffffffu, ls > 0.f && incl > target);
+        const int32_t lstar = cross ? (__ffs(cross) - 1) : (31 - __clz(pos));
+        float t1 = __shfl_sync(0xffffffffu, incl - ls, lstar);
+        t1 = cross ? target - t1 : INFINITY;
+        if (lane == lstar) {
+          int32_t ks = -1, klast = -1;
+          float tk = INFINITY, cum = 0.f;
+          for (int q = 0; q < per; ++q) {
+            const int k = lane * per + q;
+            if (k >= L.ncta) break;
+            float mk;
+            if (fp == 0) {
+              mk = L.mass[(int64_t)row * L.ncta + k];
+            } else {
+              const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
+              mk = p0.y * ex2f(p0.x * c - ri.Cp);
+            }
+            if (mk > 0.f) {
+              klast = k;
+              if (ks < 0 && cum + mk > t1) { ks = k; tk = t1 - cum; }
+            }
+            cum += mk;
+          }
+          if (ks < 0) { ks = klast; tk = INFINITY; }
+          ri.cstar = ks;
+          ri.tc = tk;
+          ri.from_p = fp;
+        }
+        __syncwarp();
+        break;
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- epilogue 5: the CTA holding the crossing scans its tile sequentially
+  for (int m = 0; m < mt && ok; ++m) {
+    const int32_t row = m * kBM + tid;
+    const LmSmemRow& ri = rowinfo[m * kBM + tid];
+    const bool mine = row < rows && ri.state == 1 && ri.cstar == cta;
+    const bool from_p = ri.from_p != 0;
+    const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
+    float v[32], w[32];
+    float cum = 0.f;
+    int32_t pick = -1, lastpos = -1;
+#pragma unroll 1
+    for (int ch = 0; ch < kBN / 32; ++ch) {
+      tmem_ld32(tp + ch * 32, v);
+      tmem_ld32(tq + ch * 32, w);
+      if (mine && pick < 0) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float pv = ex2f(fmaf(v[i], c, -ri.Cp));
+          const float wt = from_p ? pv : fmaxf(pv - ex2f(fmaf(w[i], c, -ri.Cq)), 0.f);
+          cum += wt;
+          if (wt > 0.f) {
+            lastpos = v0 + ch * 32 + i;
+            if (pick < 0 && cum > ri.tc) pick = lastpos;
+          }
+        }
+      }
+    }
+    if (mine) a.out_tok[row] = pick >= 0 ? pick : lastpos;
+  }
+
+  // ---- teardown: release TMEM (all MMAs have completed: `done` fired)
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, ncols);
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn_l() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 [outer][inner] matrix, box [box_outer x 64 inner], 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+              uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn_l();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int row_tiles(int32_t rows) { return (rows + kBM - 1) / kBM; }
+
+size_t smem_bytes(int mt, int stages) {
+  return 1024 + (size_t)stages * (2 * mt * kTileA + 2 * kTileB) + (2 * stages + 1) * 8 + 16 +
+         (size_t)mt * kBM * sizeof(LmSmemRow);
+}
+
+int stages_for(int mt) { return mt == 1 ? 3 : 2; }
+
+}  // namespace
+
+size_t lmhead_workspace(int32_t rows, int32_t V) {
+  const size_t ncta = (size_t)(V + kBN - 1) / kBN;
+  return al256(sizeof(unsigned int)) + al256((size_t)rows * ncta * sizeof(LmPartial)) +
+         al256((size_t)rows * ncta * sizeof(float));
+}
+
+ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K) {
+  if (rows < 1 || rows > kMaxRowTiles * kBM) return SSD_ERR_UNSUPPORTED;
+  if (K <= 0 || K % kBK != 0) return SSD_ERR_UNSUPPORTED;
+  if (V <= 0 || V % kBN != 0) return SSD_ERR_UNSUPPORTED;
+  // every CTA must be resident at once (one CTA per SM: TMEM and shared memory)
+  const int mt = row_tiles(rows);
+  int per_sm = 0;
+  const size_t smem = smem_bytes(mt, stages_for(mt));
+  if (cudaFuncSetAttribute(lmhead_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess)
+    return SSD_ERR_CUDA;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_accept_kernel, kThreadsL,
+                                                    smem) != cudaSuccess)
+    return SSD_ERR_CUDA;
+  if ((int64_t)(V / kBN) > (int64_t)per_sm * device_sm_count()) return SSD_ERR_UNSUPPORTED;
+  return SSD_OK;
+}
 
 cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
-  return cudaErrorNotSupported;
+  if (a.rows == 0) return cudaSuccess;
+  const int mt = row_tiles(a.rows);
+  LmLaunch L;
+  L.ncta = a.V / kBN;
+  L.mt = mt;
+  L.stages = stages_for(mt);
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  L.barrier = reinterpret_cast<unsigned int*>(w);
+  w += al256(sizeof(unsigned int));
+  L.part = reinterpret_cast<LmPartial*>(w);
+  w += al256((size_t)a.rows * L.ncta * sizeof(LmPartial));
+  L.mass = reinterpret_cast<float*>(w);
+  CUtensorMap ht, hd, wt, wd;
+  // hidden [rows][K]: boxes of 128 rows (rows past `rows` read as zero);
+  // weights [K][V]: boxes of 64 K-rows x 64 vocabulary entries
+  if (!make_map(&ht, a.h_tgt, (uint64_t)a.K, (uint64_t)a.rows, kBM) ||
+      !make_map(&hd, a.h_drf, (uint64_t)a.K, (uint64_t)a.rows, kBM) ||
+      !make_map(&wt, a.w_tgt, (uint64_t)a.V, (uint64_t)a.K, kBK) ||
+      !make_map(&wd, a.w_drf, (uint64_t)a.V, (uint64_t)a.K, kBK))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaMemsetAsync(L.barrier, 0, sizeof(unsigned int), stream);
+  if (e != cudaSuccess) return e;
+  const size_t smem = smem_bytes(mt, L.stages);
+  e = cudaFuncSetAttribute(lmhead_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)L.ncta, 1, 1);
+  cfg.blockDim = dim3(kThreadsL, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, lmhead_accept_kernel, ht, hd, wt, wd, a, L);
 }
 
 }  // namespace ssd

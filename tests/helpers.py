@@ -8,6 +8,12 @@ import synth
 
 ATTN_TOL = 2e-2     # normwise max relative error per (b, h), bf16 inputs
 PROB_TOL = 1e-5     # relative error of ratio / log-sum-exp, fp32 logits path
+# Fused lm_head: the logits themselves come from a bf16 x bf16 contraction over
+# K = 4096 accumulated in fp32 on the tensor cores; a logit error of ~1e-5
+# moves log p(t) - log q(t) by ~2e-5, so ratios carry ~4e-5 relative error
+# (measured 3.6e-5 at K = 4096).  2e-4 stays far inside the 2e-2 allowed for
+# bf16 inputs.
+FUSED_PROB_TOL = 2e-4
 
 
 def bf16_to_f64(bits):
@@ -20,7 +26,7 @@ def attention_error(o_gpu, o_ref):
     return np.abs(o_gpu - o_ref).max() / max(den, 1e-6)
 
 
-def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what=""):
+def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what="", tol=PROB_TOL):
     """Bit-exact comparison of accept flags and tokens, except near-tie rows.
 
     dec: oracle accept_rows() dict for the compared rows; out_tok/accepted:
@@ -37,9 +43,9 @@ def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what=""):
         ref = dec["ratio"]
         fin = np.isfinite(ref) & (ref < 1e30)
         rel = np.abs(ratio[fin] - ref[fin]) / np.maximum(np.abs(ref[fin]), 1e-30)
-        assert rel.max(initial=0) < PROB_TOL, f"{what}: ratio rel err {rel.max()}"
+        assert rel.max(initial=0) < tol, f"{what}: ratio rel err {rel.max()}"
     if lse is not None:
         for k, key in enumerate(("lse_p", "lse_q")):
             rel = np.abs(lse[:, k] - dec[key]) / np.abs(dec[key])
-            assert rel.max(initial=0) < PROB_TOL, f"{what}: {key} rel err {rel.max()}"
+            assert rel.max(initial=0) < tol, f"{what}: {key} rel err {rel.max()}"
     return int(tie.sum())
