@@ -37,7 +37,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ssd", choices=["ssd", "reference"])
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 5])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--fused-batch", type=int, default=1,
+                    help="sequences of the fused-head workload (config 4): 1, or up to 5 "
+                         "(240 draft rows) for the batched variant")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="approximate budget of the CPU-oracle sample")
@@ -45,7 +48,7 @@ def parse():
 
 
 # ----------------------------------------------------------------- workloads
-def workload(cfg: int, rank: int, set_index: int = 0):
+def workload(cfg: int, rank: int, set_index: int = 0, fused_batch: int = 1):
     """Host arrays of one input set; rank and set_index pick the seeds."""
     base = 1000 * rank + 100 * set_index
     if cfg == 1:
@@ -54,6 +57,8 @@ def workload(cfg: int, rank: int, set_index: int = 0):
         return synth.config2(seed0=base)
     if cfg == 3:
         return synth.config3(seed=3 + base)
+    if cfg == 4:
+        return synth.config4(points=[120] * fused_batch, seed0=4 + base)
     if cfg == 5:
         return synth.config5(seed=5 + base)
     raise ValueError(cfg)
@@ -64,6 +69,8 @@ WORKLOAD_NAMES = {
     2: "24x24 sweep: cache 120->696 step 24 (25 batch-1 problems as one ragged batch), "
        "prefix 120, 16x128 MHA, V=16384",
     3: "16 x 32x32 grids, prefix 64, cache U[64,1088], GQA 32/8x128, V=16384, Zipf draft",
+    4: "fused lm_head: 24x24, prefix 120, cache 120 (48 drafts per sequence), 16x128 MHA, "
+       "hidden bf16 [rows x 4096], W_t, W_d bf16 [4096 x 16384]",
     5: "8 x 64x64 grids, prefix 256, first replay step (cache = prefix), 32x128 MHA, V=65536",
 }
 
@@ -77,7 +84,11 @@ def algorithmic_bytes(c, n_drafts):
     kv = int((L * c.Hkv * c.d * 2 * 2).sum())
     qo = int((n * c.Hq * c.d * 2 * 2).sum())
     attn = kv + qo + int(n.sum()) * c.Hq * 4  # + lse
-    acc = int(n.sum()) * (2 * c.V * 4 + 4 + 1 + 4)
+    if c.hidden:
+        # both lm_head weights once, both hidden-state rows of every draft once
+        acc = 2 * c.hidden * c.V * 2 + int(n.sum()) * (2 * c.hidden * 2 + 4 + 1 + 4)
+    else:
+        acc = int(n.sum()) * (2 * c.V * 4 + 4 + 1 + 4)
     return attn, acc
 
 
@@ -146,8 +157,14 @@ def oracle_pass(c):
     v = synth.bf16_bits_to_f32(c.v).astype(np.float64)
     ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
                          q, k, v, c.Hq, c.Hkv)
+    if c.hidden:
+        from oracle import lmhead as olm
+        lp = olm.logits(synth.bf16_bits_to_f32(c.h_tgt), synth.bf16_bits_to_f32(c.w_tgt))
+        lq = olm.logits(synth.bf16_bits_to_f32(c.h_drf), synth.bf16_bits_to_f32(c.w_drf))
+    else:
+        lp, lq = c.tgt_logits, c.drf_logits
     r = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max,
-                          c.tgt_logits, c.drf_logits, c.uniforms)
+                          lp, lq, c.uniforms)
     return r
 
 
@@ -160,7 +177,11 @@ def sub_case(c, seqs):
     s.cache_len = c.cache_len[seqs]
     s.q, s.k, s.v = c.q[seqs], c.k[seqs], c.v[seqs]
     rows = (seqs[:, None] * c.D_max + np.arange(c.D_max)[None]).reshape(-1)
-    s.tgt_logits, s.drf_logits, s.uniforms = c.tgt_logits[rows], c.drf_logits[rows], c.uniforms[rows]
+    s.uniforms = c.uniforms[rows]
+    if c.hidden:
+        s.h_tgt, s.h_drf = c.h_tgt[rows], c.h_drf[rows]
+    else:
+        s.tgt_logits, s.drf_logits = c.tgt_logits[rows], c.drf_logits[rows]
     return s
 
 
@@ -223,14 +244,15 @@ def main():
     from paper_2606_20543_gb300.step import VerifyStep
 
     # two input sets alternate so that consecutive steps never reuse L2
-    cases = [workload(a.config, rank, s) for s in range(2)]
+    cases = [workload(a.config, rank, s, a.fused_batch) for s in range(2)]
     c = cases[0]
     steps_obj = []
     for cs in cases:
         st = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max,
-                        c.V, k_v=c.k_v, device=dev)
+                        c.V, k_v=c.k_v, device=dev, hidden=c.hidden)
         st.upload(cache_len=cs.cache_len, q=cs.q, k=cs.k, v=cs.v, tgt_logits=cs.tgt_logits,
-                  drf_logits=cs.drf_logits)
+                  drf_logits=cs.drf_logits, h_tgt=cs.h_tgt, h_drf=cs.h_drf, w_tgt=cs.w_tgt,
+                  w_drf=cs.w_drf)
         steps_obj.append(st)
     stream = torch.cuda.current_stream(dev)
     seed = 1234 + rank
@@ -307,11 +329,19 @@ def main():
                                  c.D_max, c.L_max, s.q, s.k, s.v, 0.0, s.o, None, ws, wsb,
                                  s.status, cs)
 
+    lm_wsb = ssd.ssd_lmhead_accept_workspace(c.B * c.D_max, c.V) if c.hidden else 0
+    lm_ws = torch.empty(max(lm_wsb, 256), dtype=torch.uint8, device=dev)
+
     def acc_call(i, cs):
         s = steps_obj[i & 1]
         s.set_rng(seed, i)
-        ssd.ssd_accept(c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0, s.rng, s.out_tok,
-                       s.accepted, s.ratio, None, s.status, cs)
+        if c.hidden:
+            ssd.ssd_lmhead_accept(c.B * c.D_max, c.V, c.hidden, s.h_tgt, s.h_drf, s.w_tgt,
+                                  s.w_drf, None, 1.0, s.rng, s.out_tok, s.accepted, s.ratio, None,
+                                  lm_ws, lm_wsb, s.status, cs)
+        else:
+            ssd.ssd_accept(c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0, s.rng, s.out_tok,
+                           s.accepted, s.ratio, None, s.status, cs)
 
     def kernel_ms(call):
         gr = torch.cuda.CUDAGraph()
@@ -332,17 +362,34 @@ def main():
     attn_ms = kernel_ms(attn_call)
     acc_ms = kernel_ms(acc_call)
     hbm_peak, peak_kind = measured_peaks()
-    # the standalone ssd_accept call processes every row of the padded batch
-    acc_bytes_all = c.B * c.D_max * (2 * c.V * 4 + 4 + 1 + 4)
-    kern = {"attention": (attn_bytes, attn_ms), "accept": (acc_bytes_all, acc_ms)}
+    # the standalone acceptance call processes every row of the padded batch
+    if c.hidden:
+        acc_bytes_all = 2 * c.hidden * c.V * 2 + c.B * c.D_max * (2 * c.hidden * 2 + 9)
+    else:
+        acc_bytes_all = c.B * c.D_max * (2 * c.V * 4 + 4 + 1 + 4)
+    kern = {"attention": (attn_bytes, attn_ms),
+            ("lmhead_accept" if c.hidden else "accept"): (acc_bytes_all, acc_ms)}
     dom = max(kern, key=lambda k: kern[k][1])
     dom_bytes, dom_ms = kern[dom]
     achieved = dom_bytes / (dom_ms / 1000.0) / 1e9
     status = int(max(s.status.item() for s in steps_obj))
+    tensor_info = None
+    if c.hidden:
+        # useful contraction work of the fused lm_head: 2 heads x 2 flop x rows x K x V
+        flops = 2 * 2 * c.B * c.D_max * c.hidden * c.V
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+            os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+        tpk = peaks.get("bf16_tflops", 1900.0)
+        tflops = flops / (acc_ms / 1000.0) / 1e12
+        tensor_info = {"kernel": "lmhead_accept", "achieved_tflops": tflops, "peak_tflops": tpk,
+                       "frac": tflops / tpk, "rows": c.B * c.D_max,
+                       "note": "rows padded to 128 per MMA tile; HBM-bound at this row count"}
 
     # ---------------- end to end: host buffers, copies inside the timed region
     host = {}
-    for name in ("cache_len", "q", "k", "v", "tgt", "drf"):
+    in_names = ("cache_len", "q", "k", "v") + (("h_tgt", "h_drf", "w_tgt", "w_drf") if c.hidden
+                                               else ("tgt", "drf"))
+    for name in in_names:
         t = getattr(st, name)
         host[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         host[name].copy_(t)
@@ -392,6 +439,7 @@ def main():
         "accepted_tokens_per_s": world * acc_tok_per_step * a.steps / (ms / 1000.0),
         "committed_tokens_per_step": committed,
         "hbm_gbs_per_step": (attn_bytes + acc_bytes) / (ms_per_step / 1000.0) / 1e9,
+        "tensor": tensor_info,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": None,
                      "peak_kind": peak_kind,

@@ -32,7 +32,10 @@ constexpr int kBM = 128;        // rows per MMA tile (TMEM lanes)
 constexpr int kBN = 128;        // vocabulary entries per CTA
 constexpr int kBK = 64;         // K per stage: one 128-byte swizzle atom of bf16
 constexpr int kMMAK = 16;       // K per tcgen05.mma (kind::f16)
-constexpr int kThreadsL = 128;  // 4 warps = 128 TMEM lanes
+constexpr int kThreadsL = 512;  // warps 0-3 own the 128 TMEM lanes; all 16 share the combines
+constexpr int kTmemWarps = 4;
+constexpr int kCombWarps = kThreadsL / 32;
+constexpr int kMaxTilesPerLane = 8;  // vocabulary tiles per lane in the combines: V <= 32768
 constexpr int kMaxRowTiles = 2; // rows <= 256
 constexpr float kLog2eL = 1.4426950408889634f;
 constexpr float kLn2L = 0.6931471805599453f;
@@ -220,8 +223,12 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // ---- main loop: warp 0 lane 0 produces, warp 1 lane 0 issues the MMAs
-  if (warp == 0 && lane == 0) {
+  // ---- main loop: warp 0 lane 0 produces, warp 1 lane 0 issues the MMAs.
+  // The other lanes of those two warps park at __syncwarp: spinning on an
+  // mbarrier in the same warp would let a suspended try_wait of theirs hold
+  // up the lane that drives the pipeline.
+  if (warp == 0) {
+    if (lane == 0) {
     const uint64_t pol = policy_evict_first();     // weights: read once
     const uint64_t pol_h = policy_evict_last();    // hidden states: read by every CTA
     const uint32_t bytes = (uint32_t)stage_bytes;
@@ -241,7 +248,10 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       tma_load_2d(bd, &tmWd, v0, kb * kBK, &full[s], pol);
       tma_load_2d(bd + kTileB / 2, &tmWd, v0 + 64, kb * kBK, &full[s], pol);
     }
-  } else if (warp == 1 && lane == 0) {
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % S;
       if (!mbar_wait(&full[s], (kb / S) & 1, a.status)) { *fail = 1; break; }
@@ -266,6 +276,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       mma_commit(&empty[s]);
     }
     mma_commit(done);
+    }
+    __syncwarp();
   }
   // every thread waits for the accumulators
   const bool mma_ok = mbar_wait(done, 0, a.status);
@@ -278,8 +290,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   // TMEM lane quarter of this warp: lanes 32*warp .. +31 (row tile m, row m*128 + tid)
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
-  // ---- epilogue 1: per-tile softmax partials of every row
-  for (int m = 0; m < mt && ok; ++m) {
+  // ---- epilogue 1: per-tile softmax partials of every row (TMEM warps)
+  for (int m = 0; m < mt && ok && warp < kTmemWarps; ++m) {
     const int32_t row = m * kBM + tid;
     const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
     float mp = -INFINITY, sp = 0.f, mq = -INFINITY, sq = 0.f;
@@ -336,10 +348,12 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   }
   ok = grid_barrier(L.barrier, (unsigned)L.ncta, a.status, flag) && ok;
 
-  // ---- epilogue 2: combine the partials of each row (warp per row, lanes over
-  // tiles in a fixed order), decide, and on rejection prepare the draw
+  // ---- epilogue 2: combine the partials of each row (warp per row, lane l
+  // merging tiles l, l + 32, ... in order, then a xor tree: the same arithmetic
+  // in every CTA), decide, and on rejection prepare the draw.  All loads of a
+  // row are issued before any merge.
   for (int m = 0; m < mt && ok; ++m) {
-    for (int rl = warp; rl < kBM; rl += kThreadsL / 32) {
+    for (int rl = warp; rl < kBM; rl += kCombWarps) {
       const int32_t row = m * kBM + rl;
       LmSmemRow& ri = rowinfo[m * kBM + rl];
       if (row >= rows) {
@@ -363,15 +377,26 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
         }
         continue;
       }
+      const float4* prow = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta);
+      float4 q0[kMaxTilesPerLane], q1[kMaxTilesPerLane];
+#pragma unroll
+      for (int j = 0; j < kMaxTilesPerLane; ++j) {
+        const int k = lane + 32 * j;
+        if (k < L.ncta) {
+          q0[j] = prow[2 * k];
+          q1[j] = prow[2 * k + 1];
+        }
+      }
       float Mp = -INFINITY, Sp = 0.f, Mq = -INFINITY, Sq = 0.f, xq = -INFINITY, xp = 0.f;
       int32_t t = 0x7fffffff;
-      for (int k = lane; k < L.ncta; k += 32) {
-        const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
-        const float4 p1 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[1];
-        merge_ms(Mp, Sp, p0.x, p0.y, c);
-        merge_ms(Mq, Sq, p0.z, p0.w, c);
-        const int32_t ck = __float_as_int(p1.z);
-        if (ck >= 0 && better(p1.x, ck, xq, t)) { xq = p1.x; xp = p1.y; t = ck; }
+#pragma unroll
+      for (int j = 0; j < kMaxTilesPerLane; ++j) {
+        if (lane + 32 * j < L.ncta) {
+          merge_ms(Mp, Sp, q0[j].x, q0[j].y, c);
+          merge_ms(Mq, Sq, q0[j].z, q0[j].w, c);
+          const int32_t ck = __float_as_int(q1[j].z);
+          if (ck >= 0 && better(q1[j].x, ck, xq, t)) { xq = q1[j].x; xp = q1[j].y; t = ck; }
+        }
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
@@ -417,8 +442,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   __syncthreads();
 
   // ---- epilogue 3: residual mass of this tile for every rejected row
-  // (sequential over the tile in vocabulary order)
-  for (int m = 0; m < mt && ok; ++m) {
+  // (sequential over the tile in vocabulary order; TMEM warps)
+  for (int m = 0; m < mt && ok && warp < kTmemWarps; ++m) {
     const int32_t row = m * kBM + tid;
     const LmSmemRow& ri = rowinfo[m * kBM + tid];
     const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
@@ -441,28 +466,33 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   }
   ok = grid_barrier(L.barrier, 2u * (unsigned)L.ncta, a.status, flag) && ok;
 
-  // ---- epilogue 4: locate the tile holding u_res * Z (warp per row, lanes over
-  // tiles in order; the same arithmetic in every CTA)
+  // ---- epilogue 4: locate the tile holding u_res * Z (warp per row; lane l
+  // owns tiles [l*per, (l+1)*per) and keeps their masses in registers; the
+  // same arithmetic in every CTA)
+  const int32_t per = (L.ncta + 31) / 32;  // <= kMaxTilesPerLane
   for (int m = 0; m < mt && ok; ++m) {
-    for (int rl = warp; rl < kBM; rl += kThreadsL / 32) {
+    for (int rl = warp; rl < kBM; rl += kCombWarps) {
       LmSmemRow& ri = rowinfo[m * kBM + rl];
       if (ri.state != 1) continue;
       const int32_t row = m * kBM + rl;
-      const int32_t per = (L.ncta + 31) / 32;
       for (int fp = 0; fp < 2; ++fp) {
-        // lane l owns tiles [l*per, (l+1)*per); fp = 1: masses of p itself
-        float ls = 0.f;
-        for (int q = 0; q < per; ++q) {
+        float mk[kMaxTilesPerLane];
+#pragma unroll
+        for (int q = 0; q < kMaxTilesPerLane; ++q) {
           const int k = lane * per + q;
-          if (k < L.ncta) {
+          mk[q] = 0.f;
+          if (q < per && k < L.ncta) {
             if (fp == 0) {
-              ls += L.mass[(int64_t)row * L.ncta + k];
-            } else {
+              mk[q] = L.mass[(int64_t)row * L.ncta + k];
+            } else {  // masses of p itself, from the tile partials
               const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
-              ls += p0.y * ex2f(p0.x * c - ri.Cp);
+              mk[q] = p0.y * ex2f(p0.x * c - ri.Cp);
             }
           }
         }
+        float ls = 0.f;
+#pragma unroll
+        for (int q = 0; q < kMaxTilesPerLane; ++q) ls += mk[q];
         float incl = ls;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -486,21 +516,15 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
         if (lane == lstar) {
           int32_t ks = -1, klast = -1;
           float tk = INFINITY, cum = 0.f;
-          for (int q = 0; q < per; ++q) {
-            const int k = lane * per + q;
-            if (k >= L.ncta) break;
-            float mk;
-            if (fp == 0) {
-              mk = L.mass[(int64_t)row * L.ncta + k];
-            } else {
-              const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
-              mk = p0.y * ex2f(p0.x * c - ri.Cp);
+#pragma unroll
+          for (int q = 0; q < kMaxTilesPerLane; ++q) {
+            if (q < per && lane * per + q < L.ncta) {
+              if (mk[q] > 0.f) {
+                klast = lane * per + q;
+                if (ks < 0 && cum + mk[q] > t1) { ks = klast; tk = t1 - cum; }
+              }
+              cum += mk[q];
             }
-            if (mk > 0.f) {
-              klast = k;
-              if (ks < 0 && cum + mk > t1) { ks = k; tk = t1 - cum; }
-            }
-            cum += mk;
           }
           if (ks < 0) { ks = klast; tk = INFINITY; }
           ri.cstar = ks;
@@ -515,7 +539,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   __syncthreads();
 
   // ---- epilogue 5: the CTA holding the crossing scans its tile sequentially
-  for (int m = 0; m < mt && ok; ++m) {
+  for (int m = 0; m < mt && ok && warp < kTmemWarps; ++m) {
     const int32_t row = m * kBM + tid;
     const LmSmemRow& ri = rowinfo[m * kBM + tid];
     const bool mine = row < rows && ri.state == 1 && ri.cstar == cta;
@@ -608,6 +632,7 @@ ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K) {
   if (rows < 1 || rows > kMaxRowTiles * kBM) return SSD_ERR_UNSUPPORTED;
   if (K <= 0 || K % kBK != 0) return SSD_ERR_UNSUPPORTED;
   if (V <= 0 || V % kBN != 0) return SSD_ERR_UNSUPPORTED;
+  if (V / kBN > 32 * kMaxTilesPerLane) return SSD_ERR_UNSUPPORTED;
   // every CTA must be resident at once (one CTA per SM: TMEM and shared memory)
   const int mt = row_tiles(rows);
   int per_sm = 0;
