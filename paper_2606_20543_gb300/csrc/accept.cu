@@ -4,27 +4,49 @@
 //   accept t with probability min(p(t) / q(t), 1); otherwise draw from
 //   [p - q]_+ / sum [p - q]_+ (inverse CDF in vocabulary order, one uniform).
 //
-// Design (GB300): one CTA of 256 threads per row, no shared-memory copy of
-// the row (so many rows stream at once).  Pass A reads both logit rows from
-// HBM once with 16-byte loads, four per row per thread in flight, and keeps
-// online (max, sum of 2^x) statistics and the first argmax in registers; one
-// block reduction in a fixed order gives the log-sum-exps and the draft
-// token, and thread 0 takes the decision.  Only rejected rows run pass B: the
-// rows are re-read from L2 (they were read microseconds earlier; these loads
-// mark the lines evict-first), the residual weights are formed with MUFU
-// exp2, and the mass of every 128-entry chunk goes to shared memory in
-// vocabulary order.  Warp 0 scans the chunk masses, finds the chunk holding
-// u_res * Z, and re-walks that chunk to pick the token.
+// Design (GB300): a persistent grid of several CTAs per SM, each walking rows
+// blockIdx.x, blockIdx.x + gridDim.x, ...  A dedicated producer warp streams
+// every row twice with bulk TMA copies, 256 entries per consumer warp of both
+// logit rows per stage, through a shared-memory ring: once from HBM for the
+// statistics, and once more (from L2, microseconds later) for the residual
+// draw; it runs ahead into the next row while the consumers finish the
+// current one.  Eight consumer warps fold each first-pass chunk into online
+// (max, sum of 2^x) statistics, one max and at most one rescale per chunk, and
+// the first argmax (carrying the target logit at it); a block reduction in a fixed order gives the log-sum-exps
+// and the draft token, and one thread takes the decision.  For rejected rows
+// the second-pass chunks give the residual weights (MUFU exp2) and the mass
+// of every 256-entry block in vocabulary order; warp 0 scans the block masses,
+// finds the block holding u_res * Z and re-walks it to pick the token.
+// Accepted rows only release their second-pass chunks.
+#include <algorithm>
+
 #include "kernels.cuh"
 
 namespace ssd {
 
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-constexpr int kUnroll = 4;             // float4 loads per row per thread in flight
-constexpr int kMaxV = 1 << 20;         // chunk-mass table: V / 128 floats of shared memory
+#ifndef SSD_ACCEPT_CWARPS
+#define SSD_ACCEPT_CWARPS 8
+#endif
+#ifndef SSD_ACCEPT_STAGES
+#define SSD_ACCEPT_STAGES 4
+#endif
+#ifndef SSD_ACCEPT_CTAS
+#define SSD_ACCEPT_CTAS 3
+#endif
+constexpr int kCWarps = SSD_ACCEPT_CWARPS;    // consumer warps
+constexpr int kConsumers = kCWarps * 32;
+constexpr int kThreads = kConsumers + 32;     // + the producer warp
+// Entries of each row per ring stage.  Pass A gives every consumer thread two
+// float4 of each row per chunk and pass B gives every consumer warp one
+// 256-entry block per chunk, so a chunk is exactly 256 entries per warp.
+constexpr int kChunk = 256 * kCWarps;
+constexpr int kStages = SSD_ACCEPT_STAGES;
+constexpr int kCtasPerSm = SSD_ACCEPT_CTAS;
+static_assert(kChunk == 2 * 4 * kConsumers, "pass A covers two float4 per thread per chunk");
+static_assert(kCWarps == 4 || kCWarps == 8, "consumer warps");
+constexpr int kMaxV = 1 << 20;                // block-mass table: V / 128 floats of shared memory
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -35,37 +57,13 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Streaming 16-byte loads: the first read of a row keeps it in L2 for the
-// residual pass; the residual pass marks its lines evict-first (last use).
-__device__ __forceinline__ float4 ld_keep(const float4* p) {
-  float4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
-  return v;
-}
-__device__ __forceinline__ float4 ld_last(const float4* p, uint64_t pol) {
-  float4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p), "l"(pol));
-  return v;
+// Barrier among the consumer warps only (the producer warp never joins it).
+__device__ __forceinline__ void consumers_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory");
 }
 
 __device__ __forceinline__ bool better_arg(float v, int32_t i, float bv, int32_t bi) {
   return v > bv || (v == bv && (uint32_t)i < (uint32_t)bi);
-}
-
-// Online (max, sum of exp2((x - max) * c)) over 4 more entries.
-__device__ __forceinline__ void online4(float& m, float& s, const float4& x, float c) {
-  const float mx = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
-  if (mx > m) {
-    s *= ex2((m - mx) * c);  // m == -inf: s is 0 and stays 0
-    m = mx;
-  }
-  if (m != -INFINITY) {
-    const float mc = m * c;
-    s += (ex2(fmaf(x.x, c, -mc)) + ex2(fmaf(x.y, c, -mc))) +
-         (ex2(fmaf(x.z, c, -mc)) + ex2(fmaf(x.w, c, -mc)));
-  }
 }
 
 // Merge two (max, sum) pairs.
@@ -96,260 +94,367 @@ __device__ __forceinline__ float4 weights4(const float4& xp, const float4& xq, f
 }
 
 struct Shared {
-  float red[kWarps][4];
-  int32_t red_i[kWarps];
+  uint64_t full[kStages], empty[kStages];
+  float red[kCWarps][5];
+  int32_t red_i[kCWarps];
   float Cp, Cq;      // log2-domain normalisers: max * c + log2(sum)
-  int32_t accept;    // 1 accepted, 0 rejected, 2 no valid draft token
+  int32_t accept;    // 1 accepted, 0 rejected, 2 no valid draft token, 3 drawn
   float u_res;
+  float xp_t, xq_t;  // logits at a caller-given draft token (pass A)
 };
 
-// One CTA per row.  Pass A streams both logit rows once from HBM and keeps
-// online statistics; pass B (rejected rows only) re-reads them from L2,
-// computes the residual weights and the mass of every 128-entry chunk (warp w
-// of iteration k owns entries [(8k + w) * 128, +128), so chunks are in
-// vocabulary order); warp 0 then scans the chunk masses and re-walks the
-// chunk holding the CDF crossing.
-__global__ void __launch_bounds__(kThreads, 4) accept_kernel(AcceptArgs a) {
-  extern __shared__ float chunk_mass[];  // [V / 128] (rounded up to whole iterations)
-  __shared__ Shared sh;
-  const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t r = blockIdx.x;
-
-  // ---- rows outside the frontier (padding slots of a verification step)
+// Rows that stream: frontier rows with an in-range (or absent) draft token.
+// Producer and consumers walk the same rows and skip the same ones.
+__device__ __forceinline__ int row_kind(const AcceptArgs& a, int64_t r) {
   if (a.n_drafts != nullptr) {
     const int32_t b = (int32_t)(r / a.D_max), j = (int32_t)(r % a.D_max);
-    if (j >= a.n_drafts[b]) {
-      if (tid == 0) {
-        a.out_tok[r] = -1;
-        a.accepted[r] = 0;
-        if (a.ratio) a.ratio[r] = 0.f;
-        if (a.lse) { a.lse[2 * r] = 0.f; a.lse[2 * r + 1] = 0.f; }
-      }
-      return;
-    }
+    if (j >= a.n_drafts[b]) return 1;  // padding slot
   }
-  int32_t given_t = -1;
   if (a.draft_tok != nullptr) {
-    given_t = a.draft_tok[r];
-    if (given_t < 0 || given_t >= a.V) {
+    const int32_t t = a.draft_tok[r];
+    if (t < 0 || t >= a.V) return 2;   // draft token out of range
+  }
+  return 0;
+}
+
+// Block of 256 entries (64 float4) inside a ring chunk, one per consumer warp:
+// warp w holds the chunk's float4 w * 64 + lane (first half of the block) and
+// w * 64 + 32 + lane (second half).
+constexpr int kBlocksPerChunk = kChunk / 256;  // one per consumer warp
+static_assert(kBlocksPerChunk == kCWarps, "pass B: one block per consumer warp per chunk");
+// Initial running maximum: finite, so exp2 arguments never meet (-inf) - (-inf).
+constexpr float kLowest = -1.0e30f;
+
+// Scan the block masses in vocabulary order (warp 0): returns the block
+// holding target = u * Z and the remaining target inside it (INF: take the
+// last positive entry), or -1 if Z == 0.
+__device__ __forceinline__ int32_t find_block(const float* mass, int32_t nblocks, float u,
+                                              float* t_in_block, int lane) {
+  const int32_t per = (nblocks + 31) / 32;
+  float ls = 0.f;
+  for (int32_t q = 0; q < per; ++q) {
+    const int32_t bk = lane * per + q;
+    ls += (bk < nblocks) ? mass[bk] : 0.f;
+  }
+  float incl = ls;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  const float Z = __shfl_sync(0xffffffffu, incl, 31);
+  if (!(Z > 0.f)) return -1;
+  const float target = u * Z;
+  const uint32_t pos = __ballot_sync(0xffffffffu, ls > 0.f);
+  const uint32_t cross = __ballot_sync(0xffffffffu, ls > 0.f && incl > target);
+  const int32_t ls_star = cross ? (__ffs(cross) - 1) : (31 - __clz(pos));
+  float t1 = __shfl_sync(0xffffffffu, incl - ls, ls_star);
+  t1 = cross ? target - t1 : INFINITY;
+  int32_t bs = -1, blast = -1;
+  float tb = INFINITY;
+  if (lane == ls_star) {
+    float cum = 0.f;
+    for (int32_t q = 0; q < per; ++q) {
+      const int32_t bk = lane * per + q;
+      const float m = (bk < nblocks) ? mass[bk] : 0.f;
+      if (m > 0.f) {
+        blast = bk;
+        if (bs < 0 && cum + m > t1) { bs = bk; tb = t1 - cum; }
+      }
+      cum += m;
+    }
+    if (bs < 0) { bs = blast; tb = INFINITY; }
+  }
+  bs = __shfl_sync(0xffffffffu, bs, ls_star);
+  *t_in_block = __shfl_sync(0xffffffffu, tb, ls_star);
+  return bs;
+}
+
+// Warp 0: re-walk 256-entry block `bk` (its two 128-entry halves in order)
+// with the arithmetic of the mass pass and return the token at the crossing.
+__device__ __forceinline__ int32_t walk_block(const float4* tp, const float4* dp, int32_t bk,
+                                              int32_t nv, float c, float Cp, float Cq, bool from_p,
+                                              float tb, int lane) {
+  int32_t last_pos = -1;
+  float run = 0.f;
+  for (int half = 0; half < 2; ++half) {
+    const int32_t i = bk * 64 + half * 32 + lane;
+    float4 xp = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY), xq = xp;
+    if (i < nv) {
+      xp = tp[i];
+      xq = from_p ? xp : dp[i];
+    }
+    const float4 w = weights4(xp, xq, c, Cp, Cq, from_p);
+    const float lsum = (w.x + w.y) + (w.z + w.w);
+    float li = lsum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, li, o);
+      if (lane >= o) li += y;
+    }
+    const float hsum = __shfl_sync(0xffffffffu, li, 31);
+    const int32_t e = 4 * i;
+    int32_t lp = -1;  // last entry of this lane with positive weight
+    if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
+    else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
+    const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
+    if (hasp) last_pos = __shfl_sync(0xffffffffu, lp, 31 - __clz(hasp));
+    const float th = tb - run;  // target left for this half
+    if (hsum > 0.f && th < hsum) {
+      const uint32_t lcross = __ballot_sync(0xffffffffu, lsum > 0.f && li > th);
+      const int32_t lstar = lcross ? (__ffs(lcross) - 1) : (31 - __clz(hasp));
+      int32_t pick = -1;
+      if (lane == lstar) {
+        const float t4 = th - (li - lsum);
+        const float ws[4] = {w.x, w.y, w.z, w.w};
+        float cc = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          cc += ws[k];
+          if (pick < 0 && ws[k] > 0.f && cc > t4) pick = e + k;
+        }
+        if (pick < 0) pick = lp;
+      }
+      return __shfl_sync(0xffffffffu, pick, lstar);
+    }
+    run += hsum;
+  }
+  return last_pos;  // rounding ran past the end of the block
+}
+
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs a) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  float* ring = reinterpret_cast<float*>(smem_raw);                  // [kStages][2][kChunk]
+  float* block_mass = ring + kStages * 2 * kChunk;                   // [nch * 16]
+  __shared__ Shared sh;
+  const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int32_t nch = (a.V + kChunk - 1) / kChunk;
+
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sh.full[s], 1);
+      mbar_init(&sh.empty[s], kCWarps);
+    }
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  // ------------------------------------------------------------ producer warp
+  if (warp == kCWarps) {
+    if (lane == 0) {
+      uint32_t g = 0;  // chunks issued by this CTA
+      for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
+        if (row_kind(a, r) != 0) continue;
+        for (int32_t cc = 0; cc < 2 * nch; ++cc, ++g) {  // two passes over the row
+          const int32_t ch = cc % nch;
+          const int s = g % kStages;
+          if (g >= kStages) mbar_wait(&sh.empty[s], ((g / kStages) - 1) & 1, a.status);
+          const uint32_t bytes = (uint32_t)min(kChunk, a.V - ch * kChunk) * 4u;
+          float* dst = ring + s * 2 * kChunk;
+          mbar_arrive_expect_tx(&sh.full[s], 2u * bytes);
+          bulk_g2s(dst, a.tgt + r * a.ld + (int64_t)ch * kChunk, bytes, &sh.full[s]);
+          bulk_g2s(dst + kChunk, a.drf + r * a.ld + (int64_t)ch * kChunk, bytes, &sh.full[s]);
+        }
+      }
+    }
+    __syncwarp();
+    return;
+  }
+
+  // ---------------------------------------------------------- consumer warps
+  const float c = kLog2e / a.temperature;
+  const int32_t nv = a.V >> 2;
+  const int32_t nblocks = nch * kBlocksPerChunk;
+  uint32_t g = 0;  // chunks consumed
+  for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
+    const int kind = row_kind(a, r);
+    if (kind != 0) {
       if (tid == 0) {
-        record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         a.out_tok[r] = -1;
         a.accepted[r] = 0;
         if (a.ratio) a.ratio[r] = 0.f;
+        if (kind == 1 && a.lse) { a.lse[2 * r] = 0.f; a.lse[2 * r + 1] = 0.f; }
+        if (kind == 2) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
       }
-      return;
+      continue;
     }
-  }
+    const int32_t given_t = a.draft_tok != nullptr ? a.draft_tok[r] : -1;
 
-  const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
-  const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
-  const int32_t nv = a.V >> 2;
-  const float c = kLog2e / a.temperature;
-
-  // ---- pass A: online max / sum-exp of both rows, first argmax of the draft row
-  float mp = -INFINITY, sp = 0.f, mq = -INFINITY, sq = 0.f;
-  int32_t iq = 0x7fffffff;
-  for (int32_t base = tid; base < nv; base += kThreads * kUnroll) {
-    float4 xp[kUnroll], xq[kUnroll];
+    // ---- pass A: per chunk, each thread takes 8 entries of both rows
+    // (float4 tid and tid + 256 of the chunk, ascending): one max, at most one
+    // rescale, then the exponentials; the first argmax of q carries the p logit
+    float mp = kLowest, sp = 0.f, mq = kLowest, sq = 0.f, xpa = 0.f;
+    int32_t iq = 0x7fffffff;
+    const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    for (int32_t ch = 0; ch < nch; ++ch, ++g) {
+      const int s = g % kStages;
+      mbar_wait(&sh.full[s], (g / kStages) & 1, a.status);
+      const float4* xp4 = reinterpret_cast<const float4*>(ring + s * 2 * kChunk);
+      const float4* xq4 = reinterpret_cast<const float4*>(ring + s * 2 * kChunk + kChunk);
+      const int32_t cv = min(kChunk, a.V - ch * kChunk) >> 2;
+      const bool in0 = tid < cv, in1 = tid + kConsumers < cv;
+      const float4 p0 = in0 ? xp4[tid] : ninf, p1 = in1 ? xp4[tid + kConsumers] : ninf;
+      const float4 q0 = in0 ? xq4[tid] : ninf, q1 = in1 ? xq4[tid + kConsumers] : ninf;
+      const float cmp = fmaxf(fmaxf(fmaxf(p0.x, p0.y), fmaxf(p0.z, p0.w)),
+                              fmaxf(fmaxf(p1.x, p1.y), fmaxf(p1.z, p1.w)));
+      const float cmq = fmaxf(fmaxf(fmaxf(q0.x, q0.y), fmaxf(q0.z, q0.w)),
+                              fmaxf(fmaxf(q1.x, q1.y), fmaxf(q1.z, q1.w)));
+      if (cmp > mp) {
+        sp *= ex2((mp - cmp) * c);
+        mp = cmp;
+      }
+      if (cmq > mq) {
+        sq *= ex2((mq - cmq) * c);
+        mq = cmq;
+        const int32_t e0 = ch * kChunk + 4 * tid, e1 = e0 + 4 * kConsumers;
+        if (q0.x == cmq) { iq = e0; xpa = p0.x; }
+        else if (q0.y == cmq) { iq = e0 + 1; xpa = p0.y; }
+        else if (q0.z == cmq) { iq = e0 + 2; xpa = p0.z; }
+        else if (q0.w == cmq) { iq = e0 + 3; xpa = p0.w; }
+        else if (q1.x == cmq) { iq = e1; xpa = p1.x; }
+        else if (q1.y == cmq) { iq = e1 + 1; xpa = p1.y; }
+        else if (q1.z == cmq) { iq = e1 + 2; xpa = p1.z; }
+        else { iq = e1 + 3; xpa = p1.w; }
+      }
+      // a thread that has seen only -inf keeps kLowest: its terms are exp2(-inf) = 0
+      const float mpc = (mp == kLowest) ? 0.f : mp * c, mqc = (mq == kLowest) ? 0.f : mq * c;
+      sp += ((ex2(fmaf(p0.x, c, -mpc)) + ex2(fmaf(p0.y, c, -mpc))) +
+             (ex2(fmaf(p0.z, c, -mpc)) + ex2(fmaf(p0.w, c, -mpc)))) +
+            ((ex2(fmaf(p1.x, c, -mpc)) + ex2(fmaf(p1.y, c, -mpc))) +
+             (ex2(fmaf(p1.z, c, -mpc)) + ex2(fmaf(p1.w, c, -mpc))));
+      sq += ((ex2(fmaf(q0.x, c, -mqc)) + ex2(fmaf(q0.y, c, -mqc))) +
+             (ex2(fmaf(q0.z, c, -mqc)) + ex2(fmaf(q0.w, c, -mqc)))) +
+            ((ex2(fmaf(q1.x, c, -mqc)) + ex2(fmaf(q1.y, c, -mqc))) +
+             (ex2(fmaf(q1.z, c, -mqc)) + ex2(fmaf(q1.w, c, -mqc))));
+      if (given_t >= 0 && (given_t / kChunk) == ch) {
+        const int32_t off = given_t - ch * kChunk;  // entry inside the chunk
+        const int32_t f = off >> 2, k = off & 3;
+        if (f == tid || f == tid + kConsumers) {
+          const float4 gp = (f == tid) ? p0 : p1, gq = (f == tid) ? q0 : q1;
+          sh.xp_t = k == 0 ? gp.x : k == 1 ? gp.y : k == 2 ? gp.z : gp.w;
+          sh.xq_t = k == 0 ? gq.x : k == 1 ? gq.y : k == 2 ? gq.z : gq.w;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sh.empty[s]);
+    }
+    // block reduction in a fixed order: xor tree in warps, then warps 0..7
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int32_t i = base + u * kThreads;
-      if (i < nv) {
-        xp[u] = ld_keep(tp + i);
-        xq[u] = ld_keep(dp + i);
+    for (int o = 16; o > 0; o >>= 1) {
+      merge(mp, sp, __shfl_xor_sync(0xffffffffu, mp, o), __shfl_xor_sync(0xffffffffu, sp, o), c);
+      const float om = __shfl_xor_sync(0xffffffffu, mq, o);
+      const float os = __shfl_xor_sync(0xffffffffu, sq, o);
+      const int32_t oi = __shfl_xor_sync(0xffffffffu, iq, o);
+      const float op = __shfl_xor_sync(0xffffffffu, xpa, o);
+      const bool take = better_arg(om, oi, mq, iq);
+      merge(mq, sq, om, os, c);
+      if (take) { iq = oi; xpa = op; }
+    }
+    if (lane == 0) {
+      sh.red[warp][0] = mp;
+      sh.red[warp][1] = sp;
+      sh.red[warp][2] = mq;
+      sh.red[warp][3] = sq;
+      sh.red[warp][4] = xpa;
+      sh.red_i[warp] = iq;
+    }
+    consumers_sync();
+    if (tid == 0) {
+      float Mp = sh.red[0][0], Sp = sh.red[0][1], Mq = sh.red[0][2], Sq = sh.red[0][3];
+      float xp_t = sh.red[0][4];
+      int32_t t = sh.red_i[0];
+      for (int w = 1; w < kCWarps; ++w) {
+        merge(Mp, Sp, sh.red[w][0], sh.red[w][1], c);
+        const bool take = better_arg(sh.red[w][2], sh.red_i[w], Mq, t);
+        merge(Mq, Sq, sh.red[w][2], sh.red[w][3], c);
+        if (take) { t = sh.red_i[w]; xp_t = sh.red[w][4]; }
+      }
+      float xq_t = Mq;
+      if (given_t >= 0) {
+        t = given_t;
+        xp_t = sh.xp_t;
+        xq_t = sh.xq_t;
+      }
+      const bool valid_t = t >= 0 && t < a.V;
+      float ratio = 0.f;
+      bool acc = false;
+      const float2 u = row_uniforms(a.rng, r);
+      if (valid_t) {
+        const float l2p = (xp_t - Mp) * c - log2f(Sp);
+        const float l2q = (xq_t - Mq) * c - log2f(Sq);
+        ratio = exp2f(l2p - l2q);
+        acc = u.x < fminf(ratio, 1.0f);
       } else {
-        xp[u] = xq[u] = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
+      }
+      sh.accept = acc ? 1 : (valid_t ? 0 : 2);
+      sh.u_res = u.y;
+      sh.Cp = Mp * c + log2f(Sp);
+      sh.Cq = Mq * c + log2f(Sq);
+      a.accepted[r] = acc ? 1 : 0;
+      if (acc) a.out_tok[r] = t;
+      else if (!valid_t) a.out_tok[r] = -1;
+      if (a.ratio) a.ratio[r] = ratio;
+      if (a.lse) {
+        a.lse[2 * r] = Mp / a.temperature + log2f(Sp) * kLn2;
+        a.lse[2 * r + 1] = Mq / a.temperature + log2f(Sq) * kLn2;
       }
     }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      online4(mp, sp, xp[u], c);
-      // draft row: entries visited in ascending order, strict '>' keeps the first max
-      const float4 x = xq[u];
-      const float mx = fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w));
-      if (mx > mq) {
-        const int32_t e = 4 * (base + u * kThreads);
-        iq = e + (x.x == mx ? 0 : x.y == mx ? 1 : x.z == mx ? 2 : 3);
-      }
-      online4(mq, sq, x, c);
-    }
-  }
-  // block reduction (fixed order: xor tree in warps, then warps 0..7)
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    merge(mp, sp, __shfl_xor_sync(0xffffffffu, mp, o), __shfl_xor_sync(0xffffffffu, sp, o), c);
-    const float om = __shfl_xor_sync(0xffffffffu, mq, o);
-    const float os = __shfl_xor_sync(0xffffffffu, sq, o);
-    const int32_t oi = __shfl_xor_sync(0xffffffffu, iq, o);
-    const bool take = better_arg(om, oi, mq, iq);
-    merge(mq, sq, om, os, c);
-    if (take) iq = oi;
-  }
-  if (lane == 0) {
-    sh.red[warp][0] = mp;
-    sh.red[warp][1] = sp;
-    sh.red[warp][2] = mq;
-    sh.red[warp][3] = sq;
-    sh.red_i[warp] = iq;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    float Mp = sh.red[0][0], Sp = sh.red[0][1], Mq = sh.red[0][2], Sq = sh.red[0][3];
-    int32_t t = sh.red_i[0];
-    for (int w = 1; w < kWarps; ++w) {
-      merge(Mp, Sp, sh.red[w][0], sh.red[w][1], c);
-      const bool take = better_arg(sh.red[w][2], sh.red_i[w], Mq, t);
-      merge(Mq, Sq, sh.red[w][2], sh.red[w][3], c);
-      if (take) t = sh.red_i[w];
-    }
-    if (given_t >= 0) t = given_t;
-    const bool valid_t = t >= 0 && t < a.V;
-    float ratio = 0.f;
-    bool acc = false;
-    const float2 u = row_uniforms(a.rng, r);
-    if (valid_t) {
-      const float xp_t = a.tgt[r * a.ld + t];  // L2-resident after pass A
-      const float xq_t = a.drf[r * a.ld + t];
-      const float l2p = (xp_t - Mp) * c - log2f(Sp);
-      const float l2q = (xq_t - Mq) * c - log2f(Sq);
-      ratio = exp2f(l2p - l2q);
-      acc = u.x < fminf(ratio, 1.0f);
-    } else {
-      record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
-    }
-    sh.accept = acc ? 1 : (valid_t ? 0 : 2);
-    sh.u_res = u.y;
-    sh.Cp = Mp * c + log2f(Sp);
-    sh.Cq = Mq * c + log2f(Sq);
-    a.accepted[r] = acc ? 1 : 0;
-    if (acc) a.out_tok[r] = t;
-    else if (!valid_t) a.out_tok[r] = -1;
-    if (a.ratio) a.ratio[r] = ratio;
-    if (a.lse) {
-      a.lse[2 * r] = Mp / a.temperature + log2f(Sp) * kLn2;
-      a.lse[2 * r + 1] = Mq / a.temperature + log2f(Sq) * kLn2;
-    }
-  }
-  __syncthreads();
-  if (sh.accept != 0) return;
+    consumers_sync();
+    const bool draw = (sh.accept == 0);
+    const float Cp = sh.Cp, Cq = sh.Cq;
 
-  // ---- pass B: residual draw from [p - q]_+ (or from p when that mass is zero)
-  const float Cp = sh.Cp, Cq = sh.Cq;
-  const uint64_t pol = policy_evict_first();
-  const int32_t iters = (nv + kThreads - 1) / kThreads;  // 1024 entries per iteration
-  const int32_t nchunks = iters * kWarps;
-  for (int pass = 0; pass < 2; ++pass) {
-    const bool from_p = (pass == 1);
-    for (int32_t k0 = 0; k0 < iters; k0 += kUnroll) {
-      float4 xp[kUnroll], xq[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int32_t i = (k0 + u) * kThreads + tid;
-        if (k0 + u < iters && i < nv) {
-          xp[u] = ld_last(tp + i, pol);
-          xq[u] = from_p ? xp[u] : ld_last(dp + i, pol);
-        } else {
-          xp[u] = xq[u] = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-        }
+    // ---- pass B: second-pass chunks; residual mass of every 256-entry block
+    for (int32_t ch = 0; ch < nch; ++ch, ++g) {
+      const int s = g % kStages;
+      mbar_wait(&sh.full[s], (g / kStages) & 1, a.status);
+      if (draw) {
+        const float4* xp4 = reinterpret_cast<const float4*>(ring + s * 2 * kChunk);
+        const float4* xq4 = reinterpret_cast<const float4*>(ring + s * 2 * kChunk + kChunk);
+        const int32_t cv = min(kChunk, a.V - ch * kChunk) >> 2;
+        const int32_t i0 = warp * 64 + lane, i1 = i0 + 32;
+        float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
+        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], c, Cp, Cq, false);
+        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], c, Cp, Cq, false);
+        const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
+        if (lane == 0) block_mass[ch * kBlocksPerChunk + warp] = m;
       }
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        if (k0 + u < iters) {
-          const float4 w = weights4(xp[u], xq[u], c, Cp, Cq, from_p);
-          const float m = warp_sum((w.x + w.y) + (w.z + w.w));
-          if (lane == 0) chunk_mass[(k0 + u) * kWarps + warp] = m;
-        }
-      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sh.empty[s]);
     }
-    __syncthreads();
+    if (!draw) continue;  // uniform
+    consumers_sync();
+    const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
+    const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
     if (warp == 0) {
-      // chunk masses in vocabulary order: lane l owns chunks [l*per, (l+1)*per)
-      const int32_t per = (nchunks + 31) / 32;
-      float ls = 0.f;
-      for (int32_t q = 0; q < per; ++q) {
-        const int32_t ch = lane * per + q;
-        ls += (ch < nchunks) ? chunk_mass[ch] : 0.f;
+      float tb;
+      int32_t bk = find_block(block_mass, nblocks, sh.u_res, &tb, lane);
+      bool from_p = false;
+      if (bk < 0) {
+        // zero residual mass: the same draw from p (block masses of p itself)
+        from_p = true;
+        for (int32_t b0 = 0; b0 < nblocks; ++b0) {
+          const int32_t i0 = b0 * 64 + lane, i1 = i0 + 32;
+          float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
+          if (i0 < nv) w0 = weights4(tp[i0], tp[i0], c, Cp, Cq, true);
+          if (i1 < nv) w1 = weights4(tp[i1], tp[i1], c, Cp, Cq, true);
+          const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
+          if (lane == 0) block_mass[b0] = m;
+        }
+        __syncwarp();
+        bk = find_block(block_mass, nblocks, sh.u_res, &tb, lane);
       }
-      float incl = ls;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const float y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      const float Z = __shfl_sync(0xffffffffu, incl, 31);
-      if (!(Z > 0.f)) {
-        if (from_p && lane == 0) {  // no positive mass at all (non-finite logits)
+      if (bk < 0) {
+        if (lane == 0) {  // no positive mass at all (non-finite logits)
           a.out_tok[r] = -1;
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
       } else {
-        const float target = sh.u_res * Z;
-        // lane holding the crossing (else the last lane with mass)
-        const uint32_t pos = __ballot_sync(0xffffffffu, ls > 0.f);
-        const uint32_t cross = __ballot_sync(0xffffffffu, ls > 0.f && incl > target);
-        const int32_t ls_star = cross ? (__ffs(cross) - 1) : (31 - __clz(pos));
-        float t1 = __shfl_sync(0xffffffffu, incl - ls, ls_star);
-        t1 = cross ? target - t1 : INFINITY;
-        // chunk inside that lane's range (same order as its sum)
-        int32_t chs = -1, chlast = -1;
-        float tch = INFINITY;
-        if (lane == ls_star) {
-          float cum = 0.f;
-          for (int32_t q = 0; q < per; ++q) {
-            const int32_t ch = lane * per + q;
-            const float m = (ch < nchunks) ? chunk_mass[ch] : 0.f;
-            if (m > 0.f) {
-              chlast = ch;
-              if (chs < 0 && cum + m > t1) { chs = ch; tch = t1 - cum; }
-            }
-            cum += m;
-          }
-          if (chs < 0) { chs = chlast; tch = INFINITY; }
-        }
-        chs = __shfl_sync(0xffffffffu, chs, ls_star);
-        tch = __shfl_sync(0xffffffffu, tch, ls_star);
-        // re-walk chunk chs = 8k + w: entries 4 * (k * 256 + w * 32 + lane) + 0..3
-        const int32_t kk = chs / kWarps, ww = chs % kWarps;
-        const int32_t i = kk * kThreads + ww * 32 + lane;
-        float4 xp = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY), xq = xp;
-        if (i < nv) {
-          xp = ld_keep(tp + i);
-          xq = from_p ? xp : ld_keep(dp + i);
-        }
-        const float4 w = weights4(xp, xq, c, Cp, Cq, from_p);
-        const float lsum = (w.x + w.y) + (w.z + w.w);
-        float li = lsum;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const float y = __shfl_up_sync(0xffffffffu, li, o);
-          if (lane >= o) li += y;
-        }
-        const int32_t e = 4 * i;
-        int32_t lp = -1;  // last entry of this lane with positive weight
-        if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
-        else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
-        const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
-        const uint32_t lcross = __ballot_sync(0xffffffffu, lsum > 0.f && li > tch);
-        const int32_t lstar = lcross ? (__ffs(lcross) - 1) : (hasp ? 31 - __clz(hasp) : 0);
-        if (lane == lstar) {
-          const float t4 = tch - (li - lsum);
-          const float ws[4] = {w.x, w.y, w.z, w.w};
-          float cc = 0.f;
-          int32_t pick = -1;
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            cc += ws[k];
-            if (pick < 0 && ws[k] > 0.f && cc > t4) pick = e + k;
-          }
-          if (pick < 0) pick = lp;
-          a.out_tok[r] = pick;
-        }
+        const int32_t pick = walk_block(tp, dp, bk, nv, c, Cp, Cq, from_p, tb, lane);
+        if (lane == 0) a.out_tok[r] = pick;
       }
-      if (lane == 0) sh.accept = (Z > 0.f) ? 3 : 0;  // 3: drawn
     }
-    __syncthreads();
-    if (sh.accept == 3 || from_p) break;
+    consumers_sync();  // block masses and sh are reused by the next row
   }
 }
 
@@ -359,15 +464,14 @@ bool accept_supported(int32_t V) { return V <= kMaxV; }
 
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
   if (a.rows == 0) return cudaSuccess;
-  const int32_t nv = a.V / 4;
-  const int32_t iters = (nv + kThreads - 1) / kThreads;
-  const size_t smem = (size_t)iters * kWarps * sizeof(float);
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  accept_kernel<<<(unsigned)a.rows, kThreads, smem, stream>>>(a);
+  const int32_t nch = (a.V + kChunk - 1) / kChunk;
+  const size_t smem = (size_t)kStages * 2 * kChunk * sizeof(float) +
+                      (size_t)nch * kBlocksPerChunk * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  const int64_t grid = std::min<int64_t>(a.rows, (int64_t)kCtasPerSm * device_sm_count());
+  accept_kernel<<<(unsigned)grid, kThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
