@@ -285,3 +285,16 @@ WORKLOADS = {
     4: config4,
     5: config5,
 }
+
+
+def replay_pool(B, D_max, V, seed, sets=2, logits="zipf"):
+    """Logit sets for a replay: step t uses set t % sets (rows b * D_max + j)
+    and Philox uniforms with offset t.  Returns a list of (tgt, drf) pairs."""
+    out = []
+    for k in range(sets):
+        rng = np.random.default_rng(np.random.PCG64(seed * 1000 + k))
+        if logits == "zipf":
+            out.append(_logits_zipf(rng, B * D_max, V))
+        else:
+            out.append(_logits_normal(rng, B * D_max, V))
+    return out
