@@ -13,8 +13,8 @@
 // g) sit in the CTA's warps, 16 query rows per warp, so each K/V tile is
 // read from HBM once per KV head.  K/V tiles of 64 keys are staged by TMA
 // (2D tensor maps, 128-byte swizzle, evict-first L2 policy) through a
-// 3-stage mbarrier ring; QK^T and PV run on the tensor cores (bf16 inputs,
-// fp32 accumulation), the mask predicate is evaluated in registers only on
+// 3-stage mbarrier ring; QK^T and PV run as mma.sync (bf16 inputs, fp32
+// accumulation), the mask predicate is evaluated in registers only on
 // tiles that reach the drafted block, and the softmax is the online
 // (running max / running sum) form with quad shuffles.  Long caches are split
 // over CTAs; a combine kernel merges the splits by their log-sum-exp.
@@ -409,10 +409,20 @@ bool make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int32_t d) {
 
 struct Plan {
   int32_t nwarps, mtiles, splits, kps;
+  bool tc;  // tcgen05 kernel (attention_tc.cu)
 };
 
-Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
+Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max, int32_t L_max) {
   Plan p;
+  p.tc = attention_tc_supported(Hq, Hkv, d, D_max);
+  if (p.tc) {
+    const TcPlan t = attention_tc_plan(B, Hq, Hkv, D_max, L_max);
+    p.nwarps = 0;
+    p.mtiles = t.mtiles;
+    p.splits = t.splits;
+    p.kps = t.kps;
+    return p;
+  }
   const int32_t G = Hq / Hkv;
   const int32_t rows = D_max * G;
   p.nwarps = min(kMaxWarps, (rows + 15) / 16);
@@ -442,7 +452,7 @@ int device_sm_count() {
 
 size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
                            int32_t L_max) {
-  const Plan p = make_plan(B, Hq, Hkv, D_max, L_max);
+  const Plan p = make_plan(B, Hq, Hkv, d, D_max, L_max);
   size_t bytes = align256((size_t)B * sizeof(int32_t));
   if (p.splits > 1) {
     const size_t prow = (size_t)B * Hq * D_max * p.splits;
@@ -451,14 +461,16 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
   return bytes;
 }
 
+static cudaError_t launch_combine(const AttnArgs& a, const AttnLaunch& L, cudaStream_t stream);
+
 int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
   if (B == 0) return 0;
-  return make_plan(B, Hq, Hkv, D_max, L_max).splits > 1 ? 2 : 1;
+  return make_plan(B, Hq, Hkv, 128, D_max, L_max).splits > 1 ? 2 : 1;
 }
 
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
-  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.D_max, a.L_max);
+  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max);
   AttnLaunch L;
   L.splits = p.splits;
   L.kps = p.kps;
@@ -474,13 +486,19 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
     w += align256(prow * a.d * sizeof(float));
     L.part_lse = reinterpret_cast<float*>(w);
   }
+  cudaError_t e;
+  if (p.tc) {
+    e = launch_attention_tc(a, TcPlan{p.splits, p.kps, p.mtiles}, L.seq_ok, L.part_o, L.part_lse,
+                            stream);
+    if (e != cudaSuccess) return e;
+    return p.splits == 1 ? cudaSuccess : launch_combine(a, L, stream);
+  }
   CUtensorMap tmK, tmV;
   const int64_t rows = (int64_t)a.B * a.Hkv * a.L_max;
   if (!make_kv_map(&tmK, a.k, rows, a.d) || !make_kv_map(&tmV, a.v, rows, a.d))
     return cudaErrorInvalidValue;
   const dim3 grid(p.splits, a.B * a.Hkv, p.mtiles);
   const dim3 block(p.nwarps * 32);
-  cudaError_t e;
   if (a.d == 128) {
     const size_t smem = 1024 + kStages * 2 * (KT * 128 * 2) + kStages * 8 + 129 * 4;
     e = cudaFuncSetAttribute(frontier_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -496,6 +514,10 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
   }
   e = cudaGetLastError();
   if (e != cudaSuccess || p.splits == 1) return e;
+  return launch_combine(a, L, stream);
+}
+
+static cudaError_t launch_combine(const AttnArgs& a, const AttnLaunch& L, cudaStream_t stream) {
   const int64_t rows_c = (int64_t)a.B * a.D_max * a.Hq;
   const int wpb = 8;
   const unsigned blocks = (unsigned)((rows_c + wpb - 1) / wpb);

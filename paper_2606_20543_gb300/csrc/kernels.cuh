@@ -53,6 +53,16 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
                            int32_t L_max);
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
 int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
+
+// ---- attention_tc.cu (tcgen05 frontier attention: query groups dividing 128,
+// more than 64 query rows per KV group)
+struct TcPlan {
+  int32_t splits, kps, mtiles;
+};
+bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max);
+TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
+cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
+                                float* part_lse, cudaStream_t stream);
 // Same as launch_attention with the library's static device scratch as the
 // workspace (ssd_verify_attention_noalloc); cudaErrorMemoryAllocation if the
 // problem needs more than SSD_NOALLOC_SCRATCH_BYTES.

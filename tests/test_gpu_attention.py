@@ -112,3 +112,22 @@ def test_bad_cache_length_sets_status(ssd):
     c.cache_len = np.array([10], np.int32)  # below the prefix
     o, lse, nd, st = run_attention(ssd, c)
     assert st == 6 and nd[0] == 0
+
+
+def test_head_dim_64_gqa_tensor_core_path(ssd):
+    # 32 drafts x 4 query heads per KV head = 128 rows per KV group, d = 64
+    c = synth.make_case("d64gqa", grid_h=16, grid_w=16, prefix_len=32, cache_len=[32, 96, 200],
+                        Hq=8, Hkv=2, d=64, V=64, seed=9, with_logits=False)
+    check_case(ssd, c)
+
+
+def test_mma_sync_and_tensor_core_paths_agree(ssd):
+    """The same MHA problem on both kernels: 48 drafts per sequence (mma.sync)
+    and the identical heads split as 2 query heads per KV head with 96 rows per
+    group (tcgen05); both must match the oracle."""
+    c = synth.make_case("mha48", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
+                        Hq=16, Hkv=16, d=128, V=64, seed=10, with_logits=False)
+    check_case(ssd, c)
+    c2 = synth.make_case("gqa96", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
+                         Hq=16, Hkv=8, d=128, V=64, seed=10, with_logits=False)
+    check_case(ssd, c2)
