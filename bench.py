@@ -140,6 +140,30 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of each dominant
+# kernel from one ncu capture (profiles/), valid only while the kernel's source
+# is the one that was captured: (source file, sha256 prefix, bytes, rows the
+# captured launch processed or None for a launch of the bench's own shape).
+MEASURED_TRAFFIC = {
+    ("accept", 2): ("accept.cu", "805e0d129edcc135", 148113408 + 3194880, 1128),
+    ("attention", 3): ("attention_tc.cu", "6ca0a2b87c88eb22", 53335296 + 427520, None),
+    ("lmhead_accept", 4): ("lmhead.cu", "a5b28d8ac7ea5800", 269327616 + 3034112, None),
+}
+
+
+def measured_traffic(kernel, cfg, rows):
+    """Traffic per launch of `kernel` for `rows` processed rows, or None."""
+    import hashlib
+    entry = MEASURED_TRAFFIC.get((kernel, cfg))
+    if entry is None:
+        return None
+    src, sha, nbytes, cap_rows = entry
+    path = os.path.join(ROOT, "paper_2606_20543_gb300", "csrc", src)
+    if not os.path.exists(path) or not hashlib.sha256(open(path, "rb").read()).hexdigest().startswith(sha):
+        return None
+    return nbytes if cap_rows is None else nbytes * rows / cap_rows
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -333,7 +357,8 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
         "accepted_drafts_per_s": world * accepted / (ms / 1000.0),
         "replay_ms": ms,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
-                     "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": None,
+                     "unit": "GB/s", "frac": achieved / hbm_peak,
+                     "traffic": measured_traffic(dom, a.config, c.B * c.D_max),
                      "peak_kind": peak_kind, "state": "first replay step (cache = prefix)",
                      "kernels": {k: {"bytes": b, "ms": m, "gbs": b / (m / 1000.0) / 1e9}
                                  for k, (b, m) in kern.items()}},
@@ -592,7 +617,8 @@ def main():
         "hbm_gbs_per_step": (attn_bytes + acc_bytes) / (ms_per_step / 1000.0) / 1e9,
         "tensor": tensor_info,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
-                     "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": None,
+                     "unit": "GB/s", "frac": achieved / hbm_peak,
+                     "traffic": measured_traffic(dom, a.config, c.B * c.D_max),
                      "peak_kind": peak_kind,
                      "kernels": {k: {"bytes": b, "ms": m, "gbs": b / (m / 1000.0) / 1e9}
                                  for k, (b, m) in kern.items()}},
