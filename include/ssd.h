@@ -229,6 +229,12 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * Logits path: tgt_logits/drf_logits non-NULL ([B*D_max] rows of ld floats).
  * Fused path:  logits NULL and h_tgt, h_drf, w_tgt, w_drf non-NULL (hidden
  *              = K of ssd_lmhead_accept).
+ * Streams: the attention runs on `stream`; the acceptance, which shares no
+ * data with it, runs concurrently on a side stream the library creates once
+ * per device and host thread (with two events) and joins back into `stream`
+ * before the counts, so all outputs are ordered on `stream` as usual.  Make
+ * the first call on each device and host thread outside any stream capture;
+ * later calls may be captured (the fork and join become graph edges).
  * ------------------------------------------------------------------------- */
 typedef struct {
   ssd_grid grid;

@@ -15,6 +15,31 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Side stream of ssd_verify_step: acceptance runs on it, concurrently with the
+// attention of the same step on the caller's stream (they share no data).
+// One per device and host thread, created on first use and kept until exit.
+struct SideStream {
+  cudaStream_t stream = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+constexpr int kMaxSideDevices = 64;
+
+cudaError_t side_stream(SideStream** out) {
+  thread_local SideStream side[kMaxSideDevices];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxSideDevices) return cudaErrorInvalidDevice;
+  SideStream& s = side[dev];
+  if (s.stream == nullptr) {
+    if ((e = cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&s.fork, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&s.join, cudaEventDisableTiming)) != cudaSuccess) return e;
+  }
+  *out = &s;
+  return cudaSuccess;
+}
+
 ssd_status check_grid(const ssd_grid* g) {
   if (g == nullptr) return SSD_ERR_INVALID_ARG;
   if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 1) return SSD_ERR_SHAPE;
@@ -295,11 +320,17 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
   unsigned char* ws = static_cast<unsigned char*>(workspace);
   const size_t attn_ws = align256(attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max));
+  SideStream* side = nullptr;
+  if (side_stream(&side) != cudaSuccess) return SSD_ERR_CUDA;
 
   // a1: frontier
   cudaError_t e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts, y->draft_pos,
                                   y->status, stream);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
+  // fork: acceptance on the side stream, after the frontier, beside the attention
+  if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
+      cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
+    return SSD_ERR_CUDA;
   // a2: attention of the drafted block
   AttnArgs a;
   a.grid = x->grid;
@@ -341,7 +372,7 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     h.status = y->status;
     h.n_drafts = y->n_drafts;
     h.D_max = x->D_max;
-    e = launch_lmhead(h, ws + attn_ws, workspace_bytes - attn_ws, stream);
+    e = launch_lmhead(h, ws + attn_ws, workspace_bytes - attn_ws, side->stream);
   } else {
     AcceptArgs c;
     c.rows = rows;
@@ -359,9 +390,13 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     c.status = y->status;
     c.n_drafts = y->n_drafts;
     c.D_max = x->D_max;
-    e = launch_accept(c, stream);
+    e = launch_accept(c, side->stream);
   }
   if (e != cudaSuccess) return SSD_ERR_CUDA;
+  // join: the counts need the decisions
+  if (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
+      cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess)
+    return SSD_ERR_CUDA;
   // a7: counts and the next cache length
   e = launch_counts(x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted, y->accepted_count,
                     y->accepted_prefix, y->next_cache_len, stream);
