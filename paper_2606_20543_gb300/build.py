@@ -18,6 +18,8 @@ LIB = os.path.join(HERE, "libssd.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "-I" + os.path.join(ROOT, "include")]
+# Extra nvcc flags (for example -DSSD_ACCEPT_RSTAGES=8 to retune a kernel).
+FLAGS += os.environ.get("SSD_NVCC_EXTRA", "").split()
 
 
 def nvcc() -> str:

@@ -4,20 +4,25 @@
 //   accept t with probability min(p(t) / q(t), 1); otherwise draw from
 //   [p - q]_+ / sum [p - q]_+ (inverse CDF in vocabulary order, one uniform).
 //
-// Design (GB300): a persistent grid of several CTAs per SM, each walking rows
+// Design (GB300): a persistent grid of four CTAs per SM, each walking rows
 // blockIdx.x, blockIdx.x + gridDim.x, ...  A dedicated producer warp streams
 // every row twice with bulk TMA copies, 256 entries per consumer warp of both
 // logit rows per stage, through a shared-memory ring: once from HBM for the
 // statistics, and once more (from L2, microseconds later) for the residual
 // draw; it runs ahead into the next row while the consumers finish the
-// current one.  Eight consumer warps fold each first-pass chunk into online
-// (max, sum of 2^x) statistics, one max and at most one rescale per chunk, and
-// the first argmax (carrying the target logit at it); a block reduction in a fixed order gives the log-sum-exps
-// and the draft token, and one thread takes the decision.  For rejected rows
-// the second-pass chunks give the residual weights (MUFU exp2) and the mass
-// of every 256-entry block in vocabulary order; warp 0 scans the block masses,
-// finds the block holding u_res * Z and re-walks it to pick the token.
-// Accepted rows only release their second-pass chunks.
+// current one.  The consumers are latency-bound, so the arithmetic is kept
+// short: per first-pass chunk each thread folds its 8 entries of both rows
+// into online (max, sum of 2^x) statistics with a branch-free rescale,
+// three-input maxima and packed fp32 pairs (fma/add .f32x2) for the exponent
+// arguments and the sums, and tracks the first argmax of q with the target
+// logit at it.  A fixed-order reduction (xor tree in each warp, then a
+// three-level tree over the warps) gives the log-sum-exps and the draft
+// token, and one thread takes the decision with the row's uniforms drawn
+// before the row's data arrived.  For rejected rows the second-pass chunks
+// give the residual weights and the mass of every 256-entry block in
+// vocabulary order; warp 0 scans the block masses, finds the block holding
+// u_res * Z and re-walks it to pick the token.  Accepted rows only release
+// their second-pass chunks.
 #include <algorithm>
 
 #include "kernels.cuh"
@@ -30,10 +35,10 @@ namespace {
 #define SSD_ACCEPT_CWARPS 8
 #endif
 #ifndef SSD_ACCEPT_STAGES
-#define SSD_ACCEPT_STAGES 4
+#define SSD_ACCEPT_STAGES 3
 #endif
 #ifndef SSD_ACCEPT_CTAS
-#define SSD_ACCEPT_CTAS 3
+#define SSD_ACCEPT_CTAS 4
 #endif
 constexpr int kCWarps = SSD_ACCEPT_CWARPS;    // consumer warps
 constexpr int kConsumers = kCWarps * 32;
@@ -75,22 +80,38 @@ __device__ __forceinline__ void merge(float& m, float& s, float m2, float s2, fl
 }
 
 // Residual weights of 4 entries: [p - q]_+ with p = 2^(x_p c - Cp), q = 2^(x_q c - Cq),
-// or p itself for the draw from p.
-__device__ __forceinline__ float4 weights4(const float4& xp, const float4& xq, float c, float Cp,
-                                           float Cq, bool from_p) {
+// or p itself for the draw from p.  cc = (c, c), ncp = (-Cp, -Cp), ncq = (-Cq, -Cq).
+__device__ __forceinline__ float4 weights4(const float4& xp, const float4& xq, float2 cc,
+                                           float2 ncp, float2 ncq, bool from_p) {
+  const float2 a0 = ffma2(make_float2(xp.x, xp.y), cc, ncp);
+  const float2 a1 = ffma2(make_float2(xp.z, xp.w), cc, ncp);
   float4 w;
   if (from_p) {
-    w.x = ex2(fmaf(xp.x, c, -Cp));
-    w.y = ex2(fmaf(xp.y, c, -Cp));
-    w.z = ex2(fmaf(xp.z, c, -Cp));
-    w.w = ex2(fmaf(xp.w, c, -Cp));
+    w.x = ex2(a0.x);
+    w.y = ex2(a0.y);
+    w.z = ex2(a1.x);
+    w.w = ex2(a1.y);
   } else {
-    w.x = fmaxf(ex2(fmaf(xp.x, c, -Cp)) - ex2(fmaf(xq.x, c, -Cq)), 0.f);
-    w.y = fmaxf(ex2(fmaf(xp.y, c, -Cp)) - ex2(fmaf(xq.y, c, -Cq)), 0.f);
-    w.z = fmaxf(ex2(fmaf(xp.z, c, -Cp)) - ex2(fmaf(xq.z, c, -Cq)), 0.f);
-    w.w = fmaxf(ex2(fmaf(xp.w, c, -Cp)) - ex2(fmaf(xq.w, c, -Cq)), 0.f);
+    const float2 b0 = ffma2(make_float2(xq.x, xq.y), cc, ncq);
+    const float2 b1 = ffma2(make_float2(xq.z, xq.w), cc, ncq);
+    w.x = fmaxf(ex2(a0.x) - ex2(b0.x), 0.f);
+    w.y = fmaxf(ex2(a0.y) - ex2(b0.y), 0.f);
+    w.z = fmaxf(ex2(a1.x) - ex2(b1.x), 0.f);
+    w.w = fmaxf(ex2(a1.y) - ex2(b1.y), 0.f);
   }
   return w;
+}
+
+// Sum of 2^(x c - mc) over 8 entries, as a pair of partial sums.
+__device__ __forceinline__ float2 exp_sum8(const float4& x0, const float4& x1, float2 cc,
+                                           float2 nmc) {
+  const float2 a0 = ffma2(make_float2(x0.x, x0.y), cc, nmc);
+  const float2 a1 = ffma2(make_float2(x0.z, x0.w), cc, nmc);
+  const float2 a2 = ffma2(make_float2(x1.x, x1.y), cc, nmc);
+  const float2 a3 = ffma2(make_float2(x1.z, x1.w), cc, nmc);
+  const float2 e0 = make_float2(ex2(a0.x), ex2(a0.y)), e1 = make_float2(ex2(a1.x), ex2(a1.y));
+  const float2 e2 = make_float2(ex2(a2.x), ex2(a2.y)), e3 = make_float2(ex2(a3.x), ex2(a3.y));
+  return fadd2(fadd2(e0, e1), fadd2(e2, e3));
 }
 
 struct Shared {
@@ -170,54 +191,68 @@ __device__ __forceinline__ int32_t find_block(const float* mass, int32_t nblocks
   return bs;
 }
 
+// Warp-wide scan of one 128-entry span whose lane l holds the residual
+// weights w of entries e .. e + 3 (e ascending with l).  If the target th
+// falls inside the span's mass, returns the token at the crossing; otherwise
+// returns -1 and leaves the span's mass in *hsum.  *last_pos is updated to
+// the last entry with positive weight seen so far.
+__device__ __forceinline__ int32_t walk_half(const float4& w, int32_t e, float th, float* hsum,
+                                             int32_t* last_pos, int lane) {
+  const float lsum = (w.x + w.y) + (w.z + w.w);
+  float li = lsum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, li, o);
+    if (lane >= o) li += y;
+  }
+  *hsum = __shfl_sync(0xffffffffu, li, 31);
+  int32_t lp = -1;  // last entry of this lane with positive weight
+  if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
+  else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
+  const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
+  if (hasp) *last_pos = __shfl_sync(0xffffffffu, lp, 31 - __clz(hasp));
+  if (!(*hsum > 0.f && th < *hsum)) return -1;
+  const uint32_t lcross = __ballot_sync(0xffffffffu, lsum > 0.f && li > th);
+  const int32_t lstar = lcross ? (__ffs(lcross) - 1) : (31 - __clz(hasp));
+  int32_t pick = -1;
+  if (lane == lstar) {
+    const float t4 = th - (li - lsum);
+    const float ws[4] = {w.x, w.y, w.z, w.w};
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      acc += ws[k];
+      if (pick < 0 && ws[k] > 0.f && acc > t4) pick = e + k;
+    }
+    if (pick < 0) pick = lp;
+  }
+  return __shfl_sync(0xffffffffu, pick, lstar);
+}
+
 // Warp 0: re-walk 256-entry block `bk` (its two 128-entry halves in order)
 // with the arithmetic of the mass pass and return the token at the crossing.
+// Both halves are loaded before the first is walked (one L2 round trip).
 __device__ __forceinline__ int32_t walk_block(const float4* tp, const float4* dp, int32_t bk,
-                                              int32_t nv, float c, float Cp, float Cq, bool from_p,
-                                              float tb, int lane) {
-  int32_t last_pos = -1;
-  float run = 0.f;
+                                              int32_t nv, float2 cc, float2 ncp, float2 ncq,
+                                              bool from_p, float tb, int lane) {
+  const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+  float4 xp[2], xq[2];
+#pragma unroll
   for (int half = 0; half < 2; ++half) {
     const int32_t i = bk * 64 + half * 32 + lane;
-    float4 xp = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY), xq = xp;
-    if (i < nv) {
-      xp = tp[i];
-      xq = from_p ? xp : dp[i];
-    }
-    const float4 w = weights4(xp, xq, c, Cp, Cq, from_p);
-    const float lsum = (w.x + w.y) + (w.z + w.w);
-    float li = lsum;
+    xp[half] = i < nv ? tp[i] : ninf;
+    xq[half] = (i < nv && !from_p) ? dp[i] : xp[half];
+  }
+  int32_t last_pos = -1;
+  float run = 0.f;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float y = __shfl_up_sync(0xffffffffu, li, o);
-      if (lane >= o) li += y;
-    }
-    const float hsum = __shfl_sync(0xffffffffu, li, 31);
-    const int32_t e = 4 * i;
-    int32_t lp = -1;  // last entry of this lane with positive weight
-    if (w.w > 0.f) lp = e + 3; else if (w.z > 0.f) lp = e + 2;
-    else if (w.y > 0.f) lp = e + 1; else if (w.x > 0.f) lp = e;
-    const uint32_t hasp = __ballot_sync(0xffffffffu, lp >= 0);
-    if (hasp) last_pos = __shfl_sync(0xffffffffu, lp, 31 - __clz(hasp));
-    const float th = tb - run;  // target left for this half
-    if (hsum > 0.f && th < hsum) {
-      const uint32_t lcross = __ballot_sync(0xffffffffu, lsum > 0.f && li > th);
-      const int32_t lstar = lcross ? (__ffs(lcross) - 1) : (31 - __clz(hasp));
-      int32_t pick = -1;
-      if (lane == lstar) {
-        const float t4 = th - (li - lsum);
-        const float ws[4] = {w.x, w.y, w.z, w.w};
-        float cc = 0.f;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          cc += ws[k];
-          if (pick < 0 && ws[k] > 0.f && cc > t4) pick = e + k;
-        }
-        if (pick < 0) pick = lp;
-      }
-      return __shfl_sync(0xffffffffu, pick, lstar);
-    }
-    run += hsum;
+  for (int half = 0; half < 2; ++half) {
+    const int32_t i = bk * 64 + half * 32 + lane;
+    float hs;
+    const int32_t pick = walk_half(weights4(xp[half], xq[half], cc, ncp, ncq, from_p), 4 * i,
+                                   tb - run, &hs, &last_pos, lane);
+    if (pick >= 0) return pick;
+    run += hs;
   }
   return last_pos;  // rounding ran past the end of the block
 }
@@ -263,8 +298,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
 
   // ---------------------------------------------------------- consumer warps
   const float c = kLog2e / a.temperature;
+  const float2 cc = make_float2(c, c);
   const int32_t nv = a.V >> 2;
   const int32_t nblocks = nch * kBlocksPerChunk;
+  const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
   uint32_t g = 0;  // chunks consumed
   for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
     const int kind = row_kind(a, r);
@@ -279,13 +316,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       continue;
     }
     const int32_t given_t = a.draft_tok != nullptr ? a.draft_tok[r] : -1;
+    // the row's uniforms, drawn while its first chunk is still in flight
+    const float2 u = (tid == 0) ? row_uniforms(a.rng, r) : make_float2(0.f, 0.f);
 
     // ---- pass A: per chunk, each thread takes 8 entries of both rows
-    // (float4 tid and tid + 256 of the chunk, ascending): one max, at most one
-    // rescale, then the exponentials; the first argmax of q carries the p logit
-    float mp = kLowest, sp = 0.f, mq = kLowest, sq = 0.f, xpa = 0.f;
+    // (float4 tid and tid + 256 of the chunk, ascending): new running maxima
+    // (three-input max), one rescale per row, packed exponent arguments and
+    // sums; the first argmax of q carries the p logit
+    float mp = kLowest, mq = kLowest, xpa = 0.f;
+    float2 sp2 = make_float2(0.f, 0.f), sq2 = sp2;
     int32_t iq = 0x7fffffff;
-    const float4 ninf = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
     for (int32_t ch = 0; ch < nch; ++ch, ++g) {
       const int s = g % kStages;
       mbar_wait(&sh.full[s], (g / kStages) & 1, a.status);
@@ -295,17 +335,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       const bool in0 = tid < cv, in1 = tid + kConsumers < cv;
       const float4 p0 = in0 ? xp4[tid] : ninf, p1 = in1 ? xp4[tid + kConsumers] : ninf;
       const float4 q0 = in0 ? xq4[tid] : ninf, q1 = in1 ? xq4[tid + kConsumers] : ninf;
-      const float cmp = fmaxf(fmaxf(fmaxf(p0.x, p0.y), fmaxf(p0.z, p0.w)),
-                              fmaxf(fmaxf(p1.x, p1.y), fmaxf(p1.z, p1.w)));
-      const float cmq = fmaxf(fmaxf(fmaxf(q0.x, q0.y), fmaxf(q0.z, q0.w)),
-                              fmaxf(fmaxf(q1.x, q1.y), fmaxf(q1.z, q1.w)));
-      if (cmp > mp) {
-        sp *= ex2((mp - cmp) * c);
-        mp = cmp;
-      }
+      const float nmp = fmax3(fmax3(p0.x, p0.y, p0.z), fmax3(p0.w, p1.x, p1.y), fmax3(p1.z, p1.w, mp));
+      const float cmq = fmax3(fmax3(q0.x, q0.y, q0.z), fmax3(q0.w, q1.x, q1.y), fmaxf(q1.z, q1.w));
       if (cmq > mq) {
-        sq *= ex2((mq - cmq) * c);
-        mq = cmq;
         const int32_t e0 = ch * kChunk + 4 * tid, e1 = e0 + 4 * kConsumers;
         if (q0.x == cmq) { iq = e0; xpa = p0.x; }
         else if (q0.y == cmq) { iq = e0 + 1; xpa = p0.y; }
@@ -316,16 +348,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         else if (q1.z == cmq) { iq = e1 + 2; xpa = p1.z; }
         else { iq = e1 + 3; xpa = p1.w; }
       }
-      // a thread that has seen only -inf keeps kLowest: its terms are exp2(-inf) = 0
-      const float mpc = (mp == kLowest) ? 0.f : mp * c, mqc = (mq == kLowest) ? 0.f : mq * c;
-      sp += ((ex2(fmaf(p0.x, c, -mpc)) + ex2(fmaf(p0.y, c, -mpc))) +
-             (ex2(fmaf(p0.z, c, -mpc)) + ex2(fmaf(p0.w, c, -mpc)))) +
-            ((ex2(fmaf(p1.x, c, -mpc)) + ex2(fmaf(p1.y, c, -mpc))) +
-             (ex2(fmaf(p1.z, c, -mpc)) + ex2(fmaf(p1.w, c, -mpc))));
-      sq += ((ex2(fmaf(q0.x, c, -mqc)) + ex2(fmaf(q0.y, c, -mqc))) +
-             (ex2(fmaf(q0.z, c, -mqc)) + ex2(fmaf(q0.w, c, -mqc)))) +
-            ((ex2(fmaf(q1.x, c, -mqc)) + ex2(fmaf(q1.y, c, -mqc))) +
-             (ex2(fmaf(q1.z, c, -mqc)) + ex2(fmaf(q1.w, c, -mqc))));
+      const float nmq = fmaxf(mq, cmq);
+      // rescale of the running sums (exactly 1 when the maximum did not move;
+      // the initial kLowest is finite, so no -inf - -inf)
+      const float rp = ex2((mp - nmp) * c), rq = ex2((mq - nmq) * c);
+      mp = nmp;
+      mq = nmq;
+      const float2 ep = exp_sum8(p0, p1, cc, make_float2(-mp * c, -mp * c));
+      const float2 eq = exp_sum8(q0, q1, cc, make_float2(-mq * c, -mq * c));
+      sp2 = ffma2(sp2, make_float2(rp, rp), ep);
+      sq2 = ffma2(sq2, make_float2(rq, rq), eq);
       if (given_t >= 0 && (given_t / kChunk) == ch) {
         const int32_t off = given_t - ch * kChunk;  // entry inside the chunk
         const int32_t f = off >> 2, k = off & 3;
@@ -338,7 +370,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       __syncwarp();
       if (lane == 0) mbar_arrive(&sh.empty[s]);
     }
-    // block reduction in a fixed order: xor tree in warps, then warps 0..7
+    float sp = sp2.x + sp2.y, sq = sq2.x + sq2.y;
+    // block reduction in a fixed order: xor tree in each warp, then a
+    // three-level xor tree over the warps' results in warp 0
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       merge(mp, sp, __shfl_xor_sync(0xffffffffu, mp, o), __shfl_xor_sync(0xffffffffu, sp, o), c);
@@ -359,50 +393,59 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       sh.red_i[warp] = iq;
     }
     consumers_sync();
-    if (tid == 0) {
-      float Mp = sh.red[0][0], Sp = sh.red[0][1], Mq = sh.red[0][2], Sq = sh.red[0][3];
-      float xp_t = sh.red[0][4];
-      int32_t t = sh.red_i[0];
-      for (int w = 1; w < kCWarps; ++w) {
-        merge(Mp, Sp, sh.red[w][0], sh.red[w][1], c);
-        const bool take = better_arg(sh.red[w][2], sh.red_i[w], Mq, t);
-        merge(Mq, Sq, sh.red[w][2], sh.red[w][3], c);
-        if (take) { t = sh.red_i[w]; xp_t = sh.red[w][4]; }
+    if (warp == 0) {
+      const bool have = lane < kCWarps;
+      float Mp = have ? sh.red[lane][0] : kLowest, Sp = have ? sh.red[lane][1] : 0.f;
+      float Mq = have ? sh.red[lane][2] : kLowest, Sq = have ? sh.red[lane][3] : 0.f;
+      float xp_t = have ? sh.red[lane][4] : 0.f;
+      int32_t t = have ? sh.red_i[lane] : 0x7fffffff;
+#pragma unroll
+      for (int o = kCWarps / 2; o > 0; o >>= 1) {
+        merge(Mp, Sp, __shfl_xor_sync(0xffffffffu, Mp, o), __shfl_xor_sync(0xffffffffu, Sp, o), c);
+        const float om = __shfl_xor_sync(0xffffffffu, Mq, o);
+        const float os = __shfl_xor_sync(0xffffffffu, Sq, o);
+        const int32_t oi = __shfl_xor_sync(0xffffffffu, t, o);
+        const float op = __shfl_xor_sync(0xffffffffu, xp_t, o);
+        const bool take = better_arg(om, oi, Mq, t);
+        merge(Mq, Sq, om, os, c);
+        if (take) { t = oi; xp_t = op; }
       }
-      float xq_t = Mq;
-      if (given_t >= 0) {
-        t = given_t;
-        xp_t = sh.xp_t;
-        xq_t = sh.xq_t;
-      }
-      const bool valid_t = t >= 0 && t < a.V;
-      float ratio = 0.f;
-      bool acc = false;
-      const float2 u = row_uniforms(a.rng, r);
-      if (valid_t) {
-        const float l2p = (xp_t - Mp) * c - log2f(Sp);
-        const float l2q = (xq_t - Mq) * c - log2f(Sq);
-        ratio = exp2f(l2p - l2q);
-        acc = u.x < fminf(ratio, 1.0f);
-      } else {
-        record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
-      }
-      sh.accept = acc ? 1 : (valid_t ? 0 : 2);
-      sh.u_res = u.y;
-      sh.Cp = Mp * c + log2f(Sp);
-      sh.Cq = Mq * c + log2f(Sq);
-      a.accepted[r] = acc ? 1 : 0;
-      if (acc) a.out_tok[r] = t;
-      else if (!valid_t) a.out_tok[r] = -1;
-      if (a.ratio) a.ratio[r] = ratio;
-      if (a.lse) {
-        a.lse[2 * r] = Mp / a.temperature + log2f(Sp) * kLn2;
-        a.lse[2 * r + 1] = Mq / a.temperature + log2f(Sq) * kLn2;
+      if (lane == 0) {
+        float xq_t = Mq;
+        if (given_t >= 0) {
+          t = given_t;
+          xp_t = sh.xp_t;
+          xq_t = sh.xq_t;
+        }
+        const bool valid_t = t >= 0 && t < a.V;
+        const float lsp = log2f(Sp), lsq = log2f(Sq);
+        float ratio = 0.f;
+        bool acc = false;
+        if (valid_t) {
+          const float l2p = (xp_t - Mp) * c - lsp;
+          const float l2q = (xq_t - Mq) * c - lsq;
+          ratio = exp2f(l2p - l2q);
+          acc = u.x < fminf(ratio, 1.0f);
+        } else {
+          record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
+        }
+        sh.accept = acc ? 1 : (valid_t ? 0 : 2);
+        sh.u_res = u.y;
+        sh.Cp = Mp * c + lsp;
+        sh.Cq = Mq * c + lsq;
+        a.accepted[r] = acc ? 1 : 0;
+        if (acc) a.out_tok[r] = t;
+        else if (!valid_t) a.out_tok[r] = -1;
+        if (a.ratio) a.ratio[r] = ratio;
+        if (a.lse) {
+          a.lse[2 * r] = Mp / a.temperature + lsp * kLn2;
+          a.lse[2 * r + 1] = Mq / a.temperature + lsq * kLn2;
+        }
       }
     }
     consumers_sync();
     const bool draw = (sh.accept == 0);
-    const float Cp = sh.Cp, Cq = sh.Cq;
+    const float2 ncp = make_float2(-sh.Cp, -sh.Cp), ncq = make_float2(-sh.Cq, -sh.Cq);
 
     // ---- pass B: second-pass chunks; residual mass of every 256-entry block
     for (int32_t ch = 0; ch < nch; ++ch, ++g) {
@@ -414,8 +457,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         const int32_t cv = min(kChunk, a.V - ch * kChunk) >> 2;
         const int32_t i0 = warp * 64 + lane, i1 = i0 + 32;
         float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
-        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], c, Cp, Cq, false);
-        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], c, Cp, Cq, false);
+        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], cc, ncp, ncq, false);
+        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], cc, ncp, ncq, false);
         const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
         if (lane == 0) block_mass[ch * kBlocksPerChunk + warp] = m;
       }
@@ -436,8 +479,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         for (int32_t b0 = 0; b0 < nblocks; ++b0) {
           const int32_t i0 = b0 * 64 + lane, i1 = i0 + 32;
           float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
-          if (i0 < nv) w0 = weights4(tp[i0], tp[i0], c, Cp, Cq, true);
-          if (i1 < nv) w1 = weights4(tp[i1], tp[i1], c, Cp, Cq, true);
+          if (i0 < nv) w0 = weights4(tp[i0], tp[i0], cc, ncp, ncq, true);
+          if (i1 < nv) w1 = weights4(tp[i1], tp[i1], cc, ncp, ncq, true);
           const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
           if (lane == 0) block_mass[b0] = m;
         }
@@ -450,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
       } else {
-        const int32_t pick = walk_block(tp, dp, bk, nv, c, Cp, Cq, from_p, tb, lane);
+        const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
         if (lane == 0) a.out_tok[r] = pick;
       }
     }
@@ -467,8 +510,8 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
   const int32_t nch = (a.V + kChunk - 1) / kChunk;
   const size_t smem = (size_t)kStages * 2 * kChunk * sizeof(float) +
                       (size_t)nch * kBlocksPerChunk * sizeof(float);
-  cudaError_t e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(accept_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t grid = std::min<int64_t>(a.rows, (int64_t)kCtasPerSm * device_sm_count());
   accept_kernel<<<(unsigned)grid, kThreads, smem, stream>>>(a);

@@ -1,6 +1,6 @@
 // common.cuh — small device helpers shared by the libssd kernels: status
 // recording, shared-memory addresses, mbarriers, bulk / tensor copies (TMA),
-// thread-block-cluster helpers and bf16 packing.  sm_103a only.
+// packed fp32 arithmetic and bf16 packing.  sm_103a only.
 #pragma once
 
 #include <cuda.h>
@@ -68,12 +68,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// A slow wait gives up early once any error has been recorded (another wait
+// timed out, or the inputs were bad), so a broken launch ends after one
+// timeout instead of one per wait.
+__device__ __forceinline__ bool give_up(uint32_t poll, const int32_t* status) {
+  return (poll & 4095u) == 0 && status != nullptr &&
+         *reinterpret_cast<const volatile int32_t*>(status) != (int32_t)SSD_OK;
+}
+
 // Bounded wait on an mbarrier phase.  Returns false (and records
 // SSD_ERR_TIMEOUT) if the phase did not complete within kMaxPolls polls.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status) {
   for (uint32_t i = 0; i < kMaxPolls; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (i > 4096) __nanosleep(128);
+    if (i > 4096) {
+      __nanosleep(128);
+      if (give_up(i, status)) return false;
+    }
   }
   record_status(status, SSD_ERR_TIMEOUT);
   return false;
@@ -88,6 +99,16 @@ __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gmem_src, u
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
           smem_u32(smem_dst)),
       "l"(gmem_src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Untiled bulk copy global -> shared with an L2 cache policy.
+__device__ __forceinline__ void bulk_g2s_hint(void* smem_dst, const void* gmem_src, uint32_t bytes,
+                                              uint64_t* bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(smem_dst)),
+      "l"(gmem_src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
 }
 
@@ -118,6 +139,35 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// ------------------------------------------------- packed fp32 (sm_100+)
+// One instruction for two lanes of fp32 work (fma/add on .f32x2), and the
+// three-input maximum.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rc, rd;\n"
+      " mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+      " fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rd;\n"
+      " mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " add.rn.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 // ----------------------------------------------------------------- misc

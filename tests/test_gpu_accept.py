@@ -44,12 +44,14 @@ def run_accept(ssd, tgt, drf, uniforms=None, seed=0, offset=0, draft_tok=None, T
 
 
 @pytest.mark.parametrize("V,rows,logits,seed", [
-    (4096, 64, "normal", 0),      # one CTA per row
-    (16384, 48, "normal", 1),     # cluster of 4
+    (4096, 64, "normal", 0),      # two 2048-entry chunks per row
+    (16384, 48, "normal", 1),     # eight chunks, one row per CTA
     (16384, 40, "zipf", 2),       # skewed draft vs perturbed target
-    (4100, 30, "normal", 3),      # ragged: 2 CTAs, uneven slices
-    (65536, 8, "zipf", 4),        # cluster of 8
+    (4100, 30, "normal", 3),      # ragged: a 4-entry last chunk
+    (65536, 8, "zipf", 4),        # 32 chunks per row
     (12, 16, "normal", 5),        # tiny vocabulary
+    (16384, 700, "normal", 6),    # more rows than CTAs: each CTA walks several
+    (100000, 6, "normal", 7),     # large vocabulary, ragged last chunk
 ])
 def test_accept_matches_oracle(ssd, V, rows, logits, seed):
     rng = np.random.default_rng(seed)

@@ -131,3 +131,18 @@ def test_counts_all_accept_and_all_reject(ssd):
     assert r["accepted_count"][0] == 0 and r["accepted_prefix"][0] == 0
     assert r["next_cache_len"][0] == 193
     assert np.all(r["out_tok"][:32] < 2048)
+
+
+def test_step_more_sequences_than_the_row_table(ssd):
+    """More than 1024 sequences: the acceptance walks the padded rows and
+    skips padding slots instead of using its prefix table of frontier rows."""
+    rng = np.random.default_rng(21)
+    H = W = 4
+    P = 8
+    cls = rng.integers(P, P + H * W + 1, size=1100).astype(np.int32)
+    c = synth.make_case("many", grid_h=H, grid_w=W, prefix_len=P, cache_len=cls, Hq=1, Hkv=1,
+                        d=64, V=64, seed=21)
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    check_step(c, s.results(), attention_seqs=[0, 1, 550, 1099])
