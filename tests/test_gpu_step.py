@@ -133,9 +133,9 @@ def test_counts_all_accept_and_all_reject(ssd):
     assert np.all(r["out_tok"][:32] < 2048)
 
 
-def test_step_more_sequences_than_the_row_table(ssd):
-    """More than 1024 sequences: the acceptance walks the padded rows and
-    skips padding slots instead of using its prefix table of frontier rows."""
+def test_step_large_batch_of_small_grids(ssd):
+    """1100 sequences of 4x4 grids with mixed cache lengths (some complete,
+    n_drafts = 0): far more rows than CTAs, padding slots among them."""
     rng = np.random.default_rng(21)
     H = W = 4
     P = 8
