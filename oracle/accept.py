@@ -2,8 +2,12 @@
 
 TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).
 
-Sec. 3.3 "Verification as Auto Correction", strategy (C), applied to every
-drafted position independently:
+Sec. 3.3 "Verification as Auto Correction" names three ways to select the
+final token of every drafted position, applied independently per position:
+  (A) greedy selection: argmax_v p_k(v);
+  (B) sampling: a draw from p_k;
+  (C) acceptance-rejection sampling (the default), below.
+Strategy (C):
   * q_k is the draft distribution, p_k the backbone's distribution;
   * the draft token is t_hat = argmax_v q_k(v);
   * t_hat is accepted with probability alpha = min(p_k(t_hat) / q_k(t_hat), 1);
@@ -21,12 +25,18 @@ Readings (the paper states the distributions, not the mechanism):
   * the residual draw is the inverse CDF in ascending vocabulary order with
     one uniform u_res: the smallest v with sum_{v' <= v} w_v' > u_res * Z,
     w = [p - q]_+, Z = sum w; if rounding runs past the end the last v with
-    w_v > 0 is taken; if Z == 0 the draw is made from p instead.
+    w_v > 0 is taken; if Z == 0 the draw is made from p instead;
+  * (A) takes the argmax of the raw target logits, lowest index on ties;
+  * (B) draws from p by the same inverse CDF with u_res;
+  * under (A) and (B) a position counts as accepted when the selected token
+    equals the draft token t_hat (so the commit rule of one round is the
+    same prefix rule for all three strategies).
 """
 from __future__ import annotations
 
 import numpy as np
 
+STRATEGIES = ("accept_reject", "greedy", "sample")  # (C), (A), (B) of Sec. 3.3
 NEAR_TIE = 1e-4      # |alpha - u_acc| below this: the accept decision is a near-tie
 NEAR_TIE_CDF = 1e-6  # u_res * Z within this fraction of Z of a CDF boundary: resample near-tie
 
@@ -63,8 +73,9 @@ def inverse_cdf(w: np.ndarray, u: float):
     return v, margin
 
 
-def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.0):
-    """Strategy (C) on every row.
+def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.0,
+                strategy="accept_reject"):
+    """One of the strategies of Sec. 3.3 on every row (default (C)).
 
     tgt_logits, drf_logits: [rows, V]; uniforms: [rows, 2] = (u_acc, u_res);
     draft_tok: [rows] or None (then t_hat = argmax q).
@@ -72,8 +83,12 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
     lse_p, lse_q, resampled_from_p (Z == 0 fallback), accept_margin = |alpha -
     u_acc|, tie_accept (accept_margin < NEAR_TIE), cdf_margin (distance of
     u_res * Z to the nearest boundary of the chosen bin, over Z), tie_resample
-    (cdf_margin < NEAR_TIE_CDF).
+    (cdf_margin < NEAR_TIE_CDF).  Under "greedy" out_tok is the argmax of the
+    target logits; under "sample" it is the inverse-CDF draw from p with
+    u_res; under both, accepted = (out_tok == t_hat) and tie_accept is False.
     """
+    if strategy not in STRATEGIES:
+        raise ValueError(f"unknown strategy {strategy!r}")
     lp = np.asarray(tgt_logits, dtype=np.float64)
     lq = np.asarray(drf_logits, dtype=np.float64)
     u = np.asarray(uniforms, dtype=np.float64)
@@ -93,6 +108,18 @@ def accept_rows(tgt_logits, drf_logits, uniforms, draft_tok=None, temperature=1.
         alpha = min(ratio, 1.0)
         out["ratio"][r] = ratio
         out["alpha"][r] = alpha
+        if strategy == "greedy":
+            v = int(np.argmax(lp[r]))
+            out["out_tok"][r] = v
+            out["accepted"][r] = v == tr
+            continue
+        if strategy == "sample":
+            v, margin = inverse_cdf(p[r], u[r, 1])
+            out["out_tok"][r] = v
+            out["accepted"][r] = v == tr
+            out["cdf_margin"][r] = margin
+            out["tie_resample"][r] = margin < NEAR_TIE_CDF
+            continue
         out["accept_margin"][r] = abs(alpha - u[r, 0])
         out["tie_accept"][r] = abs(alpha - u[r, 0]) < NEAR_TIE
         if u[r, 0] < alpha:

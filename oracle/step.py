@@ -22,7 +22,7 @@ def sequence_frontier(grid_h, grid_w, prefix_len, cache_len, k_v=1):
 
 
 def accept_step(grid_h, grid_w, prefix_len, k_v, cache_len, D_max, tgt_logits, drf_logits,
-                uniforms, draft_tok=None, temperature=1.0):
+                uniforms, draft_tok=None, temperature=1.0, strategy="accept_reject"):
     """Frontier + acceptance + counts for a batch (no attention).
 
     Row b*D_max + j of the logit / uniform arrays belongs to draft j of
@@ -41,7 +41,7 @@ def accept_step(grid_h, grid_w, prefix_len, k_v, cache_len, D_max, tgt_logits, d
     if rows.size:
         dt = None if draft_tok is None else np.asarray(draft_tok)[rows]
         dec = acc.accept_rows(np.asarray(tgt_logits)[rows], np.asarray(drf_logits)[rows],
-                              np.asarray(uniforms)[rows], dt, temperature)
+                              np.asarray(uniforms)[rows], dt, temperature, strategy)
     else:
         dec = {k: np.zeros(0) for k in ("out_tok", "accepted", "tie_accept", "tie_resample")}
     dec["rows"] = rows

@@ -174,3 +174,70 @@ def test_monte_carlo_marginal_chi2():
     counts = np.bincount(out["out_tok"], minlength=V)
     chi2 = ((counts - N * p) ** 2 / (N * p)).sum()
     assert chi2 < 25.0  # 5 degrees of freedom; p-value ~1e-4
+
+
+# ---------------------------------------------------------------------------
+# Strategies (A) greedy and (B) sampling of Sec. 3.3.
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_greedy_is_the_library_argmax_of_the_target(seed):
+    rng = np.random.default_rng(seed)
+    rows, V = 64, 300
+    lp = rng.standard_normal((rows, V))
+    lq = rng.standard_normal((rows, V))
+    # planted ties of the target maximum: the lower index must win
+    lp[0, [7, 200]] = lp[0].max() + 1.0
+    lp[1, [0, 299]] = lp[1].max() + 1.0
+    u = rng.random((rows, 2))
+    d = acc.accept_rows(lp, lq, u, strategy="greedy")
+    assert np.array_equal(d["out_tok"], np.argmax(lp, axis=1))
+    assert d["out_tok"][0] == 7 and d["out_tok"][1] == 0
+    assert np.array_equal(d["accepted"], np.argmax(lp, 1) == np.argmax(lq, 1))
+    # the uniforms and the draft distribution do not move the greedy token
+    d2 = acc.accept_rows(lp, lq[::-1], 1.0 - u, strategy="greedy")
+    assert np.array_equal(d2["out_tok"], d["out_tok"])
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_sampling_is_the_library_inverse_cdf_of_p_with_u_res(seed):
+    rng = np.random.default_rng(seed)
+    rows, V = 200, 97
+    lp = rng.standard_normal((rows, V)) * 2
+    lq = rng.standard_normal((rows, V)) * 2
+    u = np.stack([rng.random(rows), rng.random(rows)], 1)  # u_acc differs from u_res
+    d = acc.accept_rows(lp, lq, u, strategy="sample")
+    p = scipy.special.softmax(lp, axis=1)
+    c = np.cumsum(p, axis=1)
+    ref = np.array([np.searchsorted(c[r], u[r, 1] * c[r, -1], side="right") for r in range(rows)])
+    ok = ~d["tie_resample"]
+    assert ok.sum() > rows * 0.95
+    assert np.array_equal(d["out_tok"][ok], ref[ok])
+    assert np.array_equal(d["accepted"], d["out_tok"] == np.argmax(lq, 1))
+
+
+def test_sampling_law_on_a_stratified_grid_of_uniforms():
+    """N midpoint uniforms through an inverse CDF give each token a count
+    within one of N * p (the grid points falling in an interval of length p)."""
+    rng = np.random.default_rng(5)
+    V, N = 11, 4096
+    lp = rng.standard_normal(V) * 1.5
+    lq = rng.standard_normal(V)
+    grid = (np.arange(N) + 0.5) / N
+    u = np.stack([np.zeros(N), grid], 1)
+    d = acc.accept_rows(np.repeat(lp[None], N, 0), np.repeat(lq[None], N, 0), u,
+                        strategy="sample")
+    counts = np.bincount(d["out_tok"], minlength=V)
+    p = scipy.special.softmax(lp)
+    assert np.all(np.abs(counts - N * p) <= 1.0 + 1e-9)
+
+
+def test_strategies_share_ratio_and_lse():
+    rng = np.random.default_rng(8)
+    lp, lq = rng.standard_normal((16, 50)), rng.standard_normal((16, 50))
+    u = rng.random((16, 2))
+    base = acc.accept_rows(lp, lq, u)
+    for s in ("greedy", "sample"):
+        d = acc.accept_rows(lp, lq, u, strategy=s)
+        assert np.allclose(d["ratio"], base["ratio"]) and np.allclose(d["lse_p"], base["lse_p"])
+    with pytest.raises(ValueError):
+        acc.accept_rows(lp, lq, u, strategy="top_k")
