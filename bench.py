@@ -41,10 +41,17 @@ def parse():
     ap.add_argument("--fused-batch", type=int, default=1,
                     help="sequences of the fused-head workload (config 4): 1, or up to 5 "
                          "(240 draft rows) for the batched variant")
+    ap.add_argument("--strategy", default="accept_reject",
+                    choices=["accept_reject", "greedy", "sample"],
+                    help="token selection of Sec. 3.3: (C) accept-reject (default), (A) greedy, "
+                         "(B) sampling; logits workloads only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="approximate budget of the CPU-oracle sample")
-    return ap.parse_args()
+    a = ap.parse_args()
+    if a.strategy != "accept_reject" and a.config in (4, 5):
+        ap.error("--strategy other than accept_reject needs a logits workload (configs 1-3)")
+    return a
 
 
 # ----------------------------------------------------------------- workloads
@@ -173,7 +180,7 @@ def measured_peaks():
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_pass(c):
+def oracle_pass(c, strategy="accept_reject"):
     """One verification pass of the CPU oracle over every sequence of c."""
     from oracle import step as ostep
     q = synth.bf16_bits_to_f32(c.q).astype(np.float64)
@@ -188,7 +195,7 @@ def oracle_pass(c):
     else:
         lp, lq = c.tgt_logits, c.drf_logits
     r = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max,
-                          lp, lq, c.uniforms)
+                          lp, lq, c.uniforms, strategy=strategy)
     return r
 
 
@@ -209,7 +216,7 @@ def sub_case(c, seqs):
     return s
 
 
-def cpu_oracle_rate(c, budget_s):
+def cpu_oracle_rate(c, budget_s, strategy="accept_reject"):
     """Sequence verify steps/s of the oracle on a bounded sample of the
     workload: whole sequences of the batch, one after another (cycling over
     the batch), until about budget_s seconds of CPU work are done."""
@@ -217,7 +224,7 @@ def cpu_oracle_rate(c, budget_s):
     t0 = time.perf_counter()
     done = 0
     while True:
-        oracle_pass(sub_case(c, [done % c.B]))
+        oracle_pass(sub_case(c, [done % c.B]), strategy)
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
@@ -382,7 +389,7 @@ def main():
         if rank != 0:
             return 0
         c = workload(a.config, 0)
-        cpu = cpu_oracle_rate(c, a.cpu_seconds)
+        cpu = cpu_oracle_rate(c, a.cpu_seconds, a.strategy)
         line = {"impl": "reference", "metric": METRIC, "value": cpu["value"], "unit": UNIT,
                 "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
                 "ms_per_step": 1000.0 * c.B / cpu["value"], "higher_is_better": True,
@@ -425,7 +432,7 @@ def main():
     steps_obj = []
     for cs in cases:
         st = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max,
-                        c.V, k_v=c.k_v, device=dev, hidden=c.hidden)
+                        c.V, k_v=c.k_v, device=dev, hidden=c.hidden, strategy=a.strategy)
         st.upload(cache_len=cs.cache_len, q=cs.q, k=cs.k, v=cs.v, tgt_logits=cs.tgt_logits,
                   drf_logits=cs.drf_logits, h_tgt=cs.h_tgt, h_drf=cs.h_drf, w_tgt=cs.w_tgt,
                   w_drf=cs.w_drf)
@@ -516,8 +523,8 @@ def main():
                                   s.w_drf, None, 1.0, s.rng, s.out_tok, s.accepted, s.ratio, None,
                                   lm_ws, lm_wsb, s.status, cs)
         else:
-            ssd.ssd_accept(c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0, s.rng, s.out_tok,
-                           s.accepted, s.ratio, None, s.status, cs)
+            ssd.ssd_accept_strategy(a.strategy, c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0,
+                                    s.rng, s.out_tok, s.accepted, s.ratio, None, s.status, cs)
 
     def kernel_ms(call):
         gr = torch.cuda.CUDAGraph()
@@ -597,14 +604,15 @@ def main():
 
     cpu = None
     if not a.no_cpu_baseline:
-        cpu = cpu_oracle_rate(cases[0], a.cpu_seconds)
+        cpu = cpu_oracle_rate(cases[0], a.cpu_seconds, a.strategy)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps_done,
         "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 attention / f32 acceptance",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD_NAMES[a.config], "sequences_per_step": c.B,
+        "config": {"workload": WORKLOAD_NAMES[a.config], "strategy": a.strategy,
+                   "sequences_per_step": c.B,
                    "drafts_per_step": int(n_drafts[0].sum()), "vocab": c.V,
                    "heads": f"{c.Hq}/{c.Hkv}x{c.d}",
                    "l2": "two input sets alternate; each step streams "

@@ -81,7 +81,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 1
+#define SSD_ABI_VERSION 2
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -195,6 +195,29 @@ ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const fl
                       int32_t* status, ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * The three token-selection strategies of Sec. 3.3, applied to every row
+ * independently with the p, q, t, ratio and lse of ssd_accept():
+ *   SSD_STRATEGY_ACCEPT_REJECT  (C) the rule of ssd_accept() (the default)
+ *   SSD_STRATEGY_GREEDY         (A) out = argmax_v tgt[r][v] (lowest index
+ *                               on ties); accepted = (out == t)
+ *   SSD_STRATEGY_SAMPLE         (B) out = smallest v with
+ *                               sum_{v' <= v} p(v') > u_res * sum_v p(v);
+ *                               accepted = (out == t)
+ * ratio and lse are filled as by ssd_accept() under every strategy.
+ * An unknown strategy returns SSD_ERR_INVALID_ARG before any launch.
+ * ------------------------------------------------------------------------- */
+typedef enum {
+  SSD_STRATEGY_ACCEPT_REJECT = 0,
+  SSD_STRATEGY_GREEDY = 1,
+  SSD_STRATEGY_SAMPLE = 2
+} ssd_strategy;
+ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const float* tgt_logits,
+                               const float* drf_logits, int64_t ld, const int32_t* draft_tok,
+                               float temperature, const ssd_rng* rng, int32_t* out_tok,
+                               uint8_t* accepted, float* ratio, float* lse, int32_t* status,
+                               ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * a6. Fused lm_head + acceptance (Sec. 3.3, after Eq. 2: tokens are decoded
  * through the base model's GenHead).  Logits l_p = H_t W_t and l_q = H_d W_d
  * are formed on chip (tcgen05, fp32 accumulation) and fed to the rule of
@@ -229,6 +252,8 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * Logits path: tgt_logits/drf_logits non-NULL ([B*D_max] rows of ld floats).
  * Fused path:  logits NULL and h_tgt, h_drf, w_tgt, w_drf non-NULL (hidden
  *              = K of ssd_lmhead_accept).
+ * strategy: an ssd_strategy for the logits path; the fused path supports
+ * SSD_STRATEGY_ACCEPT_REJECT only (others: SSD_ERR_UNSUPPORTED).
  * Streams: the attention runs on `stream`; the acceptance, which shares no
  * data with it, runs concurrently on a side stream the library creates once
  * per device and host thread (with two events) and joins back into `stream`
@@ -255,6 +280,7 @@ typedef struct {
   const int32_t* draft_tok;   /* dev int32 [B*D_max] or NULL (argmax q)*/
   float temperature;
   ssd_rng rng;
+  int32_t strategy;           /* ssd_strategy (0: accept-reject)       */
 } ssd_verify_args;
 
 typedef struct {

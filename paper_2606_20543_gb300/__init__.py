@@ -22,8 +22,14 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
                 7: "SSD_ERR_WORKSPACE"}
 
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
-            "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
+            "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
+            "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
             "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
+
+
+STRATEGY_ACCEPT_REJECT, STRATEGY_GREEDY, STRATEGY_SAMPLE = 0, 1, 2
+STRATEGIES = {"accept_reject": STRATEGY_ACCEPT_REJECT, "greedy": STRATEGY_GREEDY,
+              "sample": STRATEGY_SAMPLE}
 
 
 class SsdError(RuntimeError):
@@ -56,7 +62,7 @@ class VerifyArgs(ctypes.Structure):
                 ("w_tgt", ctypes.c_void_p), ("w_drf", ctypes.c_void_p),
                 ("hidden", ctypes.c_int32),
                 ("draft_tok", ctypes.c_void_p), ("temperature", ctypes.c_float),
-                ("rng", Rng)]
+                ("rng", Rng), ("strategy", ctypes.c_int32)]
 
 
 class VerifyOut(ctypes.Structure):
@@ -91,6 +97,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_verify_attention_noalloc": (I32, [ctypes.POINTER(Grid), I32, I32, I32, I32, P, P, P,
                                                I32, I32, P, P, P, F, P, P, P, P]),
         "ssd_accept": (I32, [I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P, P, P, P]),
+        "ssd_accept_strategy": (I32, [I32, I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P,
+                                      P, P, P]),
         "ssd_lmhead_accept_workspace": (SZ, [I32, I32]),
         "ssd_lmhead_accept": (I32, [I32, I32, I32, P, P, P, P, P, F, ctypes.POINTER(Rng), P, P, P,
                                     P, P, SZ, P, P]),
@@ -180,6 +188,17 @@ def ssd_accept(rows, V, tgt_logits, drf_logits, ld, draft_tok, temperature, r: R
                accepted, ratio, lse, status, stream=None) -> None:
     _check("ssd_accept", load().ssd_accept(
         rows, V, _ptr(tgt_logits), _ptr(drf_logits), ld, _ptr(draft_tok), temperature,
+        ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
+        _stream(stream)))
+
+
+def ssd_accept_strategy(strategy, rows, V, tgt_logits, drf_logits, ld, draft_tok, temperature,
+                        r: Rng, out_tok, accepted, ratio, lse, status, stream=None) -> None:
+    """ssd_accept() under one of the strategies of Sec. 3.3: STRATEGY_ACCEPT_REJECT
+    (C), STRATEGY_GREEDY (A) or STRATEGY_SAMPLE (B); also accepts their names."""
+    strategy = STRATEGIES.get(strategy, strategy)
+    _check("ssd_accept_strategy", load().ssd_accept_strategy(
+        strategy, rows, V, _ptr(tgt_logits), _ptr(drf_logits), ld, _ptr(draft_tok), temperature,
         ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
         _stream(stream)))
 

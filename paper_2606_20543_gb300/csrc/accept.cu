@@ -3,6 +3,10 @@
 // residual draw (Sec. 3.3 "Verification as Auto Correction", strategy (C)):
 //   accept t with probability min(p(t) / q(t), 1); otherwise draw from
 //   [p - q]_+ / sum [p - q]_+ (inverse CDF in vocabulary order, one uniform).
+// The same kernel runs the paper's other two strategies: (A) greedy, the
+// argmax of p (tracked in the first pass), and (B) sampling, a draw from p
+// (the second pass with the weights of p); under both a row is "accepted"
+// when the selected token is the draft token.
 //
 // Design (GB300): a persistent grid of four CTAs per SM, each walking rows
 // blockIdx.x, blockIdx.x + gridDim.x, ...  A dedicated producer warp streams
@@ -118,6 +122,9 @@ struct Shared {
   uint64_t full[kStages], empty[kStages];
   float red[kCWarps][5];
   int32_t red_i[kCWarps];
+  float red_pm[kCWarps];  // greedy: per-warp maximum of p and its first index
+  int32_t red_pi[kCWarps];
+  int32_t t_hat;          // sampling: the draft token, for the accepted flag
   float Cp, Cq;      // log2-domain normalisers: max * c + log2(sum)
   int32_t accept;    // 1 accepted, 0 rejected, 2 no valid draft token, 3 drawn
   float u_res;
@@ -297,6 +304,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   }
 
   // ---------------------------------------------------------- consumer warps
+  const bool greedy = a.strategy == SSD_STRATEGY_GREEDY;
+  const bool sample = a.strategy == SSD_STRATEGY_SAMPLE;
   const float c = kLog2e / a.temperature;
   const float2 cc = make_float2(c, c);
   const int32_t nv = a.V >> 2;
@@ -325,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     // sums; the first argmax of q carries the p logit
     float mp = kLowest, mq = kLowest, xpa = 0.f;
     float2 sp2 = make_float2(0.f, 0.f), sq2 = sp2;
-    int32_t iq = 0x7fffffff;
+    int32_t iq = 0x7fffffff, ip = 0x7fffffff;
     for (int32_t ch = 0; ch < nch; ++ch, ++g) {
       const int s = g % kStages;
       mbar_wait(&sh.full[s], (g / kStages) & 1, a.status);
@@ -335,8 +344,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       const bool in0 = tid < cv, in1 = tid + kConsumers < cv;
       const float4 p0 = in0 ? xp4[tid] : ninf, p1 = in1 ? xp4[tid + kConsumers] : ninf;
       const float4 q0 = in0 ? xq4[tid] : ninf, q1 = in1 ? xq4[tid + kConsumers] : ninf;
-      const float nmp = fmax3(fmax3(p0.x, p0.y, p0.z), fmax3(p0.w, p1.x, p1.y), fmax3(p1.z, p1.w, mp));
+      const float cmp = fmax3(fmax3(p0.x, p0.y, p0.z), fmax3(p0.w, p1.x, p1.y), fmaxf(p1.z, p1.w));
       const float cmq = fmax3(fmax3(q0.x, q0.y, q0.z), fmax3(q0.w, q1.x, q1.y), fmaxf(q1.z, q1.w));
+      if (greedy && cmp > mp) {  // first argmax of p (strategy A)
+        const int32_t e0 = ch * kChunk + 4 * tid, e1 = e0 + 4 * kConsumers;
+        if (p0.x == cmp) ip = e0;
+        else if (p0.y == cmp) ip = e0 + 1;
+        else if (p0.z == cmp) ip = e0 + 2;
+        else if (p0.w == cmp) ip = e0 + 3;
+        else if (p1.x == cmp) ip = e1;
+        else if (p1.y == cmp) ip = e1 + 1;
+        else if (p1.z == cmp) ip = e1 + 2;
+        else ip = e1 + 3;
+      }
+      const float nmp = fmaxf(mp, cmp);
       if (cmq > mq) {
         const int32_t e0 = ch * kChunk + 4 * tid, e1 = e0 + 4 * kConsumers;
         if (q0.x == cmq) { iq = e0; xpa = p0.x; }
@@ -371,6 +392,19 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       if (lane == 0) mbar_arrive(&sh.empty[s]);
     }
     float sp = sp2.x + sp2.y, sq = sq2.x + sq2.y;
+    if (greedy) {  // first argmax of p over the CTA (warp tree, then the warps in order)
+      float pm = mp;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, pm, o);
+        const int32_t oi = __shfl_xor_sync(0xffffffffu, ip, o);
+        if (better_arg(om, oi, pm, ip)) { pm = om; ip = oi; }
+      }
+      if (lane == 0) {
+        sh.red_pm[warp] = pm;
+        sh.red_pi[warp] = ip;
+      }
+    }
     // block reduction in a fixed order: xor tree in each warp, then a
     // three-level xor tree over the warps' results in warp 0
 #pragma unroll
@@ -429,13 +463,29 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         } else {
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);  // non-finite logits
         }
-        sh.accept = acc ? 1 : (valid_t ? 0 : 2);
+        int32_t out = acc ? t : -1;
+        if (greedy && valid_t) {  // (A): the first argmax of p over the warps, in order
+          float pm = sh.red_pm[0];
+          int32_t pi = sh.red_pi[0];
+          for (int w = 1; w < kCWarps; ++w)
+            if (better_arg(sh.red_pm[w], sh.red_pi[w], pm, pi)) { pm = sh.red_pm[w]; pi = sh.red_pi[w]; }
+          out = pi;
+          acc = pi == t;
+        }
+        // (C) draws on rejection, (B) always; (A) never
+        sh.accept = !valid_t ? 2 : (sample ? 0 : (greedy || acc) ? 1 : 0);
+        sh.t_hat = t;
         sh.u_res = u.y;
         sh.Cp = Mp * c + lsp;
         sh.Cq = Mq * c + lsq;
-        a.accepted[r] = acc ? 1 : 0;
-        if (acc) a.out_tok[r] = t;
-        else if (!valid_t) a.out_tok[r] = -1;
+        if (!sample) {
+          a.accepted[r] = acc ? 1 : 0;
+          if (acc || greedy) a.out_tok[r] = out;
+        }
+        if (!valid_t) {
+          a.accepted[r] = 0;
+          a.out_tok[r] = -1;
+        }
         if (a.ratio) a.ratio[r] = ratio;
         if (a.lse) {
           a.lse[2 * r] = Mp / a.temperature + lsp * kLn2;
@@ -457,8 +507,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         const int32_t cv = min(kChunk, a.V - ch * kChunk) >> 2;
         const int32_t i0 = warp * 64 + lane, i1 = i0 + 32;
         float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
-        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], cc, ncp, ncq, false);
-        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], cc, ncp, ncq, false);
+        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], cc, ncp, ncq, sample);
+        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], cc, ncp, ncq, sample);
         const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
         if (lane == 0) block_mass[ch * kBlocksPerChunk + warp] = m;
       }
@@ -472,8 +522,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     if (warp == 0) {
       float tb;
       int32_t bk = find_block(block_mass, nblocks, sh.u_res, &tb, lane);
-      bool from_p = false;
-      if (bk < 0) {
+      bool from_p = sample;
+      if (bk < 0 && !sample) {
         // zero residual mass: the same draw from p (block masses of p itself)
         from_p = true;
         for (int32_t b0 = 0; b0 < nblocks; ++b0) {
@@ -490,11 +540,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       if (bk < 0) {
         if (lane == 0) {  // no positive mass at all (non-finite logits)
           a.out_tok[r] = -1;
+          if (sample) a.accepted[r] = 0;
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
       } else {
         const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
-        if (lane == 0) a.out_tok[r] = pick;
+        if (lane == 0) {
+          a.out_tok[r] = pick;
+          if (sample) a.accepted[r] = pick == sh.t_hat ? 1 : 0;
+        }
       }
     }
     consumers_sync();  // block masses and sh are reused by the next row

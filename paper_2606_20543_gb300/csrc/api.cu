@@ -73,6 +73,11 @@ ssd_status check_accept_common(int32_t rows, int32_t V, float temperature, const
   return SSD_OK;
 }
 
+bool strategy_ok(int32_t strategy) {
+  return strategy == SSD_STRATEGY_ACCEPT_REJECT || strategy == SSD_STRATEGY_GREEDY ||
+         strategy == SSD_STRATEGY_SAMPLE;
+}
+
 ssd_status check_logits(int32_t rows, int32_t V, const float* tgt, const float* drf, int64_t ld) {
   if (rows == 0) return SSD_OK;
   if (tgt == nullptr || drf == nullptr) return SSD_ERR_INVALID_ARG;
@@ -200,10 +205,12 @@ ssd_status ssd_verify_attention_noalloc(const ssd_grid* grid, int32_t B, int32_t
   return from_cuda(e);
 }
 
-ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
-                      int64_t ld, const int32_t* draft_tok, float temperature, const ssd_rng* rng,
-                      int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
-                      int32_t* status, ssd_stream_t stream) {
+ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const float* tgt_logits,
+                               const float* drf_logits, int64_t ld, const int32_t* draft_tok,
+                               float temperature, const ssd_rng* rng, int32_t* out_tok,
+                               uint8_t* accepted, float* ratio, float* lse, int32_t* status,
+                               ssd_stream_t stream) {
+  if (!strategy_ok(strategy)) return SSD_ERR_INVALID_ARG;
   ssd_status s = check_accept_common(rows, V, temperature, rng, out_tok, accepted, status);
   if (s != SSD_OK) return s;
   s = check_logits(rows, V, tgt_logits, drf_logits, ld);
@@ -225,7 +232,17 @@ ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const fl
   a.status = status;
   a.n_drafts = nullptr;
   a.D_max = 1;
+  a.strategy = strategy;
   return from_cuda(launch_accept(a, (cudaStream_t)stream));
+}
+
+ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
+                      int64_t ld, const int32_t* draft_tok, float temperature, const ssd_rng* rng,
+                      int32_t* out_tok, uint8_t* accepted, float* ratio, float* lse,
+                      int32_t* status, ssd_stream_t stream) {
+  return ssd_accept_strategy(SSD_STRATEGY_ACCEPT_REJECT, rows, V, tgt_logits, drf_logits, ld,
+                             draft_tok, temperature, rng, out_tok, accepted, ratio, lse, status,
+                             stream);
 }
 
 size_t ssd_lmhead_accept_workspace(int32_t rows, int32_t V) {
@@ -305,10 +322,12 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   const int32_t rows = x->B * x->D_max;
   s = check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
   if (s != SSD_OK) return s;
+  if (!strategy_ok(x->strategy)) return SSD_ERR_INVALID_ARG;
   const bool fused = (x->tgt_logits == nullptr);
   if (fused) {
     if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
       return SSD_ERR_INVALID_ARG;
+    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT) return SSD_ERR_UNSUPPORTED;
     s = lmhead_check(rows, x->V, x->hidden);
     if (s != SSD_OK) return s;
   } else {
@@ -390,6 +409,7 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     c.status = y->status;
     c.n_drafts = y->n_drafts;
     c.D_max = x->D_max;
+    c.strategy = x->strategy;
     e = launch_accept(c, side->stream);
   }
   if (e != cudaSuccess) return SSD_ERR_CUDA;

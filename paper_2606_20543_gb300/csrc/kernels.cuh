@@ -30,6 +30,7 @@ struct AcceptArgs {
   int32_t* status;
   const int32_t* n_drafts;   // nullable: row r valid iff r % D_max < n_drafts[r / D_max]
   int32_t D_max;
+  int32_t strategy;          // ssd_strategy: (C) accept-reject, (A) greedy, (B) sampling
 };
 bool accept_supported(int32_t V);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);

@@ -10,7 +10,7 @@ from __future__ import annotations
 import numpy as np
 import torch
 
-from . import (Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid, ssd_verify_step,
+from . import (STRATEGIES, Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid, ssd_verify_step,
                ssd_verify_step_workspace)
 
 
@@ -35,12 +35,14 @@ class VerifyStep:
     lm_head weights [hidden, V] (bf16)."""
 
     def __init__(self, grid_h, grid_w, prefix_len, B, Hq, Hkv, d, D_max, L_max, V,
-                 hidden=0, k_v=1, row_stride=None, device="cuda", scale=0.0, temperature=1.0):
+                 hidden=0, k_v=1, row_stride=None, device="cuda", scale=0.0, temperature=1.0,
+                 strategy="accept_reject"):
         self.g: Grid = make_grid(grid_h, grid_w, prefix_len, row_stride, k_v)
         self.B, self.Hq, self.Hkv, self.d = B, Hq, Hkv, d
         self.D_max, self.L_max, self.V, self.hidden = D_max, L_max, V, hidden
         self.device = device
         self.scale, self.temperature = scale, temperature
+        self.strategy = STRATEGIES.get(strategy, strategy)
         rows = B * D_max
         self.rows = rows
         dv = device
@@ -101,6 +103,7 @@ class VerifyStep:
         a.draft_tok = None if self.draft_tok is None else self.draft_tok.data_ptr()
         a.temperature = self.temperature
         a.rng = self.rng
+        a.strategy = self.strategy
         return a
 
     def _out(self) -> VerifyOut:

@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 1
+    assert lib.ssd_abi_version() == 2
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 
@@ -77,6 +77,16 @@ def test_host_side_validation(lib):
     # zero rows is a no-op
     assert so.ssd_accept(0, 4096, None, None, 4096, None, 1.0, ctypes.byref(r), fake, fake, None,
                          None, fake, None) == 0
+    # strategies: unknown codes are rejected before anything else; known ones
+    # reach the same argument checks as ssd_accept
+    for bad in (-1, 3, 99):
+        assert so.ssd_accept_strategy(bad, 0, 4096, None, None, 4096, None, 1.0, ctypes.byref(r),
+                                      fake, fake, None, None, fake, None) == 1
+    for good in (lib.STRATEGY_ACCEPT_REJECT, lib.STRATEGY_GREEDY, lib.STRATEGY_SAMPLE):
+        assert so.ssd_accept_strategy(good, 0, 4096, None, None, 4096, None, 1.0,
+                                      ctypes.byref(r), fake, fake, None, None, fake, None) == 0
+        assert so.ssd_accept_strategy(good, 4, 4098, fake, fake, 4100, None, 1.0,
+                                      ctypes.byref(r), fake, fake, None, None, fake, None) == 2
     # frontier: D_max too small for (k_v + 1) * W, end-of-line stride unsupported
     assert so.ssd_frontier(ctypes.byref(g), 1, fake, 31, fake, fake, fake, None) == 2
     g2 = lib.grid(16, 16, 32, row_stride=17)

@@ -21,7 +21,8 @@ def ssd():
     return m
 
 
-def run_accept(ssd, tgt, drf, uniforms=None, seed=0, offset=0, draft_tok=None, T=1.0, ld=None):
+def run_accept(ssd, tgt, drf, uniforms=None, seed=0, offset=0, draft_tok=None, T=1.0, ld=None,
+               strategy="accept_reject"):
     rows, V = tgt.shape
     ld = V if ld is None else ld
     dev = "cuda"
@@ -36,8 +37,8 @@ def run_accept(ssd, tgt, drf, uniforms=None, seed=0, offset=0, draft_tok=None, T
     ratio = torch.zeros((rows,), dtype=torch.float32, device=dev)
     lse = torch.zeros((rows, 2), dtype=torch.float32, device=dev)
     status = torch.zeros((1,), dtype=torch.int32, device=dev)
-    ssd.ssd_accept(rows, V, tg, dg, ld, dt, T, ssd.rng(seed, offset, u), out_tok, acc, ratio, lse,
-                   status)
+    ssd.ssd_accept_strategy(strategy, rows, V, tg, dg, ld, dt, T, ssd.rng(seed, offset, u),
+                            out_tok, acc, ratio, lse, status)
     torch.cuda.synchronize()
     return (out_tok.cpu().numpy(), acc.cpu().numpy(), ratio.cpu().numpy(), lse.cpu().numpy(),
             int(status.item()))
@@ -139,3 +140,58 @@ def test_out_of_range_draft_token_sets_status(ssd):
     assert st == 6
     assert tok[1] == -1 and tok[3] == -1 and acc[1] == 0 and acc[3] == 0
     assert tok[0] >= 0 and tok[2] >= 0
+
+
+# ---------------------------------------------------------------------------
+# Strategies (A) greedy and (B) sampling of Sec. 3.3.
+
+@pytest.mark.parametrize("strategy", ["greedy", "sample"])
+@pytest.mark.parametrize("V,rows,logits,seed", [
+    (16384, 48, "normal", 21),
+    (16384, 40, "zipf", 22),
+    (4100, 30, "normal", 23),     # ragged last chunk
+    (12, 16, "normal", 24),       # tiny vocabulary
+    (65536, 8, "zipf", 25),
+])
+def test_strategy_matches_oracle(ssd, strategy, V, rows, logits, seed):
+    rng = np.random.default_rng(seed)
+    if logits == "normal":
+        tgt, drf = synth._logits_normal(rng, rows, V)
+    else:
+        tgt, drf = synth._logits_zipf(rng, rows, V)
+    u = synth.philox_uniforms(seed, 3, rows)
+    tok, acc, ratio, lse, st = run_accept(ssd, tgt, drf, u, strategy=strategy)
+    assert st == 0
+    dec = oacc.accept_rows(tgt, drf, u, strategy=strategy)
+    ties = compare_decisions(dec, tok, acc, ratio, lse, what=f"{strategy} V={V}")
+    if strategy == "greedy":
+        assert ties == 0  # an argmax of raw fp32 logits has no rounding to excuse
+    assert ties <= max(2, rows // 10)
+
+
+def test_greedy_ties_and_given_tokens(ssd):
+    rng = np.random.default_rng(26)
+    rows, V = 32, 8192
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    for r in range(rows):  # the target maximum appears twice; the lower index wins
+        i, j = sorted(rng.choice(V, 2, replace=False))
+        tgt[r, [i, j]] = tgt[r].max() + 0.5
+    dt = np.argmax(tgt, 1).astype(np.int64)
+    dt[::2] = rng.integers(0, V, rows // 2)  # half the rows with another draft token
+    u = synth.philox_uniforms(7, 0, rows)
+    tok, acc, _, _, st = run_accept(ssd, tgt, drf, u, draft_tok=dt, strategy="greedy")
+    assert st == 0
+    assert np.array_equal(tok, np.argmax(tgt, 1))
+    assert np.array_equal(acc.astype(bool), np.argmax(tgt, 1) == dt)
+
+
+def test_sampling_with_given_tokens_and_temperature(ssd):
+    rng = np.random.default_rng(27)
+    rows, V = 64, 16384
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    dt = rng.integers(0, V, rows).astype(np.int64)
+    u = synth.philox_uniforms(8, 0, rows)
+    tok, acc, ratio, _, st = run_accept(ssd, tgt, drf, u, draft_tok=dt, T=0.7, strategy="sample")
+    assert st == 0
+    dec = oacc.accept_rows(tgt, drf, u, draft_tok=dt, temperature=0.7, strategy="sample")
+    compare_decisions(dec, tok, acc, ratio, what="sample T=0.7")

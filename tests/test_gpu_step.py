@@ -22,18 +22,18 @@ def ssd():
     return m
 
 
-def make_step(c):
+def make_step(c, strategy="accept_reject"):
     from paper_2606_20543_gb300.step import VerifyStep
     s = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V,
-                   k_v=c.k_v)
+                   k_v=c.k_v, strategy=strategy)
     s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=c.tgt_logits,
              drf_logits=c.drf_logits, uniforms=c.uniforms)
     return s
 
 
-def check_step(c, res, attention_seqs=None):
+def check_step(c, res, attention_seqs=None, strategy="accept_reject"):
     ref = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max,
-                            c.tgt_logits, c.drf_logits, c.uniforms)
+                            c.tgt_logits, c.drf_logits, c.uniforms, strategy=strategy)
     assert res["status"][0] == 0
     assert np.array_equal(res["n_drafts"], ref["n_drafts"])
     assert np.array_equal(res["draft_pos"], ref["draft_pos"])
@@ -146,3 +146,14 @@ def test_step_large_batch_of_small_grids(ssd):
     s.run()
     torch.cuda.synchronize()
     check_step(c, s.results(), attention_seqs=[0, 1, 550, 1099])
+
+
+@pytest.mark.parametrize("strategy", ["greedy", "sample"])
+def test_step_strategies(ssd, strategy):
+    """The whole step under strategies (A) and (B): the prefix rule of the
+    counts reads the accepted flags (selected token == draft token)."""
+    for c in (synth.config1(cache_len=192, seed=3), synth.config2(points=[120, 480, 672])):
+        s = make_step(c, strategy)
+        s.run()
+        torch.cuda.synchronize()
+        check_step(c, s.results(), strategy=strategy)
