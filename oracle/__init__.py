@@ -24,6 +24,10 @@ Modules and the passage each follows:
              (horizontal prefix acceptance): accepted counts and the next
              cache length of a single-round replay.
   lmhead     Sec. 3.3, Eq. 2's GenHead: logits = hidden @ W, then accept.
+  rounds     Sec. 3.3 (r verify-and-correct rounds: rejected positions take
+             the residual sample and this round's p as their reference; the
+             commit after the last round) and App. multi-row drafting (the
+             staged b / i schedule).
   step       the above chained in the order of Sec. 3.3, and the
              single-round replay to grid completion.
 
