@@ -45,12 +45,26 @@ def parse():
                     choices=["accept_reject", "greedy", "sample"],
                     help="token selection of Sec. 3.3: (C) accept-reject (default), (A) greedy, "
                          "(B) sampling; logits workloads only")
+    ap.add_argument("--rounds", type=int, default=1,
+                    help="verify-and-correct rounds per step (Sec. 3.3); > 1 commits the whole "
+                         "block after the last round")
+    ap.add_argument("--staged", default=None, metavar="B,I",
+                    help="staged two-row schedule: B base rounds, commit the first row, I rounds "
+                         "on the trailing row (configs 1-2, whose frontiers start at a row)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="approximate budget of the CPU-oracle sample")
     a = ap.parse_args()
     if a.strategy != "accept_reject" and a.config in (4, 5):
         ap.error("--strategy other than accept_reject needs a logits workload (configs 1-3)")
+    if (a.rounds != 1 or a.staged) and a.config in (4, 5):
+        ap.error("--rounds / --staged need a logits workload (configs 1-3)")
+    if a.staged:
+        a.staged = tuple(int(x) for x in a.staged.split(","))
+        if len(a.staged) != 2 or a.staged[0] < 1 or a.staged[1] < 1 or a.config not in (1, 2):
+            ap.error("--staged B,I with B, I >= 1 on config 1 or 2")
+    if a.rounds < 1:
+        ap.error("--rounds >= 1")
     return a
 
 
@@ -440,16 +454,46 @@ def main():
     stream = torch.cuda.current_stream(dev)
     seed = 1234 + rank
 
+    # verify-and-correct rounds: every round has its own target logits (the
+    # backbone's output for the corrected block), drifting from round to round
+    R = sum(a.staged) if a.staged else a.rounds
+    rounds_objs = None
+    if R > 1:
+        from paper_2606_20543_gb300.step import VerifyRounds
+        rounds_objs = [VerifyRounds(st) for st in steps_obj]
+        tgt_sets = []
+        for si, st in enumerate(steps_obj):
+            gen = np.random.default_rng(77 + si + 100 * rank)
+            prev, bufs = cases[si].tgt_logits, [st.tgt]
+            for _ in range(1, R):
+                prev = (0.6 * prev + 0.4 * synth._logits_normal(gen, prev.shape[0], c.V)[0]
+                        ).astype(np.float32)
+                bufs.append(torch.from_numpy(prev).to(dev))
+            tgt_sets.append(bufs)
+        init_cache = [st.cache_len.clone() for st in steps_obj]
+
     def run(i):
         st = steps_obj[i & 1]
-        st.set_rng(seed, i)
-        st.run()  # torch's current stream (the capture stream inside a graph)
+        if rounds_objs is None:
+            st.set_rng(seed, i)
+            st.run()  # torch's current stream (the capture stream inside a graph)
+        elif a.staged:
+            rounds_objs[i & 1].run_staged(a.staged[0], a.staged[1], tgt_sets[i & 1], seed=seed,
+                                          offset0=i * R)
+            st.cache_len.copy_(init_cache[i & 1])  # every step verifies the same blocks
+        else:
+            rounds_objs[i & 1].run(tgt_sets[i & 1], "block", seed=seed, offset0=i * R)
 
+    if a.staged:  # the two-row frontiers, before the staged rounds narrow them
+        for st in steps_obj:
+            st.run()
+        torch.cuda.synchronize(dev)
+        full_drafts = [st.n_drafts.cpu().numpy() for st in steps_obj]
     for i in range(a.warmup):
         run(i)
     torch.cuda.synchronize(dev)
-    n_drafts = [st.n_drafts.cpu().numpy() for st in steps_obj]
-    launches = ssd.ssd_verify_step_launches(steps_obj[0].args)
+    n_drafts = full_drafts if a.staged else [st.n_drafts.cpu().numpy() for st in steps_obj]
+    launches = ssd.ssd_verify_step_launches(steps_obj[0].args) * R + (1 if a.staged else 0)
     attn_bytes, acc_bytes = algorithmic_bytes(c, n_drafts[0])
 
     # The K timed passes are captured once as a CUDA graph (each pass with its
@@ -496,6 +540,8 @@ def main():
         accepted_tok.append(int(st.accepted_count.sum().item()))
     acc_tok_per_step = float(np.mean(accepted_tok))
     committed = float(np.mean([(st.next_cache_len - st.cache_len).sum().item() for st in steps_obj]))
+    if a.staged:  # both rows are committed (the cache is restored after each step)
+        committed = float(np.mean([nd.sum() for nd in n_drafts]))
 
     # ---------------- per-kernel durations: each kernel's entry point captured
     # as a graph of back-to-back launches on the two alternating input sets,
@@ -612,6 +658,8 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 attention / f32 acceptance",
         "data": "synthetic",
         "config": {"workload": WORKLOAD_NAMES[a.config], "strategy": a.strategy,
+                   "verify_rounds": (f"staged b={a.staged[0]}, i={a.staged[1]}" if a.staged
+                                     else a.rounds),
                    "sequences_per_step": c.B,
                    "drafts_per_step": int(n_drafts[0].sum()), "vocab": c.V,
                    "heads": f"{c.Hq}/{c.Hkv}x{c.d}",

@@ -66,7 +66,8 @@ typedef struct {
   int32_t grid_w;     /* W: grid columns                                  */
   int32_t row_stride; /* W or W + 1                                       */
   int32_t prefix_len; /* text-prefix tokens before grid token (0, 0)      */
-  int32_t k_v;        /* rows drafted below the current row, >= 1         */
+  int32_t k_v;        /* rows drafted below the current row, >= 0 (0: the
+                         rest of the current row only)                  */
 } ssd_grid;
 
 /* Per-draft uniforms (u_acc, u_res).  If `uniforms` (dev, float32
@@ -81,7 +82,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 2
+#define SSD_ABI_VERSION 3
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -218,6 +219,52 @@ ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const 
                                ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * One verify-and-correct round (Sec. 3.3: "We repeat this verify-and-correct
+ * procedure for a fixed number of rounds r ... For a rejected position, the
+ * previous-round backbone distribution becomes its reference distribution in
+ * the next round, while accepted positions retain their current reference").
+ * For every row r the rule of ssd_accept_strategy() is applied with
+ *     q = softmax(ref_rows[r][0 .. V) / T)   (the row's current reference)
+ *     t = tok[r]                             (the position's current token;
+ *                                             NULL: argmax of the reference row,
+ *                                             the draft token of round 1)
+ * and, when the row is not accepted, ref_rows[r] is set to tgt + r * ld, so
+ * this round's distribution is the row's reference in the next round.  Round
+ * 1 passes pointers to the draft rows and the draft tokens; out_tok is the
+ * next round's tok.  Give every round its own rng offset.
+ *   ref_rows  dev [rows] of const float* (in/out), each 16-byte aligned
+ *   tok       dev int32 [rows] or NULL
+ *   other arguments as ssd_accept_strategy().
+ * ------------------------------------------------------------------------- */
+ssd_status ssd_accept_round(int32_t strategy, int32_t rows, int32_t V, const float* tgt_logits,
+                            int64_t ld, const float** ref_rows, const int32_t* tok,
+                            float temperature, const ssd_rng* rng, int32_t* out_tok,
+                            uint8_t* accepted, float* ratio, float* lse, int32_t* status,
+                            ssd_stream_t stream);
+
+/* Commit rule of the counts of ssd_verify_step() (a7):
+ *   SSD_COMMIT_PREFIX     one round: the drafts up to and including the first
+ *                         rejected one (the horizontal stage; the default)
+ *   SSD_COMMIT_NONE       a round before the last: nothing is committed
+ *   SSD_COMMIT_BLOCK      the last of r rounds: the whole corrected block
+ *   SSD_COMMIT_FIRST_ROW  the staged schedule's first commit: the frontier's
+ *                         first row, W - (cache_len - prefix_len) % W drafts */
+typedef enum {
+  SSD_COMMIT_PREFIX = 0,
+  SSD_COMMIT_NONE = 1,
+  SSD_COMMIT_BLOCK = 2,
+  SSD_COMMIT_FIRST_ROW = 3
+} ssd_commit;
+
+/* Staged schedule (App. multi-row, "commit the first row, then refine the
+ * trailing row"): for every sequence b and j < W, slot b * D_max + j of tok
+ * and of ref_rows (may be NULL) takes slot b * D_max + W + j, so the
+ * trailing row of a two-row frontier becomes the frontier of the incremental
+ * rounds (k_v = 0).  Requires 2 * W <= D_max. */
+ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
+                           const float** ref_rows, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * a6. Fused lm_head + acceptance (Sec. 3.3, after Eq. 2: tokens are decoded
  * through the base model's GenHead).  Logits l_p = H_t W_t and l_q = H_d W_d
  * are formed on chip (tcgen05, fp32 accumulation) and fed to the rule of
@@ -254,6 +301,12 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  *              = K of ssd_lmhead_accept).
  * strategy: an ssd_strategy for the logits path; the fused path supports
  * SSD_STRATEGY_ACCEPT_REJECT only (others: SSD_ERR_UNSUPPORTED).
+ * ref_rows: NULL, or the per-row references of a verify-and-correct round
+ * (see ssd_accept_round(); logits path only).  ref_init = 1 marks round 1:
+ * the references are the draft rows (drf_logits) and every entry of
+ * ref_rows is written (the draft row, or the target row when the row is
+ * not accepted), so no pass over ref_rows is needed before a block.
+ * commit: an ssd_commit; the counts' next_cache_len follows it.
  * Streams: the attention runs on `stream`; the acceptance, which shares no
  * data with it, runs concurrently on a side stream the library creates once
  * per device and host thread (with two events) and joins back into `stream`
@@ -281,6 +334,9 @@ typedef struct {
   float temperature;
   ssd_rng rng;
   int32_t strategy;           /* ssd_strategy (0: accept-reject)       */
+  const float** ref_rows;     /* dev [B*D_max] or NULL (round refs)    */
+  int32_t ref_init;           /* 1: round 1 (writes every ref_rows)    */
+  int32_t commit;             /* ssd_commit (0: prefix rule)           */
 } ssd_verify_args;
 
 typedef struct {

@@ -23,11 +23,15 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
 
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
             "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
+            "ssd_accept_round", "ssd_stage_shift",
             "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
             "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
 
 
 STRATEGY_ACCEPT_REJECT, STRATEGY_GREEDY, STRATEGY_SAMPLE = 0, 1, 2
+COMMIT_PREFIX, COMMIT_NONE, COMMIT_BLOCK, COMMIT_FIRST_ROW = 0, 1, 2, 3
+COMMITS = {"prefix": COMMIT_PREFIX, "none": COMMIT_NONE, "block": COMMIT_BLOCK,
+           "first_row": COMMIT_FIRST_ROW}
 STRATEGIES = {"accept_reject": STRATEGY_ACCEPT_REJECT, "greedy": STRATEGY_GREEDY,
               "sample": STRATEGY_SAMPLE}
 
@@ -62,7 +66,8 @@ class VerifyArgs(ctypes.Structure):
                 ("w_tgt", ctypes.c_void_p), ("w_drf", ctypes.c_void_p),
                 ("hidden", ctypes.c_int32),
                 ("draft_tok", ctypes.c_void_p), ("temperature", ctypes.c_float),
-                ("rng", Rng), ("strategy", ctypes.c_int32)]
+                ("rng", Rng), ("strategy", ctypes.c_int32), ("ref_rows", ctypes.c_void_p),
+                ("ref_init", ctypes.c_int32), ("commit", ctypes.c_int32)]
 
 
 class VerifyOut(ctypes.Structure):
@@ -99,6 +104,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_accept": (I32, [I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P, P, P, P]),
         "ssd_accept_strategy": (I32, [I32, I32, I32, P, P, I64, P, F, ctypes.POINTER(Rng), P, P, P,
                                       P, P, P]),
+        "ssd_accept_round": (I32, [I32, I32, I32, P, I64, P, P, F, ctypes.POINTER(Rng), P, P, P, P,
+                                   P, P]),
+        "ssd_stage_shift": (I32, [I32, I32, I32, P, P, P]),
         "ssd_lmhead_accept_workspace": (SZ, [I32, I32]),
         "ssd_lmhead_accept": (I32, [I32, I32, I32, P, P, P, P, P, F, ctypes.POINTER(Rng), P, P, P,
                                     P, P, SZ, P, P]),
@@ -201,6 +209,30 @@ def ssd_accept_strategy(strategy, rows, V, tgt_logits, drf_logits, ld, draft_tok
         strategy, rows, V, _ptr(tgt_logits), _ptr(drf_logits), ld, _ptr(draft_tok), temperature,
         ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
         _stream(stream)))
+
+
+def ssd_accept_round(strategy, rows, V, tgt_logits, ld, ref_rows, tok, temperature, r: Rng,
+                     out_tok, accepted, ratio, lse, status, stream=None) -> None:
+    """One verify-and-correct round: ref_rows is a device int64 tensor of row
+    addresses (updated in place for rows the round does not accept)."""
+    strategy = STRATEGIES.get(strategy, strategy)
+    _check("ssd_accept_round", load().ssd_accept_round(
+        strategy, rows, V, _ptr(tgt_logits), ld, _ptr(ref_rows), _ptr(tok), temperature,
+        ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
+        _stream(stream)))
+
+
+def ssd_stage_shift(B, D_max, W, tok, ref_rows, stream=None) -> None:
+    _check("ssd_stage_shift", load().ssd_stage_shift(B, D_max, W, _ptr(tok), _ptr(ref_rows),
+                                                     _stream(stream)))
+
+
+def row_addresses(t, ld=None):
+    """Device int64 tensor of the addresses of the rows of a 2D float32 tensor
+    (the reference pointers of round 1)."""
+    import torch
+    ld = t.shape[1] if ld is None else ld
+    return t.data_ptr() + torch.arange(t.shape[0], device=t.device, dtype=torch.int64) * (ld * 4)
 
 
 def ssd_lmhead_accept_workspace(rows, V) -> int:

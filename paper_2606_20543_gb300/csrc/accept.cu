@@ -287,6 +287,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       uint32_t g = 0;  // chunks issued by this CTA
       for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
         if (row_kind(a, r) != 0) continue;
+        // the row's reference is read once: the consumers may redirect it for
+        // the next round while this row's second pass is still being issued
+        const float* drow =
+            (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
         for (int32_t cc = 0; cc < 2 * nch; ++cc, ++g) {  // two passes over the row
           const int32_t ch = cc % nch;
           const int s = g % kStages;
@@ -295,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
           float* dst = ring + s * 2 * kChunk;
           mbar_arrive_expect_tx(&sh.full[s], 2u * bytes);
           bulk_g2s(dst, a.tgt + r * a.ld + (int64_t)ch * kChunk, bytes, &sh.full[s]);
-          bulk_g2s(dst + kChunk, a.drf + r * a.ld + (int64_t)ch * kChunk, bytes, &sh.full[s]);
+          bulk_g2s(dst + kChunk, drow + (int64_t)ch * kChunk, bytes, &sh.full[s]);
         }
       }
     }
@@ -321,10 +325,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         if (a.ratio) a.ratio[r] = 0.f;
         if (kind == 1 && a.lse) { a.lse[2 * r] = 0.f; a.lse[2 * r + 1] = 0.f; }
         if (kind == 2) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+        if (a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = a.drf + r * a.ld;
       }
       continue;
     }
     const int32_t given_t = a.draft_tok != nullptr ? a.draft_tok[r] : -1;
+    const float* drow =
+        (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
     // the row's uniforms, drawn while its first chunk is still in flight
     const float2 u = (tid == 0) ? row_uniforms(a.rng, r) : make_float2(0.f, 0.f);
 
@@ -478,9 +485,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         sh.u_res = u.y;
         sh.Cp = Mp * c + lsp;
         sh.Cq = Mq * c + lsq;
+        // round 1 starts every reference at the draft row; a draw that differs
+        // from the token redirects it below (sampling) or here (the others)
+        if (sample && a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = drow;
         if (!sample) {
           a.accepted[r] = acc ? 1 : 0;
           if (acc || greedy) a.out_tok[r] = out;
+          // the next round's reference of a row this round did not accept
+          if (a.ref_rows != nullptr && valid_t && !acc) a.ref_rows[r] = a.tgt + r * a.ld;
+          else if (a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = drow;
         }
         if (!valid_t) {
           a.accepted[r] = 0;
@@ -518,7 +531,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     if (!draw) continue;  // uniform
     consumers_sync();
     const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
-    const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
+    const float4* dp = reinterpret_cast<const float4*>(drow);
     if (warp == 0) {
       float tb;
       int32_t bk = find_block(block_mass, nblocks, sh.u_res, &tb, lane);
@@ -547,7 +560,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
         if (lane == 0) {
           a.out_tok[r] = pick;
-          if (sample) a.accepted[r] = pick == sh.t_hat ? 1 : 0;
+          if (sample) {
+            a.accepted[r] = pick == sh.t_hat ? 1 : 0;
+            if (a.ref_rows != nullptr && pick != sh.t_hat) a.ref_rows[r] = a.tgt + r * a.ld;
+            else if (a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = drow;
+          }
         }
       }
     }

@@ -42,7 +42,7 @@ cudaError_t side_stream(SideStream** out) {
 
 ssd_status check_grid(const ssd_grid* g) {
   if (g == nullptr) return SSD_ERR_INVALID_ARG;
-  if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 1) return SSD_ERR_SHAPE;
+  if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 0) return SSD_ERR_SHAPE;
   if (g->row_stride != g->grid_w && g->row_stride != g->grid_w + 1) return SSD_ERR_SHAPE;
   if ((int64_t)g->grid_h * g->row_stride + g->prefix_len > INT32_MAX / 2) return SSD_ERR_SHAPE;
   return SSD_OK;
@@ -233,7 +233,53 @@ ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const 
   a.n_drafts = nullptr;
   a.D_max = 1;
   a.strategy = strategy;
+  a.ref_rows = nullptr;
+  a.ref_init = 0;
   return from_cuda(launch_accept(a, (cudaStream_t)stream));
+}
+
+ssd_status ssd_accept_round(int32_t strategy, int32_t rows, int32_t V, const float* tgt_logits,
+                            int64_t ld, const float** ref_rows, const int32_t* tok,
+                            float temperature, const ssd_rng* rng, int32_t* out_tok,
+                            uint8_t* accepted, float* ratio, float* lse, int32_t* status,
+                            ssd_stream_t stream) {
+  if (!strategy_ok(strategy)) return SSD_ERR_INVALID_ARG;
+  ssd_status s = check_accept_common(rows, V, temperature, rng, out_tok, accepted, status);
+  if (s != SSD_OK) return s;
+  if (rows == 0) return SSD_OK;
+  if (ref_rows == nullptr) return SSD_ERR_INVALID_ARG;
+  // the reference rows are only known on the device; the target is checked
+  // like the draft logits of ssd_accept_strategy()
+  s = check_logits(rows, V, tgt_logits, tgt_logits, ld);
+  if (s != SSD_OK) return s;
+  AcceptArgs a;
+  a.rows = rows;
+  a.V = V;
+  a.tgt = tgt_logits;
+  a.drf = nullptr;
+  a.ld = ld;
+  a.draft_tok = tok;
+  a.temperature = temperature;
+  a.rng = *rng;
+  a.out_tok = out_tok;
+  a.accepted = accepted;
+  a.ratio = ratio;
+  a.lse = lse;
+  a.status = status;
+  a.n_drafts = nullptr;
+  a.D_max = 1;
+  a.strategy = strategy;
+  a.ref_rows = ref_rows;
+  a.ref_init = 0;
+  return from_cuda(launch_accept(a, (cudaStream_t)stream));
+}
+
+ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
+                           const float** ref_rows, ssd_stream_t stream) {
+  if (B < 0 || D_max <= 0 || W < 0 || 2 * (int64_t)W > D_max) return SSD_ERR_SHAPE;
+  if (B == 0 || W == 0) return SSD_OK;
+  if (tok == nullptr) return SSD_ERR_INVALID_ARG;
+  return from_cuda(launch_stage_shift(B, D_max, W, tok, ref_rows, (cudaStream_t)stream));
 }
 
 ssd_status ssd_accept(int32_t rows, int32_t V, const float* tgt_logits, const float* drf_logits,
@@ -323,11 +369,15 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   s = check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
   if (s != SSD_OK) return s;
   if (!strategy_ok(x->strategy)) return SSD_ERR_INVALID_ARG;
+  if (x->commit < SSD_COMMIT_PREFIX || x->commit > SSD_COMMIT_FIRST_ROW) return SSD_ERR_INVALID_ARG;
+  if (x->ref_init != 0 && (x->ref_rows == nullptr || x->drf_logits == nullptr))
+    return SSD_ERR_INVALID_ARG;
   const bool fused = (x->tgt_logits == nullptr);
   if (fused) {
     if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
       return SSD_ERR_INVALID_ARG;
-    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT) return SSD_ERR_UNSUPPORTED;
+    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT || x->ref_rows != nullptr)
+      return SSD_ERR_UNSUPPORTED;
     s = lmhead_check(rows, x->V, x->hidden);
     if (s != SSD_OK) return s;
   } else {
@@ -410,6 +460,8 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     c.n_drafts = y->n_drafts;
     c.D_max = x->D_max;
     c.strategy = x->strategy;
+    c.ref_rows = x->ref_rows;
+    c.ref_init = x->ref_init;
     e = launch_accept(c, side->stream);
   }
   if (e != cudaSuccess) return SSD_ERR_CUDA;
@@ -418,7 +470,8 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
       cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess)
     return SSD_ERR_CUDA;
   // a7: counts and the next cache length
-  e = launch_counts(x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted, y->accepted_count,
+  e = launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted,
+                    y->accepted_count,
                     y->accepted_prefix, y->next_cache_len, stream);
   return from_cuda(e);
 }

@@ -9,7 +9,10 @@
 //
 // Counts (Sec. 3.3 and Sec. 4 "SSD Configuration", one verification round):
 // the drafts up to and including the first rejected one are committed, the
-// rejected one carrying its resampled token.
+// rejected one carrying its resampled token.  With r verify-and-correct
+// rounds (Sec. 3.3) the rounds before the last commit nothing and the last
+// commits the whole corrected block; the staged schedule (App. multi-row)
+// commits the frontier's first row after its base rounds.
 #include "kernels.cuh"
 
 namespace ssd {
@@ -44,7 +47,8 @@ __global__ void frontier_kernel(ssd_grid g, const int32_t* __restrict__ cache_le
 }
 
 // One warp per sequence: accepted count, leading accepted run, next length.
-__global__ void counts_kernel(int32_t B, int32_t D_max, const int32_t* __restrict__ cache_len,
+__global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_max,
+                              const int32_t* __restrict__ cache_len,
                               const int32_t* __restrict__ n_drafts,
                               const uint8_t* __restrict__ accepted,
                               int32_t* __restrict__ accepted_count,
@@ -75,7 +79,31 @@ __global__ void counts_kernel(int32_t B, int32_t D_max, const int32_t* __restric
   if (lane == 0) {
     accepted_count[b] = count;
     accepted_prefix[b] = prefix;
-    next_cache_len[b] = cache_len[b] + (n > 0 ? min(prefix + 1, n) : 0);
+    int32_t advance = n > 0 ? min(prefix + 1, n) : 0;  // SSD_COMMIT_PREFIX
+    if (commit == SSD_COMMIT_NONE) {
+      advance = 0;
+    } else if (commit == SSD_COMMIT_BLOCK) {
+      advance = n;
+    } else if (commit == SSD_COMMIT_FIRST_ROW) {
+      const int32_t n_c = cache_len[b] - g.prefix_len;
+      advance = min(n, g.grid_w - n_c % g.grid_w);  // the frontier's first row
+    }
+    next_cache_len[b] = cache_len[b] + advance;
+  }
+}
+
+// Staged schedule: the trailing row (slots W .. 2W-1) becomes the frontier of
+// the incremental rounds (slots 0 .. W-1), with its tokens and references.
+__global__ void stage_shift_kernel(int32_t B, int32_t D_max, int32_t W, int32_t* __restrict__ tok,
+                                   const float** __restrict__ ref_rows) {
+  const int32_t b = blockIdx.x;
+  for (int32_t j = threadIdx.x; j < W; j += blockDim.x) {
+    const int64_t dst = (int64_t)b * D_max + j, src = dst + W;
+    // destination slots 0 .. W-1 and source slots W .. 2W-1 do not overlap
+    const int32_t t = tok[src];
+    const float* p = ref_rows != nullptr ? ref_rows[src] : nullptr;
+    tok[dst] = t;
+    if (ref_rows != nullptr) ref_rows[dst] = p;
   }
 }
 
@@ -87,13 +115,22 @@ cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_l
   return cudaGetLastError();
 }
 
-cudaError_t launch_counts(int32_t B, int32_t D_max, const int32_t* cache_len,
-                          const int32_t* n_drafts, const uint8_t* accepted, int32_t* accepted_count,
+cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
+                          const int32_t* cache_len, const int32_t* n_drafts,
+                          const uint8_t* accepted, int32_t* accepted_count,
                           int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
   const int warps = 4;
   counts_kernel<<<(B + warps - 1) / warps, warps * 32, 0, stream>>>(
-      B, D_max, cache_len, n_drafts, accepted, accepted_count, accepted_prefix, next_cache_len);
+      g, commit, B, D_max, cache_len, n_drafts, accepted, accepted_count, accepted_prefix,
+      next_cache_len);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
+                               const float** ref_rows, cudaStream_t stream) {
+  if (B == 0 || W == 0) return cudaSuccess;
+  stage_shift_kernel<<<B, 128, 0, stream>>>(B, D_max, W, tok, ref_rows);
   return cudaGetLastError();
 }
 

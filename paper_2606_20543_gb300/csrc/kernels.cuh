@@ -10,9 +10,14 @@ namespace ssd {
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
                             cudaStream_t stream);
-cudaError_t launch_counts(int32_t B, int32_t D_max, const int32_t* cache_len,
-                          const int32_t* n_drafts, const uint8_t* accepted, int32_t* accepted_count,
+cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
+                          const int32_t* cache_len, const int32_t* n_drafts,
+                          const uint8_t* accepted, int32_t* accepted_count,
                           int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream);
+// Staged schedule: slot j of every sequence takes slot W + j (j < W) of the
+// per-row tokens and reference pointers.
+cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
+                               const float** ref_rows, cudaStream_t stream);
 
 // ---- accept.cu
 struct AcceptArgs {
@@ -31,6 +36,9 @@ struct AcceptArgs {
   const int32_t* n_drafts;   // nullable: row r valid iff r % D_max < n_drafts[r / D_max]
   int32_t D_max;
   int32_t strategy;          // ssd_strategy: (C) accept-reject, (A) greedy, (B) sampling
+  const float** ref_rows;    // nullable: reference (draft) row of row r; a rejected row's entry
+                             // is set to its target row (the next round's reference)
+  int32_t ref_init;          // round 1: references are the draft rows; every entry is written
 };
 bool accept_supported(int32_t V);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);

@@ -10,8 +10,8 @@ from __future__ import annotations
 import numpy as np
 import torch
 
-from . import (STRATEGIES, Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid, ssd_verify_step,
-               ssd_verify_step_workspace)
+from . import (COMMITS, STRATEGIES, Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid,
+               row_addresses, ssd_stage_shift, ssd_verify_step, ssd_verify_step_workspace)
 
 
 def _dev(shape, dtype, device):
@@ -161,3 +161,85 @@ class VerifyStep:
         r["o"] = self.o.float().cpu().numpy()
         r["lse"] = self.lse.cpu().numpy()
         return r
+
+
+class VerifyRounds:
+    """r verify-and-correct rounds (Sec. 3.3) and the staged b / i schedule
+    (App. multi-row drafting) over the buffers of a VerifyStep.
+
+    Every round is one ssd_verify_step with the round's target logits, the
+    rows' current reference pointers (ref_rows, redirected by the library to
+    the round's target row when a row is not accepted) and the tokens the
+    previous round left (two device buffers used in turn).  The caller keeps
+    each round's target logits alive and unchanged until the block is
+    committed: later rounds read them as references."""
+
+    def __init__(self, step: "VerifyStep"):
+        if step.hidden:
+            raise ValueError("verify-and-correct rounds need the logits path")
+        self.s = step
+        self.ref_rows = row_addresses(step.drf)
+        self.tok = [_dev((step.rows,), torch.int32, step.device) for _ in range(2)]
+        self.cur = 0
+
+    def reset(self):
+        """Back to round 1 (which rewrites every reference itself)."""
+        self.cur = 0
+
+    @property
+    def tokens(self):
+        """Device tensor of the tokens after the last round run."""
+        return self.tok[self.cur]
+
+    def run(self, tgt_rounds, commit_last="block", uniforms_rounds=None, seed=0, offset0=0,
+            first_round=True, stream=None) -> None:
+        """One round per entry of tgt_rounds (device float32 [rows, V]): the
+        rounds before the last commit nothing, the last commits per
+        commit_last (an ssd_commit name).  Round 1 (first_round) verifies the
+        draft tokens (argmax of the draft rows); later rounds the tokens the
+        previous round left.  Each round draws its uniforms from Philox at
+        offset offset0 + round, or from uniforms_rounds[round] if given."""
+        s = self.s
+        a, y = s.args, s.out
+        n = len(tgt_rounds)
+        for rho, tgt in enumerate(tgt_rounds):
+            a.tgt_logits = tgt.data_ptr()
+            a.ld = s.V
+            a.ref_rows = self.ref_rows.data_ptr()
+            a.ref_init = 1 if (first_round and rho == 0) else 0
+            a.draft_tok = None if (first_round and rho == 0) else self.tok[self.cur].data_ptr()
+            y.out_tok = self.tok[1 - self.cur].data_ptr()
+            a.commit = COMMITS["none"] if rho < n - 1 else COMMITS[commit_last]
+            s.rng.seed, s.rng.offset = seed, offset0 + rho
+            s.rng.uniforms = None if uniforms_rounds is None else uniforms_rounds[rho].data_ptr()
+            a.rng = s.rng
+            ssd_verify_step(a, y, s.workspace, s.ws_bytes, stream)
+            self.cur = 1 - self.cur
+        # leave the VerifyStep as it was for plain steps
+        a.tgt_logits, a.ref_rows, a.commit, a.ref_init = s.tgt.data_ptr(), None, COMMITS["prefix"], 0
+        a.draft_tok = None if s.draft_tok is None else s.draft_tok.data_ptr()
+        y.out_tok = s.out_tok.data_ptr()
+
+    def run_staged(self, b, i, tgt_rounds, uniforms_rounds=None, seed=0, offset0=0,
+                   stream=None) -> None:
+        """The staged schedule of the paper's two-row vertical stage: from a
+        row start the frontier with k_v = 1 is the two drafted rows (the
+        current row and the row below).  b base rounds on both, commit the
+        first row, move the trailing row to the front (ssd_stage_shift),
+        advance the cache, then i rounds on the trailing row alone (k_v = 0)
+        and commit it."""
+        s = self.s
+        if s.g.k_v != 1:
+            raise ValueError("the staged schedule verifies a two-row frontier (k_v = 1)")
+        W = s.g.grid_w
+        u = uniforms_rounds
+        self.run(tgt_rounds[:b], "first_row", None if u is None else u[:b], seed, offset0,
+                 True, stream)
+        ssd_stage_shift(s.B, s.D_max, W, self.tok[self.cur], self.ref_rows, stream)
+        s.cache_len.copy_(s.next_cache_len)
+        s.args.grid.k_v = 0
+        try:
+            self.run(tgt_rounds[b:], "block", None if u is None else u[b:], seed, offset0 + b,
+                     False, stream)
+        finally:
+            s.args.grid.k_v = 1

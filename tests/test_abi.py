@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 2
+    assert lib.ssd_abi_version() == 3
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 
@@ -82,6 +82,13 @@ def test_host_side_validation(lib):
     for bad in (-1, 3, 99):
         assert so.ssd_accept_strategy(bad, 0, 4096, None, None, 4096, None, 1.0, ctypes.byref(r),
                                       fake, fake, None, None, fake, None) == 1
+    # rounds: the reference pointers are required; shift: 2W must fit D_max
+    assert so.ssd_accept_round(0, 4, 4096, fake, 4096, None, None, 1.0, ctypes.byref(r), fake,
+                               fake, None, None, fake, None) == 1
+    assert so.ssd_accept_round(5, 4, 4096, fake, 4096, fake, None, 1.0, ctypes.byref(r), fake,
+                               fake, None, None, fake, None) == 1
+    assert so.ssd_stage_shift(2, 48, 25, fake, None, None) == 2
+    assert so.ssd_stage_shift(0, 48, 24, None, None, None) == 0
     for good in (lib.STRATEGY_ACCEPT_REJECT, lib.STRATEGY_GREEDY, lib.STRATEGY_SAMPLE):
         assert so.ssd_accept_strategy(good, 0, 4096, None, None, 4096, None, 1.0,
                                       ctypes.byref(r), fake, fake, None, None, fake, None) == 0

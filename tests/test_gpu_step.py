@@ -87,9 +87,9 @@ def test_step_config3_shape(ssd):
 
 
 def test_frontier_all_cache_lengths(ssd):
-    """Every cache length of a 24x24 grid, k_v = 1 and 2, bit-exact."""
+    """Every cache length of a 24x24 grid, k_v = 0, 1 and 2, bit-exact."""
     dev = "cuda"
-    for k_v in (1, 2):
+    for k_v in (0, 1, 2):
         H = W = 24
         P = 120
         cls = np.arange(P, P + H * W + 1, dtype=np.int32)

@@ -24,7 +24,7 @@ def test_golden_spatial_offsets():
         assert b - a == off
 
 
-@pytest.mark.parametrize("H,W,k_v", [(16, 16, 1), (24, 24, 1), (8, 5, 2), (3, 7, 3)])
+@pytest.mark.parametrize("H,W,k_v", [(16, 16, 1), (24, 24, 1), (8, 5, 2), (3, 7, 3), (6, 9, 0)])
 def test_frontier_sizes(H, W, k_v):
     P = 11
     for n_c in range(H * W + 1):
