@@ -29,3 +29,14 @@ def step_counts(accepted_row: np.ndarray, n_d: int, cache_len: int):
         prefix += 1
     advance = min(prefix + 1, n_d) if n_d > 0 else 0
     return count, prefix, cache_len + advance
+
+
+def step_counts_bonus(accepted_row: np.ndarray, n_d: int, cache_len: int, bonus_exists: bool):
+    """The horizontal stage (Sec. 4 "SSD Configuration": k_h drafts, one
+    verification round): the prefix rule, and when every draft is accepted
+    the token at the next position, drawn from the backbone's distribution
+    there, is committed as well (reading: only if that position exists)."""
+    count, prefix, nxt = step_counts(accepted_row, n_d, cache_len)
+    if n_d > 0 and prefix == n_d and bonus_exists:
+        nxt = cache_len + n_d + 1
+    return count, prefix, nxt

@@ -21,23 +21,29 @@ from __future__ import annotations
 import numpy as np
 
 
-def frontier(grid_h: int, grid_w: int, prefix_len: int, cache_len: int, k_v: int = 1):
+def frontier(grid_h: int, grid_w: int, prefix_len: int, cache_len: int, k_v: int = 1,
+             k_h: int = 0):
     """Return the drafted grid coordinates [(y, x), ...] in raster order.
 
     Horizontal part: (y0, x) for x = c .. W-1, where the first uncommitted
-    token sits at (y0, c).  Vertical part: rows y0+1 .. y0+k_v, all columns.
-    Rows at or beyond grid_h do not exist and are dropped.
+    token sits at (y0, c); with k_h > 0 only the first k_h of them (Sec. 3.3:
+    k_h horizontal heads draft offsets +1 .. +k_h along the row).  Vertical
+    part: rows y0+1 .. y0+k_v, all columns -- reading: only when the
+    horizontal part completes the row, so the frontier stays contiguous in
+    raster order.  Rows at or beyond grid_h do not exist and are dropped.
     """
     n_c = cache_len - prefix_len  # committed image tokens
     if n_c < 0 or n_c > grid_h * grid_w:
         raise ValueError("cache_len outside [prefix_len, prefix_len + H*W]")
     y0, c = divmod(n_c, grid_w)
     coords = []
+    h = grid_w - c if k_h <= 0 else min(k_h, grid_w - c)
     if y0 < grid_h:
-        coords += [(y0, x) for x in range(c, grid_w)]          # horizontal heads
-    for dy in range(1, k_v + 1):                                # vertical heads
-        if y0 + dy < grid_h:
-            coords += [(y0 + dy, x) for x in range(grid_w)]
+        coords += [(y0, x) for x in range(c, c + h)]            # horizontal heads
+    if c + h == grid_w:
+        for dy in range(1, k_v + 1):                            # vertical heads
+            if y0 + dy < grid_h:
+                coords += [(y0 + dy, x) for x in range(grid_w)]
     return coords
 
 

@@ -16,24 +16,30 @@ from . import counts as cnt
 from . import frontier as fr
 
 
-def sequence_frontier(grid_h, grid_w, prefix_len, cache_len, k_v=1):
-    coords = fr.frontier(grid_h, grid_w, prefix_len, int(cache_len), k_v)
+def sequence_frontier(grid_h, grid_w, prefix_len, cache_len, k_v=1, k_h=0):
+    coords = fr.frontier(grid_h, grid_w, prefix_len, int(cache_len), k_v, k_h)
     return coords, fr.grid_index(coords, grid_w)
 
 
 def accept_step(grid_h, grid_w, prefix_len, k_v, cache_len, D_max, tgt_logits, drf_logits,
-                uniforms, draft_tok=None, temperature=1.0, strategy="accept_reject"):
+                uniforms, draft_tok=None, temperature=1.0, strategy="accept_reject", k_h=0,
+                bonus=False):
     """Frontier + acceptance + counts for a batch (no attention).
 
     Row b*D_max + j of the logit / uniform arrays belongs to draft j of
     sequence b.  Returns per-sequence lists and the per-row decision dict
-    restricted to valid rows (key "rows" lists their global row indices)."""
+    restricted to valid rows (key "rows" lists their global row indices).
+    With bonus (the horizontal stage), row b*D_max + n_d holds the backbone's
+    logits at the position after the last draft: its token is the argmax
+    under strategy (A) and otherwise the inverse-CDF draw from p with u_res
+    (keys bonus_tok, bonus_tie, bonus_row); when every draft is accepted and
+    that position exists it is committed too."""
     B = len(cache_len)
     n_d = np.zeros(B, np.int64)
     pos = np.full((B, D_max), -1, np.int64)
     rows = []
     for b in range(B):
-        coords, g = sequence_frontier(grid_h, grid_w, prefix_len, cache_len[b], k_v)
+        coords, g = sequence_frontier(grid_h, grid_w, prefix_len, cache_len[b], k_v, k_h)
         n_d[b] = len(coords)
         pos[b, :len(g)] = g
         rows += [b * D_max + j for j in range(len(g))]
@@ -50,15 +56,31 @@ def accept_step(grid_h, grid_w, prefix_len, k_v, cache_len, D_max, tgt_logits, d
     counts = np.zeros(B, np.int64)
     prefix = np.zeros(B, np.int64)
     nxt = np.zeros(B, np.int64)
+    bonus_tok = np.full(B, -1, np.int64)
+    bonus_tie = np.zeros(B, bool)
+    bonus_row = np.full(B, -1, np.int64)
     for b in range(B):
-        counts[b], prefix[b], nxt[b] = cnt.step_counts(
-            accepted_full[b * D_max:(b + 1) * D_max], int(n_d[b]), int(cache_len[b]))
+        exists = False
+        if bonus and 0 < n_d[b] < D_max:
+            row = b * D_max + int(n_d[b])
+            bonus_row[b] = row
+            lp = np.asarray(tgt_logits, dtype=np.float64)[row]
+            if strategy == "greedy":
+                bonus_tok[b] = int(np.argmax(lp))
+            else:
+                p, _ = acc.softmax(lp[None], temperature)
+                bonus_tok[b], margin = acc.inverse_cdf(p[0], float(np.asarray(uniforms)[row, 1]))
+                bonus_tie[b] = margin < acc.NEAR_TIE_CDF
+            exists = int(cache_len[b]) - prefix_len + int(n_d[b]) < grid_h * grid_w
+        counts[b], prefix[b], nxt[b] = cnt.step_counts_bonus(
+            accepted_full[b * D_max:(b + 1) * D_max], int(n_d[b]), int(cache_len[b]), exists)
     return dict(n_drafts=n_d, draft_pos=pos, accepted_count=counts, accepted_prefix=prefix,
-                next_cache_len=nxt, decisions=dec)
+                next_cache_len=nxt, decisions=dec, bonus_tok=bonus_tok, bonus_tie=bonus_tie,
+                bonus_row=bonus_row)
 
 
 def attention_step(grid_h, grid_w, prefix_len, row_stride, k_v, cache_len, q, k, v, Hq, Hkv,
-                   scale=None, seqs=None):
+                   scale=None, seqs=None, k_h=0):
     """Frontier attention for the sequences in ``seqs`` (default: all).
 
     q [B, D_max, Hq, d], k/v [B, Hkv, L_max, d] (float).  Returns
@@ -66,7 +88,7 @@ def attention_step(grid_h, grid_w, prefix_len, row_stride, k_v, cache_len, q, k,
     B = len(cache_len)
     res = {}
     for b in (range(B) if seqs is None else seqs):
-        coords, _ = sequence_frontier(grid_h, grid_w, prefix_len, cache_len[b], k_v)
+        coords, _ = sequence_frontier(grid_h, grid_w, prefix_len, cache_len[b], k_v, k_h)
         n = len(coords)
         res[b] = att.verify_attention(q[b, :n], k[b], v[b], int(cache_len[b]), coords,
                                       prefix_len, row_stride, Hq, Hkv, scale)
