@@ -51,6 +51,9 @@ def parse():
     ap.add_argument("--staged", default=None, metavar="B,I",
                     help="staged two-row schedule: B base rounds, commit the first row, I rounds "
                          "on the trailing row (configs 1-2, whose frontiers start at a row)")
+    ap.add_argument("--horizontal", type=int, default=0, metavar="K_H",
+                    help="the horizontal stage: K_H drafts along the row per step (k_v = 0), one "
+                         "round, prefix acceptance plus the bonus token (logits workloads)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="approximate budget of the CPU-oracle sample")
@@ -65,6 +68,8 @@ def parse():
             ap.error("--staged B,I with B, I >= 1 on config 1 or 2")
     if a.rounds < 1:
         ap.error("--rounds >= 1")
+    if a.horizontal and (a.config in (4, 5) or a.rounds != 1 or a.staged or a.horizontal < 0):
+        ap.error("--horizontal K_H > 0 on a logits workload (configs 1-3), one round")
     return a
 
 
@@ -96,10 +101,11 @@ WORKLOAD_NAMES = {
 }
 
 
-def algorithmic_bytes(c, n_drafts):
+def algorithmic_bytes(c, n_drafts, bonus=False):
     """Bytes one verification pass must move: every K/V row of the visible
     keys once per KV head, Q and O of each draft, both logit rows of each
-    draft, and the per-row / per-sequence outputs."""
+    draft (and of each sequence's bonus row in the horizontal stage), and the
+    per-row / per-sequence outputs."""
     n = np.asarray(n_drafts, dtype=np.int64)
     L = c.cache_len.astype(np.int64) + n
     kv = int((L * c.Hkv * c.d * 2 * 2).sum())
@@ -109,7 +115,8 @@ def algorithmic_bytes(c, n_drafts):
         # both lm_head weights once, both hidden-state rows of every draft once
         acc = 2 * c.hidden * c.V * 2 + int(n.sum()) * (2 * c.hidden * 2 + 4 + 1 + 4)
     else:
-        acc = int(n.sum()) * (2 * c.V * 4 + 4 + 1 + 4)
+        rows = int(n.sum()) + (int((n > 0).sum()) if bonus else 0)
+        acc = rows * (2 * c.V * 4 + 4 + 1 + 4)
     return attn, acc
 
 
@@ -446,7 +453,9 @@ def main():
     steps_obj = []
     for cs in cases:
         st = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max,
-                        c.V, k_v=c.k_v, device=dev, hidden=c.hidden, strategy=a.strategy)
+                        c.V, k_v=0 if a.horizontal else c.k_v, device=dev, hidden=c.hidden,
+                        strategy=a.strategy, k_h=a.horizontal,
+                        commit="prefix_bonus" if a.horizontal else "prefix")
         st.upload(cache_len=cs.cache_len, q=cs.q, k=cs.k, v=cs.v, tgt_logits=cs.tgt_logits,
                   drf_logits=cs.drf_logits, h_tgt=cs.h_tgt, h_drf=cs.h_drf, w_tgt=cs.w_tgt,
                   w_drf=cs.w_drf)
@@ -494,7 +503,7 @@ def main():
     torch.cuda.synchronize(dev)
     n_drafts = full_drafts if a.staged else [st.n_drafts.cpu().numpy() for st in steps_obj]
     launches = ssd.ssd_verify_step_launches(steps_obj[0].args) * R + (1 if a.staged else 0)
-    attn_bytes, acc_bytes = algorithmic_bytes(c, n_drafts[0])
+    attn_bytes, acc_bytes = algorithmic_bytes(c, n_drafts[0], bonus=a.horizontal > 0)
 
     # The K timed passes are captured once as a CUDA graph (each pass with its
     # own Philox offset) and replayed: one eager ctypes call per pass would
@@ -660,6 +669,8 @@ def main():
         "config": {"workload": WORKLOAD_NAMES[a.config], "strategy": a.strategy,
                    "verify_rounds": (f"staged b={a.staged[0]}, i={a.staged[1]}" if a.staged
                                      else a.rounds),
+                   "stage": (f"horizontal: k_h={a.horizontal} drafts, prefix + bonus token"
+                             if a.horizontal else "frontier: rest of the row + k_v rows"),
                    "sequences_per_step": c.B,
                    "drafts_per_step": int(n_drafts[0].sum()), "vocab": c.V,
                    "heads": f"{c.Hq}/{c.Hkv}x{c.d}",

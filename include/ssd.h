@@ -68,6 +68,9 @@ typedef struct {
   int32_t prefix_len; /* text-prefix tokens before grid token (0, 0)      */
   int32_t k_v;        /* rows drafted below the current row, >= 0 (0: the
                          rest of the current row only)                  */
+  int32_t k_h;        /* horizontal drafts per step, >= 0 (0: the rest of
+                         the row); with k_h < W - c the frontier is the
+                         next k_h positions and no rows below            */
 } ssd_grid;
 
 /* Per-draft uniforms (u_acc, u_res).  If `uniforms` (dev, float32
@@ -82,7 +85,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 3
+#define SSD_ABI_VERSION 4
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -94,6 +97,8 @@ const char* ssd_status_string(ssd_status s);
  * For each sequence b, with n_c = cache_len[b] - prefix_len committed grid
  * tokens and the first uncommitted token at (y0, c) = (n_c / W, n_c % W):
  *     n_drafts[b] = (W - c) + k_v * W, clipped at the grid's last row,
+ *     or, with k_h > 0, h = min(k_h, W - c) horizontal drafts plus the k_v
+ *     rows only when h = W - c (Sec. 3.3: k_h horizontal heads);
  *     draft_pos[b][j] = n_c + j (grid index y * W + x), j < n_drafts[b];
  * padding slots get -1.
  *   cache_len  dev int32 [B]
@@ -248,12 +253,22 @@ ssd_status ssd_accept_round(int32_t strategy, int32_t rows, int32_t V, const flo
  *   SSD_COMMIT_NONE       a round before the last: nothing is committed
  *   SSD_COMMIT_BLOCK      the last of r rounds: the whole corrected block
  *   SSD_COMMIT_FIRST_ROW  the staged schedule's first commit: the frontier's
- *                         first row, W - (cache_len - prefix_len) % W drafts */
+ *                         first row, W - (cache_len - prefix_len) % W drafts
+ *   SSD_COMMIT_PREFIX_BONUS the horizontal stage (Sec. 4: one round): the
+ *                         prefix rule, and when every draft is accepted the
+ *                         bonus token as well, so next = cache + n_d + 1 if
+ *                         the position after the last draft exists.  Row
+ *                         b * D_max + n_d of the target logits then holds the
+ *                         backbone's logits at that position (n_d < D_max);
+ *                         its out_tok is the bonus token: under (A) the argmax
+ *                         of p, otherwise a draw from p with the row's u_res;
+ *                         its accepted flag is 1.  Logits path only. */
 typedef enum {
   SSD_COMMIT_PREFIX = 0,
   SSD_COMMIT_NONE = 1,
   SSD_COMMIT_BLOCK = 2,
-  SSD_COMMIT_FIRST_ROW = 3
+  SSD_COMMIT_FIRST_ROW = 3,
+  SSD_COMMIT_PREFIX_BONUS = 4
 } ssd_commit;
 
 /* Staged schedule (App. multi-row, "commit the first row, then refine the

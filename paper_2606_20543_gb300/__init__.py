@@ -29,9 +29,9 @@ EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_
 
 
 STRATEGY_ACCEPT_REJECT, STRATEGY_GREEDY, STRATEGY_SAMPLE = 0, 1, 2
-COMMIT_PREFIX, COMMIT_NONE, COMMIT_BLOCK, COMMIT_FIRST_ROW = 0, 1, 2, 3
+COMMIT_PREFIX, COMMIT_NONE, COMMIT_BLOCK, COMMIT_FIRST_ROW, COMMIT_PREFIX_BONUS = 0, 1, 2, 3, 4
 COMMITS = {"prefix": COMMIT_PREFIX, "none": COMMIT_NONE, "block": COMMIT_BLOCK,
-           "first_row": COMMIT_FIRST_ROW}
+           "first_row": COMMIT_FIRST_ROW, "prefix_bonus": COMMIT_PREFIX_BONUS}
 STRATEGIES = {"accept_reject": STRATEGY_ACCEPT_REJECT, "greedy": STRATEGY_GREEDY,
               "sample": STRATEGY_SAMPLE}
 
@@ -45,7 +45,7 @@ class SsdError(RuntimeError):
 class Grid(ctypes.Structure):
     _fields_ = [("grid_h", ctypes.c_int32), ("grid_w", ctypes.c_int32),
                 ("row_stride", ctypes.c_int32), ("prefix_len", ctypes.c_int32),
-                ("k_v", ctypes.c_int32)]
+                ("k_v", ctypes.c_int32), ("k_h", ctypes.c_int32)]
 
 
 class Rng(ctypes.Structure):
@@ -144,8 +144,8 @@ def _check(fn: str, code: int) -> None:
 
 
 def grid(grid_h: int, grid_w: int, prefix_len: int, row_stride: Optional[int] = None,
-         k_v: int = 1) -> Grid:
-    return Grid(grid_h, grid_w, grid_w if row_stride is None else row_stride, prefix_len, k_v)
+         k_v: int = 1, k_h: int = 0) -> Grid:
+    return Grid(grid_h, grid_w, grid_w if row_stride is None else row_stride, prefix_len, k_v, k_h)
 
 
 def rng(seed: int = 0, offset: int = 0, uniforms=None) -> Rng:

@@ -131,12 +131,15 @@ struct Shared {
   float xp_t, xq_t;  // logits at a caller-given draft token (pass A)
 };
 
-// Rows that stream: frontier rows with an in-range (or absent) draft token.
-// Producer and consumers walk the same rows and skip the same ones.
+// Rows that stream: frontier rows with an in-range (or absent) draft token
+// (kind 0) and, in the horizontal stage, the bonus row after a sequence's
+// last draft (kind 3).  Producer and consumers walk the same rows and skip
+// the same ones.
 __device__ __forceinline__ int row_kind(const AcceptArgs& a, int64_t r) {
   if (a.n_drafts != nullptr) {
     const int32_t b = (int32_t)(r / a.D_max), j = (int32_t)(r % a.D_max);
-    if (j >= a.n_drafts[b]) return 1;  // padding slot
+    const int32_t n = a.n_drafts[b];
+    if (j >= n) return (a.bonus && j == n && n > 0) ? 3 : 1;  // bonus row / padding slot
   }
   if (a.draft_tok != nullptr) {
     const int32_t t = a.draft_tok[r];
@@ -286,7 +289,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     if (lane == 0) {
       uint32_t g = 0;  // chunks issued by this CTA
       for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
-        if (row_kind(a, r) != 0) continue;
+        const int kind = row_kind(a, r);
+        if (kind == 1 || kind == 2) continue;
         // the row's reference is read once: the consumers may redirect it for
         // the next round while this row's second pass is still being issued
         const float* drow =
@@ -318,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   uint32_t g = 0;  // chunks consumed
   for (int64_t r = blockIdx.x; r < a.rows; r += gridDim.x) {
     const int kind = row_kind(a, r);
-    if (kind != 0) {
+    if (kind == 1 || kind == 2) {
       if (tid == 0) {
         a.out_tok[r] = -1;
         a.accepted[r] = 0;
@@ -329,7 +333,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       }
       continue;
     }
-    const int32_t given_t = a.draft_tok != nullptr ? a.draft_tok[r] : -1;
+    // the bonus row draws from p alone (its draft logits are not read for it)
+    const bool is_bonus = kind == 3;
+    const bool row_p = sample || is_bonus;  // second pass over the weights of p
+    const int32_t given_t = (a.draft_tok != nullptr && !is_bonus) ? a.draft_tok[r] : -1;
     const float* drow =
         (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
     // the row's uniforms, drawn while its first chunk is still in flight
@@ -451,7 +458,29 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         merge(Mq, Sq, om, os, c);
         if (take) { t = oi; xp_t = op; }
       }
-      if (lane == 0) {
+      if (lane == 0 && is_bonus) {
+        // the position after the last draft (horizontal stage): no draft
+        // token; (A) the argmax of p, otherwise a draw from p
+        const float lsp = log2f(Sp);
+        if (greedy) {
+          float pm = sh.red_pm[0];
+          int32_t pi = sh.red_pi[0];
+          for (int w = 1; w < kCWarps; ++w)
+            if (better_arg(sh.red_pm[w], sh.red_pi[w], pm, pi)) { pm = sh.red_pm[w]; pi = sh.red_pi[w]; }
+          a.out_tok[r] = pi;
+        }
+        sh.accept = greedy ? 1 : 0;
+        sh.t_hat = -1;
+        sh.u_res = u.y;
+        sh.Cp = Mp * c + lsp;
+        sh.Cq = 0.f;
+        a.accepted[r] = 1;
+        if (a.ratio) a.ratio[r] = 0.f;
+        if (a.lse) {
+          a.lse[2 * r] = Mp / a.temperature + lsp * kLn2;
+          a.lse[2 * r + 1] = 0.f;
+        }
+      } else if (lane == 0) {
         float xq_t = Mq;
         if (given_t >= 0) {
           t = given_t;
@@ -520,8 +549,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         const int32_t cv = min(kChunk, a.V - ch * kChunk) >> 2;
         const int32_t i0 = warp * 64 + lane, i1 = i0 + 32;
         float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
-        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], cc, ncp, ncq, sample);
-        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], cc, ncp, ncq, sample);
+        if (i0 < cv) w0 = weights4(xp4[i0], xq4[i0], cc, ncp, ncq, row_p);
+        if (i1 < cv) w1 = weights4(xp4[i1], xq4[i1], cc, ncp, ncq, row_p);
         const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
         if (lane == 0) block_mass[ch * kBlocksPerChunk + warp] = m;
       }
@@ -535,8 +564,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     if (warp == 0) {
       float tb;
       int32_t bk = find_block(block_mass, nblocks, sh.u_res, &tb, lane);
-      bool from_p = sample;
-      if (bk < 0 && !sample) {
+      bool from_p = row_p;
+      if (bk < 0 && !row_p) {
         // zero residual mass: the same draw from p (block masses of p itself)
         from_p = true;
         for (int32_t b0 = 0; b0 < nblocks; ++b0) {
@@ -553,14 +582,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       if (bk < 0) {
         if (lane == 0) {  // no positive mass at all (non-finite logits)
           a.out_tok[r] = -1;
-          if (sample) a.accepted[r] = 0;
+          if (sample || is_bonus) a.accepted[r] = 0;
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
       } else {
         const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
         if (lane == 0) {
           a.out_tok[r] = pick;
-          if (sample) {
+          if (sample && !is_bonus) {
             a.accepted[r] = pick == sh.t_hat ? 1 : 0;
             if (a.ref_rows != nullptr && pick != sh.t_hat) a.ref_rows[r] = a.tgt + r * a.ld;
             else if (a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = drow;

@@ -42,7 +42,8 @@ cudaError_t side_stream(SideStream** out) {
 
 ssd_status check_grid(const ssd_grid* g) {
   if (g == nullptr) return SSD_ERR_INVALID_ARG;
-  if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 0) return SSD_ERR_SHAPE;
+  if (g->grid_h <= 0 || g->grid_w <= 0 || g->prefix_len < 0 || g->k_v < 0 || g->k_h < 0)
+    return SSD_ERR_SHAPE;
   if (g->row_stride != g->grid_w && g->row_stride != g->grid_w + 1) return SSD_ERR_SHAPE;
   if ((int64_t)g->grid_h * g->row_stride + g->prefix_len > INT32_MAX / 2) return SSD_ERR_SHAPE;
   return SSD_OK;
@@ -235,6 +236,7 @@ ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const 
   a.strategy = strategy;
   a.ref_rows = nullptr;
   a.ref_init = 0;
+  a.bonus = 0;
   return from_cuda(launch_accept(a, (cudaStream_t)stream));
 }
 
@@ -271,6 +273,7 @@ ssd_status ssd_accept_round(int32_t strategy, int32_t rows, int32_t V, const flo
   a.strategy = strategy;
   a.ref_rows = ref_rows;
   a.ref_init = 0;
+  a.bonus = 0;
   return from_cuda(launch_accept(a, (cudaStream_t)stream));
 }
 
@@ -369,14 +372,15 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   s = check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
   if (s != SSD_OK) return s;
   if (!strategy_ok(x->strategy)) return SSD_ERR_INVALID_ARG;
-  if (x->commit < SSD_COMMIT_PREFIX || x->commit > SSD_COMMIT_FIRST_ROW) return SSD_ERR_INVALID_ARG;
+  if (x->commit < SSD_COMMIT_PREFIX || x->commit > SSD_COMMIT_PREFIX_BONUS) return SSD_ERR_INVALID_ARG;
   if (x->ref_init != 0 && (x->ref_rows == nullptr || x->drf_logits == nullptr))
     return SSD_ERR_INVALID_ARG;
   const bool fused = (x->tgt_logits == nullptr);
   if (fused) {
     if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
       return SSD_ERR_INVALID_ARG;
-    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT || x->ref_rows != nullptr)
+    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT || x->ref_rows != nullptr ||
+        x->commit == SSD_COMMIT_PREFIX_BONUS)
       return SSD_ERR_UNSUPPORTED;
     s = lmhead_check(rows, x->V, x->hidden);
     if (s != SSD_OK) return s;
@@ -462,6 +466,7 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     c.strategy = x->strategy;
     c.ref_rows = x->ref_rows;
     c.ref_init = x->ref_init;
+    c.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
     e = launch_accept(c, side->stream);
   }
   if (e != cudaSuccess) return SSD_ERR_CUDA;

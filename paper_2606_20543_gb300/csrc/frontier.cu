@@ -5,14 +5,18 @@
 // the vertical heads draft the k_v rows below it in one column-parallel step.
 // With n_c committed grid tokens and the first uncommitted one at
 // (y0, c) = (n_c / W, n_c % W), the frontier is the next
-// (W - c) + k_v * W raster positions, clipped at the last grid row.
+// (W - c) + k_v * W raster positions, clipped at the last grid row.  With
+// k_h > 0 the horizontal part is the next min(k_h, W - c) positions (k_h
+// horizontal heads), and the vertical rows follow only when it completes
+// the row, so the frontier stays one contiguous raster run.
 //
 // Counts (Sec. 3.3 and Sec. 4 "SSD Configuration", one verification round):
 // the drafts up to and including the first rejected one are committed, the
 // rejected one carrying its resampled token.  With r verify-and-correct
 // rounds (Sec. 3.3) the rounds before the last commit nothing and the last
 // commits the whole corrected block; the staged schedule (App. multi-row)
-// commits the frontier's first row after its base rounds.
+// commits the frontier's first row after its base rounds.  The horizontal
+// stage (Sec. 4, one round) adds the bonus token when every draft is kept.
 #include "kernels.cuh"
 
 namespace ssd {
@@ -21,8 +25,9 @@ __device__ __forceinline__ int32_t frontier_size(const ssd_grid& g, int32_t n_c)
   const int32_t y0 = n_c / g.grid_w;
   const int32_t c = n_c - y0 * g.grid_w;
   if (y0 >= g.grid_h) return 0;
-  const int32_t rows_below = min(g.k_v, g.grid_h - 1 - y0);
-  return (g.grid_w - c) + rows_below * g.grid_w;
+  const int32_t h = g.k_h > 0 ? min(g.k_h, g.grid_w - c) : g.grid_w - c;
+  const int32_t rows_below = (c + h == g.grid_w) ? min(g.k_v, g.grid_h - 1 - y0) : 0;
+  return h + rows_below * g.grid_w;
 }
 
 // One block per sequence.  Writes n_drafts[b] and draft_pos[b][0..D_max).
@@ -87,6 +92,11 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
     } else if (commit == SSD_COMMIT_FIRST_ROW) {
       const int32_t n_c = cache_len[b] - g.prefix_len;
       advance = min(n, g.grid_w - n_c % g.grid_w);  // the frontier's first row
+    } else if (commit == SSD_COMMIT_PREFIX_BONUS) {
+      // horizontal stage: every draft accepted -> the bonus token as well, if
+      // the position after the last draft exists (and has a row slot)
+      const int32_t n_c = cache_len[b] - g.prefix_len;
+      if (n > 0 && prefix == n && n < D_max && n_c + n < g.grid_h * g.grid_w) advance = n + 1;
     }
     next_cache_len[b] = cache_len[b] + advance;
   }

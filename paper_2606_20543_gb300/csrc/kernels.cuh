@@ -39,6 +39,7 @@ struct AcceptArgs {
   const float** ref_rows;    // nullable: reference (draft) row of row r; a rejected row's entry
                              // is set to its target row (the next round's reference)
   int32_t ref_init;          // round 1: references are the draft rows; every entry is written
+  int32_t bonus;             // horizontal stage: row j == n_drafts[b] draws the bonus token
 };
 bool accept_supported(int32_t V);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);

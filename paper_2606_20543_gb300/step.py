@@ -36,13 +36,14 @@ class VerifyStep:
 
     def __init__(self, grid_h, grid_w, prefix_len, B, Hq, Hkv, d, D_max, L_max, V,
                  hidden=0, k_v=1, row_stride=None, device="cuda", scale=0.0, temperature=1.0,
-                 strategy="accept_reject"):
-        self.g: Grid = make_grid(grid_h, grid_w, prefix_len, row_stride, k_v)
+                 strategy="accept_reject", k_h=0, commit="prefix"):
+        self.g: Grid = make_grid(grid_h, grid_w, prefix_len, row_stride, k_v, k_h)
         self.B, self.Hq, self.Hkv, self.d = B, Hq, Hkv, d
         self.D_max, self.L_max, self.V, self.hidden = D_max, L_max, V, hidden
         self.device = device
         self.scale, self.temperature = scale, temperature
         self.strategy = STRATEGIES.get(strategy, strategy)
+        self.commit = COMMITS.get(commit, commit)
         rows = B * D_max
         self.rows = rows
         dv = device
@@ -104,6 +105,7 @@ class VerifyStep:
         a.temperature = self.temperature
         a.rng = self.rng
         a.strategy = self.strategy
+        a.commit = self.commit
         return a
 
     def _out(self) -> VerifyOut:
@@ -216,7 +218,7 @@ class VerifyRounds:
             ssd_verify_step(a, y, s.workspace, s.ws_bytes, stream)
             self.cur = 1 - self.cur
         # leave the VerifyStep as it was for plain steps
-        a.tgt_logits, a.ref_rows, a.commit, a.ref_init = s.tgt.data_ptr(), None, COMMITS["prefix"], 0
+        a.tgt_logits, a.ref_rows, a.commit, a.ref_init = s.tgt.data_ptr(), None, s.commit, 0
         a.draft_tok = None if s.draft_tok is None else s.draft_tok.data_ptr()
         y.out_tok = s.out_tok.data_ptr()
 

@@ -157,3 +157,65 @@ def test_step_strategies(ssd, strategy):
         s.run()
         torch.cuda.synchronize()
         check_step(c, s.results(), strategy=strategy)
+
+
+def test_frontier_with_k_h_all_cache_lengths(ssd):
+    """The horizontal stage's frontier (k_h = 5) for every cache length of a
+    24x24 grid, with and without rows below, bit-exact."""
+    dev = "cuda"
+    H = W = 24
+    P = 120
+    cls = np.arange(P, P + H * W + 1, dtype=np.int32)
+    for k_v in (0, 1):
+        D_max = (k_v + 1) * W
+        g = ssd.grid(H, W, P, k_v=k_v, k_h=5)
+        nd = torch.empty(len(cls), dtype=torch.int32, device=dev)
+        pos = torch.empty((len(cls), D_max), dtype=torch.int32, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        ssd.ssd_frontier(g, len(cls), torch.from_numpy(cls).to(dev), D_max, nd, pos, st)
+        torch.cuda.synchronize()
+        nd, pos = nd.cpu().numpy(), pos.cpu().numpy()
+        assert st.item() == 0
+        for i, cl in enumerate(cls):
+            gidx = ofr.grid_index(ofr.frontier(H, W, P, int(cl), k_v, 5), W)
+            assert nd[i] == len(gidx)
+            assert np.array_equal(pos[i, :nd[i]], gidx)
+
+
+@pytest.mark.parametrize("strategy", ["accept_reject", "greedy", "sample"])
+def test_horizontal_stage_with_bonus(ssd, strategy):
+    """k_h = 5 drafts, one round, prefix acceptance plus the bonus token."""
+    from paper_2606_20543_gb300.step import VerifyStep
+    H = W = 16
+    P = 32
+    cls = [P + 3, P + W * 2, P + W * 5 + 13, P + H * W - 2, P + W * 7 + 11]
+    c = synth.make_case("horizontal", grid_h=H, grid_w=W, prefix_len=P, cache_len=cls, Hq=4,
+                        Hkv=4, d=64, V=4096, seed=61, k_v=0)
+    for same in (False, True):  # True: p = q, every draft accepted, the bonus committed
+        tgt = c.drf_logits.copy() if same else c.tgt_logits
+        s = VerifyStep(H, W, P, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V, k_v=0, k_h=5,
+                       strategy=strategy, commit="prefix_bonus")
+        s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=tgt,
+                 drf_logits=c.drf_logits, uniforms=c.uniforms)
+        s.run()
+        torch.cuda.synchronize()
+        res = s.results()
+        assert res["status"][0] == 0
+        ref = ostep.accept_step(H, W, P, 0, c.cache_len, c.D_max, tgt, c.drf_logits, c.uniforms,
+                                strategy=strategy, k_h=5, bonus=True)
+        assert np.array_equal(res["n_drafts"], ref["n_drafts"])
+        assert np.array_equal(res["n_drafts"], [5, 5, 3, 2, 5])
+        rows = ref["decisions"]["rows"]
+        ties = compare_decisions(ref["decisions"], res["out_tok"][rows], res["accepted"][rows],
+                                 what=f"horizontal {strategy}")
+        for b in range(c.B):
+            if ref["bonus_row"][b] >= 0 and not ref["bonus_tie"][b]:
+                assert res["out_tok"][ref["bonus_row"][b]] == ref["bonus_tok"][b]
+                assert res["accepted"][ref["bonus_row"][b]] == 1
+        if ties == 0:
+            assert np.array_equal(res["next_cache_len"], ref["next_cache_len"])
+        if same and strategy != "sample":
+            # every draft accepted: the bonus is committed except at the grid's end
+            assert np.array_equal(res["next_cache_len"][[0, 1, 2, 4]],
+                                  c.cache_len[[0, 1, 2, 4]] + res["n_drafts"][[0, 1, 2, 4]] + 1)
+            assert res["next_cache_len"][3] == c.cache_len[3] + 2
