@@ -173,7 +173,7 @@ class ClockSampler:
 # is the one that was captured: (source file, sha256 prefix, bytes, rows the
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
-    ("accept", 2): ("accept.cu", "5f684b006ac1eeb1", 152679680 + 3432448, 1128),
+    ("accept", 2): ("accept.cu", "5ccfccad7a2ff8ae", 152415232 + 3548416, 1128),
     ("attention", 3): ("attention_tc.cu", "6ca0a2b87c88eb22", 53335296 + 427520, None),
     ("lmhead_accept", 4): ("lmhead.cu", "a5b28d8ac7ea5800", 269327616 + 3034112, None),
 }

@@ -267,6 +267,7 @@ __device__ __forceinline__ int32_t walk_block(const float4* tp, const float4* dp
   return last_pos;  // rounding ran past the end of the block
 }
 
+template <int STRATEGY>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs a) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   float* ring = reinterpret_cast<float*>(smem_raw);                  // [kStages][2][kChunk]
@@ -312,8 +313,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   }
 
   // ---------------------------------------------------------- consumer warps
-  const bool greedy = a.strategy == SSD_STRATEGY_GREEDY;
-  const bool sample = a.strategy == SSD_STRATEGY_SAMPLE;
+  constexpr bool greedy = STRATEGY == SSD_STRATEGY_GREEDY;
+  constexpr bool sample = STRATEGY == SSD_STRATEGY_SAMPLE;
   const float c = kLog2e / a.temperature;
   const float2 cc = make_float2(c, c);
   const int32_t nv = a.V >> 2;
@@ -337,8 +338,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     const bool is_bonus = kind == 3;
     const bool row_p = sample || is_bonus;  // second pass over the weights of p
     const int32_t given_t = (a.draft_tok != nullptr && !is_bonus) ? a.draft_tok[r] : -1;
-    const float* drow =
-        (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
     // the row's uniforms, drawn while its first chunk is still in flight
     const float2 u = (tid == 0) ? row_uniforms(a.rng, r) : make_float2(0.f, 0.f);
 
@@ -406,6 +405,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       if (lane == 0) mbar_arrive(&sh.empty[s]);
     }
     float sp = sp2.x + sp2.y, sq = sq2.x + sq2.y;
+    // the row's reference (draft) row: read here, before the barrier after
+    // which this row's decision may redirect it for the next round
+    const float* drow =
+        (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
     if (greedy) {  // first argmax of p over the CTA (warp tree, then the warps in order)
       float pm = mp;
 #pragma unroll
@@ -610,12 +613,19 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
   const int32_t nch = (a.V + kChunk - 1) / kChunk;
   const size_t smem = (size_t)kStages * 2 * kChunk * sizeof(float) +
                       (size_t)nch * kBlocksPerChunk * sizeof(float);
-  cudaError_t e = cudaFuncSetAttribute(accept_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
   const int64_t grid = std::min<int64_t>(a.rows, (int64_t)kCtasPerSm * device_sm_count());
-  accept_kernel<<<(unsigned)grid, kThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  auto launch = [&](auto kernel) {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    kernel<<<(unsigned)grid, kThreads, smem, stream>>>(a);
+    return cudaGetLastError();
+  };
+  switch (a.strategy) {
+    case SSD_STRATEGY_GREEDY: return launch(accept_kernel<SSD_STRATEGY_GREEDY>);
+    case SSD_STRATEGY_SAMPLE: return launch(accept_kernel<SSD_STRATEGY_SAMPLE>);
+    default: return launch(accept_kernel<SSD_STRATEGY_ACCEPT_REJECT>);
+  }
 }
 
 }  // namespace ssd

@@ -26,6 +26,9 @@ namespace ssd {
 
 namespace {
 
+#ifndef SSD_ATTN_CTAS_PER_SM
+#define SSD_ATTN_CTAS_PER_SM 2  // KV splits are added until the grid has this many CTAs per SM
+#endif
 constexpr int KT = 64;        // keys per tile
 constexpr int kStages = 3;
 constexpr int kMaxWarps = 8;  // 128 query rows per CTA
@@ -428,7 +431,7 @@ Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max, int
   p.nwarps = min(kMaxWarps, (rows + 15) / 16);
   p.mtiles = (rows + p.nwarps * 16 - 1) / (p.nwarps * 16);
   const int64_t base = (int64_t)B * Hkv * p.mtiles;
-  const int32_t target = 2 * device_sm_count();
+  const int32_t target = SSD_ATTN_CTAS_PER_SM * device_sm_count();
   const int32_t max_splits = max(1, (L_max + 2 * KT - 1) / (2 * KT));  // >= 2 tiles per split
   int32_t splits = (int32_t)((target + base - 1) / base);
   splits = max(1, min(splits, max_splits));
