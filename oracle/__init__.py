@@ -24,6 +24,8 @@ Modules and the passage each follows:
              (horizontal prefix acceptance): accepted counts and the next
              cache length of a single-round replay.
   lmhead     Sec. 3.3, Eq. 2's GenHead: logits = hidden @ W, then accept.
+  predictor  Sec. 3.3 "Draft Prediction in Latent Space", Eq. 2: the spatial
+             draft predictor f_phi and the draft token argmax GenHead(RMSNorm).
   rounds     Sec. 3.3 (r verify-and-correct rounds: rejected positions take
              the residual sample and this round's p as their reference; the
              commit after the last round) and App. multi-row drafting (the
