@@ -54,6 +54,9 @@ def parse():
     ap.add_argument("--horizontal", type=int, default=0, metavar="K_H",
                     help="the horizontal stage: K_H drafts along the row per step (k_v = 0), one "
                          "round, prefix acceptance plus the bonus token (logits workloads)")
+    ap.add_argument("--predictor", type=int, default=0, metavar="ROWS",
+                    help="time the spatial draft predictor (Eq. 2) and its draft tokens for ROWS "
+                         "positions at the paper's head size (d = 4096, m = 2d, V = 16384)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="approximate budget of the CPU-oracle sample")
@@ -399,6 +402,139 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
     return 0
 
 
+# ------------------------------------------------------- the draft predictor
+PRED_D, PRED_M, PRED_V = 4096, 8192, 16384
+
+
+def predictor_inputs(rows, seed=80):
+    """Synthetic predictor weights at the paper's head size (bf16 bits) and a
+    row of source states; trained heads do not exist here."""
+    rng = np.random.default_rng(seed)
+    d, m, V = PRED_D, PRED_M, PRED_V
+    b = lambda shape, std: synth.bf16_normal(rng, shape, std)  # noqa: E731
+    w = dict(z=b((rows, 2 * d), 1.0), w0=b((d, 2 * d), 1 / np.sqrt(2 * d)),
+             w1=b((m, d), 1 / np.sqrt(d)), w3=b((m, d), 1 / np.sqrt(d)),
+             w2=b((d, m), 1 / np.sqrt(m)), wh=b((d, V), 1 / np.sqrt(d)))
+    g1 = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    g2 = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    return w, g1, g2
+
+
+def predictor_oracle_rate(rows, budget_s):
+    """Draft predictor calls/s of the oracle (float64 NumPy) on the host cores."""
+    from oracle import predictor as pr
+    w, g1, g2 = predictor_inputs(rows)
+    f = {k: synth.bf16_bits_to_f32(v).astype(np.float64) for k, v in w.items()}
+    t0 = time.perf_counter()
+    done = 0
+    while True:
+        pr.predict(f["z"], f["w0"], f["w1"], f["w2"], f["w3"], g1, g2, f["wh"], 1e-5)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
+    return {"value": done / (time.perf_counter() - t0), "unit": "draft predictor calls/s",
+            "cores": int(threads) if threads else (os.cpu_count() or 1), "kind": "oracle",
+            "sample": f"{done} whole calls ({rows} rows, d = {PRED_D}, m = {PRED_M}, "
+                      f"V = {PRED_V}) in float64 NumPy"}
+
+
+def run_predictor(a, world, rank, dev, torch, ssd):
+    rows, d, m, V = a.predictor, PRED_D, PRED_M, PRED_V
+    w, g1, g2 = predictor_inputs(rows)
+
+    def bf(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(
+            torch.bfloat16).to(dev)
+    t = {k: bf(v) for k, v in w.items()}
+    dg1, dg2 = torch.from_numpy(g1).to(dev), torch.from_numpy(g2).to(dev)
+    tok = torch.empty(rows, dtype=torch.int32, device=dev)
+    hid = torch.empty((rows, d), dtype=torch.float32, device=dev)
+    wsb = ssd.ssd_draft_predict_workspace(rows, d, m, V)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def call(z):
+        ssd.ssd_draft_predict(rows, d, m, V, z, t["w0"], t["w1"], t["w3"], t["w2"], dg1, dg2,
+                              t["wh"], 1e-5, tok, hid, ws, wsb, st)
+
+    for _ in range(max(a.warmup, 3)):  # the first call creates the cuBLAS handle
+        call(t["z"])
+    torch.cuda.synchronize(dev)
+    chunk = min(a.steps, 200)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for _ in range(chunk):
+            call(t["z"])
+    g.replay()
+    torch.cuda.synchronize(dev)
+    reps = -(-a.steps // chunk)
+    clocks = ClockSampler(dev.index or 0)
+    clocks.start()
+    time.sleep(0.2)
+    if world > 1:
+        torch.distributed.barrier()
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    calls = reps * chunk
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    # end to end: the source states in from pinned host memory, the tokens back
+    z_host = torch.from_numpy(np.ascontiguousarray(w["z"]).view(np.int16)).view(
+        torch.bfloat16).pin_memory()
+    tok_host = torch.empty(rows, dtype=torch.int32).pin_memory()
+    ne = 20
+    torch.cuda.synchronize(dev)
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2.record(stream)
+    for _ in range(ne):
+        t["z"].copy_(z_host, non_blocking=True)
+        call(t["z"])
+        tok_host.copy_(tok, non_blocking=True)
+    e3.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e2.elapsed_time(e3) / ne
+    wbytes = 2 * (d * 2 * d + 3 * m * d + d * V)  # the four projections and GenHead, bf16
+    abytes = rows * (2 * d * 2 + d * 4 * 3 + 2 * m * 4 * 2 + V * 4 * 2 + 4)
+    hbm_peak, peak_kind = measured_peaks()
+    achieved = (wbytes + abytes) / (ms / calls / 1000.0) / 1e9
+    if rank != 0:
+        return 0
+    cpu = None if a.no_cpu_baseline else predictor_oracle_rate(rows, min(a.cpu_seconds, 20.0))
+    line = {
+        "metric": "draft predictor calls/s (Eq. 2 + argmax GenHead, one row)",
+        "value": world * calls / (ms / 1000.0), "unit": "draft predictor calls/s",
+        "n_gpus": world, "steps": calls, "warmup": max(a.warmup, 3), "ms_per_step": ms / calls,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16 GEMM inputs / f32 accumulation", "data": "synthetic weights",
+        "config": {"workload": f"spatial draft predictor: {rows} positions, d = {d}, m = {m}, "
+                               f"V = {V} (134.2 M parameters per head + GenHead)",
+                   "l2": f"every call streams {wbytes / 1e6:.0f} MB of weights > 129 MB L2",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "kernel": "draft_predict", "achieved": achieved,
+                     "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                     "traffic": None, "peak_kind": peak_kind},
+        "clocks": clk,
+        "e2e": {"value": world * 1000.0 / e2e_ms, "unit": "draft predictor calls/s",
+                "h2d_bytes_per_step": rows * 2 * d * 2, "d2h_bytes_per_step": rows * 4},
+        "gpu_launches": 4 * calls,  # rmsnorm x 2, swiglu, argmax (+ 5 cuBLAS GEMMs)
+        "device_status": int(st.item()), "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    return 0
+
+
 # -------------------------------------------------------------------- main
 def main():
     a = parse()
@@ -406,6 +542,18 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
 
+    if a.impl == "reference" and a.predictor:
+        if rank != 0:
+            return 0
+        cpu = predictor_oracle_rate(a.predictor, a.cpu_seconds)
+        print(json.dumps({"impl": "reference", "metric": "draft predictor calls/s (Eq. 2 + argmax "
+                          "GenHead, one row)", "value": cpu["value"], "unit": cpu["unit"],
+                          "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
+                          "ms_per_step": 1000.0 / cpu["value"], "higher_is_better": True,
+                          "cpu_baseline": cpu, "e2e": {"value": cpu["value"], "unit": cpu["unit"],
+                                                      "h2d_bytes_per_step": 0,
+                                                      "d2h_bytes_per_step": 0}}))
+        return 0
     if a.impl == "reference":
         if rank != 0:
             return 0
@@ -437,6 +585,12 @@ def main():
     build.build()
     import paper_2606_20543_gb300 as ssd
     from paper_2606_20543_gb300.step import VerifyStep
+
+    if a.predictor:
+        rc = run_predictor(a, world, rank, dev, torch, ssd)
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return rc
 
     if a.config == 5:
         cpu = None

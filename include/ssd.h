@@ -85,7 +85,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 4
+#define SSD_ABI_VERSION 5
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -374,6 +374,35 @@ size_t ssd_verify_step_workspace(const ssd_verify_args* args);
 int32_t ssd_verify_step_launches(const ssd_verify_args* args);
 ssd_status ssd_verify_step(const ssd_verify_args* args, const ssd_verify_out* out,
                            void* workspace, size_t workspace_bytes, ssd_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * The spatial draft predictor (Sec. 3.3 "Draft Prediction in Latent Space",
+ * Eq. 2) and its draft tokens, for `rows` positions at once (one grid row of
+ * W columns for a vertical head, or the k_h horizontal offsets):
+ *     h_hat = W0 z + W2 (silu(W1 a) * W3 a),  a = RMSNorm(W0 z; gamma1),
+ *     out_tok = argmax_v (RMSNorm(h_hat; gamma2) W_head)_v  (lowest index on
+ *     ties), RMSNorm(x; g) = x / sqrt(mean(x^2) + eps) * g.
+ *   z        dev bf16 [rows][2d]: [h ; e], the hidden state and the token
+ *            embedding of each source position
+ *   w0       dev bf16 [d][2d]; w1, w3 dev bf16 [m][d]; w2 dev bf16 [d][m]
+ *            ([out][in], as a linear layer stores them)
+ *   gamma1, gamma2  dev float32 [d]; w_head dev bf16 [d][V] (GenHead)
+ *   out_tok  dev int32 [rows] (out); out_hidden dev float32 [rows][d] or NULL
+ *            (out: h_hat, the predicted pre-norm hidden state)
+ *   workspace dev, >= ssd_draft_predict_workspace(rows, d, m, V) bytes
+ * Every GEMM input is bf16 with fp32 accumulation (the four projections run
+ * as cuBLAS GEMMs: the library creates one cuBLAS handle per device and host
+ * thread on the first call, which must be outside any stream capture; the
+ * handle works in `workspace` and allocates nothing afterwards).
+ * Supported: rows >= 1, d, m multiples of 8, V a multiple of 4, every
+ * pointer 16-byte aligned.  A cuBLAS failure returns SSD_ERR_CUDA.
+ * ------------------------------------------------------------------------- */
+size_t ssd_draft_predict_workspace(int32_t rows, int32_t d, int32_t m, int32_t V);
+ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, const void* z,
+                             const void* w0, const void* w1, const void* w3, const void* w2,
+                             const float* gamma1, const float* gamma2, const void* w_head,
+                             float eps, int32_t* out_tok, float* out_hidden, void* workspace,
+                             size_t workspace_bytes, int32_t* status, ssd_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -23,7 +23,8 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
 
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
             "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
-            "ssd_accept_round", "ssd_stage_shift",
+            "ssd_accept_round", "ssd_stage_shift", "ssd_draft_predict_workspace",
+            "ssd_draft_predict",
             "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
             "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
 
@@ -107,6 +108,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_accept_round": (I32, [I32, I32, I32, P, I64, P, P, F, ctypes.POINTER(Rng), P, P, P, P,
                                    P, P]),
         "ssd_stage_shift": (I32, [I32, I32, I32, P, P, P]),
+        "ssd_draft_predict_workspace": (SZ, [I32, I32, I32, I32]),
+        "ssd_draft_predict": (I32, [I32, I32, I32, I32, P, P, P, P, P, P, P, P, F, P, P, P, SZ,
+                                    P, P]),
         "ssd_lmhead_accept_workspace": (SZ, [I32, I32]),
         "ssd_lmhead_accept": (I32, [I32, I32, I32, P, P, P, P, P, F, ctypes.POINTER(Rng), P, P, P,
                                     P, P, SZ, P, P]),
@@ -225,6 +229,19 @@ def ssd_accept_round(strategy, rows, V, tgt_logits, ld, ref_rows, tok, temperatu
 def ssd_stage_shift(B, D_max, W, tok, ref_rows, stream=None) -> None:
     _check("ssd_stage_shift", load().ssd_stage_shift(B, D_max, W, _ptr(tok), _ptr(ref_rows),
                                                      _stream(stream)))
+
+
+def ssd_draft_predict_workspace(rows, d, m, V) -> int:
+    return load().ssd_draft_predict_workspace(rows, d, m, V)
+
+
+def ssd_draft_predict(rows, d, m, V, z, w0, w1, w3, w2, gamma1, gamma2, w_head, eps, out_tok,
+                      out_hidden, workspace, workspace_bytes, status, stream=None) -> None:
+    """Eq. 2's spatial draft predictor and argmax GenHead(RMSNorm(h_hat))."""
+    _check("ssd_draft_predict", load().ssd_draft_predict(
+        rows, d, m, V, _ptr(z), _ptr(w0), _ptr(w1), _ptr(w3), _ptr(w2), _ptr(gamma1),
+        _ptr(gamma2), _ptr(w_head), eps, _ptr(out_tok), _ptr(out_hidden), _ptr(workspace),
+        workspace_bytes, _ptr(status), _stream(stream)))
 
 
 def row_addresses(t, ld=None):

@@ -277,6 +277,49 @@ ssd_status ssd_accept_round(int32_t strategy, int32_t rows, int32_t V, const flo
   return from_cuda(launch_accept(a, (cudaStream_t)stream));
 }
 
+size_t ssd_draft_predict_workspace(int32_t rows, int32_t d, int32_t m, int32_t V) {
+  if (rows <= 0 || d <= 0 || m <= 0 || V <= 0) return 0;
+  return predictor_workspace(rows, d, m, V, true);
+}
+
+ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, const void* z,
+                             const void* w0, const void* w1, const void* w3, const void* w2,
+                             const float* gamma1, const float* gamma2, const void* w_head,
+                             float eps, int32_t* out_tok, float* out_hidden, void* workspace,
+                             size_t workspace_bytes, int32_t* status, ssd_stream_t stream) {
+  if (rows <= 0 || d <= 0 || m <= 0 || V <= 0) return SSD_ERR_SHAPE;
+  if (d % 8 != 0 || m % 8 != 0 || V % 4 != 0) return SSD_ERR_SHAPE;
+  if ((int64_t)rows * 2 * m >= (int64_t)1 << 31 || (int64_t)rows * V >= (int64_t)1 << 31)
+    return SSD_ERR_UNSUPPORTED;
+  const void* ptrs[] = {z, w0, w1, w3, w2, gamma1, gamma2, w_head, out_tok, status};
+  for (const void* q : ptrs)
+    if (q == nullptr) return SSD_ERR_INVALID_ARG;
+  for (const void* q : {z, w0, w1, w3, w2, w_head, (const void*)gamma1, (const void*)gamma2,
+                        (const void*)out_hidden})
+    if (q != nullptr && !aligned16(q)) return SSD_ERR_INVALID_ARG;
+  if (!(eps >= 0.f) || !isfinite(eps)) return SSD_ERR_INVALID_ARG;
+  if (workspace == nullptr ||
+      workspace_bytes < predictor_workspace(rows, d, m, V, out_hidden == nullptr))
+    return SSD_ERR_WORKSPACE;
+  PredictorArgs p;
+  p.rows = rows;
+  p.d = d;
+  p.m = m;
+  p.V = V;
+  p.z = z;
+  p.w0 = w0;
+  p.w1 = w1;
+  p.w3 = w3;
+  p.w2 = w2;
+  p.gamma1 = gamma1;
+  p.gamma2 = gamma2;
+  p.w_head = w_head;
+  p.eps = eps;
+  p.out_tok = out_tok;
+  p.out_hidden = out_hidden;
+  return from_cuda(launch_predictor(p, workspace, workspace_bytes, (cudaStream_t)stream));
+}
+
 ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
                            const float** ref_rows, ssd_stream_t stream) {
   if (B < 0 || D_max <= 0 || W < 0 || 2 * (int64_t)W > D_max) return SSD_ERR_SHAPE;

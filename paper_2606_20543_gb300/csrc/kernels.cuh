@@ -100,6 +100,25 @@ size_t lmhead_workspace(int32_t rows, int32_t V);
 ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K);
 cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
 
+// ---- predictor.cu (Eq. 2: the spatial draft predictor and its draft tokens)
+struct PredictorArgs {
+  int32_t rows, d, m, V;
+  const void* z;        // bf16 [rows][2d] = [h ; e]
+  const void* w0;       // bf16 [d][2d]
+  const void* w1;       // bf16 [m][d]
+  const void* w3;       // bf16 [m][d]
+  const void* w2;       // bf16 [d][m]
+  const float* gamma1;  // [d]
+  const float* gamma2;  // [d]
+  const void* w_head;   // bf16 [d][V]
+  float eps;
+  int32_t* out_tok;     // [rows]
+  float* out_hidden;    // fp32 [rows][d] or nullptr (then in the workspace)
+};
+size_t predictor_workspace(int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden);
+cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
+                             cudaStream_t stream);
+
 int device_sm_count();
 
 }  // namespace ssd

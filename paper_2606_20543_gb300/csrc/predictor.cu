@@ -1,0 +1,197 @@
+// predictor.cu — the spatial draft predictor f_phi (Sec. 3.3 "Draft
+// Prediction in Latent Space", Eq. 2) and the draft tokens it yields:
+//
+//   h_hat = W0 z + SwiGLU(RMSNorm(W0 z)),  z = [h ; e],
+//   SwiGLU(x) = W2 (silu(W1 x) * W3 x),    t_hat = argmax GenHead(RMSNorm(h_hat)).
+//
+// Design (GB300): for one row of W grid columns the predictor is a chain of
+// skinny products (rows <= a few hundred) that stream 268 MB of weights per
+// head plus the 4096 x V GenHead, so it is bound by HBM, not by the tensor
+// cores.  The four projections are plain GEMMs and run as cuBLAS bf16 GEMMs
+// (fp32 accumulation on the tensor cores, fp32 or bf16 outputs); everything
+// between them is a kernel of this file, and the data flow needs no copies:
+//   H  = W0 z                 GEMM into the caller's hidden-state buffer (fp32)
+//   At = RMSNorm(H) * gamma1  rmsnorm_kernel (bf16, the next GEMM's input)
+//   UV = At [W1 | W3]^T       two GEMMs into the halves of one fp32 buffer
+//   G  = silu(U) * V          swiglu_kernel (bf16)
+//   H  = H + G W2^T           GEMM with beta = 1: the residual in place
+//   Hn = RMSNorm(H) * gamma2  rmsnorm_kernel (bf16)
+//   L  = Hn W_head            GEMM (fp32 logits, rows x V)
+//   t  = argmax L             argmax_kernel (lowest index on ties)
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "kernels.cuh"
+
+namespace ssd {
+
+namespace {
+
+constexpr int kNormThreads = 256;
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_sum(v);
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+  if (warp == 0) {
+    t = lane < (int)(blockDim.x >> 5) ? red[lane] : 0.f;
+    t = warp_sum(t);
+    if (lane == 0) red[0] = t;
+  }
+  __syncthreads();
+  return red[0];
+}
+
+// One CTA per row: y = x / sqrt(mean(x^2) + eps) * gamma, rounded to bf16.
+__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __restrict__ x,
+                                                               const float* __restrict__ gamma,
+                                                               float eps, int32_t d,
+                                                               __nv_bfloat16* __restrict__ y) {
+  __shared__ float red[32];
+  const float* xr = x + (int64_t)blockIdx.x * d;
+  __nv_bfloat16* yr = y + (int64_t)blockIdx.x * d;
+  float ss = 0.f;
+  for (int32_t i = threadIdx.x; i < d; i += blockDim.x) ss += xr[i] * xr[i];
+  const float inv = 1.0f / sqrtf(block_sum(ss, red) / (float)d + eps);
+  for (int32_t i = threadIdx.x; i < d; i += blockDim.x)
+    yr[i] = __float2bfloat16_rn(xr[i] * inv * gamma[i]);
+}
+
+// g = silu(u) * v over rows x m; uv holds [u | v] per row (2m floats).
+__global__ void swiglu_kernel(const float* __restrict__ uv, int32_t rows, int32_t m,
+                              __nv_bfloat16* __restrict__ g) {
+  const int64_t n = (int64_t)rows * m;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / m, j = i - r * m;
+    const float u = uv[r * 2 * m + j], v = uv[r * 2 * m + m + j];
+    g[i] = __float2bfloat16_rn(u / (1.0f + expf(-u)) * v);
+  }
+}
+
+// One CTA per row: the first index of the maximum logit.
+__global__ void __launch_bounds__(kNormThreads) argmax_kernel(const float* __restrict__ logits,
+                                                              int32_t V,
+                                                              int32_t* __restrict__ out_tok) {
+  __shared__ float sv[32];
+  __shared__ int32_t si[32];
+  const float* lr = logits + (int64_t)blockIdx.x * V;
+  float bv = -INFINITY;
+  int32_t bi = 0x7fffffff;
+  for (int32_t i = threadIdx.x; i < V; i += blockDim.x) {
+    const float v = lr[i];
+    if (v > bv) { bv = v; bi = i; }  // ascending i per thread: first max kept
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const int32_t oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+  }
+  if (lane == 0) { sv[warp] = bv; si[warp] = bi; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+      if (sv[w] > bv || (sv[w] == bv && si[w] < bi)) { bv = sv[w]; bi = si[w]; }
+    out_tok[blockIdx.x] = bi;
+  }
+}
+
+// cuBLAS handle per device and host thread, created on first use.
+constexpr int kMaxDevices = 64;
+cublasStatus_t blas_handle(cublasHandle_t* out) {
+  thread_local cublasHandle_t handles[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return CUBLAS_STATUS_NOT_INITIALIZED;
+  if (handles[dev] == nullptr) {
+    const cublasStatus_t s = cublasCreate(&handles[dev]);
+    if (s != CUBLAS_STATUS_SUCCESS) return s;
+  }
+  *out = handles[dev];
+  return CUBLAS_STATUS_SUCCESS;
+}
+
+// Row-major Y[rows][N] (+)= X[rows][K] W[N][K]^T  (torch Linear layout), as the
+// column-major product Y^T = W X^T.
+cublasStatus_t linear(cublasHandle_t h, int32_t rows, int32_t N, int32_t K, const void* X,
+                      const void* W, float beta, void* Y, cudaDataType ytype) {
+  const float alpha = 1.0f;
+  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, N, rows, K, &alpha, W, CUDA_R_16BF, K, X,
+                      CUDA_R_16BF, K, &beta, Y, ytype, N, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+}
+
+size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+constexpr size_t kBlasWorkspace = (size_t)32 << 20;
+
+}  // namespace
+
+size_t predictor_workspace(int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden) {
+  size_t b = al256(kBlasWorkspace);
+  b += al256((size_t)rows * d * 2);       // At / Hn (bf16)
+  b += al256((size_t)rows * 2 * m * 4);   // [U | V] (fp32)
+  b += al256((size_t)rows * m * 2);       // G (bf16)
+  b += al256((size_t)rows * V * 4);       // logits (fp32)
+  if (own_hidden) b += al256((size_t)rows * d * 4);
+  return b;
+}
+
+cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
+                             cudaStream_t stream) {
+  if (ws_bytes < predictor_workspace(p.rows, p.d, p.m, p.V, p.out_hidden == nullptr))
+    return cudaErrorInvalidValue;
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  void* blas_ws = w;
+  w += al256(kBlasWorkspace);
+  __nv_bfloat16* nrm = reinterpret_cast<__nv_bfloat16*>(w);
+  w += al256((size_t)p.rows * p.d * 2);
+  float* uv = reinterpret_cast<float*>(w);
+  w += al256((size_t)p.rows * 2 * p.m * 4);
+  __nv_bfloat16* g = reinterpret_cast<__nv_bfloat16*>(w);
+  w += al256((size_t)p.rows * p.m * 2);
+  float* logits = reinterpret_cast<float*>(w);
+  w += al256((size_t)p.rows * p.V * 4);
+  float* H = p.out_hidden;
+  if (H == nullptr) H = reinterpret_cast<float*>(w);
+
+  cublasHandle_t h;
+  if (blas_handle(&h) != CUBLAS_STATUS_SUCCESS) return cudaErrorUnknown;
+  if (cublasSetStream(h, stream) != CUBLAS_STATUS_SUCCESS ||
+      cublasSetWorkspace(h, blas_ws, kBlasWorkspace) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  const int32_t rows = p.rows, d = p.d, m = p.m;
+  const int swg_blocks = (int)std::min<int64_t>(((int64_t)rows * m + 255) / 256,
+                                                4 * (int64_t)device_sm_count());
+  // H = W0 z
+  if (linear(h, rows, d, 2 * d, p.z, p.w0, 0.f, H, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma1, p.eps, d, nrm);
+  // [U | V] = At [W1 | W3]^T: two GEMMs into the halves of each row of uv
+  const float alpha = 1.0f, zero = 0.0f;
+  if (cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, rows, d, &alpha, p.w1, CUDA_R_16BF, d, nrm,
+                   CUDA_R_16BF, d, &zero, uv, CUDA_R_32F, 2 * m, CUBLAS_COMPUTE_32F,
+                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS ||
+      cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, rows, d, &alpha, p.w3, CUDA_R_16BF, d, nrm,
+                   CUDA_R_16BF, d, &zero, uv + m, CUDA_R_32F, 2 * m, CUBLAS_COMPUTE_32F,
+                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  swiglu_kernel<<<swg_blocks, 256, 0, stream>>>(uv, rows, m, g);
+  // H = H + G W2^T
+  if (linear(h, rows, d, m, g, p.w2, 1.f, H, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma2, p.eps, d, nrm);
+  // logits[rows][V] = Hn[rows][d] W_head[d][V]: column-major L^T = W_head^T' Hn^T
+  if (cublasGemmEx(h, CUBLAS_OP_N, CUBLAS_OP_N, p.V, rows, d, &alpha, p.w_head, CUDA_R_16BF, p.V,
+                   nrm, CUDA_R_16BF, d, &zero, logits, CUDA_R_32F, p.V, CUBLAS_COMPUTE_32F,
+                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  argmax_kernel<<<rows, kNormThreads, 0, stream>>>(logits, p.V, p.out_tok);
+  return cudaGetLastError();
+}
+
+}  // namespace ssd

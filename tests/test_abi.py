@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 4
+    assert lib.ssd_abi_version() == 5
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 
@@ -89,6 +89,20 @@ def test_host_side_validation(lib):
                                fake, None, None, fake, None) == 1
     assert so.ssd_stage_shift(2, 48, 25, fake, None, None) == 2
     assert so.ssd_stage_shift(0, 48, 24, None, None, None) == 0
+    # draft predictor: shapes, null pointers, workspace
+    W = so.ssd_draft_predict
+    assert W(0, 64, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, 1 << 30, fake, None) == 2
+    assert W(4, 60, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, 1 << 30, fake, None) == 2
+    assert W(4, 64, 128, 256, None, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, 1 << 30, fake, None) == 1
+    assert W(4, 64, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, -1.0, fake, None,
+             fake, 1 << 30, fake, None) == 1
+    need = so.ssd_draft_predict_workspace(4, 64, 128, 256)
+    assert need > 0
+    assert W(4, 64, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, need - 1, fake, None) == 7
     for good in (lib.STRATEGY_ACCEPT_REJECT, lib.STRATEGY_GREEDY, lib.STRATEGY_SAMPLE):
         assert so.ssd_accept_strategy(good, 0, 4096, None, None, 4096, None, 1.0,
                                       ctypes.byref(r), fake, fake, None, None, fake, None) == 0

@@ -1,0 +1,88 @@
+"""GPU parity of the spatial draft predictor (Eq. 2) and its draft tokens
+against the oracle: tokens bit-exact except argmax near-ties (top-2 logit gap
+below 1e-3 of the row's logit scale, counted), the predicted hidden state
+within bf16-level error; at a small size and at the paper's head size
+(d = 4096, m = 2d, V = 16384, one 24-column row)."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import predictor as pr
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ssd():
+    import paper_2606_20543_gb300 as m
+    from paper_2606_20543_gb300 import build
+    build.build()
+    m.load()
+    return m
+
+
+def _bf_dev(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def _case(seed, rows, d, m, V):
+    rng = np.random.default_rng(seed)
+    b = lambda shape, std: synth.bf16_normal(rng, shape, std)  # noqa: E731
+    w = dict(z=b((rows, 2 * d), 1.0), w0=b((d, 2 * d), 1 / np.sqrt(2 * d)),
+             w1=b((m, d), 1 / np.sqrt(d)), w3=b((m, d), 1 / np.sqrt(d)),
+             w2=b((d, m), 1 / np.sqrt(m)), wh=b((d, V), 1 / np.sqrt(d)))
+    g1 = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    g2 = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    return w, g1, g2
+
+
+def _run(ssd, rows, d, m, V, w, g1, g2, eps, with_hidden=True):
+    dev = {k: _bf_dev(v) for k, v in w.items()}
+    tok = torch.full((rows,), -7, dtype=torch.int32, device="cuda")
+    hid = torch.zeros((rows, d), dtype=torch.float32, device="cuda") if with_hidden else None
+    wsb = ssd.ssd_draft_predict_workspace(rows, d, m, V)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ssd.ssd_draft_predict(rows, d, m, V, dev["z"], dev["w0"], dev["w1"], dev["w3"], dev["w2"],
+                          torch.from_numpy(g1).cuda(), torch.from_numpy(g2).cuda(), dev["wh"],
+                          eps, tok, hid, ws, wsb, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    return tok.cpu().numpy(), None if hid is None else hid.cpu().numpy()
+
+
+def _check(w, g1, g2, eps, tok, hid):
+    f = {k: synth.bf16_bits_to_f32(v).astype(np.float64) for k, v in w.items()}
+    h, logits, ref = pr.predict(f["z"], f["w0"], f["w1"], f["w2"], f["w3"], g1, g2, f["wh"], eps)
+    if hid is not None:
+        rel = np.abs(hid - h).max() / np.abs(h).max()
+        assert rel < 2e-3, f"hidden state rel err {rel}"
+    tie = pr.top2_gap(logits) < 1e-3 * np.abs(logits).max(axis=1)
+    bad = np.nonzero((tok != ref) & ~tie)[0]
+    assert bad.size == 0, f"tokens differ at rows {bad[:5]}: gpu {tok[bad[:5]]} ref {ref[bad[:5]]}"
+    return int(tie.sum())
+
+
+@pytest.mark.parametrize("rows,d,m,V", [(24, 256, 512, 4096), (5, 128, 256, 1000)])
+def test_predictor_small(ssd, rows, d, m, V):
+    w, g1, g2 = _case(70 + rows, rows, d, m, V)
+    tok, hid = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6)
+    ties = _check(w, g1, g2, 1e-6, tok, hid)
+    assert ties <= max(1, rows // 10)
+
+
+def test_predictor_paper_head_size(ssd):
+    """d = 4096, m = 8192 (134.2 M parameters), GenHead over V = 16384, a row of 24."""
+    rows, d, m, V = 24, 4096, 8192, 16384
+    w, g1, g2 = _case(80, rows, d, m, V)
+    tok, hid = _run(ssd, rows, d, m, V, w, g1, g2, 1e-5)
+    ties = _check(w, g1, g2, 1e-5, tok, hid)
+    assert ties <= 2
+
+
+def test_predictor_without_hidden_output(ssd):
+    rows, d, m, V = 16, 256, 512, 2048
+    w, g1, g2 = _case(90, rows, d, m, V)
+    tok, _ = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6, with_hidden=False)
+    _check(w, g1, g2, 1e-6, tok, None)
