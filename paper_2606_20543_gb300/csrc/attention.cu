@@ -8,16 +8,17 @@
 //   M(s, j) = 0 iff pos(s) <= pos(j), pos(s) = s for cache slots s < cache_len,
 //   pos(cache_len + j') = prefix + y' * row_stride + x' of draft j'.
 //
-// Design (GB300): one CTA per (KV split, sequence b, KV head g, query tile).
-// All draft queries of the KV group (drafts x the Hq/Hkv query heads sharing
-// g) sit in the CTA's warps, 16 query rows per warp, so each K/V tile is
-// read from HBM once per KV head.  K/V tiles of 64 keys are staged by TMA
-// (2D tensor maps, 128-byte swizzle, evict-first L2 policy) through a
-// 3-stage mbarrier ring; QK^T and PV run as mma.sync (bf16 inputs, fp32
-// accumulation), the mask predicate is evaluated in registers only on
-// tiles that reach the drafted block, and the softmax is the online
-// (running max / running sum) form with quad shuffles.  Long caches are split
-// over CTAs; a combine kernel merges the splits by their log-sum-exp.
+// Design (GB300): one CTA per (KV split, sequence b, KV head g, query tile),
+// sequences taken longest first.  All draft queries of the KV group (drafts x
+// the Hq/Hkv query heads sharing g) sit in the CTA's warps, 16 query rows per
+// warp, so each K/V tile is read from HBM once per KV head.  K/V tiles of 64
+// keys are staged by TMA (2D tensor maps, 128-byte swizzle, evict-first L2
+// policy) through a 2-stage mbarrier ring (three CTAs per SM); QK^T and PV
+// run as mma.sync (bf16 inputs, fp32 accumulation), the mask predicate is
+// evaluated in registers only on tiles that reach the drafted block, and the
+// softmax is the online (running max / running sum) form with quad shuffles.
+// Long caches are split over CTAs; a combine kernel merges the splits by
+// their log-sum-exp.
 #include <mutex>
 
 #include "kernels.cuh"
@@ -29,8 +30,11 @@ namespace {
 #ifndef SSD_ATTN_CTAS_PER_SM
 #define SSD_ATTN_CTAS_PER_SM 2  // KV splits are added until the grid has this many CTAs per SM
 #endif
+#ifndef SSD_ATTN_STAGES
+#define SSD_ATTN_STAGES 2  // K/V ring depth: 2 lets three CTAs share an SM
+#endif
 constexpr int KT = 64;        // keys per tile
-constexpr int kStages = 3;
+constexpr int kStages = SSD_ATTN_STAGES;
 constexpr int kMaxWarps = 8;  // 128 query rows per CTA
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -107,9 +111,11 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   int32_t* kflat = reinterpret_cast<int32_t*>(full + kStages);  // [128]
   int32_t* bad = kflat + 128;
 
+  __shared__ int32_t s_order[kLptMax + 1];
   const int32_t split = blockIdx.x;
   const int32_t bg = blockIdx.y;
-  const int32_t b = bg / a.Hkv, g = bg - b * a.Hkv;
+  const int32_t g = bg % a.Hkv;
+  const int32_t b = longest_first(a, bg / a.Hkv, s_order);
   const int32_t G = a.Hq / a.Hkv;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 

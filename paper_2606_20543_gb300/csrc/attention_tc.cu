@@ -173,9 +173,11 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   int32_t* bad = kflat + 128;
   float* xch = reinterpret_cast<float*>(bad + 4);   // [2 parities][2 halves][128 rows]
 
+  __shared__ int32_t s_order[kLptMax + 1];
   const int32_t split = blockIdx.x;
   const int32_t bg = blockIdx.y;
-  const int32_t b = bg / a.Hkv, g = bg - b * a.Hkv;
+  const int32_t g = bg % a.Hkv;
+  const int32_t b = longest_first(a, bg / a.Hkv, s_order);
   const int32_t G = a.Hq / a.Hkv;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 

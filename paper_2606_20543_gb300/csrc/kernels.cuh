@@ -59,6 +59,31 @@ struct AttnArgs {
   float* lse;  // nullable
   int32_t* status;
 };
+// Longest-first work order for the attention grids: CTA row `rank` (of B)
+// takes the sequence with the rank-th most keys (cache_len + n_drafts, ties by
+// index), so the longest sequences start in the first wave instead of being
+// left for the last one.  Batches above kLptMax keep their order.  Every
+// thread of the block must call it; `skey` is shared memory of kLptMax + 1 ints.
+constexpr int kLptMax = 256;
+__device__ __forceinline__ int32_t longest_first(const AttnArgs& a, int32_t rank, int32_t* skey) {
+  if (a.B > kLptMax) return rank;
+  for (int32_t i = threadIdx.x; i < a.B; i += blockDim.x) {
+    const int32_t c = a.cache_len[i], n = a.n_drafts[i];
+    skey[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
+  }
+  __syncthreads();
+  for (int32_t i = threadIdx.x; i < a.B; i += blockDim.x) {
+    const int32_t k = skey[i];
+    int32_t r = 0;
+    for (int32_t j = 0; j < a.B; ++j) {
+      const int32_t kj = skey[j];
+      r += (kj > k) || (kj == k && j < i);
+    }
+    if (r == rank) skey[kLptMax] = i;  // the ranks form a permutation: one writer
+  }
+  __syncthreads();
+  return skey[kLptMax];
+}
 size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
                            int32_t L_max);
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
