@@ -144,10 +144,13 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     const int s = t % kStages;
     mbar_arrive_expect_tx(&full[s], 2 * TILE_BYTES);
     const int32_t row = kvrow0 + k_lo + t * KT;
-#pragma unroll
-    for (int c = 0; c < NSUB; ++c) {
-      tma_load_2d(sK + s * TILE_BYTES + c * (KT * 128), &tmK, c * 64, row, &full[s], policy);
-      tma_load_2d(sV + s * TILE_BYTES + c * (KT * 128), &tmV, c * 64, row, &full[s], policy);
+    // one copy per tile: for d = 128 the map is the 3D view {64, rows, 2}
+    if constexpr (NSUB == 2) {
+      tma_load_3d(sK + s * TILE_BYTES, &tmK, 0, row, 0, &full[s], policy);
+      tma_load_3d(sV + s * TILE_BYTES, &tmV, 0, row, 0, &full[s], policy);
+    } else {
+      tma_load_2d(sK + s * TILE_BYTES, &tmK, 0, row, &full[s], policy);
+      tma_load_2d(sV + s * TILE_BYTES, &tmV, 0, row, &full[s], policy);
     }
   };
   const int32_t n_pre = min(kStages - 1, ntiles);
@@ -403,16 +406,20 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2D view [rows, d] of a bf16 [B][Hkv][L_max][d] tensor, box [KT rows x 64 cols].
+// View of a bf16 [B][Hkv][L_max][d] tensor whose box is one K (or V) tile of
+// KT rows in the layout [d / 64][KT rows][128 B]: for d = 128 the 3D view
+// {64 columns, rows, 2 halves} with the halves 128 B apart inside a row; for
+// d = 64 the 2D view {64, rows}.
 bool make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int32_t d) {
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)d * 2};
-  cuuint32_t box[2] = {64, KT};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  const cuuint32_t rank = d == 128 ? 3 : 2;
+  cuuint64_t dims[3] = {64, (cuuint64_t)rows, 2};
+  cuuint64_t strides[2] = {(cuuint64_t)d * 2, 128};
+  cuuint32_t box[3] = {64, KT, 2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 

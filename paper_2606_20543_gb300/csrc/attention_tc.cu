@@ -5,24 +5,45 @@
 // drafts before it in raster order):
 //   O[b][j][h] = softmax_s(scale * Q[b][j][h] . K[b][g][s] + M(s, j)) V[b][g][s]
 //
-// Design (GB300, tcgen05 + TMEM), one CTA per (KV split, sequence, KV head,
-// tile of 128 query rows = drafts x the Hq/Hkv heads sharing the KV head):
-//  * warp 8 (producer): Q once through a 3D tensor map, then K and V tiles of
-//    64 keys through a 4-stage mbarrier ring (TMA, 128-byte swizzle);
-//  * warp 9 (MMA): S_t = Q K_t^T into one of two TMEM S buffers, then, once
-//    the softmax has written P_t, O += P_t V_t into the TMEM O accumulator;
-//    tcgen05.commit releases each K/V stage and signals each product;
+// Design (GB300, tcgen05 + TMEM): a persistent kernel, one CTA per SM, that
+// walks work items (KV split, sequence, KV head, tile of 128 query rows =
+// drafts x the Hq/Hkv heads sharing the KV head).  Sequences are taken
+// longest first and the items are dealt to the CTAs in snake order, so the
+// long items start early and every CTA gets a similar share.
+//  * warp 8 (producer): decodes the next item, checks and converts its draft
+//    positions into an item slot (two slots), loads Q into one of two Q
+//    buffers through a 3D tensor map, then the item's K tiles of 64 keys;
+//    warp 10 streams its V tiles (TMA, 128-byte swizzle, one copy per tile,
+//    issued by two threads because one thread issues only a few million copies
+//    per second).  The producers run ahead of the other warps by up to two
+//    items, so the next item's loads overlap the current item's last tiles
+//    and its epilogue;
+//  * warp 9 issues S_t = Q K_t^T into one of three TMEM S buffers; warp 11,
+//    once the softmax has written P_t, O += P_t V_t into the item's TMEM O
+//    buffer (two buffers, so an item's epilogue overlaps the next item's
+//    products);
 //  * warps 0-7 (softmax; query row = TMEM lane, warp w owns lane quarter w % 4
 //    and the half w / 4 of every row's columns): tcgen05.ld of its half of the
 //    row of S_t, the spatial mask predicate in registers, the partial maxima of
 //    the two halves exchanged through a named barrier per warp pair, the
 //    running max and sum, P_t as swizzled bf16 in shared memory (the A operand
-//    of the PV product).  Warps whose rows are all padding skip the math.
-//    The running max is only moved (and O in TMEM rescaled with tcgen05.ld/st)
-//    when it grows by more than 2^8; otherwise the exponentials use the stale
-//    max, which the final sum shares, so the result is exact.
-// Every barrier a thread waits on is at most one phase ahead of it (S, P and
-// PV barriers are per buffer), so parity waits are unambiguous.
+//    of the PV product), and the item's epilogue.  Warps whose rows are all
+//    padding skip the math.  The running max is only moved (and O in TMEM
+//    rescaled with tcgen05.ld/st) when it grows by more than 2^8; otherwise
+//    the exponentials use the stale max, which the final sum shares, so the
+//    result is exact.
+// The K stages and S buffers, and the V stages and P buffers, form rings of
+// three indexed by tile t mod 3, so that one barrier per ring slot covers
+// several conditions: "K_t loaded, S buffer free and P buffer free (PV of
+// tile t - 3 done)", whence S_t done implies its P buffer is free, and "V_t
+// loaded and P_t written".  An mbarrier poll costs a few hundred cycles even when the phase is
+// complete and a tcgen05.mma tens of cycles to issue, so each issuing thread
+// has one wait, one group of products and one commit per tile.
+// Every barrier a thread waits on is at most one phase ahead of it (tile
+// barriers are per tile parity, item barriers per item slot), so parity
+// waits are unambiguous.
+#include <algorithm>
+
 #include "kernels.cuh"
 
 namespace ssd {
@@ -31,9 +52,10 @@ namespace {
 
 constexpr int kBM = 128;          // query rows per CTA (TMEM lanes)
 constexpr int KTC = 64;           // keys per tile
-constexpr int kNS = 4;            // K/V ring stages
+constexpr int kNB = 3;            // ring depth: K stages = TMEM S buffers, V stages = P buffers
+constexpr uint32_t kTmemCols = 512;  // S x 3 (64 columns each), O x 2 (128 columns each) at 256
 constexpr int kSoftWarps = 8;     // two per TMEM lane quarter, each taking half of every row
-constexpr int kThreadsTC = (kSoftWarps + 2) * 32;
+constexpr int kThreadsTC = (kSoftWarps + 4) * 32;  // + K/Q producer, S, V producer, PV
 constexpr float kLog2eTC = 1.4426950408889634f;
 constexpr float kRescale = 8.0f;  // log2 growth of the running max that forces a rescale
 
@@ -120,6 +142,13 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t
   return d;
 }
 
+// The descriptor of base + off: the start address field is (address >> 4) in
+// the low 14 bits, so a 16-byte-multiple offset that keeps the address below
+// 256 KB (all of shared memory) is a plain add.
+__device__ __forceinline__ uint64_t sdesc_at(uint64_t d, uint32_t off) {
+  return d + (uint64_t)(off >> 4);
+}
+
 // kind::f16 instruction descriptor: fp32 D, bf16 A and B, A K-major, M = 128.
 __host__ __device__ constexpr uint32_t idesc_f16(int n, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
@@ -133,10 +162,29 @@ struct TcLaunch {
   int32_t* seq_ok;
 };
 
+// One work item (KV split, sequence, KV head, query tile) as the producer
+// hands it to the MMA and softmax warps; ntiles < 0 ends the CTA's work.
+struct TcItem {
+  int32_t b, g, split, row0, rows_total, cache, Lk, k_lo, k_hi, ntiles, direct, pad[5];
+  int32_t kflat[128];  // raster position of each draft of b
+};
+
 template <int D>
 constexpr size_t tc_smem_bytes() {
-  return 1024 + (size_t)kBM * D * 2 + (size_t)2 * kNS * KTC * D * 2 + (size_t)2 * kBM * KTC * 2 +
-         256 + 132 * 4 + (size_t)4 * kBM * 4 + 16;
+  return 1024 + (size_t)2 * kBM * D * 2 + (size_t)2 * kNB * KTC * D * 2 +
+         (size_t)kNB * kBM * KTC * 2 + 320 + 2 * sizeof(TcItem) + (size_t)6 * kBM * 4;
+}
+
+// One K or V tile of KTC keys in the MMA's layout [d / 64][KTC rows][128 B]
+// (128-byte swizzle) with one copy: for d = 128 the tensor map is the 3D view
+// {64, rows, 2} whose last dimension steps 128 B inside a row.
+template <int D>
+__device__ __forceinline__ void load_kv_tile(void* dst, const CUtensorMap* map, int32_t row,
+                                             uint64_t* bar, uint64_t pol) {
+  if constexpr (D == 128)
+    tma_load_3d(dst, map, 0, row, 0, bar, pol);
+  else
+    tma_load_2d(dst, map, 0, row, bar, pol);
 }
 
 template <int D>
@@ -149,308 +197,477 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   constexpr int P_BYTES = kBM * KTC * 2;     // one P buffer
   constexpr uint32_t kIdescS = idesc_f16(KTC, false);
   constexpr uint32_t kIdescO = idesc_f16(D, true);
-  constexpr uint32_t kTmemCols = 256;        // S x 2 (64 each) + O (<= 128)
   constexpr int HC = KTC / 2;                // S columns per softmax thread
   constexpr int HD = D / 2;                  // O columns per softmax thread
 
   extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ int32_t s_order[kLptMax];
+  __shared__ int32_t s_key[kLptMax];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  unsigned char* sQ = smem;
-  unsigned char* sK = sQ + Q_BYTES;                 // [kNS][KV_BYTES]
-  unsigned char* sV = sK + kNS * KV_BYTES;          // [kNS][KV_BYTES]
-  unsigned char* sP = sV + kNS * KV_BYTES;          // [2][P_BYTES]
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sP + 2 * P_BYTES);
-  uint64_t* q_full = bar;
-  uint64_t* kv_full = bar + 1;                      // [kNS]
-  uint64_t* kv_empty = kv_full + kNS;               // [kNS]
-  uint64_t* s_full = kv_empty + kNS;                // [2]
-  uint64_t* s_free = s_full + 2;                    // [2]
-  uint64_t* p_full = s_free + 2;                    // [2]
-  uint64_t* pv_done = p_full + 2;                   // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_done + 2);
-  int32_t* kflat = reinterpret_cast<int32_t*>(tmem_slot + 4);  // [128]
-  int32_t* bad = kflat + 128;
-  float* xch = reinterpret_cast<float*>(bad + 4);   // [2 parities][2 halves][128 rows]
+  unsigned char* sQ = smem;                         // [2][Q_BYTES]
+  unsigned char* sK = sQ + 2 * Q_BYTES;             // [kNB][KV_BYTES]
+  unsigned char* sV = sK + kNB * KV_BYTES;          // [kNB][KV_BYTES]
+  unsigned char* sP = sV + kNB * KV_BYTES;          // [kNB][P_BYTES]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sP + kNB * P_BYTES);
+  uint64_t* q_full = bar;                           // [2] per item slot
+  uint64_t* q_empty = q_full + 2;                   // [2]
+  uint64_t* it_full = q_empty + 2;                  // [2]
+  uint64_t* it_empty = it_full + 2;                 // [2]
+  uint64_t* o_empty = it_empty + 2;                 // [2]
+  // per ring slot t % kNB: k_ready = K_t loaded, S buffer free (S_{t-kNB} read)
+  // and P buffer free (PV_{t-kNB} done); s_full = S_t done (K stage free);
+  // v_ready = V_t loaded and P_t written; pv_done = PV_t done (V stage free)
+  uint64_t* k_ready = o_empty + 2;                  // [kNB]
+  uint64_t* s_full = k_ready + kNB;                 // [kNB]
+  uint64_t* v_ready = s_full + kNB;                 // [kNB]
+  uint64_t* pv_done = v_ready + kNB;                // [kNB]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_done + kNB);
+  TcItem* items = reinterpret_cast<TcItem*>(bar + 40);  // [2]
+  float* xch = reinterpret_cast<float*>(items + 2);     // [3 slots][2 halves][128 rows]
 
-  __shared__ int32_t s_order[kLptMax + 1];
-  const int32_t split = blockIdx.x;
-  const int32_t bg = blockIdx.y;
-  const int32_t g = bg % a.Hkv;
-  const int32_t b = longest_first(a, bg / a.Hkv, s_order);
   const int32_t G = a.Hq / a.Hkv;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int32_t per_b = a.Hkv * L.splits * L.mtiles;
+  const int64_t n_items = (int64_t)a.B * per_b;
 
-  const int32_t cache = a.cache_len[b];
-  const int32_t nd = a.n_drafts[b];
-  const int32_t Lk = cache + nd;
-  const bool shape_ok = !(nd < 0 || nd > a.D_max || cache < 0 || Lk > a.L_max);
-  const int32_t rows_total = shape_ok ? nd * G : 0;
-  const int32_t row0 = blockIdx.z * kBM;
-  const int32_t k_lo = split * L.kps;
-  const int32_t k_hi = min(Lk, k_lo + L.kps);
-  const bool has_work = shape_ok && nd > 0 && row0 < rows_total && k_lo < Lk;
-  const int32_t ntiles = has_work ? (k_hi - k_lo + KTC - 1) / KTC : 0;
-  const int32_t n_active = (Lk + L.kps - 1) / L.kps;
-
-  // ---- draft positions (validity is identical in every CTA of b)
-  if (tid == 0) *bad = shape_ok ? 0 : 1;
-  __syncthreads();
-  bool seq_valid = shape_ok;
-  if (shape_ok) {
-    const int32_t HW = a.grid.grid_h * a.grid.grid_w;
-    for (int32_t j = tid; j < nd; j += blockDim.x) {
-      const int32_t gidx = a.draft_pos[(int64_t)b * a.D_max + j];
-      if (gidx < 0 || gidx >= HW) {
-        *bad = 1;
-        kflat[j] = 0;
-      } else {
-        const int32_t y = gidx / a.grid.grid_w, x = gidx - y * a.grid.grid_w;
-        kflat[j] = a.grid.prefix_len + y * a.grid.row_stride + x;
-      }
-    }
-    __syncthreads();
-    seq_valid = (*bad == 0);
-  }
-  if (split == 0 && g == 0 && blockIdx.z == 0 && tid == 0) {
-    L.seq_ok[b] = seq_valid ? 1 : 0;
-    if (!seq_valid) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
-  }
-  if (!seq_valid || !has_work) return;
-
-  // ---- set-up: barriers, TMEM
+  // ---- set-up: barriers, TMEM, the longest-first order of the sequences
   if (tid == 0) {
-    mbar_init(q_full, 1);
-    for (int s = 0; s < kNS; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
-    }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], kSoftWarps);
-      mbar_init(&p_full[i], kSoftWarps);
-      mbar_init(&pv_done[i], 1);
+      mbar_init(&q_full[i], 1);
+      mbar_init(&q_empty[i], 1);
+      mbar_init(&it_full[i], 1);
+      mbar_init(&it_empty[i], kSoftWarps);
+      mbar_init(&o_empty[i], kSoftWarps);
+    }
+    for (int s = 0; s < kNB; ++s) {
+      mbar_init(&k_ready[s], 2 + kSoftWarps);
+      mbar_init(&s_full[s], 1);
+      mbar_init(&v_ready[s], 1 + kSoftWarps);
+      mbar_init(&pv_done[s], 1);
     }
     fence_barrier_init();
+    // every S and P buffer starts free: the softmax and PV arrivals of the first round
+    for (int s = 0; s < kNB; ++s)
+      for (int w = 0; w < kSoftWarps + 1; ++w) mbar_arrive(&k_ready[s]);
   }
   if (warp == 0) {
     tmem_alloc_tc(tmem_slot, kTmemCols);
     tmem_relinquish_tc();
   }
+  if (a.B <= kLptMax) {
+    // s_order[rank] = the sequence with the rank-th most keys (ties by index)
+    for (int32_t i = tid; i < a.B; i += blockDim.x) {
+      const int32_t c = a.cache_len[i], n = a.n_drafts[i];
+      s_key[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
+    }
+    __syncthreads();
+    for (int32_t i = tid; i < a.B; i += blockDim.x) {
+      const int32_t key = s_key[i];
+      int32_t r = 0;
+      for (int32_t j = 0; j < a.B; ++j) {
+        const int32_t kj = s_key[j];
+        r += (kj > key) || (kj == key && j < i);
+      }
+      s_order[r] = i;
+    }
+  }
   tc_before();
   __syncthreads();
   tc_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + 2 * KTC;
+  const uint32_t tS = tmem;            // [kNB] x KTC columns
+  const uint32_t tO0 = tmem + 256;     // [2] x 128 columns
 
   const float c2 = (a.scale != 0.f ? a.scale : rsqrtf((float)D)) * kLog2eTC;
-  const int32_t kvrow0 = (b * a.Hkv + g) * a.L_max + k_lo;  // 2D row of the first key
 
   if (warp == kSoftWarps) {
     // ------------------------------------------------------------ producer
+    // Items in snake order over the longest-first list: round k takes items
+    // k * gridDim.x + (blockIdx.x, or its mirror on odd rounds).
+    const uint64_t pol = policy_evict_first();
+    const uint64_t polq = policy_evict_last();
+    const int32_t HW = a.grid.grid_h * a.grid.grid_w;
+    bool ok = true;
+    int32_t k = 0;        // items handed out
+    uint32_t T = 0;       // K/V tiles issued
+    for (int64_t round = 0; ok; ++round) {
+      const int64_t base = round * gridDim.x;
+      if (base >= n_items) break;
+      const int64_t i = base + ((round & 1) ? (gridDim.x - 1 - blockIdx.x) : blockIdx.x);
+      if (i >= n_items) continue;
+      const int32_t rank_b = (int32_t)(i / per_b);
+      int32_t rem = (int32_t)(i - (int64_t)rank_b * per_b);
+      const int32_t mtile = rem % L.mtiles;
+      rem /= L.mtiles;
+      const int32_t split = rem % L.splits, g = rem / L.splits;
+      const int32_t b = (a.B <= kLptMax) ? s_order[rank_b] : rank_b;
+      const int32_t cache = a.cache_len[b], nd = a.n_drafts[b];
+      const bool shape_ok = nd >= 0 && nd <= a.D_max && cache >= 0 && cache <= a.L_max - nd;
+      // draft positions (validity is identical in every item of b)
+      int32_t kfv[4];
+      bool bad = !shape_ok;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int32_t j = lane + 32 * u;
+        kfv[u] = 0;
+        if (shape_ok && j < nd) {
+          const int32_t gidx = a.draft_pos[(int64_t)b * a.D_max + j];
+          if (gidx < 0 || gidx >= HW) {
+            bad = true;
+          } else {
+            const int32_t y = gidx / a.grid.grid_w, x = gidx - y * a.grid.grid_w;
+            kfv[u] = a.grid.prefix_len + y * a.grid.row_stride + x;
+          }
+        }
+      }
+      const bool valid = !__any_sync(0xffffffffu, bad);
+      if (split == 0 && g == 0 && mtile == 0 && lane == 0) {
+        L.seq_ok[b] = valid ? 1 : 0;
+        if (!valid) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+      }
+      const int32_t Lk = valid ? cache + nd : 0;
+      const int32_t rows_total = valid ? nd * G : 0;
+      const int32_t row0 = mtile * kBM;
+      const int32_t k_lo = split * L.kps;
+      const int32_t k_hi = min(Lk, k_lo + L.kps);
+      if (!valid || nd == 0 || row0 >= rows_total || k_lo >= Lk) continue;
+      const int32_t ntiles = (k_hi - k_lo + KTC - 1) / KTC;
+      const int s = k & 1;
+      if (k >= 2 && lane == 0) ok = mbar_wait(&it_empty[s], ((k >> 1) - 1) & 1, a.status);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      TcItem& it = items[s];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (lane + 32 * u < nd) it.kflat[lane + 32 * u] = kfv[u];
+      if (lane == 0) {
+        it.b = b;
+        it.g = g;
+        it.split = split;
+        it.row0 = row0;
+        it.rows_total = rows_total;
+        it.cache = cache;
+        it.Lk = Lk;
+        it.k_lo = k_lo;
+        it.k_hi = k_hi;
+        it.ntiles = ntiles;
+        it.direct = ((Lk + L.kps - 1) / L.kps) == 1;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&it_full[s]);
+        // Q of this item into slot s once the S products of item k - 2 are done
+        if (k >= 2) ok = mbar_wait(&q_empty[s], ((k >> 1) - 1) & 1, a.status);
+        if (ok) {
+          mbar_arrive_expect_tx(&q_full[s], Q_BYTES);
+          for (int c = 0; c < NSUB; ++c) {
+            // 3D Q view {d, Hq, B * D_max}: box {64, G, 128 / G} -> rows (j, hg)
+            asm volatile(
+                "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+                " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(
+                    smem_u32(sQ + s * Q_BYTES + c * (kBM * 128))),
+                "l"(reinterpret_cast<uint64_t>(&tmQ)), "r"(c * 64), "r"(g * G),
+                "r"(b * a.D_max + row0 / G), "r"(smem_u32(&q_full[s])), "l"(polq)
+                : "memory");
+          }
+        }
+        const int32_t kvrow0 = (b * a.Hkv + g) * a.L_max + k_lo;  // 2D row of the first key
+        for (int t = 0; t < ntiles && ok; ++t, ++T) {
+          const int sb = T % kNB;
+          // K stage sb is free once S_{T-kNB} is done
+          if (T >= (uint32_t)kNB && !mbar_wait(&s_full[sb], ((T / kNB) - 1) & 1, a.status)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&k_ready[sb], KV_BYTES);
+          load_kv_tile<D>(sK + sb * KV_BYTES, &tmK, kvrow0 + t * KTC, &k_ready[sb], pol);
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      T = __shfl_sync(0xffffffffu, T, 0);
+      ++k;
+    }
+    if (ok) {
+      // end marker
+      const int s = k & 1;
+      if (k >= 2 && lane == 0) ok = mbar_wait(&it_empty[s], ((k >> 1) - 1) & 1, a.status);
+      if (lane == 0 && ok) {
+        items[s].ntiles = -1;
+        mbar_arrive(&it_full[s]);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kSoftWarps + 2) {
+    // ---------------------------------------------------------- V producer
+    // Follows the item slots like the MMA warp; a slot is not rewritten before
+    // the softmax has finished its item, which needs every V tile of it.
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
-      const uint64_t polq = policy_evict_last();
-      mbar_arrive_expect_tx(q_full, Q_BYTES);
-      for (int c = 0; c < NSUB; ++c) {
-        // 3D Q view {d, Hq, B * D_max}: box {64, G, 128 / G} -> rows (j, hg)
-        asm volatile(
-            "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-            " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(sQ + c * (kBM * 128))),
-            "l"(reinterpret_cast<uint64_t>(&tmQ)), "r"(c * 64), "r"(g * G),
-            "r"(b * a.D_max + row0 / G), "r"(smem_u32(q_full)), "l"(polq)
-            : "memory");
-      }
-      for (int t = 0; t < ntiles; ++t) {
-        const int s = t % kNS;
-        if (t >= kNS && !mbar_wait(&kv_empty[s], ((t / kNS) - 1) & 1, a.status)) break;
-        mbar_arrive_expect_tx(&kv_full[s], 2 * KV_BYTES);
-        const int32_t row = kvrow0 + t * KTC;
-        for (int c = 0; c < NSUB; ++c) {
-          tma_load_2d(sK + s * KV_BYTES + c * (KTC * 128), &tmK, c * 64, row, &kv_full[s], pol);
-          tma_load_2d(sV + s * KV_BYTES + c * (KTC * 128), &tmV, c * 64, row, &kv_full[s], pol);
+      uint32_t T = 0;
+      bool ok = true;
+      for (int32_t k = 0; ok; ++k) {
+        const int s = k & 1;
+        if (!mbar_wait(&it_full[s], (k >> 1) & 1, a.status)) break;
+        const TcItem& it = items[s];
+        const int32_t ntiles = it.ntiles;
+        if (ntiles < 0) break;
+        const int32_t kvrow0 = (it.b * a.Hkv + it.g) * a.L_max + it.k_lo;
+        for (int t = 0; t < ntiles; ++t, ++T) {
+          const int sb = T % kNB;
+          // V stage sb is free once PV_{T-kNB} is done
+          if (T >= (uint32_t)kNB && !mbar_wait(&pv_done[sb], ((T / kNB) - 1) & 1, a.status)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&v_ready[sb], KV_BYTES);
+          load_kv_tile<D>(sV + sb * KV_BYTES, &tmV, kvrow0 + t * KTC, &v_ready[sb], pol);
         }
       }
     }
     __syncwarp();
   } else if (warp == kSoftWarps + 1) {
-    // ----------------------------------------------------------------- MMA
+    // ----------------------------------------------------------- S products
     if (lane == 0) {
-      bool ok = mbar_wait(q_full, 0, a.status);
-      const uint32_t q0 = smem_u32(sQ);
-      auto issue_pv = [&](int t) {
-        const int bb = t & 1, s = t % kNS;
-        if (!mbar_wait(&p_full[bb], (t >> 1) & 1, a.status)) return false;
+      uint32_t T = 0;
+      for (int32_t k = 0;; ++k) {
+        const int s = k & 1;
+        if (!mbar_wait(&it_full[s], (k >> 1) & 1, a.status)) break;
+        const int32_t ntiles = items[s].ntiles;
+        if (ntiles < 0) break;
+        if (!mbar_wait(&q_full[s], (k >> 1) & 1, a.status)) break;
         tc_after();
-        const uint32_t p0 = smem_u32(sP + bb * P_BYTES);
-        const uint32_t v0 = smem_u32(sV + s * KV_BYTES);
+        const uint64_t dq = sdesc(smem_u32(sQ + s * Q_BYTES), 16, 1024);
+        bool ok = true;
+        for (int t = 0; t < ntiles; ++t, ++T) {
+          const int sb = T % kNB;
+          if (!mbar_wait(&k_ready[sb], (T / kNB) & 1, a.status)) { ok = false; break; }
+          tc_after();
+          const uint64_t dk = sdesc(smem_u32(sK + sb * KV_BYTES), 16, 1024);
 #pragma unroll
-        for (int kk = 0; kk < KTC / 16; ++kk) {
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const int sub = ks >> 2, kin = (ks & 3) * 32;
+            umma(tS + sb * KTC, sdesc_at(dq, sub * (kBM * 128) + kin),
+                 sdesc_at(dk, sub * (KTC * 128) + kin), kIdescS, ks > 0 ? 1u : 0u);
+          }
+          umma_commit(&s_full[sb]);
+          if (t == ntiles - 1) umma_commit(&q_empty[s]);
+        }
+        if (!ok) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kSoftWarps + 3) {
+    // ---------------------------------------------------------- PV products
+    // Issued by a thread of its own: a tcgen05.mma takes tens of cycles to
+    // issue and an mbarrier poll a few hundred, so one thread issuing both
+    // products would be the slowest stage of the tile loop.
+    if (lane == 0) {
+      uint32_t T = 0;
+      for (int32_t k = 0;; ++k) {
+        const int s = k & 1;
+        if (!mbar_wait(&it_full[s], (k >> 1) & 1, a.status)) break;
+        const int32_t ntiles = items[s].ntiles;
+        if (ntiles < 0) break;
+        // the first product of the item overwrites O[s]: the epilogue of item k - 2 must be done
+        if (k >= 2 && !mbar_wait(&o_empty[s], ((k >> 1) - 1) & 1, a.status)) break;
+        bool ok = true;
+        for (int t = 0; t < ntiles; ++t, ++T) {
+          const int sb = T % kNB;
+          if (!mbar_wait(&v_ready[sb], (T / kNB) & 1, a.status)) { ok = false; break; }
+          tc_after();
           // A = P (K-major, 128-byte rows), B = V (MN-major: d atoms KTC*128 bytes
           // apart, 8-key groups 1 KB apart; 16 keys = 2 KB per step)
-          umma(tO, sdesc(p0 + kk * 32, 16, 1024), sdesc(v0 + kk * 2048, KTC * 128, 1024), kIdescO,
-               (t > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&kv_empty[s]);
-        umma_commit(&pv_done[bb]);
-        return true;
-      };
-      for (int t = 0; t < ntiles && ok; ++t) {
-        const int s = t % kNS, bb = t & 1;
-        if (!mbar_wait(&kv_full[s], (t / kNS) & 1, a.status)) { ok = false; break; }
-        if (t >= 2 && !mbar_wait(&s_free[bb], ((t >> 1) - 1) & 1, a.status)) { ok = false; break; }
-        tc_after();
-        const uint32_t k0 = smem_u32(sK + s * KV_BYTES);
+          const uint64_t dp = sdesc(smem_u32(sP + sb * P_BYTES), 16, 1024);
+          const uint64_t dv = sdesc(smem_u32(sV + sb * KV_BYTES), KTC * 128, 1024);
 #pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const int sub = ks >> 2, kin = (ks & 3) * 32;
-          umma(tS + bb * KTC, sdesc(q0 + sub * (kBM * 128) + kin, 16, 1024),
-               sdesc(k0 + sub * (KTC * 128) + kin, 16, 1024), kIdescS, ks > 0 ? 1u : 0u);
+          for (int kk = 0; kk < KTC / 16; ++kk)
+            umma(tO0 + s * 128, sdesc_at(dp, kk * 32), sdesc_at(dv, kk * 2048), kIdescO,
+                 (t == 0 && kk == 0) ? 0u : 1u);
+          umma_commit(&pv_done[sb]);
+          umma_commit(&k_ready[sb]);  // S_{T+kNB} may start: P buffer sb is free again
         }
-        umma_commit(&s_full[bb]);
-        if (t >= 1 && !issue_pv(t - 1)) { ok = false; break; }
+        if (!ok) break;
       }
-      if (ok && ntiles > 0) issue_pv(ntiles - 1);
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------- softmax
     const int quarter = warp & 3, half = warp >> 2;
     const int32_t rl = quarter * 32 + lane;   // row inside the tile = TMEM lane
-    const int32_t r = row0 + rl;              // this thread's query row
-    const bool live = r < rows_total;
-    const bool warp_live = row0 + quarter * 32 < rows_total;  // same for both warps of a pair
-    const int32_t qpos = live ? kflat[r / G] : 0x7fffffff;
-    // cache slots below every query position of this CTA are visible to all rows
-    int32_t minq = 0x7fffffff;
-    for (int32_t rr = row0; rr < min(rows_total, row0 + kBM); ++rr) minq = min(minq, kflat[rr / G]);
-    const int32_t mask_from = min(cache, minq + 1);
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's partial sum
-    bool ok = true;
-    // partial values of the two halves of a row, double-buffered by tile parity
-    auto xslot = [&](int parity, int hf) -> float& { return xch[(parity * 2 + hf) * kBM + rl]; };
+    // partial values of the two halves of a row: slots 0 / 1 by tile parity, 2 for the epilogue
+    auto xslot = [&](int slot, int hf) -> float& { return xch[(slot * 2 + hf) * kBM + rl]; };
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory"); };
-    for (int t = 0; t < ntiles; ++t) {
-      const int bb = t & 1;
-      if (!mbar_wait(&s_full[bb], (t >> 1) & 1, a.status)) ok = false;
+    bool ok = true;
+    uint32_t T = 0;
+    for (int32_t k = 0; ok; ++k) {
+      const int s = k & 1;
+      if (!mbar_wait(&it_full[s], (k >> 1) & 1, a.status)) { ok = false; break; }
+      const TcItem& it = items[s];
+      const int32_t ntiles = it.ntiles;
+      if (ntiles < 0) break;
+      const int32_t b = it.b, g = it.g, split = it.split, row0 = it.row0;
+      const int32_t rows_total = it.rows_total, cache = it.cache, Lk = it.Lk;
+      const int32_t k_lo = it.k_lo, k_hi = it.k_hi;
+      const bool direct = it.direct != 0;
+      const int32_t* kflat = it.kflat;
+      const uint32_t tO = tO0 + s * 128;
+      const int32_t r = row0 + rl;              // this thread's query row
+      const bool live = r < rows_total;
+      const bool warp_live = row0 + quarter * 32 < rows_total;  // same for both warps of a pair
+      const int32_t qpos = live ? kflat[r / G] : 0x7fffffff;
+      // cache slots below every query position of this item are visible to all rows
+      int32_t minq = 0x7fffffff;
+      {
+        const int32_t j_lo = row0 / G, j_end = (min(rows_total, row0 + kBM) + G - 1) / G;
+        for (int32_t j = j_lo + lane; j < j_end; j += 32) minq = min(minq, kflat[j]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) minq = min(minq, __shfl_xor_sync(0xffffffffu, minq, o));
+      }
+      const int32_t mask_from = min(cache, minq + 1);
+      float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's partial sum
+      for (int t = 0; t < ntiles; ++t, ++T) {
+        const int bb = T & 1, sb = T % kNB;
+        // S_T is done; S_T started after PV_{T-kNB}, so P buffer sb is free too
+        if (!mbar_wait(&s_full[sb], (T / kNB) & 1, a.status)) ok = false;
+        tc_after();
+        float sv[HC];
+        if (warp_live) tld32(tS + lane_off + sb * KTC + half * HC, sv);
+        tc_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&k_ready[sb]);  // S buffer sb is free for S_{T+kNB}
+        bool moved = false;
+        float alpha = 1.f;
+        uint32_t pk[HC / 2];
+        if (warp_live) {
+          // mask: keys past this split / the sequence, and the spatial predicate
+          const int32_t c0 = k_lo + t * KTC + half * HC;
+          if (c0 + HC > k_hi || c0 + HC > mask_from) {
+#pragma unroll
+            for (int jj = 0; jj < HC; ++jj) {
+              const int32_t key = c0 + jj;
+              const int32_t kp = key < cache ? key : (key < Lk ? kflat[key - cache] : 0x7fffffff);
+              if (!(key < k_hi && kp <= qpos)) sv[jj] = -INFINITY;
+            }
+          }
+          // tree reductions: short dependency chains
+          float m8[HC / 4];
+#pragma unroll
+          for (int i = 0; i < HC / 4; ++i)
+            m8[i] = fmaxf(fmaxf(sv[4 * i], sv[4 * i + 1]), fmaxf(sv[4 * i + 2], sv[4 * i + 3]));
+#pragma unroll
+          for (int w = HC / 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) m8[i] = fmaxf(m8[i], m8[i + w]);
+          float mx = m8[0];
+          xslot(bb, half) = mx;
+          pair_sync();
+          mx = fmaxf(mx, xslot(bb, half ^ 1));
+          // move the running max only when it grows by more than 2^kRescale
+          if (mx != -INFINITY && (m_run == -INFINITY || (mx - m_run) * c2 > kRescale)) {
+            alpha = (m_run == -INFINITY) ? 0.f : ex2a((m_run - mx) * c2);
+            m_run = mx;
+            moved = true;
+          }
+          const float moff = (m_run == -INFINITY) ? 0.f : m_run * c2;
+          float r8[HC / 4];
+#pragma unroll
+          for (int i = 0; i < HC / 4; ++i) {
+            const float e0 = ex2a(fmaf(sv[4 * i], c2, -moff));
+            const float e1 = ex2a(fmaf(sv[4 * i + 1], c2, -moff));
+            const float e2 = ex2a(fmaf(sv[4 * i + 2], c2, -moff));
+            const float e3 = ex2a(fmaf(sv[4 * i + 3], c2, -moff));
+            r8[i] = (e0 + e1) + (e2 + e3);
+            pk[2 * i] = pack_bf16x2(e0, e1);
+            pk[2 * i + 1] = pack_bf16x2(e2, e3);
+          }
+#pragma unroll
+          for (int w = HC / 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) r8[i] += r8[i + w];
+          l_run = l_run * alpha + r8[0];
+        }
+        // O may be rescaled once PV_{T-1} is done
+        if (warp_live) {
+          unsigned char* prow = sP + sb * P_BYTES + rl * 128;
+#pragma unroll
+          for (int cq = 0; cq < HC / 8; ++cq) {  // 16-byte chunks of this half
+            const int cch = half * (HC / 8) + cq;
+            const uint4 v4 = make_uint4(pk[4 * cq], pk[4 * cq + 1], pk[4 * cq + 2], pk[4 * cq + 3]);
+            *reinterpret_cast<uint4*>(prow + ((cch ^ (rl & 7)) << 4)) = v4;
+          }
+          if (__any_sync(0xffffffffu, moved && t > 0)) {
+            if (!mbar_wait(&pv_done[(T - 1) % kNB], ((T - 1) / kNB) & 1, a.status)) ok = false;
+            tc_after();
+            float ov[32];
+#pragma unroll 1
+            for (int cc = 0; cc < HD / 32; ++cc) {
+              const uint32_t ta = tO + lane_off + half * HD + cc * 32;
+              tld32(ta, ov);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+              tst32(ta, ov);
+            }
+          }
+        }
+        fence_proxy_async();  // P stores -> visible to the tensor core
+        tc_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&v_ready[sb]);
+      }
+      // ---- epilogue: wait for the item's last PV product, normalise, write this half
+      const uint32_t Tl = T - 1;
+      if (!mbar_wait(&pv_done[Tl % kNB], (Tl / kNB) & 1, a.status)) ok = false;
       tc_after();
-      float sv[HC];
-      if (warp_live) tld32(tS + lane_off + bb * KTC + half * HC, sv);
-      tc_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[bb]);
-      bool moved = false;
-      float alpha = 1.f;
-      uint32_t pk[HC / 2];
       if (warp_live) {
-        // mask: keys past this split / the sequence, and the spatial predicate
-        const int32_t c0 = k_lo + t * KTC + half * HC;
-        if (c0 + HC > k_hi || c0 + HC > mask_from) {
-#pragma unroll
-          for (int jj = 0; jj < HC; ++jj) {
-            const int32_t key = c0 + jj;
-            const int32_t kp = key < cache ? key : (key < Lk ? kflat[key - cache] : 0x7fffffff);
-            if (!(key < k_hi && kp <= qpos)) sv[jj] = -INFINITY;
-          }
-        }
-        float mx = -INFINITY;
-#pragma unroll
-        for (int jj = 0; jj < HC; ++jj) mx = fmaxf(mx, sv[jj]);
-        xslot(bb, half) = mx;
+        xslot(2, half) = l_run;
         pair_sync();
-        mx = fmaxf(mx, xslot(bb, half ^ 1));
-        // move the running max only when it grows by more than 2^kRescale
-        if (mx != -INFINITY && (m_run == -INFINITY || (mx - m_run) * c2 > kRescale)) {
-          alpha = (m_run == -INFINITY) ? 0.f : ex2a((m_run - mx) * c2);
-          m_run = mx;
-          moved = true;
-        }
-        const float moff = (m_run == -INFINITY) ? 0.f : m_run * c2;
-        float rs = 0.f;
-#pragma unroll
-        for (int jj = 0; jj < HC; jj += 2) {
-          const float e0 = ex2a(fmaf(sv[jj], c2, -moff));
-          const float e1 = ex2a(fmaf(sv[jj + 1], c2, -moff));
-          rs += e0 + e1;
-          pk[jj / 2] = pack_bf16x2(e0, e1);
-        }
-        l_run = l_run * alpha + rs;
-      }
-      // P_t may overwrite the buffer PV(t-2) read; O may be rescaled once PV(t-1) is done
-      if (t >= 2 && !mbar_wait(&pv_done[bb], ((t >> 1) - 1) & 1, a.status)) ok = false;
-      if (warp_live) {
-        unsigned char* prow = sP + bb * P_BYTES + rl * 128;
-#pragma unroll
-        for (int cq = 0; cq < HC / 8; ++cq) {  // 16-byte chunks of this half
-          const int cch = half * (HC / 8) + cq;
-          const uint4 v4 = make_uint4(pk[4 * cq], pk[4 * cq + 1], pk[4 * cq + 2], pk[4 * cq + 3]);
-          *reinterpret_cast<uint4*>(prow + ((cch ^ (rl & 7)) << 4)) = v4;
-        }
-        if (__any_sync(0xffffffffu, moved && t > 0)) {
-          if (!mbar_wait(&pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1, a.status)) ok = false;
-          tc_after();
-          float ov[32];
+        const float l_tot = l_run + xslot(2, half ^ 1);
+        const float inv_l = l_tot > 0.f ? 1.0f / l_tot : 0.f;
+        const float lse = (l_tot > 0.f) ? (m_run * (c2 / kLog2eTC) + logf(l_tot)) : -INFINITY;
+        const int32_t jq = live ? r / G : 0, h = g * G + (live ? r % G : 0);
 #pragma unroll 1
-          for (int cc = 0; cc < HD / 32; ++cc) {
-            const uint32_t ta = tO + lane_off + half * HD + cc * 32;
-            tld32(ta, ov);
+        for (int cc = 0; cc < HD / 32; ++cc) {
+          float ov[32];
+          tld32(tO + lane_off + half * HD + cc * 32, ov);
+          if (!live || !ok) continue;
+          const int col = half * HD + cc * 32;
+          if (direct) {
+            __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.o) +
+                                (((int64_t)b * a.D_max + jq) * a.Hq + h) * D + col;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-            tst32(ta, ov);
+            for (int i = 0; i < 32; i += 8) {
+              uint4 w;
+              w.x = pack_bf16x2(ov[i] * inv_l, ov[i + 1] * inv_l);
+              w.y = pack_bf16x2(ov[i + 2] * inv_l, ov[i + 3] * inv_l);
+              w.z = pack_bf16x2(ov[i + 4] * inv_l, ov[i + 5] * inv_l);
+              w.w = pack_bf16x2(ov[i + 6] * inv_l, ov[i + 7] * inv_l);
+              *reinterpret_cast<uint4*>(ob + i) = w;
+            }
+          } else {
+            const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split;
+            float* po = L.part_o + prow * D + col;
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              *reinterpret_cast<float4*>(po + i) = make_float4(
+                  ov[i] * inv_l, ov[i + 1] * inv_l, ov[i + 2] * inv_l, ov[i + 3] * inv_l);
+          }
+        }
+        if (live && ok && half == 0) {
+          if (direct) {
+            if (a.lse != nullptr) a.lse[((int64_t)b * a.Hq + h) * a.D_max + jq] = lse;
+          } else {
+            L.part_lse[(((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split] = lse;
           }
         }
       }
-      fence_proxy_async();  // P stores -> visible to the tensor core
+      // O[s] and the item slot are free for item k + 2
       tc_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[bb]);
-    }
-    // ---- epilogue: wait for the last PV product, normalise, write this half
-    if (ntiles > 0 && !mbar_wait(&pv_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.status))
-      ok = false;
-    tc_after();
-    if (warp_live) {
-      xslot(ntiles & 1, half) = l_run;  // the parity the last tile did not use
-      pair_sync();
-      const float l_tot = l_run + xslot(ntiles & 1, half ^ 1);
-      const float inv_l = l_tot > 0.f ? 1.0f / l_tot : 0.f;
-      const float lse = (l_tot > 0.f) ? (m_run * (c2 / kLog2eTC) + logf(l_tot)) : -INFINITY;
-      const bool direct = (n_active == 1);
-      const int32_t jq = live ? r / G : 0, h = g * G + (live ? r % G : 0);
-#pragma unroll 1
-      for (int cc = 0; cc < HD / 32; ++cc) {
-        float ov[32];
-        tld32(tO + lane_off + half * HD + cc * 32, ov);
-        if (!live || !ok) continue;
-        const int col = half * HD + cc * 32;
-        if (direct) {
-          __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.o) +
-                              (((int64_t)b * a.D_max + jq) * a.Hq + h) * D + col;
-#pragma unroll
-          for (int i = 0; i < 32; i += 8) {
-            uint4 w;
-            w.x = pack_bf16x2(ov[i] * inv_l, ov[i + 1] * inv_l);
-            w.y = pack_bf16x2(ov[i + 2] * inv_l, ov[i + 3] * inv_l);
-            w.z = pack_bf16x2(ov[i + 4] * inv_l, ov[i + 5] * inv_l);
-            w.w = pack_bf16x2(ov[i + 6] * inv_l, ov[i + 7] * inv_l);
-            *reinterpret_cast<uint4*>(ob + i) = w;
-          }
-        } else {
-          const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split;
-          float* po = L.part_o + prow * D + col;
-#pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4*>(po + i) =
-                make_float4(ov[i] * inv_l, ov[i + 1] * inv_l, ov[i + 2] * inv_l, ov[i + 3] * inv_l);
-        }
-      }
-      if (live && ok && half == 0) {
-        if (direct) {
-          if (a.lse != nullptr) a.lse[((int64_t)b * a.Hq + h) * a.D_max + jq] = lse;
-        } else {
-          L.part_lse[(((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split] = lse;
-        }
+      if (lane == 0) {
+        mbar_arrive(&o_empty[s]);
+        mbar_arrive(&it_empty[s]);
       }
     }
   }
@@ -483,11 +700,14 @@ EncodeTiledFnTc encode_tc() {
 
 }  // namespace
 
+#ifndef SSD_ATTN_TC_MIN_ROWS
+#define SSD_ATTN_TC_MIN_ROWS 64  // query rows per KV group above which the tcgen05 kernel runs
+#endif
+
 bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max) {
   const int32_t G = Hq / Hkv;
-  // Below 64 query rows per KV group the 128-row MMA tile is mostly padding and
-  // the mma.sync kernel (several CTAs per SM) is faster.
-  return (d == 64 || d == 128) && G >= 1 && G <= kBM && (kBM % G) == 0 && D_max * G > 64;
+  return (d == 64 || d == 128) && G >= 1 && G <= kBM && (kBM % G) == 0 &&
+         D_max * G > SSD_ATTN_TC_MIN_ROWS;
 }
 
 TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
@@ -524,11 +744,14 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq
   }
   const int64_t rows = (int64_t)a.B * a.Hkv * a.L_max;
   for (int w = 0; w < 2; ++w) {
-    cuuint64_t dims[2] = {(cuuint64_t)a.d, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)a.d * 2};
-    cuuint32_t box[2] = {64, KTC};
-    cuuint32_t estr[2] = {1, 1};
-    if (fn(w == 0 ? &tk : &tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+    // d = 128: {64 columns, rows, 2 halves}, the halves 128 B apart inside a row,
+    // so one box {64, KTC, 2} is a whole tile; d = 64: {64, rows}, box {64, KTC}
+    const cuuint32_t rank = a.d == 128 ? 3 : 2;
+    cuuint64_t dims[3] = {64, (cuuint64_t)rows, 2};
+    cuuint64_t strides[2] = {(cuuint64_t)a.d * 2, 128};
+    cuuint32_t box[3] = {64, KTC, 2};
+    cuuint32_t estr[3] = {1, 1, 1};
+    if (fn(w == 0 ? &tk : &tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank,
            const_cast<void*>(w == 0 ? a.k : a.v), dims, strides, box, estr,
            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
@@ -541,7 +764,9 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq
   L.part_o = part_o;
   L.part_lse = part_lse;
   L.seq_ok = seq_ok;
-  const dim3 grid(p.splits, a.B * a.Hkv, p.mtiles);
+  // persistent: one CTA per SM (at most one per work item)
+  const int64_t n_items = (int64_t)a.B * a.Hkv * p.mtiles * p.splits;
+  const dim3 grid((unsigned)std::min<int64_t>(n_items, device_sm_count()));
   const dim3 block(kThreadsTC);
   cudaError_t e;
   if (a.d == 128) {

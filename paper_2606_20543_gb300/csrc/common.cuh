@@ -90,6 +90,39 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_
   return false;
 }
 
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on two mbarrier phases at once.  A poll of an mbarrier takes a
+// few hundred cycles even when the phase is long complete; both polls are
+// issued back to back so their latencies overlap.
+__device__ __forceinline__ bool mbar_wait2(uint64_t* bar1, uint32_t parity1, uint64_t* bar2,
+                                           uint32_t parity2, int32_t* status) {
+  bool done1 = false, done2 = false;
+  for (uint32_t i = 0; i < kMaxPolls; ++i) {
+    const bool t1 = done1 || mbar_test_wait(bar1, parity1);
+    const bool t2 = done2 || mbar_test_wait(bar2, parity2);
+    done1 = t1;
+    done2 = t2;
+    if (done1 && done2) return true;
+    if (i > 4096) {
+      __nanosleep(128);
+      if (give_up(i, status)) return false;
+    }
+  }
+  record_status(status, SSD_ERR_TIMEOUT);
+  return false;
+}
+
 // ------------------------------------------------------------- bulk copies
 // Untiled bulk copy global -> shared (TMA engine); both addresses 16-byte
 // aligned, bytes a multiple of 16.  Completion is signalled on `bar`.
@@ -134,6 +167,17 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+// Tiled 3D tensor copy global -> shared through a CUtensorMap (c0 innermost).
+__device__ __forceinline__ void tma_load_3d(void* smem_dst, const CUtensorMap* map, int32_t c0,
+                                            int32_t c1, int32_t c2, uint64_t* bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar)),
+      "l"(policy)
       : "memory");
 }
 

@@ -25,7 +25,7 @@ def _bf(x):
     return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).cuda()
 
 
-def run_attention(ssd, c, scale=0.0):
+def run_attention(ssd, c, scale=0.0, edit_pos=None):
     dev = "cuda"
     g = ssd.grid(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v)
     cl = torch.from_numpy(c.cache_len.astype(np.int32)).to(dev)
@@ -33,6 +33,8 @@ def run_attention(ssd, c, scale=0.0):
     pos = torch.empty((c.B, c.D_max), dtype=torch.int32, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     ssd.ssd_frontier(g, c.B, cl, c.D_max, nd, pos, status)
+    if edit_pos is not None:
+        edit_pos(pos)
     q, k, v = _bf(c.q), _bf(c.k), _bf(c.v)
     o = torch.zeros((c.B, c.D_max, c.Hq, c.d), dtype=torch.bfloat16, device=dev)
     lse = torch.zeros((c.B, c.Hq, c.D_max), dtype=torch.float32, device=dev)
@@ -44,9 +46,9 @@ def run_attention(ssd, c, scale=0.0):
     return (o.float().cpu().numpy(), lse.cpu().numpy(), nd.cpu().numpy(), int(status.item()))
 
 
-def check_case(ssd, c, seqs=None, scale=0.0):
-    o, lse, nd, st = run_attention(ssd, c, scale)
-    assert st == 0
+def check_case(ssd, c, seqs=None, scale=0.0, edit_pos=None, want_status=0):
+    o, lse, nd, st = run_attention(ssd, c, scale, edit_pos)
+    assert st == want_status
     q, k, v = bf16_to_f64(c.q), bf16_to_f64(c.k), bf16_to_f64(c.v)
     ref = ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
                                q, k, v, c.Hq, c.Hkv, scale if scale else None, seqs)
@@ -131,3 +133,38 @@ def test_mma_sync_and_tensor_core_paths_agree(ssd):
     c2 = synth.make_case("gqa96", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
                          Hq=16, Hkv=8, d=128, V=64, seed=10, with_logits=False)
     check_case(ssd, c2)
+
+
+def _gqa_batch(B, seed):
+    rng = np.random.default_rng(seed)
+    cl = rng.integers(64, 1088 + 1, size=B).astype(np.int32)
+    return synth.make_case("gqa_many", grid_h=32, grid_w=32, prefix_len=64, cache_len=cl, Hq=32,
+                           Hkv=8, d=128, V=64, seed=seed, with_logits=False)
+
+
+def test_tensor_core_items_outnumber_sms(ssd):
+    """24 sequences x 8 KV heads x 2 query tiles = 384 work items: every CTA
+    of the persistent tcgen05 kernel takes two or three items in turn (item
+    slots, Q buffers and O buffers reused)."""
+    check_case(ssd, _gqa_batch(24, 11))
+
+
+def test_tensor_core_bad_draft_position_skips_only_its_sequence(ssd):
+    c = _gqa_batch(20, 12)
+    hw = c.grid_h * c.grid_w
+
+    def corrupt(pos):
+        pos[3, 0] = hw + 5  # sequence 3 reads past the grid
+
+    o, lse, nd, st = run_attention(ssd, c, edit_pos=corrupt)
+    assert st == 6
+    q, k, v = bf16_to_f64(c.q), bf16_to_f64(c.k), bf16_to_f64(c.v)
+    seqs = [b for b in range(c.B) if b != 3]
+    ref = ostep.attention_step(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v, c.cache_len,
+                               q, k, v, c.Hq, c.Hkv, None, seqs)
+    for b, (o_ref, _) in ref.items():
+        n = o_ref.shape[0]
+        for h in range(c.Hq):
+            if n:
+                assert attention_error(o[b, :n, h], o_ref[:, h]) < ATTN_TOL, f"b={b} h={h}"
+    assert not o[3].any()  # the bad sequence is not written
