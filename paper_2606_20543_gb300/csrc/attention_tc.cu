@@ -12,33 +12,36 @@
 // long items start early and every CTA gets a similar share.
 //  * warp 8 (producer): decodes the next item, checks and converts its draft
 //    positions into an item slot (two slots), loads Q into one of two Q
-//    buffers through a 3D tensor map, then the item's K tiles of 64 keys;
+//    buffers through a 3D tensor map, then the item's K tiles of 128 keys;
 //    warp 10 streams its V tiles (TMA, 128-byte swizzle, one copy per tile,
 //    issued by two threads because one thread issues only a few million copies
 //    per second).  The producers run ahead of the other warps by up to two
 //    items, so the next item's loads overlap the current item's last tiles
 //    and its epilogue;
-//  * warp 9 issues S_t = Q K_t^T into one of three TMEM S buffers; warp 11,
-//    once the softmax has written P_t, O += P_t V_t into the item's TMEM O
-//    buffer (two buffers, so an item's epilogue overlaps the next item's
-//    products);
+//  * warp 9 issues S_t = Q K_t^T (N = 128 keys) into one of two TMEM S/P
+//    buffers; warp 11, once the softmax has written P_t, O += P_t V_t with P
+//    read from TMEM (the A operand of a tcgen05.mma may live in tensor
+//    memory) into the item's TMEM O buffer (two buffers, so an item's
+//    epilogue overlaps the next item's products);
 //  * warps 0-7 (softmax; query row = TMEM lane, warp w owns lane quarter w % 4
 //    and the half w / 4 of every row's columns): tcgen05.ld of its half of the
-//    row of S_t, the spatial mask predicate in registers, the partial maxima of
-//    the two halves exchanged through a named barrier per warp pair, the
-//    running max and sum, P_t as swizzled bf16 in shared memory (the A operand
-//    of the PV product), and the item's epilogue.  Warps whose rows are all
-//    padding skip the math.  The running max is only moved (and O in TMEM
-//    rescaled with tcgen05.ld/st) when it grows by more than 2^8; otherwise
-//    the exponentials use the stale max, which the final sum shares, so the
+//    row of S_t, the spatial mask (a per-row bitmask of the visible drafts,
+//    built once per item), the partial maxima of the two halves exchanged
+//    through a named barrier per warp pair, the running max and sum, and P_t
+//    as bf16 pairs stored with tcgen05.st over the first half of the same
+//    TMEM buffer; then the item's epilogue.  Warps whose rows are all padding
+//    skip the math.  The running max is only moved (and O in TMEM rescaled
+//    with tcgen05.ld/st) when it grows by more than 2^8; otherwise the
+//    exponentials use the stale max, which the final sum shares, so the
 //    result is exact.
-// The K stages and S buffers, and the V stages and P buffers, form rings of
-// three indexed by tile t mod 3, so that one barrier per ring slot covers
-// several conditions: "K_t loaded, S buffer free and P buffer free (PV of
-// tile t - 3 done)", whence S_t done implies its P buffer is free, and "V_t
-// loaded and P_t written".  An mbarrier poll costs a few hundred cycles even when the phase is
-// complete and a tcgen05.mma tens of cycles to issue, so each issuing thread
-// has one wait, one group of products and one commit per tile.
+// K stages, V stages and S/P buffers form rings of two indexed by tile t mod
+// 2, and one barrier per ring slot covers several conditions: "K_t loaded and
+// S/P buffer free (PV of tile t - 2 done)" and "V_t loaded and P_t written".
+// An mbarrier poll costs a few hundred cycles even when the phase is complete
+// and a tcgen05.mma tens of cycles to issue, so each issuing thread has one
+// wait, one group of products and one commit per 128-key tile.  Code that
+// runs once per item (mask, bitmask, epilogue) is kept small: unrolled cold
+// paths cost instruction-cache misses of thousands of cycles.
 // Every barrier a thread waits on is at most one phase ahead of it (tile
 // barriers are per tile parity, item barriers per item slot), so parity
 // waits are unambiguous.
@@ -51,9 +54,9 @@ namespace ssd {
 namespace {
 
 constexpr int kBM = 128;          // query rows per CTA (TMEM lanes)
-constexpr int KTC = 64;           // keys per tile
-constexpr int kNB = 3;            // ring depth: K stages = TMEM S buffers, V stages = P buffers
-constexpr uint32_t kTmemCols = 512;  // S x 3 (64 columns each), O x 2 (128 columns each) at 256
+constexpr int KTC = 128;          // keys per tile
+constexpr int kNB = 2;            // ring depth: K stages, V stages, TMEM S/P buffers
+constexpr uint32_t kTmemCols = 512;  // S/P x 2 (128 columns each), O x 2 (128 columns each) at 256
 constexpr int kSoftWarps = 8;     // two per TMEM lane quarter, each taking half of every row
 constexpr int kThreadsTC = (kSoftWarps + 4) * 32;  // + K/Q producer, S, V producer, PV
 constexpr float kLog2eTC = 1.4426950408889634f;
@@ -86,6 +89,15 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t adesc, uint64_t b
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// D (TMEM) (+)= A (TMEM, 128 lanes x 16 bf16 in 8 columns) * B (shared memory).
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                    smem_u32(bar))
@@ -106,6 +118,18 @@ __device__ __forceinline__ void tld32(uint32_t taddr, float* v) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tst32u(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+      "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]),
+      "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]),
+      "r"(v[30]), "r"(v[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tst32(uint32_t taddr, const float* v) {
   asm volatile(
@@ -171,8 +195,8 @@ struct TcItem {
 
 template <int D>
 constexpr size_t tc_smem_bytes() {
-  return 1024 + (size_t)2 * kBM * D * 2 + (size_t)2 * kNB * KTC * D * 2 +
-         (size_t)kNB * kBM * KTC * 2 + 320 + 2 * sizeof(TcItem) + (size_t)6 * kBM * 4;
+  return 1024 + (size_t)2 * kBM * D * 2 + (size_t)2 * kNB * KTC * D * 2 + 320 +
+         2 * sizeof(TcItem) + (size_t)6 * kBM * 4;
 }
 
 // One K or V tile of KTC keys in the MMA's layout [d / 64][KTC rows][128 B]
@@ -194,10 +218,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   constexpr int NSUB = D / 64;
   constexpr int Q_BYTES = kBM * D * 2;
   constexpr int KV_BYTES = KTC * D * 2;      // one K (or V) tile
-  constexpr int P_BYTES = kBM * KTC * 2;     // one P buffer
   constexpr uint32_t kIdescS = idesc_f16(KTC, false);
   constexpr uint32_t kIdescO = idesc_f16(D, true);
-  constexpr int HC = KTC / 2;                // S columns per softmax thread
+  constexpr int HC = KTC / 2;                // S columns per softmax thread (P: HC / 2)
   constexpr int HD = D / 2;                  // O columns per softmax thread
 
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -208,16 +231,15 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   unsigned char* sQ = smem;                         // [2][Q_BYTES]
   unsigned char* sK = sQ + 2 * Q_BYTES;             // [kNB][KV_BYTES]
   unsigned char* sV = sK + kNB * KV_BYTES;          // [kNB][KV_BYTES]
-  unsigned char* sP = sV + kNB * KV_BYTES;          // [kNB][P_BYTES]
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sP + kNB * P_BYTES);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + kNB * KV_BYTES);
   uint64_t* q_full = bar;                           // [2] per item slot
   uint64_t* q_empty = q_full + 2;                   // [2]
   uint64_t* it_full = q_empty + 2;                  // [2]
   uint64_t* it_empty = it_full + 2;                 // [2]
   uint64_t* o_empty = it_empty + 2;                 // [2]
-  // per ring slot t % kNB: k_ready = K_t loaded, S buffer free (S_{t-kNB} read)
-  // and P buffer free (PV_{t-kNB} done); s_full = S_t done (K stage free);
-  // v_ready = V_t loaded and P_t written; pv_done = PV_t done (V stage free)
+  // per ring slot t % kNB: k_ready = K_t loaded and the TMEM S/P buffer free
+  // (PV_{t-kNB} done); s_full = S_t done (K stage free); v_ready = V_t loaded
+  // and P_t written; pv_done = PV_t done (V stage free)
   uint64_t* k_ready = o_empty + 2;                  // [kNB]
   uint64_t* s_full = k_ready + kNB;                 // [kNB]
   uint64_t* v_ready = s_full + kNB;                 // [kNB]
@@ -241,15 +263,14 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       mbar_init(&o_empty[i], kSoftWarps);
     }
     for (int s = 0; s < kNB; ++s) {
-      mbar_init(&k_ready[s], 2 + kSoftWarps);
+      mbar_init(&k_ready[s], 2);
       mbar_init(&s_full[s], 1);
       mbar_init(&v_ready[s], 1 + kSoftWarps);
       mbar_init(&pv_done[s], 1);
     }
     fence_barrier_init();
-    // every S and P buffer starts free: the softmax and PV arrivals of the first round
-    for (int s = 0; s < kNB; ++s)
-      for (int w = 0; w < kSoftWarps + 1; ++w) mbar_arrive(&k_ready[s]);
+    // every S/P buffer starts free: the PV arrivals of the first round
+    for (int s = 0; s < kNB; ++s) mbar_arrive(&k_ready[s]);
   }
   if (warp == 0) {
     tmem_alloc_tc(tmem_slot, kTmemCols);
@@ -276,7 +297,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   __syncthreads();
   tc_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem;            // [kNB] x KTC columns
+  const uint32_t tS = tmem;            // [kNB] x KTC columns: S_t in fp32, then P_t in bf16
   const uint32_t tO0 = tmem + 256;     // [2] x 128 columns
 
   const float c2 = (a.scale != 0.f ? a.scale : rsqrtf((float)D)) * kLog2eTC;
@@ -476,16 +497,15 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           const int sb = T % kNB;
           if (!mbar_wait(&v_ready[sb], (T / kNB) & 1, a.status)) { ok = false; break; }
           tc_after();
-          // A = P (K-major, 128-byte rows), B = V (MN-major: d atoms KTC*128 bytes
-          // apart, 8-key groups 1 KB apart; 16 keys = 2 KB per step)
-          const uint64_t dp = sdesc(smem_u32(sP + sb * P_BYTES), 16, 1024);
+          // A = P in TMEM (16 keys = 8 columns per step), B = V (MN-major: d
+          // atoms KTC*128 bytes apart, 8-key groups 1 KB apart; 16 keys = 2 KB)
           const uint64_t dv = sdesc(smem_u32(sV + sb * KV_BYTES), KTC * 128, 1024);
 #pragma unroll
           for (int kk = 0; kk < KTC / 16; ++kk)
-            umma(tO0 + s * 128, sdesc_at(dp, kk * 32), sdesc_at(dv, kk * 2048), kIdescO,
-                 (t == 0 && kk == 0) ? 0u : 1u);
+            umma_ts(tO0 + s * 128, tS + sb * KTC + kk * 8, sdesc_at(dv, kk * 2048), kIdescO,
+                    (t == 0 && kk == 0) ? 0u : 1u);
           umma_commit(&pv_done[sb]);
-          umma_commit(&k_ready[sb]);  // S_{T+kNB} may start: P buffer sb is free again
+          umma_commit(&k_ready[sb]);  // S_{T+kNB} may start: the S/P buffer is free again
         }
         if (!ok) break;
       }
@@ -526,17 +546,32 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         for (int o = 16; o > 0; o >>= 1) minq = min(minq, __shfl_xor_sync(0xffffffffu, minq, o));
       }
       const int32_t mask_from = min(cache, minq + 1);
+      // visibility of the item's drafts to this row: bit j of (vis_hi:vis_lo) is
+      // kflat[j] <= qpos.  Runs once per item, so the loop is kept rolled (small
+      // code: a cold unrolled path costs instruction-cache misses).
+      uint64_t vis_lo = 0, vis_hi = 0;
+      if (warp_live) {
+        const int32_t nd = Lk - cache;
+#pragma unroll 1
+        for (int j = 0; j < nd; j += 4) {
+          const int4 kf = *reinterpret_cast<const int4*>(kflat + j);
+          const uint64_t bits = (uint64_t)((uint32_t)(kf.x <= qpos) | ((uint32_t)(kf.y <= qpos) << 1) |
+                                           ((uint32_t)(kf.z <= qpos) << 2) |
+                                           ((uint32_t)(kf.w <= qpos) << 3));
+          if (j < 64) vis_lo |= bits << j;
+          else vis_hi |= bits << (j - 64);
+        }
+      }
       float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's partial sum
       for (int t = 0; t < ntiles; ++t, ++T) {
         const int bb = T & 1, sb = T % kNB;
-        // S_T is done; S_T started after PV_{T-kNB}, so P buffer sb is free too
         if (!mbar_wait(&s_full[sb], (T / kNB) & 1, a.status)) ok = false;
         tc_after();
         float sv[HC];
-        if (warp_live) tld32(tS + lane_off + sb * KTC + half * HC, sv);
-        tc_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&k_ready[sb]);  // S buffer sb is free for S_{T+kNB}
+        if (warp_live) {
+          tld32(tS + lane_off + sb * KTC + half * HC, sv);
+          tld32(tS + lane_off + sb * KTC + half * HC + 32, sv + 32);
+        }
         bool moved = false;
         float alpha = 1.f;
         uint32_t pk[HC / 2];
@@ -544,12 +579,25 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           // mask: keys past this split / the sequence, and the spatial predicate
           const int32_t c0 = k_lo + t * KTC + half * HC;
           if (c0 + HC > k_hi || c0 + HC > mask_from) {
+            // keep bit jj: key c0 + jj is visible to this row.  Cache keys are a
+            // prefix of the window (visible up to qpos), draft keys come from the
+            // visibility bits, keys past the split are dropped.
+            auto low = [](int32_t n) -> uint64_t {
+              return n <= 0 ? 0ull : (n >= 64 ? ~0ull : ((1ull << n) - 1ull));
+            };
+            const int32_t base = c0 - cache;  // draft index of column 0
+            uint64_t win;                     // bit jj: draft base + jj is visible
+            if (base >= 128 || base <= -64) win = 0;
+            else if (base >= 64) win = vis_hi >> (base - 64);
+            else if (base > 0) win = (vis_lo >> base) | (vis_hi << (64 - base));
+            else if (base == 0) win = vis_lo;
+            else win = vis_lo << (-base);
+            const int32_t seen_end = qpos < cache ? qpos + 1 : cache;
+            const uint64_t keep =
+                (low(seen_end - c0) | (win & ~low(cache - c0))) & low(k_hi - c0);
 #pragma unroll
-            for (int jj = 0; jj < HC; ++jj) {
-              const int32_t key = c0 + jj;
-              const int32_t kp = key < cache ? key : (key < Lk ? kflat[key - cache] : 0x7fffffff);
-              if (!(key < k_hi && kp <= qpos)) sv[jj] = -INFINITY;
-            }
+            for (int jj = 0; jj < HC; ++jj)
+              if (!((keep >> jj) & 1ull)) sv[jj] = -INFINITY;
           }
           // tree reductions: short dependency chains
           float m8[HC / 4];
@@ -561,6 +609,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll
             for (int i = 0; i < w; ++i) m8[i] = fmaxf(m8[i], m8[i + w]);
           float mx = m8[0];
+          // (the pair barrier also orders the partner's tcgen05.ld of S before
+          // this warp overwrites the buffer with P)
           xslot(bb, half) = mx;
           pair_sync();
           mx = fmaxf(mx, xslot(bb, half ^ 1));
@@ -590,13 +640,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
         // O may be rescaled once PV_{T-1} is done
         if (warp_live) {
-          unsigned char* prow = sP + sb * P_BYTES + rl * 128;
-#pragma unroll
-          for (int cq = 0; cq < HC / 8; ++cq) {  // 16-byte chunks of this half
-            const int cch = half * (HC / 8) + cq;
-            const uint4 v4 = make_uint4(pk[4 * cq], pk[4 * cq + 1], pk[4 * cq + 2], pk[4 * cq + 3]);
-            *reinterpret_cast<uint4*>(prow + ((cch ^ (rl & 7)) << 4)) = v4;
-          }
           if (__any_sync(0xffffffffu, moved && t > 0)) {
             if (!mbar_wait(&pv_done[(T - 1) % kNB], ((T - 1) / kNB) & 1, a.status)) ok = false;
             tc_after();
@@ -610,8 +653,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
               tst32(ta, ov);
             }
           }
+          // P_T as bf16 pairs over the first half of its S buffer: this half's keys
+          // are columns [half * HC / 2, (half + 1) * HC / 2)
+          tst32u(tS + lane_off + sb * KTC + half * (HC / 2), pk);
         }
-        fence_proxy_async();  // P stores -> visible to the tensor core
         tc_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&v_ready[sb]);
