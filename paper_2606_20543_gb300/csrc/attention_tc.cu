@@ -536,7 +536,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       const int32_t r = row0 + rl;              // this thread's query row
       const bool live = r < rows_total;
       const bool warp_live = row0 + quarter * 32 < rows_total;  // same for both warps of a pair
-      const int32_t qpos = live ? kflat[r / G] : 0x7fffffff;
+      // this row's draft and query head (computed once per item)
+      const int32_t jq = live ? r / G : 0, h = g * G + (live ? r - (r / G) * G : 0);
+      const int32_t qpos = live ? kflat[jq] : 0x7fffffff;
       // cache slots below every query position of this item are visible to all rows
       int32_t minq = 0x7fffffff;
       {
@@ -669,9 +671,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         xslot(2, half) = l_run;
         pair_sync();
         const float l_tot = l_run + xslot(2, half ^ 1);
-        const float inv_l = l_tot > 0.f ? 1.0f / l_tot : 0.f;
-        const float lse = (l_tot > 0.f) ? (m_run * (c2 / kLog2eTC) + logf(l_tot)) : -INFINITY;
-        const int32_t jq = live ? r / G : 0, h = g * G + (live ? r % G : 0);
+        // fast reciprocal and logarithm: the epilogue runs once per item, and
+        // its instruction count is its cost
+        const float inv_l = l_tot > 0.f ? __fdividef(1.0f, l_tot) : 0.f;
+        const float lse = (l_tot > 0.f) ? (m_run * (c2 / kLog2eTC) + __logf(l_tot)) : -INFINITY;
 #pragma unroll 1
         for (int cc = 0; cc < HD / 32; ++cc) {
           float ov[32];
