@@ -189,7 +189,9 @@ struct TcLaunch {
 // One work item (KV split, sequence, KV head, query tile) as the producer
 // hands it to the MMA and softmax warps; ntiles < 0 ends the CTA's work.
 struct TcItem {
-  int32_t b, g, split, row0, rows_total, cache, Lk, k_lo, k_hi, ntiles, direct, pad[5];
+  int32_t b, g, split, row0, rows_total, cache, Lk, k_lo, k_hi, ntiles, direct;
+  int32_t increasing;  // kflat strictly increasing (the raster frontier): draft j sees draft j' iff j' <= j
+  int32_t pad[4];
   int32_t kflat[128];  // raster position of each draft of b
 };
 
@@ -343,6 +345,18 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
       }
       const bool valid = !__any_sync(0xffffffffu, bad);
+      // strictly increasing positions? (the previous draft of j = lane + 32 u is
+      // lane - 1 of the same u, or lane 31 of u - 1)
+      bool dec = false;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int32_t up = __shfl_up_sync(0xffffffffu, kfv[u], 1);
+        const int32_t prev_hi = __shfl_sync(0xffffffffu, u > 0 ? kfv[u > 0 ? u - 1 : 0] : 0, 31);
+        const int32_t prev = lane > 0 ? up : prev_hi;
+        const int32_t j = lane + 32 * u;
+        if (j >= 1 && j < nd && kfv[u] <= prev) dec = true;
+      }
+      const bool increasing = !__any_sync(0xffffffffu, dec);
       if (split == 0 && g == 0 && mtile == 0 && lane == 0) {
         L.seq_ok[b] = valid ? 1 : 0;
         if (!valid) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
@@ -374,6 +388,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         it.k_hi = k_hi;
         it.ntiles = ntiles;
         it.direct = ((Lk + L.kps - 1) / L.kps) == 1;
+        it.increasing = increasing ? 1 : 0;
       }
       __syncwarp();
       if (lane == 0) {
@@ -539,20 +554,29 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       // this row's draft and query head (computed once per item)
       const int32_t jq = live ? r / G : 0, h = g * G + (live ? r - (r / G) * G : 0);
       const int32_t qpos = live ? kflat[jq] : 0x7fffffff;
+      const bool increasing = it.increasing != 0;
       // cache slots below every query position of this item are visible to all rows
       int32_t minq = 0x7fffffff;
-      {
-        const int32_t j_lo = row0 / G, j_end = (min(rows_total, row0 + kBM) + G - 1) / G;
+      const int32_t j_lo = row0 / G;
+      if (increasing) {
+        minq = kflat[j_lo];
+      } else {
+        const int32_t j_end = (min(rows_total, row0 + kBM) + G - 1) / G;
         for (int32_t j = j_lo + lane; j < j_end; j += 32) minq = min(minq, kflat[j]);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) minq = min(minq, __shfl_xor_sync(0xffffffffu, minq, o));
       }
       const int32_t mask_from = min(cache, minq + 1);
       // visibility of the item's drafts to this row: bit j of (vis_hi:vis_lo) is
-      // kflat[j] <= qpos.  Runs once per item, so the loop is kept rolled (small
-      // code: a cold unrolled path costs instruction-cache misses).
+      // kflat[j] <= qpos, that is j <= jq for increasing positions.  Runs once
+      // per item, so the general loop is kept rolled (small code: a cold
+      // unrolled path costs instruction-cache misses).
       uint64_t vis_lo = 0, vis_hi = 0;
-      if (warp_live) {
+      if (warp_live && increasing) {
+        const int32_t n = jq + 1;  // 1 .. 128
+        vis_lo = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
+        vis_hi = n <= 64 ? 0ull : (n >= 128 ? ~0ull : ((1ull << (n - 64)) - 1ull));
+      } else if (warp_live) {
         const int32_t nd = Lk - cache;
 #pragma unroll 1
         for (int j = 0; j < nd; j += 4) {
@@ -749,7 +773,7 @@ EncodeTiledFnTc encode_tc() {
 }  // namespace
 
 #ifndef SSD_ATTN_TC_MIN_ROWS
-#define SSD_ATTN_TC_MIN_ROWS 64  // query rows per KV group above which the tcgen05 kernel runs
+#define SSD_ATTN_TC_MIN_ROWS 0  // query rows per KV group above which the tcgen05 kernel runs
 #endif
 
 bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max) {

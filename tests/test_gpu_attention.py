@@ -124,12 +124,15 @@ def test_head_dim_64_gqa_tensor_core_path(ssd):
 
 
 def test_mma_sync_and_tensor_core_paths_agree(ssd):
-    """The same MHA problem on both kernels: 48 drafts per sequence (mma.sync)
-    and the identical heads split as 2 query heads per KV head with 96 rows per
-    group (tcgen05); both must match the oracle."""
-    c = synth.make_case("mha48", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
-                        Hq=16, Hkv=16, d=128, V=64, seed=10, with_logits=False)
+    """Related problems on both kernels: 3 query heads per KV head (128 is not
+    a multiple of 3: mma.sync), and MHA and 2 heads per KV head on the same
+    caches (tcgen05); all must match the oracle."""
+    c = synth.make_case("gqa3", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
+                        Hq=12, Hkv=4, d=128, V=64, seed=10, with_logits=False)
     check_case(ssd, c)
+    c1 = synth.make_case("mha48", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
+                         Hq=16, Hkv=16, d=128, V=64, seed=10, with_logits=False)
+    check_case(ssd, c1)
     c2 = synth.make_case("gqa96", grid_h=24, grid_w=24, prefix_len=120, cache_len=[120, 408],
                          Hq=16, Hkv=8, d=128, V=64, seed=10, with_logits=False)
     check_case(ssd, c2)
@@ -168,3 +171,54 @@ def test_tensor_core_bad_draft_position_skips_only_its_sequence(ssd):
             if n:
                 assert attention_error(o[b, :n, h], o_ref[:, h]) < ATTN_TOL, f"b={b} h={h}"
     assert not o[3].any()  # the bad sequence is not written
+
+
+def _check_permuted_frontier(ssd, c):
+    """The drafts of every sequence in a shuffled order (valid, not increasing
+    positions): the kernels take the general visibility path.  The oracle gets
+    the same draft order."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(13)
+    perms = {}
+
+    def permute(pos):
+        host = pos.cpu().numpy()
+        nd_all = [len(ostep.sequence_frontier(c.grid_h, c.grid_w, c.prefix_len, c.cache_len[b],
+                                             c.k_v)[0]) for b in range(c.B)]
+        for b in range(c.B):
+            n = nd_all[b]
+            perms[b] = rng.permutation(n)
+            host[b, :n] = host[b, :n][perms[b]]
+        pos.copy_(torch.from_numpy(host))
+
+    o, lse, nd, st = run_attention(ssd, c, edit_pos=permute)
+    assert st == 0
+    q, k, v = bf16_to_f64(c.q), bf16_to_f64(c.k), bf16_to_f64(c.v)
+    for b in range(c.B):
+        coords, _ = ostep.sequence_frontier(c.grid_h, c.grid_w, c.prefix_len, c.cache_len[b], c.k_v)
+        n = len(coords)
+        if n == 0:
+            continue
+        pc = [coords[i] for i in perms[b]]
+        o_ref, lse_ref = oatt.verify_attention(q[b, :n], k[b], v[b], int(c.cache_len[b]), pc,
+                                               c.prefix_len, c.row_stride, c.Hq, c.Hkv)
+        for h in range(c.Hq):
+            assert attention_error(o[b, :n, h], o_ref[:, h]) < ATTN_TOL, f"b={b} h={h}"
+            assert np.abs(lse[b, h, :n] - lse_ref[h]).max() < 2e-2
+
+
+def test_tensor_core_shuffled_draft_order(ssd):
+    _check_permuted_frontier(ssd, _gqa_batch(6, 14))
+
+
+def test_mma_sync_shuffled_draft_order(ssd):
+    # 3 query heads per KV head: the mma.sync kernel
+    c = synth.make_case("gqa3_shuffled", grid_h=24, grid_w=24, prefix_len=120,
+                        cache_len=[120, 144, 408, 672], Hq=12, Hkv=4, d=128, V=64, seed=15,
+                        with_logits=False)
+    _check_permuted_frontier(ssd, c)
+
+
+def test_sweep_shape_shuffled_draft_order(ssd):
+    c = synth.config2(points=[120, 144, 408, 672], with_logits=False)
+    _check_permuted_frontier(ssd, c)
