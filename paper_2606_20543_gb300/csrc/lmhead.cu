@@ -13,7 +13,8 @@
 //    each epilogue thread owns one row's 128 logits of the tile;
 //  * A = hidden states (K-major), B = weights (MN-major: the vocabulary is
 //    contiguous in W[K][V]); both staged by TMA with the 128-byte swizzle
-//    through a 3-stage mbarrier ring, one thread producing, one thread
+//    through a 3-stage mbarrier ring, two threads producing (hidden states;
+//    weights, one copy per tile through a 3D view), one thread
 //    issuing tcgen05.mma (bf16 x bf16 -> fp32) into two TMEM accumulators
 //    (target, draft), tcgen05.commit releasing each stage;
 //  * epilogue: tcgen05.ld of each row's tile, per-tile softmax partials to a
@@ -228,25 +229,37 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   // mbarrier in the same warp would let a suspended try_wait of theirs hold
   // up the lane that drives the pipeline.
   if (warp == 0) {
-    if (lane == 0) {
+    // Lane 0 issues the hidden-state tiles, lane 1 the two weight tiles (one
+    // copy each through the 3D view {64, K, V / 64}): one thread issues only a
+    // few million copies per second.
+    if (lane < 2) {
     const uint64_t pol = policy_evict_first();     // weights: read once
     const uint64_t pol_h = policy_evict_last();    // hidden states: read by every CTA
     const uint32_t bytes = (uint32_t)stage_bytes;
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % S;
-      if (kb >= S && !mbar_wait(&empty[s], ((kb / S) - 1) & 1, a.status)) { *fail = 1; break; }
-      unsigned char* st = smem + s * stage_bytes;
-      mbar_arrive_expect_tx(&full[s], bytes);
-      for (int m = 0; m < mt; ++m) {
-        tma_load_2d(st + m * kTileA, &tmHt, kb * kBK, m * kBM, &full[s], pol_h);
-        tma_load_2d(st + (mt + m) * kTileA, &tmHd, kb * kBK, m * kBM, &full[s], pol_h);
+      int stop = 0;
+      if (lane == 0) {
+        if (kb >= S && !mbar_wait(&empty[s], ((kb / S) - 1) & 1, a.status)) {
+          *fail = 1;
+          stop = 1;
+        } else {
+          mbar_arrive_expect_tx(&full[s], bytes);
+        }
       }
-      unsigned char* bt = st + 2 * mt * kTileA;
-      unsigned char* bd = bt + kTileB;
-      tma_load_2d(bt, &tmWt, v0, kb * kBK, &full[s], pol);
-      tma_load_2d(bt + kTileB / 2, &tmWt, v0 + 64, kb * kBK, &full[s], pol);
-      tma_load_2d(bd, &tmWd, v0, kb * kBK, &full[s], pol);
-      tma_load_2d(bd + kTileB / 2, &tmWd, v0 + 64, kb * kBK, &full[s], pol);
+      stop = __shfl_sync(0x3u, stop, 0);  // the stage is free and its bytes expected
+      if (stop) break;
+      unsigned char* st = smem + s * stage_bytes;
+      if (lane == 0) {
+        for (int m = 0; m < mt; ++m) {
+          tma_load_2d(st + m * kTileA, &tmHt, kb * kBK, m * kBM, &full[s], pol_h);
+          tma_load_2d(st + (mt + m) * kTileA, &tmHd, kb * kBK, m * kBM, &full[s], pol_h);
+        }
+      } else {
+        unsigned char* bt = st + 2 * mt * kTileA;
+        tma_load_3d(bt, &tmWt, 0, kb * kBK, v0 / 64, &full[s], pol);
+        tma_load_3d(bt + kTileB, &tmWd, 0, kb * kBK, v0 / 64, &full[s], pol);
+      }
     }
     }
     __syncwarp();
@@ -609,6 +622,21 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// bf16 [K][V] weights as the 3D view {64 vocabulary entries, K rows, V / 64
+// column blocks} (the last dimension steps 128 B along a row); a box
+// {64, kBK, 2} is one CTA's [2 blocks][kBK rows][128 B] weight tile in one copy.
+bool make_weight_map(CUtensorMap* map, const void* base, uint64_t V, uint64_t K) {
+  EncodeTiledFn fn = encode_fn_l();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[3] = {64, K, V / 64};
+  cuuint64_t strides[2] = {V * 2, 128};
+  cuuint32_t box[3] = {64, kBK, kBN / 64};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 
 int row_tiles(int32_t rows) { return (rows + kBM - 1) / kBM; }
@@ -662,11 +690,11 @@ cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaSt
   L.mass = reinterpret_cast<float*>(w);
   CUtensorMap ht, hd, wt, wd;
   // hidden [rows][K]: boxes of 128 rows (rows past `rows` read as zero);
-  // weights [K][V]: boxes of 64 K-rows x 64 vocabulary entries
+  // weights [K][V]: boxes of 64 K-rows x 128 vocabulary entries (3D view)
   if (!make_map(&ht, a.h_tgt, (uint64_t)a.K, (uint64_t)a.rows, kBM) ||
       !make_map(&hd, a.h_drf, (uint64_t)a.K, (uint64_t)a.rows, kBM) ||
-      !make_map(&wt, a.w_tgt, (uint64_t)a.V, (uint64_t)a.K, kBK) ||
-      !make_map(&wd, a.w_drf, (uint64_t)a.V, (uint64_t)a.K, kBK))
+      !make_weight_map(&wt, a.w_tgt, (uint64_t)a.V, (uint64_t)a.K) ||
+      !make_weight_map(&wd, a.w_drf, (uint64_t)a.V, (uint64_t)a.K))
     return cudaErrorInvalidValue;
   cudaError_t e = cudaMemsetAsync(L.barrier, 0, sizeof(unsigned int), stream);
   if (e != cudaSuccess) return e;
