@@ -7,9 +7,11 @@
 // Design (GB300): for one row of W grid columns the predictor is a chain of
 // skinny products (rows <= a few hundred) that stream 268 MB of weights per
 // head plus the 4096 x V GenHead, so it is bound by HBM, not by the tensor
-// cores.  The four projections are plain GEMMs and run as cuBLAS bf16 GEMMs
-// (fp32 accumulation on the tensor cores, fp32 or bf16 outputs); everything
-// between them is a kernel of this file, and the data flow needs no copies:
+// cores.  The four projections and the GenHead are plain GEMMs and run as
+// cuBLAS bf16 GEMMs (fp32 accumulation on the tensor cores, fp32 outputs);
+// everything between them is a kernel of this file (float4 accesses, several
+// loads in flight per thread: these kernels are latency-bound at a few dozen
+// rows), and the data flow needs no copies:
 //   H  = W0 z                 GEMM into the caller's hidden-state buffer (fp32)
 //   At = RMSNorm(H) * gamma1  rmsnorm_kernel (bf16, the next GEMM's input)
 //   UV = At [W1 | W3]^T       two GEMMs into the halves of one fp32 buffer
@@ -47,18 +49,31 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 
 // One CTA per row: y = x / sqrt(mean(x^2) + eps) * gamma, rounded to bf16.
+// float4 accesses, unrolled so that several loads are in flight (d % 4 == 0).
 __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __restrict__ x,
                                                                const float* __restrict__ gamma,
                                                                float eps, int32_t d,
                                                                __nv_bfloat16* __restrict__ y) {
   __shared__ float red[32];
-  const float* xr = x + (int64_t)blockIdx.x * d;
-  __nv_bfloat16* yr = y + (int64_t)blockIdx.x * d;
+  const float4* xr = reinterpret_cast<const float4*>(x + (int64_t)blockIdx.x * d);
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  uint2* yr = reinterpret_cast<uint2*>(y + (int64_t)blockIdx.x * d);
+  const int32_t n4 = d >> 2;
   float ss = 0.f;
-  for (int32_t i = threadIdx.x; i < d; i += blockDim.x) ss += xr[i] * xr[i];
+#pragma unroll 4
+  for (int32_t i = threadIdx.x; i < n4; i += blockDim.x) {
+    const float4 v = xr[i];
+    ss += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
+  }
   const float inv = 1.0f / sqrtf(block_sum(ss, red) / (float)d + eps);
-  for (int32_t i = threadIdx.x; i < d; i += blockDim.x)
-    yr[i] = __float2bfloat16_rn(xr[i] * inv * gamma[i]);
+#pragma unroll 4
+  for (int32_t i = threadIdx.x; i < n4; i += blockDim.x) {
+    const float4 v = xr[i], gm = g4[i];
+    uint2 o;
+    o.x = pack_bf16x2(v.x * inv * gm.x, v.y * inv * gm.y);
+    o.y = pack_bf16x2(v.z * inv * gm.z, v.w * inv * gm.w);
+    yr[i] = o;
+  }
 }
 
 // g = silu(u) * v over rows x m; uv holds [u | v] per row (2m floats).
@@ -73,18 +88,23 @@ __global__ void swiglu_kernel(const float* __restrict__ uv, int32_t rows, int32_
   }
 }
 
-// One CTA per row: the first index of the maximum logit.
+// One CTA per row: the first index of the maximum logit (V % 4 == 0; float4
+// loads, unrolled so that several are in flight).
 __global__ void __launch_bounds__(kNormThreads) argmax_kernel(const float* __restrict__ logits,
                                                               int32_t V,
                                                               int32_t* __restrict__ out_tok) {
   __shared__ float sv[32];
   __shared__ int32_t si[32];
-  const float* lr = logits + (int64_t)blockIdx.x * V;
+  const float4* lr = reinterpret_cast<const float4*>(logits + (int64_t)blockIdx.x * V);
   float bv = -INFINITY;
   int32_t bi = 0x7fffffff;
-  for (int32_t i = threadIdx.x; i < V; i += blockDim.x) {
-    const float v = lr[i];
-    if (v > bv) { bv = v; bi = i; }  // ascending i per thread: first max kept
+#pragma unroll 4
+  for (int32_t i = threadIdx.x; i < (V >> 2); i += blockDim.x) {
+    const float4 v = lr[i];  // ascending index per thread: the first maximum is kept
+    if (v.x > bv) { bv = v.x; bi = 4 * i; }
+    if (v.y > bv) { bv = v.y; bi = 4 * i + 1; }
+    if (v.z > bv) { bv = v.z; bi = 4 * i + 2; }
+    if (v.w > bv) { bv = v.w; bi = 4 * i + 3; }
   }
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
@@ -115,15 +135,6 @@ cublasStatus_t blas_handle(cublasHandle_t* out) {
   }
   *out = handles[dev];
   return CUBLAS_STATUS_SUCCESS;
-}
-
-// Row-major Y[rows][N] (+)= X[rows][K] W[N][K]^T  (torch Linear layout), as the
-// column-major product Y^T = W X^T.
-cublasStatus_t linear(cublasHandle_t h, int32_t rows, int32_t N, int32_t K, const void* X,
-                      const void* W, float beta, void* Y, cudaDataType ytype) {
-  const float alpha = 1.0f;
-  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, N, rows, K, &alpha, W, CUDA_R_16BF, K, X,
-                      CUDA_R_16BF, K, &beta, Y, ytype, N, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
 }
 
 size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -159,37 +170,42 @@ cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
   float* H = p.out_hidden;
   if (H == nullptr) H = reinterpret_cast<float*>(w);
 
+  const int32_t rows = p.rows, d = p.d, m = p.m;
+  const int swg_blocks = (int)std::min<int64_t>(((int64_t)rows * m + 255) / 256,
+                                                4 * (int64_t)device_sm_count());
   cublasHandle_t h;
   if (blas_handle(&h) != CUBLAS_STATUS_SUCCESS) return cudaErrorUnknown;
   if (cublasSetStream(h, stream) != CUBLAS_STATUS_SUCCESS ||
       cublasSetWorkspace(h, blas_ws, kBlasWorkspace) != CUBLAS_STATUS_SUCCESS)
     return cudaErrorUnknown;
-  const int32_t rows = p.rows, d = p.d, m = p.m;
-  const int swg_blocks = (int)std::min<int64_t>(((int64_t)rows * m + 255) / 256,
-                                                4 * (int64_t)device_sm_count());
+  // Y[rows][N] (ld ldy) = (accumulate ? Y : 0) + X[rows][K] op(W); W [N][K]
+  // (a linear layer's [out][in], as the column-major product Y^T = W X^T), or
+  // [K][N] when w_kn
+  auto product = [&](int32_t N, int32_t K, const void* x, const void* w, bool w_kn, float* y,
+                     int32_t ldy, bool accumulate) -> cudaError_t {
+    const float alpha = 1.0f, beta = accumulate ? 1.0f : 0.0f;
+    const cublasStatus_t st =
+        w_kn ? cublasGemmEx(h, CUBLAS_OP_N, CUBLAS_OP_N, N, rows, K, &alpha, w, CUDA_R_16BF, N, x,
+                            CUDA_R_16BF, K, &beta, y, CUDA_R_32F, ldy, CUBLAS_COMPUTE_32F,
+                            CUBLAS_GEMM_DEFAULT)
+             : cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, N, rows, K, &alpha, w, CUDA_R_16BF, K, x,
+                            CUDA_R_16BF, K, &beta, y, CUDA_R_32F, ldy, CUBLAS_COMPUTE_32F,
+                            CUBLAS_GEMM_DEFAULT);
+    return st == CUBLAS_STATUS_SUCCESS ? cudaSuccess : cudaErrorUnknown;
+  };
+  cudaError_t e;
   // H = W0 z
-  if (linear(h, rows, d, 2 * d, p.z, p.w0, 0.f, H, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
+  if ((e = product(d, 2 * d, p.z, p.w0, false, H, d, false)) != cudaSuccess) return e;
   rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma1, p.eps, d, nrm);
-  // [U | V] = At [W1 | W3]^T: two GEMMs into the halves of each row of uv
-  const float alpha = 1.0f, zero = 0.0f;
-  if (cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, rows, d, &alpha, p.w1, CUDA_R_16BF, d, nrm,
-                   CUDA_R_16BF, d, &zero, uv, CUDA_R_32F, 2 * m, CUBLAS_COMPUTE_32F,
-                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS ||
-      cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, rows, d, &alpha, p.w3, CUDA_R_16BF, d, nrm,
-                   CUDA_R_16BF, d, &zero, uv + m, CUDA_R_32F, 2 * m, CUBLAS_COMPUTE_32F,
-                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
+  // [U | V] = At [W1 | W3]^T: two products into the halves of each row of uv
+  if ((e = product(m, d, nrm, p.w1, false, uv, 2 * m, false)) != cudaSuccess) return e;
+  if ((e = product(m, d, nrm, p.w3, false, uv + m, 2 * m, false)) != cudaSuccess) return e;
   swiglu_kernel<<<swg_blocks, 256, 0, stream>>>(uv, rows, m, g);
-  // H = H + G W2^T
-  if (linear(h, rows, d, m, g, p.w2, 1.f, H, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
+  // H = H + G W2^T (the residual)
+  if ((e = product(d, m, g, p.w2, false, H, d, true)) != cudaSuccess) return e;
   rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma2, p.eps, d, nrm);
-  // logits[rows][V] = Hn[rows][d] W_head[d][V]: column-major L^T = W_head^T' Hn^T
-  if (cublasGemmEx(h, CUBLAS_OP_N, CUBLAS_OP_N, p.V, rows, d, &alpha, p.w_head, CUDA_R_16BF, p.V,
-                   nrm, CUDA_R_16BF, d, &zero, logits, CUDA_R_32F, p.V, CUBLAS_COMPUTE_32F,
-                   CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
+  // logits[rows][V] = Hn[rows][d] W_head[d][V]
+  if ((e = product(p.V, d, nrm, p.w_head, true, logits, p.V, false)) != cudaSuccess) return e;
   argmax_kernel<<<rows, kNormThreads, 0, stream>>>(logits, p.V, p.out_tok);
   return cudaGetLastError();
 }

@@ -86,3 +86,14 @@ def test_predictor_without_hidden_output(ssd):
     w, g1, g2 = _case(90, rows, d, m, V)
     tok, _ = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6, with_hidden=False)
     _check(w, g1, g2, 1e-6, tok, None)
+
+
+@pytest.mark.parametrize("rows,d,m,V", [(128, 256, 512, 2048), (130, 256, 512, 2048),
+                                        (1, 128, 256, 256)])
+def test_predictor_row_limits(ssd, rows, d, m, V):
+    """128 rows (the tcgen05 products' largest tile), 130 (the cuBLAS path)
+    and a single row."""
+    w, g1, g2 = _case(90 + rows, rows, d, m, V)
+    tok, hid = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6)
+    ties = _check(w, g1, g2, 1e-6, tok, hid)
+    assert ties <= max(1, rows // 10)
