@@ -177,8 +177,9 @@ class ClockSampler:
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
     ("accept", 2): ("accept.cu", "5ccfccad7a2ff8ae", 152415232 + 3548416, 1128),
-    ("attention", 3): ("attention_tc.cu", "6ca0a2b87c88eb22", 53335296 + 427520, None),
-    ("lmhead_accept", 4): ("lmhead.cu", "a5b28d8ac7ea5800", 269327616 + 3034112, None),
+    ("attention", 2): ("attention_tc.cu", "90f7f3d45983421a", 102310144 + 2746368, None),
+    ("attention", 3): ("attention_tc.cu", "90f7f3d45983421a", 53837312 + 197632, None),
+    ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
 }
 
 
