@@ -362,12 +362,14 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
     attn_ms = timed(lambda i, cs: ssd.ssd_verify_attention(
         s.g, c.B, c.Hq, c.Hkv, c.d, s.cache_len, s.n_drafts, s.draft_pos, c.D_max, c.L_max, s.q,
         s.k, s.v, 0.0, s.o, None, ws, wsb, s.status, cs))
-    acc_ms = timed(lambda i, cs: ssd.ssd_accept(
-        c.B * c.D_max, c.V, dpool[i % 2][0], dpool[i % 2][1], c.V, None, 1.0, ssd.rng(seed, i),
-        s.out_tok, s.accepted, s.ratio, None, s.status, cs))
+    def acc_call(i, cs):  # the step's acceptance part (decisions, committed draws, counts)
+        s.args.tgt_logits, s.args.drf_logits = dpool[i % 2][0].data_ptr(), dpool[i % 2][1].data_ptr()
+        s.set_rng(seed, i)
+        ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes, cs)
+
+    acc_ms = timed(acc_call)
     nd0 = s.n_drafts.cpu().numpy()
-    attn_bytes, _ = algorithmic_bytes(c, nd0)
-    acc_bytes = c.B * c.D_max * (2 * c.V * 4 + 9)
+    attn_bytes, acc_bytes = algorithmic_bytes(c, nd0)
     kern = {"attention": (attn_bytes, attn_ms), "accept": (acc_bytes, acc_ms)}
     dom = max(kern, key=lambda k: kern[k][1])
     hbm_peak, peak_kind = measured_peaks()
@@ -732,9 +734,8 @@ def main():
             ssd.ssd_lmhead_accept(c.B * c.D_max, c.V, c.hidden, s.h_tgt, s.h_drf, s.w_tgt,
                                   s.w_drf, None, 1.0, s.rng, s.out_tok, s.accepted, s.ratio, None,
                                   lm_ws, lm_wsb, s.status, cs)
-        else:
-            ssd.ssd_accept_strategy(a.strategy, c.B * c.D_max, c.V, s.tgt, s.drf, c.V, None, 1.0,
-                                    s.rng, s.out_tok, s.accepted, s.ratio, None, s.status, cs)
+        else:  # the step's acceptance part as the step launches it (decisions, draws, counts)
+            ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes, cs)
 
     def kernel_ms(call):
         gr = torch.cuda.CUDAGraph()
@@ -755,11 +756,12 @@ def main():
     attn_ms = kernel_ms(attn_call)
     acc_ms = kernel_ms(acc_call)
     hbm_peak, peak_kind = measured_peaks()
-    # the standalone acceptance call processes every row of the padded batch
+    # the standalone fused call processes every row of the padded batch; the
+    # logits path's acceptance part reads the frontier's rows (and bonus rows)
     if c.hidden:
         acc_bytes_all = 2 * c.hidden * c.V * 2 + c.B * c.D_max * (2 * c.hidden * 2 + 9)
     else:
-        acc_bytes_all = c.B * c.D_max * (2 * c.V * 4 + 4 + 1 + 4)
+        acc_bytes_all = acc_bytes
     kern = {"attention": (attn_bytes, attn_ms),
             ("lmhead_accept" if c.hidden else "accept"): (acc_bytes_all, acc_ms)}
     dom = max(kern, key=lambda k: kern[k][1])

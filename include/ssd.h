@@ -85,7 +85,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 5
+#define SSD_ABI_VERSION 6
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -322,6 +322,15 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * ref_rows is written (the draft row, or the target row when the row is
  * not accepted), so no pass over ref_rows is needed before a block.
  * commit: an ssd_commit; the counts' next_cache_len follows it.
+ * Draws: under strategy (C) from logits with commit SSD_COMMIT_PREFIX or
+ * SSD_COMMIT_PREFIX_BONUS and no ref_rows, the step draws only the token it
+ * commits: the residual token of each sequence's first rejected draft, or
+ * the bonus token when every draft is accepted.  out_tok of the other
+ * rejected rows (never committed: the drafts after the first rejection are
+ * discarded) and of an uncommitted bonus row is -1; accepted and ratio are
+ * written for every row.  The committed token is the one the full draw
+ * (ssd_accept_strategy) gives for that row, bit for bit.  The other commit
+ * rules, ref_rows, strategies (A) and (B) and the fused path draw every row.
  * Streams: the attention runs on `stream`; the acceptance, which shares no
  * data with it, runs concurrently on a side stream the library creates once
  * per device and host thread (with two events) and joins back into `stream`
@@ -374,6 +383,17 @@ size_t ssd_verify_step_workspace(const ssd_verify_args* args);
 int32_t ssd_verify_step_launches(const ssd_verify_args* args);
 ssd_status ssd_verify_step(const ssd_verify_args* args, const ssd_verify_out* out,
                            void* workspace, size_t workspace_bytes, ssd_stream_t stream);
+
+/* a3-a5 and a7 of ssd_verify_step() on their own, on `stream` alone: the
+ * acceptance (and committed draws) of a frontier whose out->n_drafts is
+ * already set (by ssd_frontier() or an earlier step), then the counts.
+ * Uses args->grid, B, D_max, V, cache_len, the logits (or hidden-state)
+ * fields, draft_tok, temperature, rng, strategy, ref_rows, ref_init and
+ * commit; the attention fields and out->draft_pos, o and lse are ignored.
+ * workspace: ssd_verify_step_workspace(args) bytes are enough (may be NULL
+ * when the acceptance part needs none).  Errors as ssd_verify_step(). */
+ssd_status ssd_verify_accept(const ssd_verify_args* args, const ssd_verify_out* out,
+                             void* workspace, size_t workspace_bytes, ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * The spatial draft predictor (Sec. 3.3 "Draft Prediction in Latent Space",

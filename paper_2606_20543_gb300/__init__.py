@@ -26,7 +26,8 @@ EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_
             "ssd_accept_round", "ssd_stage_shift", "ssd_draft_predict_workspace",
             "ssd_draft_predict",
             "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
-            "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step"]
+            "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step",
+            "ssd_verify_accept"]
 
 
 STRATEGY_ACCEPT_REJECT, STRATEGY_GREEDY, STRATEGY_SAMPLE = 0, 1, 2
@@ -117,6 +118,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_verify_step_workspace": (SZ, [ctypes.POINTER(VerifyArgs)]),
         "ssd_verify_step_launches": (I32, [ctypes.POINTER(VerifyArgs)]),
         "ssd_verify_step": (I32, [ctypes.POINTER(VerifyArgs), ctypes.POINTER(VerifyOut), P, SZ, P]),
+        "ssd_verify_accept": (I32, [ctypes.POINTER(VerifyArgs), ctypes.POINTER(VerifyOut), P, SZ, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -276,4 +278,10 @@ def ssd_verify_step_launches(args: VerifyArgs) -> int:
 def ssd_verify_step(args: VerifyArgs, out: VerifyOut, workspace, workspace_bytes,
                     stream=None) -> None:
     _check("ssd_verify_step", load().ssd_verify_step(
+        ctypes.byref(args), ctypes.byref(out), _ptr(workspace), workspace_bytes, _stream(stream)))
+
+
+def ssd_verify_accept(args: VerifyArgs, out: VerifyOut, workspace, workspace_bytes,
+                      stream=None) -> None:
+    _check("ssd_verify_accept", load().ssd_verify_accept(
         ctypes.byref(args), ctypes.byref(out), _ptr(workspace), workspace_bytes, _stream(stream)))

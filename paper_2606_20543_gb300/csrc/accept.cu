@@ -285,6 +285,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   }
   __syncthreads();
 
+  // (A) never draws and lazy (C) leaves its draws to launch_resolve: one pass
+  const int32_t passes = (STRATEGY == SSD_STRATEGY_GREEDY || a.lazy) ? 1 : 2;
+
   // ------------------------------------------------------------ producer warp
   if (warp == kCWarps) {
     if (lane == 0) {
@@ -296,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         // the next round while this row's second pass is still being issued
         const float* drow =
             (a.ref_rows != nullptr && !a.ref_init) ? a.ref_rows[r] : a.drf + r * a.ld;
-        for (int32_t cc = 0; cc < 2 * nch; ++cc, ++g) {  // two passes over the row
+        for (int32_t cc = 0; cc < passes * nch; ++cc, ++g) {  // one or two passes over the row
           const int32_t ch = cc % nch;
           const int s = g % kStages;
           if (g >= kStages) mbar_wait(&sh.empty[s], ((g / kStages) - 1) & 1, a.status);
@@ -331,6 +334,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         if (kind == 1 && a.lse) { a.lse[2 * r] = 0.f; a.lse[2 * r + 1] = 0.f; }
         if (kind == 2) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         if (a.ref_rows != nullptr && a.ref_init) a.ref_rows[r] = a.drf + r * a.ld;
+        if (a.lazy) a.stats[r] = make_float2(NAN, NAN);
       }
       continue;
     }
@@ -477,6 +481,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
         sh.u_res = u.y;
         sh.Cp = Mp * c + lsp;
         sh.Cq = 0.f;
+        if (a.lazy) {  // drawn by launch_resolve if every draft is accepted
+          a.out_tok[r] = -1;
+          a.stats[r] = make_float2(sh.Cp, 0.f);
+        }
         a.accepted[r] = 1;
         if (a.ratio) a.ratio[r] = 0.f;
         if (a.lse) {
@@ -531,6 +539,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
           a.accepted[r] = 0;
           a.out_tok[r] = -1;
         }
+        if (a.lazy) {  // a rejected row's token is drawn by launch_resolve if committed
+          if (sh.accept == 0) a.out_tok[r] = -1;
+          a.stats[r] = valid_t ? make_float2(sh.Cp, sh.Cq) : make_float2(NAN, NAN);
+        }
         if (a.ratio) a.ratio[r] = ratio;
         if (a.lse) {
           a.lse[2 * r] = Mp / a.temperature + lsp * kLn2;
@@ -539,6 +551,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       }
     }
     consumers_sync();
+    if (passes == 1) continue;  // uniform; sh is rewritten only after the next row's pass A
     const bool draw = (sh.accept == 0);
     const float2 ncp = make_float2(-sh.Cp, -sh.Cp), ncq = make_float2(-sh.Cq, -sh.Cq);
 
@@ -604,6 +617,109 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   }
 }
 
+// One CTA per sequence after a lazy acceptance pass: warp 0 takes the counts,
+// then, if the counts commit a drawn token — the residual token of the first
+// rejected draft, or the bonus token after a fully accepted horizontal
+// frontier — every warp computes the residual mass of its 256-entry blocks
+// with the arithmetic of pass B (the same lane layout, weights and warp
+// sums, so every block mass is bit-identical) and warp 0 scans and re-walks
+// them exactly as the eager kernel does for that row.
+constexpr int kRWarps = 16;
+constexpr int kRBatch = 4;  // blocks per warp whose loads are issued together
+
+// Block masses of one row, block bk = warp, warp + kRWarps, ...
+__device__ __forceinline__ void resolve_masses(const float4* tp, const float4* dp, int32_t nblocks,
+                                               int32_t nv, float2 cc, float2 ncp, float2 ncq,
+                                               bool from_p, float* mass, int32_t warp, int lane) {
+  for (int32_t b0 = warp; b0 < nblocks; b0 += kRBatch * kRWarps) {
+    float4 xp[kRBatch][2], xq[kRBatch][2];
+#pragma unroll
+    for (int k = 0; k < kRBatch; ++k) {
+      const int32_t bk = b0 + k * kRWarps;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int32_t i = bk * 64 + half * 32 + lane;
+        const bool in = bk < nblocks && i < nv;
+        xp[k][half] = in ? tp[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+        xq[k][half] = (in && !from_p) ? dp[i] : xp[k][half];
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kRBatch; ++k) {
+      const int32_t bk = b0 + k * kRWarps;
+      if (bk >= nblocks) break;  // warp-uniform
+      float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
+      if (bk * 64 + lane < nv) w0 = weights4(xp[k][0], xq[k][0], cc, ncp, ncq, from_p);
+      if (bk * 64 + 32 + lane < nv) w1 = weights4(xp[k][1], xq[k][1], cc, ncp, ncq, from_p);
+      const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
+      if (lane == 0) mass[bk] = m;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kRWarps * 32) resolve_kernel(ResolveArgs a) {
+  extern __shared__ __align__(16) float rmass[];  // [nblocks]
+  __shared__ int32_t s_row;
+  const int32_t b = blockIdx.x;
+  const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int32_t n = a.n_drafts[b];
+  if (n < 0 || n > a.D_max) {  // a caller's frontier (ssd_verify_accept) out of range
+    if (tid == 0) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+    n = n < 0 ? 0 : a.D_max;
+  }
+  if (warp == 0) {
+    const int32_t prefix = sequence_counts(a.grid, a.commit, b, a.D_max, a.cache_len, n,
+                                           a.accepted, a.accepted_count, a.accepted_prefix,
+                                           a.next_cache_len, lane);
+    if (lane == 0) {
+      int32_t j = -1;
+      if (n > 0 && prefix < n) j = prefix;                              // first rejected draft
+      else if (a.bonus && n > 0 && prefix == n && n < a.D_max) j = n;   // the bonus row
+      s_row = j;
+    }
+  }
+  __syncthreads();
+  const int32_t j = s_row;
+  if (j < 0) return;  // uniform
+  const int64_t r = (int64_t)b * a.D_max + j;
+  const float2 st = a.stats[r];
+  if (!(st.x == st.x)) return;  // NaN: an invalid row, reported by the acceptance pass
+  const bool is_bonus = j == n;
+  const float c = kLog2e / a.temperature;
+  const float2 cc = make_float2(c, c);
+  const float2 ncp = make_float2(-st.x, -st.x), ncq = make_float2(-st.y, -st.y);
+  const int32_t nv = a.V >> 2;
+  const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;
+  const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
+  const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
+  const float u_res = row_uniforms(a.rng, r).y;
+
+  resolve_masses(tp, dp, nblocks, nv, cc, ncp, ncq, is_bonus, rmass, warp, lane);
+  __syncthreads();
+  float tb = 0.f;
+  int32_t bk = -1;
+  if (warp == 0) bk = find_block(rmass, nblocks, u_res, &tb, lane);
+  bool from_p = is_bonus;
+  if (!is_bonus && __syncthreads_or(warp == 0 && bk < 0 && lane == 0)) {
+    // zero residual mass: the same draw from p (block masses of p itself)
+    from_p = true;
+    resolve_masses(tp, tp, nblocks, nv, cc, ncp, ncq, true, rmass, warp, lane);
+    __syncthreads();
+    if (warp == 0) bk = find_block(rmass, nblocks, u_res, &tb, lane);
+  }
+  if (warp != 0) return;
+  if (bk < 0) {
+    if (lane == 0) {  // no positive mass at all (non-finite logits)
+      a.out_tok[r] = -1;
+      if (is_bonus) a.accepted[r] = 0;
+      record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+    }
+    return;
+  }
+  const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
+  if (lane == 0) a.out_tok[r] = pick;
+}
+
 }  // namespace
 
 bool accept_supported(int32_t V) { return V <= kMaxV; }
@@ -626,6 +742,17 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
     case SSD_STRATEGY_SAMPLE: return launch(accept_kernel<SSD_STRATEGY_SAMPLE>);
     default: return launch(accept_kernel<SSD_STRATEGY_ACCEPT_REJECT>);
   }
+}
+
+cudaError_t launch_resolve(const ResolveArgs& a, cudaStream_t stream) {
+  if (a.B == 0) return cudaSuccess;
+  const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;
+  const size_t smem = (size_t)nblocks * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(resolve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  resolve_kernel<<<a.B, kRWarps * 32, smem, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace ssd

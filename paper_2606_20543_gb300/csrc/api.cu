@@ -379,13 +379,147 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
   return from_cuda(launch_lmhead(a, workspace, workspace_bytes, (cudaStream_t)stream));
 }
 
+}  // extern "C"
+
+namespace {
+
+// Strategy (C) under a prefix rule, one round, from logits: only the tokens
+// the counts commit are drawn (AcceptArgs::lazy).
+bool lazy_draws(const ssd_verify_args* x) {
+  return x->tgt_logits != nullptr && x->strategy == SSD_STRATEGY_ACCEPT_REJECT &&
+         x->ref_rows == nullptr &&
+         (x->commit == SSD_COMMIT_PREFIX || x->commit == SSD_COMMIT_PREFIX_BONUS);
+}
+
+// Workspace of the acceptance part (a3-a7) of a step.  From logits: the
+// per-row normalisers of a lazy pass, counted under every strategy and
+// commit rule so that one workspace serves a VerifyStep's buffers in any mode.
+size_t accept_part_workspace(const ssd_verify_args* x) {
+  if (x->tgt_logits == nullptr && x->w_tgt != nullptr)
+    return align256(ssd_lmhead_accept_workspace(x->B * x->D_max, x->V));
+  return align256((size_t)x->B * x->D_max * sizeof(float2));
+}
+
+// Argument checks of the acceptance part, shared by ssd_verify_step and
+// ssd_verify_accept (shapes of the grid and the batch checked by the caller).
+ssd_status check_accept_part(const ssd_verify_args* x, const ssd_verify_out* y) {
+  if (x->cache_len == nullptr) return SSD_ERR_INVALID_ARG;
+  if (y->n_drafts == nullptr || y->out_tok == nullptr || y->accepted == nullptr ||
+      y->accepted_count == nullptr || y->accepted_prefix == nullptr ||
+      y->next_cache_len == nullptr || y->status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  const int32_t rows = x->B * x->D_max;
+  ssd_status s =
+      check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
+  if (s != SSD_OK) return s;
+  if (!strategy_ok(x->strategy)) return SSD_ERR_INVALID_ARG;
+  if (x->commit < SSD_COMMIT_PREFIX || x->commit > SSD_COMMIT_PREFIX_BONUS) return SSD_ERR_INVALID_ARG;
+  if (x->ref_init != 0 && (x->ref_rows == nullptr || x->drf_logits == nullptr))
+    return SSD_ERR_INVALID_ARG;
+  if (x->tgt_logits == nullptr) {
+    if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
+      return SSD_ERR_INVALID_ARG;
+    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT || x->ref_rows != nullptr ||
+        x->commit == SSD_COMMIT_PREFIX_BONUS)
+      return SSD_ERR_UNSUPPORTED;
+    return lmhead_check(rows, x->V, x->hidden);
+  }
+  return check_logits(rows, x->V, x->tgt_logits, x->drf_logits, x->ld);
+}
+
+// a3-a7 on one stream: acceptance from logits or through the fused lm_head,
+// then the counts (with the committed draws when lazy).  `ws` holds
+// accept_part_workspace(x) bytes.
+cudaError_t launch_accept_part(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
+                               size_t ws_bytes, cudaStream_t stream) {
+  const int32_t rows = x->B * x->D_max;
+  const bool lazy = lazy_draws(x);
+  cudaError_t e;
+  if (x->tgt_logits == nullptr) {
+    LmHeadArgs h;
+    h.rows = rows;
+    h.V = x->V;
+    h.K = x->hidden;
+    h.h_tgt = x->h_tgt;
+    h.h_drf = x->h_drf;
+    h.w_tgt = x->w_tgt;
+    h.w_drf = x->w_drf;
+    h.draft_tok = x->draft_tok;
+    h.temperature = x->temperature;
+    h.rng = x->rng;
+    h.out_tok = y->out_tok;
+    h.accepted = y->accepted;
+    h.ratio = y->ratio;
+    h.lse = nullptr;
+    h.status = y->status;
+    h.n_drafts = y->n_drafts;
+    h.D_max = x->D_max;
+    e = launch_lmhead(h, ws, ws_bytes, stream);
+  } else {
+    AcceptArgs c;
+    c.rows = rows;
+    c.V = x->V;
+    c.tgt = x->tgt_logits;
+    c.drf = x->drf_logits;
+    c.ld = x->ld;
+    c.draft_tok = x->draft_tok;
+    c.temperature = x->temperature;
+    c.rng = x->rng;
+    c.out_tok = y->out_tok;
+    c.accepted = y->accepted;
+    c.ratio = y->ratio;
+    c.lse = nullptr;
+    c.status = y->status;
+    c.n_drafts = y->n_drafts;
+    c.D_max = x->D_max;
+    c.strategy = x->strategy;
+    c.ref_rows = x->ref_rows;
+    c.ref_init = x->ref_init;
+    c.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
+    c.lazy = lazy ? 1 : 0;
+    c.stats = lazy ? static_cast<float2*>(ws) : nullptr;
+    e = launch_accept(c, stream);
+    if (e != cudaSuccess) return e;
+    if (lazy) {
+      ResolveArgs r;
+      r.grid = x->grid;
+      r.commit = x->commit;
+      r.B = x->B;
+      r.D_max = x->D_max;
+      r.V = x->V;
+      r.tgt = x->tgt_logits;
+      r.drf = x->drf_logits;
+      r.ld = x->ld;
+      r.temperature = x->temperature;
+      r.rng = x->rng;
+      r.cache_len = x->cache_len;
+      r.n_drafts = y->n_drafts;
+      r.stats = c.stats;
+      r.bonus = c.bonus;
+      r.out_tok = y->out_tok;
+      r.accepted = y->accepted;
+      r.accepted_count = y->accepted_count;
+      r.accepted_prefix = y->accepted_prefix;
+      r.next_cache_len = y->next_cache_len;
+      r.status = y->status;
+      return launch_resolve(r, stream);  // a7 with the committed draws
+    }
+  }
+  if (e != cudaSuccess) return e;
+  // a7: counts and the next cache length
+  return launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted,
+                       y->accepted_count, y->accepted_prefix, y->next_cache_len, y->status,
+                       stream);
+}
+
+}  // namespace
+
+extern "C" {
+
 size_t ssd_verify_step_workspace(const ssd_verify_args* x) {
   if (x == nullptr || x->B <= 0) return 0;
-  size_t bytes = align256(ssd_verify_attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max,
-                                                         x->L_max));
-  if (x->tgt_logits == nullptr && x->w_tgt != nullptr)
-    bytes += align256(ssd_lmhead_accept_workspace(x->B * x->D_max, x->V));
-  return bytes;
+  return align256(ssd_verify_attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max)) +
+         accept_part_workspace(x);
 }
 
 int32_t ssd_verify_step_launches(const ssd_verify_args* x) {
@@ -393,7 +527,7 @@ int32_t ssd_verify_step_launches(const ssd_verify_args* x) {
   if (check_attention(&x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max) != SSD_OK) return -1;
   if (x->B == 0) return 0;
   // frontier + attention (+ split combine) + acceptance + counts
-  return 3 + attention_launches(x->B, x->Hq, x->Hkv, x->D_max, x->L_max);
+  return 3 + attention_launches(x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max);
 }
 
 ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, void* workspace,
@@ -405,32 +539,10 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   if (x->grid.row_stride != x->grid.grid_w) return SSD_ERR_UNSUPPORTED;
   if ((int64_t)(x->grid.k_v + 1) * x->grid.grid_w > x->D_max) return SSD_ERR_SHAPE;
   if (x->B == 0) return SSD_OK;
-  if (x->cache_len == nullptr || x->q == nullptr || x->k == nullptr || x->v == nullptr)
-    return SSD_ERR_INVALID_ARG;
-  if (y->n_drafts == nullptr || y->draft_pos == nullptr || y->o == nullptr ||
-      y->out_tok == nullptr || y->accepted == nullptr || y->accepted_count == nullptr ||
-      y->accepted_prefix == nullptr || y->next_cache_len == nullptr || y->status == nullptr)
-    return SSD_ERR_INVALID_ARG;
-  const int32_t rows = x->B * x->D_max;
-  s = check_accept_common(rows, x->V, x->temperature, &x->rng, y->out_tok, y->accepted, y->status);
+  if (x->q == nullptr || x->k == nullptr || x->v == nullptr) return SSD_ERR_INVALID_ARG;
+  if (y->draft_pos == nullptr || y->o == nullptr) return SSD_ERR_INVALID_ARG;
+  s = check_accept_part(x, y);
   if (s != SSD_OK) return s;
-  if (!strategy_ok(x->strategy)) return SSD_ERR_INVALID_ARG;
-  if (x->commit < SSD_COMMIT_PREFIX || x->commit > SSD_COMMIT_PREFIX_BONUS) return SSD_ERR_INVALID_ARG;
-  if (x->ref_init != 0 && (x->ref_rows == nullptr || x->drf_logits == nullptr))
-    return SSD_ERR_INVALID_ARG;
-  const bool fused = (x->tgt_logits == nullptr);
-  if (fused) {
-    if (x->h_tgt == nullptr || x->h_drf == nullptr || x->w_tgt == nullptr || x->w_drf == nullptr)
-      return SSD_ERR_INVALID_ARG;
-    if (x->strategy != SSD_STRATEGY_ACCEPT_REJECT || x->ref_rows != nullptr ||
-        x->commit == SSD_COMMIT_PREFIX_BONUS)
-      return SSD_ERR_UNSUPPORTED;
-    s = lmhead_check(rows, x->V, x->hidden);
-    if (s != SSD_OK) return s;
-  } else {
-    s = check_logits(rows, x->V, x->tgt_logits, x->drf_logits, x->ld);
-    if (s != SSD_OK) return s;
-  }
   if (!(x->scale >= 0.f) || !isfinite(x->scale)) return SSD_ERR_INVALID_ARG;
   const size_t need = ssd_verify_step_workspace(x);
   if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
@@ -468,60 +580,28 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   a.status = y->status;
   e = launch_attention(a, ws, attn_ws, stream);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
-  // a3-a6: acceptance
-  if (fused) {
-    LmHeadArgs h;
-    h.rows = rows;
-    h.V = x->V;
-    h.K = x->hidden;
-    h.h_tgt = x->h_tgt;
-    h.h_drf = x->h_drf;
-    h.w_tgt = x->w_tgt;
-    h.w_drf = x->w_drf;
-    h.draft_tok = x->draft_tok;
-    h.temperature = x->temperature;
-    h.rng = x->rng;
-    h.out_tok = y->out_tok;
-    h.accepted = y->accepted;
-    h.ratio = y->ratio;
-    h.lse = nullptr;
-    h.status = y->status;
-    h.n_drafts = y->n_drafts;
-    h.D_max = x->D_max;
-    e = launch_lmhead(h, ws + attn_ws, workspace_bytes - attn_ws, side->stream);
-  } else {
-    AcceptArgs c;
-    c.rows = rows;
-    c.V = x->V;
-    c.tgt = x->tgt_logits;
-    c.drf = x->drf_logits;
-    c.ld = x->ld;
-    c.draft_tok = x->draft_tok;
-    c.temperature = x->temperature;
-    c.rng = x->rng;
-    c.out_tok = y->out_tok;
-    c.accepted = y->accepted;
-    c.ratio = y->ratio;
-    c.lse = nullptr;
-    c.status = y->status;
-    c.n_drafts = y->n_drafts;
-    c.D_max = x->D_max;
-    c.strategy = x->strategy;
-    c.ref_rows = x->ref_rows;
-    c.ref_init = x->ref_init;
-    c.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
-    e = launch_accept(c, side->stream);
-  }
+  // a3-a7: acceptance and counts on the side stream
+  e = launch_accept_part(x, y, ws + attn_ws, workspace_bytes - attn_ws, side->stream);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
-  // join: the counts need the decisions
+  // join: every output is ordered on `stream`
   if (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
       cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess)
     return SSD_ERR_CUDA;
-  // a7: counts and the next cache length
-  e = launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted,
-                    y->accepted_count,
-                    y->accepted_prefix, y->next_cache_len, stream);
-  return from_cuda(e);
+  return SSD_OK;
+}
+
+ssd_status ssd_verify_accept(const ssd_verify_args* x, const ssd_verify_out* y, void* workspace,
+                             size_t workspace_bytes, ssd_stream_t stream) {
+  if (x == nullptr || y == nullptr) return SSD_ERR_INVALID_ARG;
+  ssd_status s = check_grid(&x->grid);
+  if (s != SSD_OK) return s;
+  if (x->B < 0 || x->D_max <= 0) return SSD_ERR_SHAPE;
+  if (x->B == 0) return SSD_OK;
+  s = check_accept_part(x, y);
+  if (s != SSD_OK) return s;
+  const size_t need = accept_part_workspace(x);
+  if (need > 0 && (workspace == nullptr || workspace_bytes < need)) return SSD_ERR_WORKSPACE;
+  return from_cuda(launch_accept_part(x, y, workspace, workspace_bytes, (cudaStream_t)stream));
 }
 
 }  // extern "C"

@@ -428,9 +428,13 @@ struct Plan {
   bool tc;  // tcgen05 kernel (attention_tc.cu)
 };
 
-Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max, int32_t L_max) {
+// `rows_hint` (<= D_max) bounds the drafts a sequence can have in this launch;
+// it chooses between the two kernels only, both of which size their work by
+// D_max, so a wrong hint costs time, never correctness.
+Plan make_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max, int32_t L_max,
+               int32_t rows_hint) {
   Plan p;
-  p.tc = attention_tc_supported(Hq, Hkv, d, D_max);
+  p.tc = attention_tc_supported(Hq, Hkv, d, min(D_max, rows_hint));
   if (p.tc) {
     const TcPlan t = attention_tc_plan(B, Hq, Hkv, D_max, L_max);
     p.nwarps = 0;
@@ -466,12 +470,22 @@ int device_sm_count() {
   return n;
 }
 
+int32_t attention_rows_hint(const ssd_grid& g, int32_t D_max) {
+  if (g.grid_w <= 0 || g.k_h < 0 || g.k_v < 0) return D_max;
+  const int64_t h = g.k_h > 0 ? min(g.k_h, g.grid_w) : g.grid_w;
+  const int64_t n = h + (int64_t)g.k_v * g.grid_w;
+  return n < D_max ? (int32_t)n : D_max;
+}
+
+// Large enough for the plan of either kernel, so that the kernel choice (which
+// depends on the grid) never outgrows a workspace sized without it.
 size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
                            int32_t L_max) {
-  const Plan p = make_plan(B, Hq, Hkv, d, D_max, L_max);
   size_t bytes = align256((size_t)B * sizeof(int32_t));
-  if (p.splits > 1) {
-    const size_t prow = (size_t)B * Hq * D_max * p.splits;
+  int32_t splits = 1;
+  for (int32_t hint : {D_max, 0}) splits = max(splits, make_plan(B, Hq, Hkv, d, D_max, L_max, hint).splits);
+  if (splits > 1) {
+    const size_t prow = (size_t)B * Hq * D_max * splits;
     bytes += align256(prow * d * sizeof(float)) + align256(prow * sizeof(float));
   }
   return bytes;
@@ -479,14 +493,16 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
 
 static cudaError_t launch_combine(const AttnArgs& a, const AttnLaunch& L, cudaStream_t stream);
 
-int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
+int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                       int32_t D_max, int32_t L_max) {
   if (B == 0) return 0;
-  return make_plan(B, Hq, Hkv, 128, D_max, L_max).splits > 1 ? 2 : 1;
+  return make_plan(B, Hq, Hkv, d, D_max, L_max, attention_rows_hint(g, D_max)).splits > 1 ? 2 : 1;
 }
 
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
-  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max);
+  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
+                           attention_rows_hint(a.grid, a.D_max));
   AttnLaunch L;
   L.splits = p.splits;
   L.kps = p.kps;

@@ -773,7 +773,7 @@ EncodeTiledFnTc encode_tc() {
 }  // namespace
 
 #ifndef SSD_ATTN_TC_MIN_ROWS
-#define SSD_ATTN_TC_MIN_ROWS 0  // query rows per KV group above which the tcgen05 kernel runs
+#define SSD_ATTN_TC_MIN_ROWS 16  // query rows per KV group above which the tcgen05 kernel runs
 #endif
 
 bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max) {

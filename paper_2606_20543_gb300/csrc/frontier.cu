@@ -58,48 +58,16 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
                               const uint8_t* __restrict__ accepted,
                               int32_t* __restrict__ accepted_count,
                               int32_t* __restrict__ accepted_prefix,
-                              int32_t* __restrict__ next_cache_len) {
+                              int32_t* __restrict__ next_cache_len, int32_t* status) {
   const int32_t b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int32_t lane = threadIdx.x & 31;
   if (b >= B) return;
-  const int32_t n = n_drafts[b];
-  int32_t count = 0, prefix = 0;
-  bool run = true;  // still inside the leading accepted run
-  for (int32_t j0 = 0; j0 < n; j0 += 32) {
-    const int32_t j = j0 + lane;
-    const bool a = (j < n) && accepted[(int64_t)b * D_max + j] != 0;
-    const uint32_t acc_mask = __ballot_sync(0xffffffffu, a);
-    count += __popc(acc_mask);
-    if (run) {
-      const uint32_t valid = (n - j0 >= 32) ? 0xffffffffu : ((1u << (n - j0)) - 1u);
-      const uint32_t rejected = valid & ~acc_mask;
-      if (rejected) {
-        prefix += __ffs(rejected) - 1;
-        run = false;
-      } else {
-        prefix += __popc(valid);
-      }
-    }
+  int32_t n = n_drafts[b];
+  if (n < 0 || n > D_max) {  // a caller's frontier (ssd_verify_accept) out of range
+    if ((threadIdx.x & 31) == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
+    n = n < 0 ? 0 : D_max;
   }
-  if (lane == 0) {
-    accepted_count[b] = count;
-    accepted_prefix[b] = prefix;
-    int32_t advance = n > 0 ? min(prefix + 1, n) : 0;  // SSD_COMMIT_PREFIX
-    if (commit == SSD_COMMIT_NONE) {
-      advance = 0;
-    } else if (commit == SSD_COMMIT_BLOCK) {
-      advance = n;
-    } else if (commit == SSD_COMMIT_FIRST_ROW) {
-      const int32_t n_c = cache_len[b] - g.prefix_len;
-      advance = min(n, g.grid_w - n_c % g.grid_w);  // the frontier's first row
-    } else if (commit == SSD_COMMIT_PREFIX_BONUS) {
-      // horizontal stage: every draft accepted -> the bonus token as well, if
-      // the position after the last draft exists (and has a row slot)
-      const int32_t n_c = cache_len[b] - g.prefix_len;
-      if (n > 0 && prefix == n && n < D_max && n_c + n < g.grid_h * g.grid_w) advance = n + 1;
-    }
-    next_cache_len[b] = cache_len[b] + advance;
-  }
+  sequence_counts(g, commit, b, D_max, cache_len, n, accepted, accepted_count, accepted_prefix,
+                  next_cache_len, threadIdx.x & 31);
 }
 
 // Staged schedule: the trailing row (slots W .. 2W-1) becomes the frontier of
@@ -128,12 +96,13 @@ cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_l
 cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
                           const int32_t* cache_len, const int32_t* n_drafts,
                           const uint8_t* accepted, int32_t* accepted_count,
-                          int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream) {
+                          int32_t* accepted_prefix, int32_t* next_cache_len, int32_t* status,
+                          cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
   const int warps = 4;
   counts_kernel<<<(B + warps - 1) / warps, warps * 32, 0, stream>>>(
       g, commit, B, D_max, cache_len, n_drafts, accepted, accepted_count, accepted_prefix,
-      next_cache_len);
+      next_cache_len, status);
   return cudaGetLastError();
 }
 

@@ -13,11 +13,65 @@ cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_l
 cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
                           const int32_t* cache_len, const int32_t* n_drafts,
                           const uint8_t* accepted, int32_t* accepted_count,
-                          int32_t* accepted_prefix, int32_t* next_cache_len, cudaStream_t stream);
+                          int32_t* accepted_prefix, int32_t* next_cache_len, int32_t* status,
+                          cudaStream_t stream);
 // Staged schedule: slot j of every sequence takes slot W + j (j < W) of the
 // per-row tokens and reference pointers.
 cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
                                const float** ref_rows, cudaStream_t stream);
+
+// One warp: the counts of sequence b (a7) from its n drafts' accepted flags —
+// drafts accepted, the leading accepted run and the next cache length under
+// `commit` — written by lane 0; every lane returns the leading run.  The
+// drafts up to and including the first rejected one are committed (the
+// rejected one with its resampled token); SSD_COMMIT_NONE / _BLOCK /
+// _FIRST_ROW serve the verify-and-correct rounds, _PREFIX_BONUS the
+// horizontal stage (Sec. 3.3, Sec. 4).
+__device__ __forceinline__ int32_t sequence_counts(const ssd_grid& g, int32_t commit, int32_t b,
+                                                   int32_t D_max, const int32_t* cache_len,
+                                                   int32_t n, const uint8_t* accepted,
+                                                   int32_t* accepted_count,
+                                                   int32_t* accepted_prefix,
+                                                   int32_t* next_cache_len, int32_t lane) {
+  int32_t count = 0, prefix = 0;
+  bool run = true;  // still inside the leading accepted run
+  for (int32_t j0 = 0; j0 < n; j0 += 32) {
+    const int32_t j = j0 + lane;
+    const bool a = (j < n) && accepted[(int64_t)b * D_max + j] != 0;
+    const uint32_t acc_mask = __ballot_sync(0xffffffffu, a);
+    count += __popc(acc_mask);
+    if (run) {
+      const uint32_t valid = (n - j0 >= 32) ? 0xffffffffu : ((1u << (n - j0)) - 1u);
+      const uint32_t rejected = valid & ~acc_mask;
+      if (rejected) {
+        prefix += __ffs(rejected) - 1;
+        run = false;
+      } else {
+        prefix += __popc(valid);
+      }
+    }
+  }
+  if (lane == 0) {
+    accepted_count[b] = count;
+    accepted_prefix[b] = prefix;
+    int32_t advance = n > 0 ? min(prefix + 1, n) : 0;  // SSD_COMMIT_PREFIX
+    if (commit == SSD_COMMIT_NONE) {
+      advance = 0;
+    } else if (commit == SSD_COMMIT_BLOCK) {
+      advance = n;
+    } else if (commit == SSD_COMMIT_FIRST_ROW) {
+      const int32_t n_c = cache_len[b] - g.prefix_len;
+      advance = min(n, g.grid_w - n_c % g.grid_w);  // the frontier's first row
+    } else if (commit == SSD_COMMIT_PREFIX_BONUS) {
+      // horizontal stage: every draft accepted -> the bonus token as well, if
+      // the position after the last draft exists (and has a row slot)
+      const int32_t n_c = cache_len[b] - g.prefix_len;
+      if (n > 0 && prefix == n && n < D_max && n_c + n < g.grid_h * g.grid_w) advance = n + 1;
+    }
+    next_cache_len[b] = cache_len[b] + advance;
+  }
+  return prefix;
+}
 
 // ---- accept.cu
 struct AcceptArgs {
@@ -40,9 +94,41 @@ struct AcceptArgs {
                              // is set to its target row (the next round's reference)
   int32_t ref_init;          // round 1: references are the draft rows; every entry is written
   int32_t bonus;             // horizontal stage: row j == n_drafts[b] draws the bonus token
+  // Committed draws only (strategy (C) under the prefix rules, one round): the
+  // kernel takes each row's decision in one pass, leaves out_tok = -1 on
+  // rejected and bonus rows and writes the row's log2-domain normalisers
+  // (Cp, Cq) to stats[r] (NaN: nothing to draw); launch_resolve then draws
+  // the one token per sequence that the counts commit.
+  int32_t lazy = 0;
+  float2* stats = nullptr;   // [rows] when lazy
 };
 bool accept_supported(int32_t V);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);
+// After a lazy launch_accept on the same stream: per sequence b, the counts of
+// sequence_counts() and the draw of the committed token — the residual token
+// of the first rejected draft, or (bonus) the draw from p at the row after
+// the last draft when every draft was accepted — bit-identical to the draw
+// the eager kernel makes for that row.
+struct ResolveArgs {
+  ssd_grid grid;
+  int32_t commit, B, D_max, V;
+  const float* tgt;
+  const float* drf;
+  int64_t ld;
+  float temperature;
+  ssd_rng rng;
+  const int32_t* cache_len;
+  const int32_t* n_drafts;
+  const float2* stats;
+  int32_t bonus;
+  int32_t* out_tok;
+  uint8_t* accepted;
+  int32_t* accepted_count;
+  int32_t* accepted_prefix;
+  int32_t* next_cache_len;
+  int32_t* status;
+};
+cudaError_t launch_resolve(const ResolveArgs& a, cudaStream_t stream);
 
 // ---- attention.cu
 struct AttnArgs {
@@ -87,7 +173,12 @@ __device__ __forceinline__ int32_t longest_first(const AttnArgs& a, int32_t rank
 size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
                            int32_t L_max);
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
-int attention_launches(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
+int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                       int32_t D_max, int32_t L_max);
+// Most drafts one sequence can have under grid `g` (Sec. 3.3 frontier: at most
+// min(k_h, W) horizontal positions, or W - c with k_h = 0, then k_v rows of W),
+// clipped to D_max.
+int32_t attention_rows_hint(const ssd_grid& g, int32_t D_max);
 
 // ---- attention_tc.cu (tcgen05 frontier attention: query groups dividing 128,
 // more than 64 query rows per KV group)

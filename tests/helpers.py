@@ -26,6 +26,26 @@ def attention_error(o_gpu, o_ref):
     return np.abs(o_gpu - o_ref).max() / max(den, 1e-6)
 
 
+def committed_draws(dec, accepted, D_max):
+    """The oracle's decisions with the tokens a verification step draws under
+    strategy (C) and a prefix commit rule: only the first rejected draft of a
+    sequence carries its residual token; a later rejected draft is discarded
+    by the counts and left undrawn (-1).  The first rejection is the one the
+    GPU's accepted flags give (compare_decisions checks those flags against
+    the oracle's).  dec["rows"] ascends within each sequence."""
+    tok = np.array(dec["out_tok"], copy=True)
+    seen = set()
+    for k, r in enumerate(dec["rows"]):
+        b = int(r) // D_max
+        if not accepted[k]:
+            if b in seen:
+                tok[k] = -1
+            seen.add(b)
+    out = dict(dec)
+    out["out_tok"] = tok
+    return out
+
+
 def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what="", tol=PROB_TOL):
     """Bit-exact comparison of accept flags and tokens, except near-tie rows.
 

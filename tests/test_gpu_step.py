@@ -8,7 +8,7 @@ import torch
 import synth
 from oracle import step as ostep
 from oracle import frontier as ofr
-from tests.helpers import ATTN_TOL, attention_error, bf16_to_f64, compare_decisions
+from tests.helpers import ATTN_TOL, attention_error, bf16_to_f64, committed_draws, compare_decisions
 
 pytestmark = pytest.mark.gpu
 
@@ -40,7 +40,10 @@ def check_step(c, res, attention_seqs=None, strategy="accept_reject"):
     rows = ref["decisions"]["rows"]
     ties = 0
     if rows.size:
-        ties = compare_decisions(ref["decisions"], res["out_tok"][rows], res["accepted"][rows],
+        dec = ref["decisions"]
+        if strategy == "accept_reject":  # prefix rule: only the committed rejection is drawn
+            dec = committed_draws(dec, res["accepted"][rows], c.D_max)
+        ties = compare_decisions(dec, res["out_tok"][rows], res["accepted"][rows],
                                  res["ratio"][rows], what=c.name)
     # padding rows
     pad = np.setdiff1d(np.arange(c.B * c.D_max), rows)
@@ -206,12 +209,21 @@ def test_horizontal_stage_with_bonus(ssd, strategy):
         assert np.array_equal(res["n_drafts"], ref["n_drafts"])
         assert np.array_equal(res["n_drafts"], [5, 5, 3, 2, 5])
         rows = ref["decisions"]["rows"]
-        ties = compare_decisions(ref["decisions"], res["out_tok"][rows], res["accepted"][rows],
+        lazy = strategy == "accept_reject"  # draws only what the counts commit
+        dec = committed_draws(ref["decisions"], res["accepted"][rows], c.D_max) if lazy \
+            else ref["decisions"]
+        ties = compare_decisions(dec, res["out_tok"][rows], res["accepted"][rows],
                                  what=f"horizontal {strategy}")
         for b in range(c.B):
-            if ref["bonus_row"][b] >= 0 and not ref["bonus_tie"][b]:
-                assert res["out_tok"][ref["bonus_row"][b]] == ref["bonus_tok"][b]
-                assert res["accepted"][ref["bonus_row"][b]] == 1
+            br = ref["bonus_row"][b]
+            if br < 0:
+                continue
+            all_acc = res["accepted_prefix"][b] == res["n_drafts"][b]
+            if lazy and not all_acc:
+                assert res["out_tok"][br] == -1  # not committed: not drawn
+            elif not ref["bonus_tie"][b]:
+                assert res["out_tok"][br] == ref["bonus_tok"][b]
+                assert res["accepted"][br] == 1
         if ties == 0:
             assert np.array_equal(res["next_cache_len"], ref["next_cache_len"])
         if same and strategy != "sample":
@@ -219,3 +231,91 @@ def test_horizontal_stage_with_bonus(ssd, strategy):
             assert np.array_equal(res["next_cache_len"][[0, 1, 2, 4]],
                                   c.cache_len[[0, 1, 2, 4]] + res["n_drafts"][[0, 1, 2, 4]] + 1)
             assert res["next_cache_len"][3] == c.cache_len[3] + 2
+
+
+def _full_draw(ssd, s, c, strategy="accept_reject"):
+    """ssd_accept_strategy over every row of the padded batch with the step's
+    logits and uniforms: the full (eager) draw of every row."""
+    rows = c.B * c.D_max
+    out_tok = torch.full((rows,), -7, dtype=torch.int32, device="cuda")
+    acc = torch.zeros(rows, dtype=torch.uint8, device="cuda")
+    ratio = torch.zeros(rows, dtype=torch.float32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ssd.ssd_accept_strategy(strategy, rows, c.V, s.tgt, s.drf, c.V, None, 1.0, s.rng, out_tok,
+                            acc, ratio, None, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    return out_tok.cpu().numpy(), acc.cpu().numpy(), ratio.cpu().numpy()
+
+
+def test_committed_draw_is_the_full_draw_bit_for_bit(ssd):
+    """Under the prefix rule the step draws only each sequence's first
+    rejected draft; that token, every accept flag and every ratio are the
+    ones the full draw over every row gives, bit for bit (same block masses,
+    scan, re-walk and Philox counters), on a ragged multi-tile batch."""
+    c = synth.config2(points=[120, 192, 312, 480, 552, 648, 672, 696])
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    r = s.results()
+    tok_f, acc_f, ratio_f = _full_draw(ssd, s, c)
+    firsts = 0
+    for b in range(c.B):
+        n = int(r["n_drafts"][b])
+        rows = np.arange(b * c.D_max, b * c.D_max + n)
+        assert np.array_equal(r["accepted"][rows], acc_f[rows])
+        assert np.array_equal(r["ratio"][rows].view(np.uint32), ratio_f[rows].view(np.uint32))
+        rej = rows[acc_f[rows] == 0]
+        acc_rows = rows[acc_f[rows] == 1]
+        assert np.array_equal(r["out_tok"][acc_rows], tok_f[acc_rows])
+        if rej.size:
+            firsts += 1
+            assert r["out_tok"][rej[0]] == tok_f[rej[0]] >= 0
+            assert np.all(r["out_tok"][rej[1:]] == -1)
+            assert r["accepted_prefix"][b] == rej[0] - b * c.D_max
+    assert firsts >= c.B // 2  # the synthetic drafts are rejected early in most sequences
+
+
+def test_committed_bonus_is_the_full_draw_from_p(ssd):
+    """Horizontal stage with p = q (every draft accepted): the bonus row's
+    token is the draw from p that strategy (B) makes for that row."""
+    from paper_2606_20543_gb300.step import VerifyStep
+    H = W = 16
+    P = 32
+    cls = [P + 3, P + W * 2, P + W * 5 + 13, P + W * 7 + 11]
+    c = synth.make_case("horizontal", grid_h=H, grid_w=W, prefix_len=P, cache_len=cls, Hq=4,
+                        Hkv=4, d=64, V=4096, seed=62, k_v=0)
+    s = VerifyStep(H, W, P, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V, k_v=0, k_h=5,
+                   commit="prefix_bonus")
+    s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=c.drf_logits,
+             drf_logits=c.drf_logits, uniforms=c.uniforms)
+    s.run()
+    torch.cuda.synchronize()
+    r = s.results()
+    assert r["status"][0] == 0
+    tok_b, _, _ = _full_draw(ssd, s, c, "sample")
+    for b in range(c.B):
+        n = int(r["n_drafts"][b])
+        assert r["accepted_prefix"][b] == n
+        br = b * c.D_max + n
+        assert r["out_tok"][br] == tok_b[br] >= 0
+
+
+def test_verify_accept_matches_the_step(ssd):
+    """ssd_verify_accept (acceptance and counts of a drafted frontier, on one
+    stream) gives the step's outputs bit for bit."""
+    c = synth.config2(points=[120, 408, 696])
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    r = s.results()
+    for t in (s.out_tok, s.accepted, s.ratio, s.accepted_count, s.accepted_prefix,
+              s.next_cache_len):
+        t.fill_(0)
+    ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes)
+    torch.cuda.synchronize()
+    r2 = s.results()
+    for k in ("out_tok", "accepted", "accepted_count", "accepted_prefix", "next_cache_len",
+              "status"):
+        assert np.array_equal(r[k], r2[k]), k
+    assert np.array_equal(r["ratio"].view(np.uint32), r2["ratio"].view(np.uint32))
