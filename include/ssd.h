@@ -331,12 +331,19 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * written for every row.  The committed token is the one the full draw
  * (ssd_accept_strategy) gives for that row, bit for bit.  The other commit
  * rules, ref_rows, strategies (A) and (B) and the fused path draw every row.
- * Streams: the attention runs on `stream`; the acceptance, which shares no
- * data with it, runs concurrently on a side stream the library creates once
- * per device and host thread (with two events) and joins back into `stream`
- * before the counts, so all outputs are ordered on `stream` as usual.  Make
- * the first call on each device and host thread outside any stream capture;
- * later calls may be captured (the fork and join become graph edges).
+ * Streams: logits path — the acceptance pass computes the frontier itself
+ * (and writes n_drafts and draft_pos) and the attention computes the same
+ * frontier from cache_len.  With committed draws only and at least
+ * 2 x (SM count) rows, everything runs on `stream`: acceptance, attention,
+ * then the counts and committed draws as a programmatic dependent of the
+ * attention (they need only the acceptance's results, start once every
+ * attention CTA is resident and wait for the attention before they exit, so
+ * stream order holds).  Otherwise, and on the fused path (frontier first,
+ * lm_head acceptance), the acceptance and counts run on a side stream beside
+ * the attention, joined back into `stream`; the library creates that stream
+ * once per device and host thread (with two events).  Make the first call on
+ * each device and host thread outside any stream capture; later calls may
+ * be captured (the fork and join become graph edges).
  * ------------------------------------------------------------------------- */
 typedef struct {
   ssd_grid grid;
@@ -384,14 +391,14 @@ int32_t ssd_verify_step_launches(const ssd_verify_args* args);
 ssd_status ssd_verify_step(const ssd_verify_args* args, const ssd_verify_out* out,
                            void* workspace, size_t workspace_bytes, ssd_stream_t stream);
 
-/* a3-a5 and a7 of ssd_verify_step() on their own, on `stream` alone: the
- * acceptance (and committed draws) of a frontier whose out->n_drafts is
- * already set (by ssd_frontier() or an earlier step), then the counts.
- * Uses args->grid, B, D_max, V, cache_len, the logits (or hidden-state)
- * fields, draft_tok, temperature, rng, strategy, ref_rows, ref_init and
- * commit; the attention fields and out->draft_pos, o and lse are ignored.
- * workspace: ssd_verify_step_workspace(args) bytes are enough (may be NULL
- * when the acceptance part needs none).  Errors as ssd_verify_step(). */
+/* ssd_verify_step() without the attention (a1, a3-a5, a7), on `stream`
+ * alone: the frontier (written to out->n_drafts and out->draft_pos), the
+ * acceptance with its committed draws, and the counts.  Uses args->grid, B,
+ * D_max, V, cache_len, the logits (or hidden-state) fields, draft_tok,
+ * temperature, rng, strategy, ref_rows, ref_init and commit; Hq, Hkv, d,
+ * L_max, q, k, v, scale and out->o, out->lse are ignored.  workspace:
+ * ssd_verify_step_workspace(args) bytes are enough.  Errors as
+ * ssd_verify_step(). */
 ssd_status ssd_verify_accept(const ssd_verify_args* args, const ssd_verify_out* out,
                              void* workspace, size_t workspace_bytes, ssd_stream_t stream);
 

@@ -136,9 +136,10 @@ struct Shared {
 // last draft (kind 3).  Producer and consumers walk the same rows and skip
 // the same ones.
 __device__ __forceinline__ int row_kind(const AcceptArgs& a, int64_t r) {
-  if (a.n_drafts != nullptr) {
+  if (a.cache_len != nullptr || a.n_drafts != nullptr) {
     const int32_t b = (int32_t)(r / a.D_max), j = (int32_t)(r % a.D_max);
-    const int32_t n = a.n_drafts[b];
+    const int32_t n = a.cache_len != nullptr ? frontier_drafts(a.grid, a.cache_len[b], a.D_max)
+                                             : a.n_drafts[b];
     if (j >= n) return (a.bonus && j == n && n > 0) ? 3 : 1;  // bonus row / padding slot
   }
   if (a.draft_tok != nullptr) {
@@ -309,6 +310,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
           bulk_g2s(dst, a.tgt + r * a.ld + (int64_t)ch * kChunk, bytes, &sh.full[s]);
           bulk_g2s(dst + kChunk, drow + (int64_t)ch * kChunk, bytes, &sh.full[s]);
         }
+      }
+    } else if (a.cache_len != nullptr) {
+      // lanes 1-31: write the frontier of sequences blockIdx.x, + gridDim.x, ...
+      const int32_t B = (int32_t)(a.rows / a.D_max);
+      for (int32_t b = blockIdx.x; b < B; b += gridDim.x) {
+        const int32_t n = frontier_drafts(a.grid, a.cache_len[b], a.D_max);
+        const int32_t n_c = a.cache_len[b] - a.grid.prefix_len;
+        if (lane == 1) {
+          a.n_drafts_out[b] = n < 0 ? 0 : n;
+          if (a.tickets != nullptr) a.tickets[b] = 0;
+          if (n < 0) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+        }
+        for (int32_t j = lane - 1; j < a.D_max; j += 31)
+          a.draft_pos[(int64_t)b * a.D_max + j] = j < n ? n_c + j : -1;
       }
     }
     __syncwarp();
@@ -617,37 +632,39 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   }
 }
 
-// One CTA per sequence after a lazy acceptance pass: warp 0 takes the counts,
-// then, if the counts commit a drawn token — the residual token of the first
+// After a lazy acceptance pass: the counts and the one committed draw per
+// sequence.  Grid (parts, B), one warp per CTA, so that the CTAs fit in the
+// registers an attention kernel leaves free on an SM and run beside it.
+// Every CTA of sequence b takes the counts' leading run (part 0 writes the
+// counts); if they commit a drawn token — the residual token of the first
 // rejected draft, or the bonus token after a fully accepted horizontal
-// frontier — every warp computes the residual mass of its 256-entry blocks
-// with the arithmetic of pass B (the same lane layout, weights and warp
-// sums, so every block mass is bit-identical) and warp 0 scans and re-walks
-// them exactly as the eager kernel does for that row.
-constexpr int kRWarps = 16;
-constexpr int kRBatch = 4;  // blocks per warp whose loads are issued together
+// frontier — part k computes the residual masses of 256-entry blocks
+// [kRBlocks k, kRBlocks (k + 1)) with the arithmetic of pass B (same lane
+// layout, weights and warp sums, so every block mass is bit-identical) into
+// global memory; the last part to finish (a ticket per sequence) scans the
+// masses in vocabulary order and re-walks the chosen block exactly as the
+// eager kernel does for that row.
+constexpr int kRBlocks = 4;  // blocks per part
 
-// Block masses of one row, block bk = warp, warp + kRWarps, ...
-__device__ __forceinline__ void resolve_masses(const float4* tp, const float4* dp, int32_t nblocks,
-                                               int32_t nv, float2 cc, float2 ncp, float2 ncq,
-                                               bool from_p, float* mass, int32_t warp, int lane) {
-  for (int32_t b0 = warp; b0 < nblocks; b0 += kRBatch * kRWarps) {
-    float4 xp[kRBatch][2], xq[kRBatch][2];
+__device__ __forceinline__ void resolve_part_masses(const float4* tp, const float4* dp, int32_t bk0,
+                                                    int32_t bk1, int32_t nv, float2 cc, float2 ncp,
+                                                    float2 ncq, bool from_p, float* mass, int lane) {
+  for (int32_t b0 = bk0; b0 < bk1; b0 += 2) {
+    float4 xp[2][2], xq[2][2];
 #pragma unroll
-    for (int k = 0; k < kRBatch; ++k) {
-      const int32_t bk = b0 + k * kRWarps;
+    for (int k = 0; k < 2; ++k) {
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
-        const int32_t i = bk * 64 + half * 32 + lane;
-        const bool in = bk < nblocks && i < nv;
+        const int32_t i = (b0 + k) * 64 + half * 32 + lane;
+        const bool in = b0 + k < bk1 && i < nv;
         xp[k][half] = in ? tp[i] : make_float4(0.f, 0.f, 0.f, 0.f);
         xq[k][half] = (in && !from_p) ? dp[i] : xp[k][half];
       }
     }
 #pragma unroll
-    for (int k = 0; k < kRBatch; ++k) {
-      const int32_t bk = b0 + k * kRWarps;
-      if (bk >= nblocks) break;  // warp-uniform
+    for (int k = 0; k < 2; ++k) {
+      const int32_t bk = b0 + k;
+      if (bk >= bk1) break;  // warp-uniform
       float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
       if (bk * 64 + lane < nv) w0 = weights4(xp[k][0], xq[k][0], cc, ncp, ncq, from_p);
       if (bk * 64 + 32 + lane < nv) w1 = weights4(xp[k][1], xq[k][1], cc, ncp, ncq, from_p);
@@ -657,67 +674,71 @@ __device__ __forceinline__ void resolve_masses(const float4* tp, const float4* d
   }
 }
 
-__global__ void __launch_bounds__(kRWarps * 32) resolve_kernel(ResolveArgs a) {
-  extern __shared__ __align__(16) float rmass[];  // [nblocks]
-  __shared__ int32_t s_row;
-  const int32_t b = blockIdx.x;
-  const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+__global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
+  extern __shared__ __align__(16) float rmass[];  // [nblocks], last part only
+  const int32_t part = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
+  const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;  // resolve_blocks(V)
   int32_t n = a.n_drafts[b];
-  if (n < 0 || n > a.D_max) {  // a caller's frontier (ssd_verify_accept) out of range
-    if (tid == 0) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
-    n = n < 0 ? 0 : a.D_max;
+  const bool bad_n = n < 0 || n > a.D_max;  // a caller's frontier (ssd_verify_accept)
+  n = bad_n ? (n < 0 ? 0 : a.D_max) : n;
+  if (part == 0 && bad_n && lane == 0) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+  const int32_t prefix = sequence_counts(a.grid, a.commit, b, a.D_max, a.cache_len, n, a.accepted,
+                                         a.accepted_count, a.accepted_prefix, a.next_cache_len,
+                                         lane, part == 0);
+  int32_t j = -1;
+  if (n > 0 && prefix < n) j = prefix;                             // first rejected draft
+  else if (a.bonus && n > 0 && prefix == n && n < a.D_max) j = n;  // the bonus row
+  const int64_t r = (int64_t)b * a.D_max + (j < 0 ? 0 : j);
+  const float2 st = j < 0 ? make_float2(NAN, NAN) : a.stats[r];
+  if (!(st.x == st.x)) {  // nothing to draw, or an invalid row the acceptance pass reported
+    pdl_wait();
+    return;
   }
-  if (warp == 0) {
-    const int32_t prefix = sequence_counts(a.grid, a.commit, b, a.D_max, a.cache_len, n,
-                                           a.accepted, a.accepted_count, a.accepted_prefix,
-                                           a.next_cache_len, lane);
-    if (lane == 0) {
-      int32_t j = -1;
-      if (n > 0 && prefix < n) j = prefix;                              // first rejected draft
-      else if (a.bonus && n > 0 && prefix == n && n < a.D_max) j = n;   // the bonus row
-      s_row = j;
-    }
-  }
-  __syncthreads();
-  const int32_t j = s_row;
-  if (j < 0) return;  // uniform
-  const int64_t r = (int64_t)b * a.D_max + j;
-  const float2 st = a.stats[r];
-  if (!(st.x == st.x)) return;  // NaN: an invalid row, reported by the acceptance pass
   const bool is_bonus = j == n;
   const float c = kLog2e / a.temperature;
   const float2 cc = make_float2(c, c);
   const float2 ncp = make_float2(-st.x, -st.x), ncq = make_float2(-st.y, -st.y);
   const int32_t nv = a.V >> 2;
-  const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;
   const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
   const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
+  float* gmass = a.mass + (int64_t)b * nblocks;
+  const int32_t bk0 = part * kRBlocks, bk1 = min(nblocks, bk0 + kRBlocks);
+  resolve_part_masses(tp, dp, bk0, bk1, nv, cc, ncp, ncq, is_bonus, gmass, lane);
+  // last part to finish: its fence orders every part's masses before its ticket
+  __threadfence();
+  int32_t last = 0;
+  if (lane == 0) last = atomicAdd(&a.tickets[b], 1) == (int32_t)gridDim.x - 1;
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) {
+    pdl_wait();
+    return;
+  }
+  __threadfence();
+  for (int32_t k = lane; k < nblocks; k += 32) rmass[k] = __ldcg(gmass + k);
+  __syncwarp();
   const float u_res = row_uniforms(a.rng, r).y;
-
-  resolve_masses(tp, dp, nblocks, nv, cc, ncp, ncq, is_bonus, rmass, warp, lane);
-  __syncthreads();
   float tb = 0.f;
-  int32_t bk = -1;
-  if (warp == 0) bk = find_block(rmass, nblocks, u_res, &tb, lane);
+  int32_t bk = find_block(rmass, nblocks, u_res, &tb, lane);
   bool from_p = is_bonus;
-  if (!is_bonus && __syncthreads_or(warp == 0 && bk < 0 && lane == 0)) {
+  if (bk < 0 && !is_bonus) {
     // zero residual mass: the same draw from p (block masses of p itself)
     from_p = true;
-    resolve_masses(tp, tp, nblocks, nv, cc, ncp, ncq, true, rmass, warp, lane);
-    __syncthreads();
-    if (warp == 0) bk = find_block(rmass, nblocks, u_res, &tb, lane);
+    __syncwarp();
+    resolve_part_masses(tp, tp, 0, nblocks, nv, cc, ncp, ncq, true, rmass, lane);
+    __syncwarp();
+    bk = find_block(rmass, nblocks, u_res, &tb, lane);
   }
-  if (warp != 0) return;
   if (bk < 0) {
     if (lane == 0) {  // no positive mass at all (non-finite logits)
       a.out_tok[r] = -1;
       if (is_bonus) a.accepted[r] = 0;
       record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
     }
-    return;
+  } else {
+    const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
+    if (lane == 0) a.out_tok[r] = pick;
   }
-  const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
-  if (lane == 0) a.out_tok[r] = pick;
+  pdl_wait();  // under a programmatic launch: exit only after the kernel before it
 }
 
 }  // namespace
@@ -744,15 +765,17 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream) {
   }
 }
 
-cudaError_t launch_resolve(const ResolveArgs& a, cudaStream_t stream) {
+int32_t resolve_blocks(int32_t V) { return ((V + kChunk - 1) / kChunk) * kBlocksPerChunk; }
+
+cudaError_t launch_resolve(const ResolveArgs& a, bool pdl, cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
-  const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;
+  const int32_t nblocks = resolve_blocks(a.V);
   const size_t smem = (size_t)nblocks * sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(resolve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  resolve_kernel<<<a.B, kRWarps * 32, smem, stream>>>(a);
-  return cudaGetLastError();
+  const dim3 grid((unsigned)((nblocks + kRBlocks - 1) / kRBlocks), (unsigned)a.B);
+  return launch_kernel(resolve_kernel, grid, dim3(32), smem, stream, pdl, a);
 }
 
 }  // namespace ssd

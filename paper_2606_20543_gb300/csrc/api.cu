@@ -391,21 +391,39 @@ bool lazy_draws(const ssd_verify_args* x) {
          (x->commit == SSD_COMMIT_PREFIX || x->commit == SSD_COMMIT_PREFIX_BONUS);
 }
 
-// Workspace of the acceptance part (a3-a7) of a step.  From logits: the
-// per-row normalisers of a lazy pass, counted under every strategy and
-// commit rule so that one workspace serves a VerifyStep's buffers in any mode.
+// Workspace of the acceptance part (a3-a7) of a step.  Fused path: the
+// lm_head's.  Logits path: the per-row normalisers of a lazy pass, a ticket
+// per sequence and the block masses of the committed rows, counted under
+// every strategy and commit rule so that one workspace serves any mode.
+struct AcceptWs {
+  float2* stats;
+  int32_t* tickets;
+  float* mass;
+};
 size_t accept_part_workspace(const ssd_verify_args* x) {
   if (x->tgt_logits == nullptr && x->w_tgt != nullptr)
     return align256(ssd_lmhead_accept_workspace(x->B * x->D_max, x->V));
-  return align256((size_t)x->B * x->D_max * sizeof(float2));
+  return align256((size_t)x->B * x->D_max * sizeof(float2)) +
+         align256((size_t)x->B * sizeof(int32_t)) +
+         align256((size_t)x->B * resolve_blocks(x->V) * sizeof(float));
+}
+AcceptWs carve_accept(const ssd_verify_args* x, void* ws) {
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  AcceptWs c;
+  c.stats = reinterpret_cast<float2*>(w);
+  w += align256((size_t)x->B * x->D_max * sizeof(float2));
+  c.tickets = reinterpret_cast<int32_t*>(w);
+  w += align256((size_t)x->B * sizeof(int32_t));
+  c.mass = reinterpret_cast<float*>(w);
+  return c;
 }
 
 // Argument checks of the acceptance part, shared by ssd_verify_step and
 // ssd_verify_accept (shapes of the grid and the batch checked by the caller).
 ssd_status check_accept_part(const ssd_verify_args* x, const ssd_verify_out* y) {
   if (x->cache_len == nullptr) return SSD_ERR_INVALID_ARG;
-  if (y->n_drafts == nullptr || y->out_tok == nullptr || y->accepted == nullptr ||
-      y->accepted_count == nullptr || y->accepted_prefix == nullptr ||
+  if (y->n_drafts == nullptr || y->draft_pos == nullptr || y->out_tok == nullptr ||
+      y->accepted == nullptr || y->accepted_count == nullptr || y->accepted_prefix == nullptr ||
       y->next_cache_len == nullptr || y->status == nullptr)
     return SSD_ERR_INVALID_ARG;
   const int32_t rows = x->B * x->D_max;
@@ -427,89 +445,102 @@ ssd_status check_accept_part(const ssd_verify_args* x, const ssd_verify_out* y) 
   return check_logits(rows, x->V, x->tgt_logits, x->drf_logits, x->ld);
 }
 
-// a3-a7 on one stream: acceptance from logits or through the fused lm_head,
-// then the counts (with the committed draws when lazy).  `ws` holds
-// accept_part_workspace(x) bytes.
-cudaError_t launch_accept_part(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
-                               size_t ws_bytes, cudaStream_t stream) {
-  const int32_t rows = x->B * x->D_max;
+// Logits path, a1 + a3-a5: the acceptance pass, which computes the frontier
+// itself and writes it out (n_drafts, draft_pos).
+cudaError_t launch_accept_phase(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
+                                cudaStream_t stream) {
   const bool lazy = lazy_draws(x);
-  cudaError_t e;
-  if (x->tgt_logits == nullptr) {
-    LmHeadArgs h;
-    h.rows = rows;
-    h.V = x->V;
-    h.K = x->hidden;
-    h.h_tgt = x->h_tgt;
-    h.h_drf = x->h_drf;
-    h.w_tgt = x->w_tgt;
-    h.w_drf = x->w_drf;
-    h.draft_tok = x->draft_tok;
-    h.temperature = x->temperature;
-    h.rng = x->rng;
-    h.out_tok = y->out_tok;
-    h.accepted = y->accepted;
-    h.ratio = y->ratio;
-    h.lse = nullptr;
-    h.status = y->status;
-    h.n_drafts = y->n_drafts;
-    h.D_max = x->D_max;
-    e = launch_lmhead(h, ws, ws_bytes, stream);
-  } else {
-    AcceptArgs c;
-    c.rows = rows;
-    c.V = x->V;
-    c.tgt = x->tgt_logits;
-    c.drf = x->drf_logits;
-    c.ld = x->ld;
-    c.draft_tok = x->draft_tok;
-    c.temperature = x->temperature;
-    c.rng = x->rng;
-    c.out_tok = y->out_tok;
-    c.accepted = y->accepted;
-    c.ratio = y->ratio;
-    c.lse = nullptr;
-    c.status = y->status;
-    c.n_drafts = y->n_drafts;
-    c.D_max = x->D_max;
-    c.strategy = x->strategy;
-    c.ref_rows = x->ref_rows;
-    c.ref_init = x->ref_init;
-    c.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
-    c.lazy = lazy ? 1 : 0;
-    c.stats = lazy ? static_cast<float2*>(ws) : nullptr;
-    e = launch_accept(c, stream);
-    if (e != cudaSuccess) return e;
-    if (lazy) {
-      ResolveArgs r;
-      r.grid = x->grid;
-      r.commit = x->commit;
-      r.B = x->B;
-      r.D_max = x->D_max;
-      r.V = x->V;
-      r.tgt = x->tgt_logits;
-      r.drf = x->drf_logits;
-      r.ld = x->ld;
-      r.temperature = x->temperature;
-      r.rng = x->rng;
-      r.cache_len = x->cache_len;
-      r.n_drafts = y->n_drafts;
-      r.stats = c.stats;
-      r.bonus = c.bonus;
-      r.out_tok = y->out_tok;
-      r.accepted = y->accepted;
-      r.accepted_count = y->accepted_count;
-      r.accepted_prefix = y->accepted_prefix;
-      r.next_cache_len = y->next_cache_len;
-      r.status = y->status;
-      return launch_resolve(r, stream);  // a7 with the committed draws
-    }
-  }
+  const AcceptWs w = carve_accept(x, ws);
+  AcceptArgs c;
+  c.rows = x->B * x->D_max;
+  c.V = x->V;
+  c.tgt = x->tgt_logits;
+  c.drf = x->drf_logits;
+  c.ld = x->ld;
+  c.draft_tok = x->draft_tok;
+  c.temperature = x->temperature;
+  c.rng = x->rng;
+  c.out_tok = y->out_tok;
+  c.accepted = y->accepted;
+  c.ratio = y->ratio;
+  c.lse = nullptr;
+  c.status = y->status;
+  c.n_drafts = nullptr;
+  c.D_max = x->D_max;
+  c.strategy = x->strategy;
+  c.ref_rows = x->ref_rows;
+  c.ref_init = x->ref_init;
+  c.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
+  c.lazy = lazy ? 1 : 0;
+  c.stats = lazy ? w.stats : nullptr;
+  c.cache_len = x->cache_len;
+  c.grid = x->grid;
+  c.n_drafts_out = y->n_drafts;
+  c.draft_pos = y->draft_pos;
+  c.tickets = w.tickets;
+  return launch_accept(c, stream);
+}
+
+// Logits path, a7: the counts, with the committed draws after a lazy pass.
+cudaError_t launch_finish_phase(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
+                                bool pdl, cudaStream_t stream) {
+  if (!lazy_draws(x))
+    return launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts,
+                         y->accepted, y->accepted_count, y->accepted_prefix, y->next_cache_len,
+                         y->status, pdl, stream);
+  const AcceptWs w = carve_accept(x, ws);
+  ResolveArgs r;
+  r.grid = x->grid;
+  r.commit = x->commit;
+  r.B = x->B;
+  r.D_max = x->D_max;
+  r.V = x->V;
+  r.tgt = x->tgt_logits;
+  r.drf = x->drf_logits;
+  r.ld = x->ld;
+  r.temperature = x->temperature;
+  r.rng = x->rng;
+  r.cache_len = x->cache_len;
+  r.n_drafts = y->n_drafts;
+  r.stats = w.stats;
+  r.bonus = x->commit == SSD_COMMIT_PREFIX_BONUS;
+  r.out_tok = y->out_tok;
+  r.accepted = y->accepted;
+  r.accepted_count = y->accepted_count;
+  r.accepted_prefix = y->accepted_prefix;
+  r.next_cache_len = y->next_cache_len;
+  r.status = y->status;
+  r.tickets = w.tickets;
+  r.mass = w.mass;
+  return launch_resolve(r, pdl, stream);
+}
+
+// Fused path, a1 + a6 + a7 on one stream (the frontier already written).
+cudaError_t launch_fused_accept(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
+                                size_t ws_bytes, cudaStream_t stream) {
+  LmHeadArgs h;
+  h.rows = x->B * x->D_max;
+  h.V = x->V;
+  h.K = x->hidden;
+  h.h_tgt = x->h_tgt;
+  h.h_drf = x->h_drf;
+  h.w_tgt = x->w_tgt;
+  h.w_drf = x->w_drf;
+  h.draft_tok = x->draft_tok;
+  h.temperature = x->temperature;
+  h.rng = x->rng;
+  h.out_tok = y->out_tok;
+  h.accepted = y->accepted;
+  h.ratio = y->ratio;
+  h.lse = nullptr;
+  h.status = y->status;
+  h.n_drafts = y->n_drafts;
+  h.D_max = x->D_max;
+  cudaError_t e = launch_lmhead(h, ws, ws_bytes, stream);
   if (e != cudaSuccess) return e;
-  // a7: counts and the next cache length
   return launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted,
                        y->accepted_count, y->accepted_prefix, y->next_cache_len, y->status,
-                       stream);
+                       false, stream);
 }
 
 }  // namespace
@@ -526,8 +557,10 @@ int32_t ssd_verify_step_launches(const ssd_verify_args* x) {
   if (x == nullptr) return -1;
   if (check_attention(&x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max) != SSD_OK) return -1;
   if (x->B == 0) return 0;
-  // frontier + attention (+ split combine) + acceptance + counts
-  return 3 + attention_launches(x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max);
+  // logits: acceptance (with the frontier) + attention (+ split combine) + counts/draws;
+  // fused: frontier + attention (+ combine) + lm_head acceptance + counts
+  const int fixed = x->tgt_logits != nullptr ? 2 : 3;
+  return fixed + attention_launches(x->grid, x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max);
 }
 
 ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, void* workspace,
@@ -548,18 +581,6 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
   unsigned char* ws = static_cast<unsigned char*>(workspace);
   const size_t attn_ws = align256(attention_workspace(x->B, x->Hq, x->Hkv, x->d, x->D_max, x->L_max));
-  SideStream* side = nullptr;
-  if (side_stream(&side) != cudaSuccess) return SSD_ERR_CUDA;
-
-  // a1: frontier
-  cudaError_t e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts, y->draft_pos,
-                                  y->status, stream);
-  if (e != cudaSuccess) return SSD_ERR_CUDA;
-  // fork: acceptance on the side stream, after the frontier, beside the attention
-  if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
-      cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
-    return SSD_ERR_CUDA;
-  // a2: attention of the drafted block
   AttnArgs a;
   a.grid = x->grid;
   a.B = x->B;
@@ -578,12 +599,59 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   a.o = y->o;
   a.lse = y->lse;
   a.status = y->status;
+  cudaError_t e;
+  SideStream* side = nullptr;
+  if (x->tgt_logits != nullptr) {
+    // Logits path: the acceptance pass computes the frontier and writes it
+    // out (a1 + a3-a5); the attention computes the same frontier from
+    // cache_len (a2), so the two need no frontier launch before them.
+    a.raster = 1;
+    if (lazy_draws(x) && x->B * x->D_max >= 2 * device_sm_count()) {
+      // A lazy pass that fills the GPU, on `stream` alone: acceptance, then
+      // attention, then a7 (counts and the committed draws) as a programmatic
+      // dependent of the attention: it needs only the acceptance's results,
+      // starts once every attention CTA is resident and runs in the registers
+      // they leave free, beside them.
+      e = launch_accept_phase(x, y, ws + attn_ws, stream);
+      if (e != cudaSuccess) return SSD_ERR_CUDA;
+      e = launch_attention(a, ws, attn_ws, stream, /*defer_combine=*/true);
+      if (e != cudaSuccess) return SSD_ERR_CUDA;
+      e = launch_finish_phase(x, y, ws + attn_ws, /*pdl=*/true, stream);
+      if (e != cudaSuccess) return SSD_ERR_CUDA;
+      return from_cuda(launch_attention_combine(a, ws, stream));
+    }
+    // Otherwise the acceptance and a7 on a side stream beside the attention:
+    // kernels that do not fill the GPU, or that draw every row, overlap.
+    if (side_stream(&side) != cudaSuccess) return SSD_ERR_CUDA;
+    if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
+        cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
+      return SSD_ERR_CUDA;
+    // (the attention first: its persistent CTAs deal their items statically,
+    // while the acceptance's rows adapt to CTAs that start late)
+    e = launch_attention(a, ws, attn_ws, stream);
+    if (e != cudaSuccess) return SSD_ERR_CUDA;
+    e = launch_accept_phase(x, y, ws + attn_ws, side->stream);
+    if (e != cudaSuccess) return SSD_ERR_CUDA;
+    e = launch_finish_phase(x, y, ws + attn_ws, /*pdl=*/false, side->stream);
+    if (e != cudaSuccess) return SSD_ERR_CUDA;
+    if (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
+        cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess)
+      return SSD_ERR_CUDA;
+    return SSD_OK;
+  }
+  // Fused path: a1, then the attention on `stream` beside the lm_head
+  // acceptance and the counts on a side stream, joined back into `stream`.
+  if (side_stream(&side) != cudaSuccess) return SSD_ERR_CUDA;
+  e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts, y->draft_pos, y->status,
+                      stream);
+  if (e != cudaSuccess) return SSD_ERR_CUDA;
+  if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
+      cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
+    return SSD_ERR_CUDA;
   e = launch_attention(a, ws, attn_ws, stream);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
-  // a3-a7: acceptance and counts on the side stream
-  e = launch_accept_part(x, y, ws + attn_ws, workspace_bytes - attn_ws, side->stream);
+  e = launch_fused_accept(x, y, ws + attn_ws, workspace_bytes - attn_ws, side->stream);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
-  // join: every output is ordered on `stream`
   if (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
       cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess)
     return SSD_ERR_CUDA;
@@ -596,12 +664,23 @@ ssd_status ssd_verify_accept(const ssd_verify_args* x, const ssd_verify_out* y, 
   ssd_status s = check_grid(&x->grid);
   if (s != SSD_OK) return s;
   if (x->B < 0 || x->D_max <= 0) return SSD_ERR_SHAPE;
+  if (x->grid.row_stride != x->grid.grid_w) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)(x->grid.k_v + 1) * x->grid.grid_w > x->D_max) return SSD_ERR_SHAPE;
   if (x->B == 0) return SSD_OK;
   s = check_accept_part(x, y);
   if (s != SSD_OK) return s;
   const size_t need = accept_part_workspace(x);
-  if (need > 0 && (workspace == nullptr || workspace_bytes < need)) return SSD_ERR_WORKSPACE;
-  return from_cuda(launch_accept_part(x, y, workspace, workspace_bytes, (cudaStream_t)stream));
+  if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (x->tgt_logits == nullptr) {
+    cudaError_t e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts,
+                                    y->draft_pos, y->status, st);
+    if (e != cudaSuccess) return SSD_ERR_CUDA;
+    return from_cuda(launch_fused_accept(x, y, workspace, workspace_bytes, st));
+  }
+  cudaError_t e = launch_accept_phase(x, y, workspace, st);
+  if (e != cudaSuccess) return SSD_ERR_CUDA;
+  return from_cuda(launch_finish_phase(x, y, workspace, /*pdl=*/false, st));
 }
 
 }  // extern "C"

@@ -80,7 +80,7 @@ __device__ __forceinline__ bool load_draft_positions(const AttnArgs& a, int32_t 
                                                      int32_t* kflat, int32_t* bad) {
   const int32_t HW = a.grid.grid_h * a.grid.grid_w;
   for (int32_t j = threadIdx.x; j < nd; j += blockDim.x) {
-    const int32_t gidx = a.draft_pos[(int64_t)b * a.D_max + j];
+    const int32_t gidx = attn_draft_pos(a, b, j);
     if (gidx < 0 || gidx >= HW) {
       *bad = 1;
       kflat[j] = 0;
@@ -101,6 +101,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   constexpr int TILE_BYTES = KT * D * 2;       // one K (or V) tile
   constexpr int KSTEPS = D / 16;               // k16 steps of QK^T
   constexpr int NT_O = D / 8;                  // n8 tiles of O
+  pdl_launch_dependents();  // as in the tcgen05 kernel: a dependent may start beside it
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the swizzle atoms
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -120,7 +121,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
   const int32_t cache = a.cache_len[b];
-  const int32_t nd = a.n_drafts[b];
+  const int32_t nd = attn_drafts(a, b);
   const int32_t Lk = cache + nd;
   const bool shape_ok = !(nd < 0 || nd > a.D_max || cache < 0 || Lk > a.L_max);
   const int32_t rows_total = shape_ok ? nd * G : 0;
@@ -357,7 +358,7 @@ __global__ void attn_combine_kernel(AttnArgs a, AttnLaunch L) {
   const int32_t j = (int32_t)((gw / a.Hq) % a.D_max);
   const int32_t b = (int32_t)(gw / ((int64_t)a.Hq * a.D_max));
   if (!L.seq_ok[b]) return;
-  const int32_t nd = a.n_drafts[b];
+  const int32_t nd = attn_drafts(a, b);
   if (j >= nd) return;
   const int32_t Lk = a.cache_len[b] + nd;
   const int32_t n_active = (Lk + L.kps - 1) / L.kps;
@@ -499,10 +500,10 @@ int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, in
   return make_plan(B, Hq, Hkv, d, D_max, L_max, attention_rows_hint(g, D_max)).splits > 1 ? 2 : 1;
 }
 
-cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
-  if (a.B == 0) return cudaSuccess;
-  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
-                           attention_rows_hint(a.grid, a.D_max));
+namespace {
+
+// The launch record of a plan over workspace `ws` (laid out as attention_workspace counts it).
+AttnLaunch carve(const AttnArgs& a, const Plan& p, void* ws) {
   AttnLaunch L;
   L.splits = p.splits;
   L.kps = p.kps;
@@ -518,12 +519,30 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
     w += align256(prow * a.d * sizeof(float));
     L.part_lse = reinterpret_cast<float*>(w);
   }
+  return L;
+}
+
+}  // namespace
+
+cudaError_t launch_attention_combine(const AttnArgs& a, void* ws, cudaStream_t stream) {
+  if (a.B == 0) return cudaSuccess;
+  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
+                           attention_rows_hint(a.grid, a.D_max));
+  return p.splits == 1 ? cudaSuccess : launch_combine(a, carve(a, p, ws), stream);
+}
+
+cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream,
+                             bool defer_combine) {
+  if (a.B == 0) return cudaSuccess;
+  const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
+                           attention_rows_hint(a.grid, a.D_max));
+  const AttnLaunch L = carve(a, p, ws);
   cudaError_t e;
   if (p.tc) {
     e = launch_attention_tc(a, TcPlan{p.splits, p.kps, p.mtiles}, L.seq_ok, L.part_o, L.part_lse,
                             stream);
     if (e != cudaSuccess) return e;
-    return p.splits == 1 ? cudaSuccess : launch_combine(a, L, stream);
+    return (p.splits == 1 || defer_combine) ? cudaSuccess : launch_combine(a, L, stream);
   }
   CUtensorMap tmK, tmV;
   const int64_t rows = (int64_t)a.B * a.Hkv * a.L_max;
@@ -545,7 +564,7 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
     frontier_attn_kernel<64><<<grid, block, smem, stream>>>(tmK, tmV, a, L);
   }
   e = cudaGetLastError();
-  if (e != cudaSuccess || p.splits == 1) return e;
+  if (e != cudaSuccess || p.splits == 1 || defer_combine) return e;
   return launch_combine(a, L, stream);
 }
 

@@ -224,6 +224,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   constexpr uint32_t kIdescO = idesc_f16(D, true);
   constexpr int HC = KTC / 2;                // S columns per softmax thread (P: HC / 2)
   constexpr int HD = D / 2;                  // O columns per softmax thread
+  // a kernel queued after this one as a programmatic dependent (the step's
+  // counts and draws, which need none of its results) may start beside it
+  pdl_launch_dependents();
 
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ int32_t s_order[kLptMax];
@@ -281,7 +284,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   if (a.B <= kLptMax) {
     // s_order[rank] = the sequence with the rank-th most keys (ties by index)
     for (int32_t i = tid; i < a.B; i += blockDim.x) {
-      const int32_t c = a.cache_len[i], n = a.n_drafts[i];
+      const int32_t c = a.cache_len[i], n = attn_drafts(a, i);
       s_key[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
     }
     __syncthreads();
@@ -325,7 +328,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       rem /= L.mtiles;
       const int32_t split = rem % L.splits, g = rem / L.splits;
       const int32_t b = (a.B <= kLptMax) ? s_order[rank_b] : rank_b;
-      const int32_t cache = a.cache_len[b], nd = a.n_drafts[b];
+      const int32_t cache = a.cache_len[b], nd = attn_drafts(a, b);
       const bool shape_ok = nd >= 0 && nd <= a.D_max && cache >= 0 && cache <= a.L_max - nd;
       // draft positions (validity is identical in every item of b)
       int32_t kfv[4];
@@ -335,7 +338,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         const int32_t j = lane + 32 * u;
         kfv[u] = 0;
         if (shape_ok && j < nd) {
-          const int32_t gidx = a.draft_pos[(int64_t)b * a.D_max + j];
+          const int32_t gidx = attn_draft_pos(a, b, j);
           if (gidx < 0 || gidx >= HW) {
             bad = true;
           } else {

@@ -22,6 +22,16 @@ namespace ssd {
 // thousand polls; 2^22 polls is well above a second of waiting.
 constexpr uint32_t kMaxPolls = 1u << 22;
 
+// Programmatic dependent launch (sm_90 and later): let the kernel queued
+// after this one on the stream be scheduled before this grid completes ...
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// ... and, in that dependent kernel, wait until the grid it depends on has
+// completed with its memory visible (a no-op in a kernel launched without
+// the programmatic attribute).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void record_status(int32_t* status, int32_t code) {
   if (status != nullptr) atomicCAS(status, (int32_t)SSD_OK, code);
 }

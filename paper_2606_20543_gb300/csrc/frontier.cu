@@ -21,32 +21,17 @@
 
 namespace ssd {
 
-__device__ __forceinline__ int32_t frontier_size(const ssd_grid& g, int32_t n_c) {
-  const int32_t y0 = n_c / g.grid_w;
-  const int32_t c = n_c - y0 * g.grid_w;
-  if (y0 >= g.grid_h) return 0;
-  const int32_t h = g.k_h > 0 ? min(g.k_h, g.grid_w - c) : g.grid_w - c;
-  const int32_t rows_below = (c + h == g.grid_w) ? min(g.k_v, g.grid_h - 1 - y0) : 0;
-  return h + rows_below * g.grid_w;
-}
-
 // One block per sequence.  Writes n_drafts[b] and draft_pos[b][0..D_max).
 __global__ void frontier_kernel(ssd_grid g, const int32_t* __restrict__ cache_len, int32_t D_max,
                                 int32_t* __restrict__ n_drafts, int32_t* __restrict__ draft_pos,
                                 int32_t* status) {
   const int32_t b = blockIdx.x;
   const int32_t n_c = cache_len[b] - g.prefix_len;
-  int32_t n = 0;
-  if (n_c < 0 || n_c > g.grid_h * g.grid_w) {
-    if (threadIdx.x == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
-  } else {
-    n = frontier_size(g, n_c);
-    if (n > D_max) {  // host checks D_max >= (k_v + 1) * W; keep the guard
-      if (threadIdx.x == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
-      n = 0;
-    }
+  const int32_t n = frontier_drafts(g, cache_len[b], D_max);
+  if (threadIdx.x == 0) {
+    n_drafts[b] = n < 0 ? 0 : n;
+    if (n < 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
   }
-  if (threadIdx.x == 0) n_drafts[b] = n;
   for (int32_t j = threadIdx.x; j < D_max; j += blockDim.x)
     draft_pos[(int64_t)b * D_max + j] = (j < n) ? (n_c + j) : -1;
 }
@@ -60,7 +45,10 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
                               int32_t* __restrict__ accepted_prefix,
                               int32_t* __restrict__ next_cache_len, int32_t* status) {
   const int32_t b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (b >= B) return;
+  if (b >= B) {
+    pdl_wait();
+    return;
+  }
   int32_t n = n_drafts[b];
   if (n < 0 || n > D_max) {  // a caller's frontier (ssd_verify_accept) out of range
     if ((threadIdx.x & 31) == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
@@ -68,6 +56,7 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
   }
   sequence_counts(g, commit, b, D_max, cache_len, n, accepted, accepted_count, accepted_prefix,
                   next_cache_len, threadIdx.x & 31);
+  pdl_wait();  // under a programmatic launch: exit only after the kernel before it
 }
 
 // Staged schedule: the trailing row (slots W .. 2W-1) becomes the frontier of
@@ -97,13 +86,12 @@ cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t 
                           const int32_t* cache_len, const int32_t* n_drafts,
                           const uint8_t* accepted, int32_t* accepted_count,
                           int32_t* accepted_prefix, int32_t* next_cache_len, int32_t* status,
-                          cudaStream_t stream) {
+                          bool pdl, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
   const int warps = 4;
-  counts_kernel<<<(B + warps - 1) / warps, warps * 32, 0, stream>>>(
-      g, commit, B, D_max, cache_len, n_drafts, accepted, accepted_count, accepted_prefix,
-      next_cache_len, status);
-  return cudaGetLastError();
+  return launch_kernel(counts_kernel, dim3((B + warps - 1) / warps), dim3(warps * 32), 0, stream,
+                       pdl, g, commit, B, D_max, cache_len, n_drafts, accepted, accepted_count,
+                       accepted_prefix, next_cache_len, status);
 }
 
 cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,

@@ -6,15 +6,60 @@
 
 namespace ssd {
 
+// Frontier size (Sec. 3.3) after n_c committed grid tokens: the horizontal
+// part completes the current grid row (at most k_h positions when k_h > 0),
+// and when it does, the k_v rows below follow, clipped at the last grid row;
+// one contiguous raster run.
+__device__ __forceinline__ int32_t frontier_size(const ssd_grid& g, int32_t n_c) {
+  const int32_t y0 = n_c / g.grid_w;
+  const int32_t c = n_c - y0 * g.grid_w;
+  if (y0 >= g.grid_h) return 0;
+  const int32_t h = g.k_h > 0 ? min(g.k_h, g.grid_w - c) : g.grid_w - c;
+  const int32_t rows_below = (c + h == g.grid_w) ? min(g.k_v, g.grid_h - 1 - y0) : 0;
+  return h + rows_below * g.grid_w;
+}
+
+// Drafts of a sequence with cache length `cache_len` (its positions are
+// n_c .. n_c + n - 1, n_c = cache_len - prefix_len), or -1 when cache_len is
+// outside the grid or the frontier does not fit D_max (reported by the caller).
+__device__ __forceinline__ int32_t frontier_drafts(const ssd_grid& g, int32_t cache_len,
+                                                   int32_t D_max) {
+  const int32_t n_c = cache_len - g.prefix_len;
+  if (n_c < 0 || n_c > g.grid_h * g.grid_w) return -1;
+  const int32_t n = frontier_size(g, n_c);
+  return n > D_max ? -1 : n;  // the host checks D_max >= (k_v + 1) W; keep the guard
+}
+
+// Launch `kernel`, optionally as a programmatic dependent of the kernel
+// before it on `stream` (cudaLaunchAttributeProgrammaticStreamSerialization).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t stream, bool pdl, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // ---- frontier.cu
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
                             cudaStream_t stream);
+// pdl: launched as a programmatic dependent of the kernel before it on the
+// stream (it may start while that kernel runs, needs none of its results and
+// waits for it before exiting, so stream order is kept).
 cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
                           const int32_t* cache_len, const int32_t* n_drafts,
                           const uint8_t* accepted, int32_t* accepted_count,
                           int32_t* accepted_prefix, int32_t* next_cache_len, int32_t* status,
-                          cudaStream_t stream);
+                          bool pdl, cudaStream_t stream);
 // Staged schedule: slot j of every sequence takes slot W + j (j < W) of the
 // per-row tokens and reference pointers.
 cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
@@ -22,7 +67,7 @@ cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok
 
 // One warp: the counts of sequence b (a7) from its n drafts' accepted flags —
 // drafts accepted, the leading accepted run and the next cache length under
-// `commit` — written by lane 0; every lane returns the leading run.  The
+// `commit` — written by lane 0 if `write`; every lane returns the leading run.  The
 // drafts up to and including the first rejected one are committed (the
 // rejected one with its resampled token); SSD_COMMIT_NONE / _BLOCK /
 // _FIRST_ROW serve the verify-and-correct rounds, _PREFIX_BONUS the
@@ -32,7 +77,8 @@ __device__ __forceinline__ int32_t sequence_counts(const ssd_grid& g, int32_t co
                                                    int32_t n, const uint8_t* accepted,
                                                    int32_t* accepted_count,
                                                    int32_t* accepted_prefix,
-                                                   int32_t* next_cache_len, int32_t lane) {
+                                                   int32_t* next_cache_len, int32_t lane,
+                                                   bool write = true) {
   int32_t count = 0, prefix = 0;
   bool run = true;  // still inside the leading accepted run
   for (int32_t j0 = 0; j0 < n; j0 += 32) {
@@ -51,7 +97,7 @@ __device__ __forceinline__ int32_t sequence_counts(const ssd_grid& g, int32_t co
       }
     }
   }
-  if (lane == 0) {
+  if (lane == 0 && write) {
     accepted_count[b] = count;
     accepted_prefix[b] = prefix;
     int32_t advance = n > 0 ? min(prefix + 1, n) : 0;  // SSD_COMMIT_PREFIX
@@ -101,6 +147,15 @@ struct AcceptArgs {
   // the one token per sequence that the counts commit.
   int32_t lazy = 0;
   float2* stats = nullptr;   // [rows] when lazy
+  // One verification step (rows = B * D_max): with cache_len non-null the
+  // kernel computes every sequence's frontier under `grid` (Sec. 3.3) itself
+  // instead of reading n_drafts, and spare lanes write it out (n_drafts_out,
+  // draft_pos, as ssd_frontier) and zero `tickets` [B] for launch_resolve.
+  const int32_t* cache_len = nullptr;
+  ssd_grid grid{};
+  int32_t* n_drafts_out = nullptr;
+  int32_t* draft_pos = nullptr;
+  int32_t* tickets = nullptr;
 };
 bool accept_supported(int32_t V);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t stream);
@@ -127,8 +182,11 @@ struct ResolveArgs {
   int32_t* accepted_prefix;
   int32_t* next_cache_len;
   int32_t* status;
+  int32_t* tickets;  // [B], zeroed by the acceptance pass
+  float* mass;       // [B][resolve_blocks(V)] block masses of the committed rows
 };
-cudaError_t launch_resolve(const ResolveArgs& a, cudaStream_t stream);
+int32_t resolve_blocks(int32_t V);
+cudaError_t launch_resolve(const ResolveArgs& a, bool pdl, cudaStream_t stream);
 
 // ---- attention.cu
 struct AttnArgs {
@@ -144,7 +202,20 @@ struct AttnArgs {
   void* o;
   float* lse;  // nullable
   int32_t* status;
+  // The step's frontier: the drafts of sequence b are its raster frontier under
+  // `grid` (Sec. 3.3), computed from cache_len; n_drafts and draft_pos unread.
+  int32_t raster = 0;
 };
+__device__ __forceinline__ int32_t attn_drafts(const AttnArgs& a, int32_t b) {
+  if (!a.raster) return a.n_drafts[b];
+  const int32_t n = frontier_drafts(a.grid, a.cache_len[b], a.D_max);
+  return n < 0 ? 0 : n;  // an out-of-grid cache length is reported by the acceptance pass
+}
+// Grid index of draft j of sequence b.
+__device__ __forceinline__ int32_t attn_draft_pos(const AttnArgs& a, int32_t b, int32_t j) {
+  return a.raster ? a.cache_len[b] - a.grid.prefix_len + j
+                  : a.draft_pos[(int64_t)b * a.D_max + j];
+}
 // Longest-first work order for the attention grids: CTA row `rank` (of B)
 // takes the sequence with the rank-th most keys (cache_len + n_drafts, ties by
 // index), so the longest sequences start in the first wave instead of being
@@ -154,7 +225,7 @@ constexpr int kLptMax = 256;
 __device__ __forceinline__ int32_t longest_first(const AttnArgs& a, int32_t rank, int32_t* skey) {
   if (a.B > kLptMax) return rank;
   for (int32_t i = threadIdx.x; i < a.B; i += blockDim.x) {
-    const int32_t c = a.cache_len[i], n = a.n_drafts[i];
+    const int32_t c = a.cache_len[i], n = attn_drafts(a, i);
     skey[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
   }
   __syncthreads();
@@ -172,7 +243,11 @@ __device__ __forceinline__ int32_t longest_first(const AttnArgs& a, int32_t rank
 }
 size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max,
                            int32_t L_max);
-cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
+// defer_combine: leave the split-KV combine (if the plan has splits) to
+// launch_attention_combine, so that another kernel can be queued between.
+cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream,
+                             bool defer_combine = false);
+cudaError_t launch_attention_combine(const AttnArgs& a, void* ws, cudaStream_t stream);
 int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
                        int32_t D_max, int32_t L_max);
 // Most drafts one sequence can have under grid `g` (Sec. 3.3 frontier: at most

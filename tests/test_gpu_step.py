@@ -302,20 +302,20 @@ def test_committed_bonus_is_the_full_draw_from_p(ssd):
 
 
 def test_verify_accept_matches_the_step(ssd):
-    """ssd_verify_accept (acceptance and counts of a drafted frontier, on one
-    stream) gives the step's outputs bit for bit."""
+    """ssd_verify_accept (the step without the attention, on one stream)
+    gives the step's frontier, decisions, draws and counts bit for bit."""
     c = synth.config2(points=[120, 408, 696])
     s = make_step(c)
     s.run()
     torch.cuda.synchronize()
     r = s.results()
     for t in (s.out_tok, s.accepted, s.ratio, s.accepted_count, s.accepted_prefix,
-              s.next_cache_len):
-        t.fill_(0)
+              s.next_cache_len, s.n_drafts, s.draft_pos):
+        t.fill_(-5 if t.dtype == torch.int32 else 0)
     ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes)
     torch.cuda.synchronize()
     r2 = s.results()
-    for k in ("out_tok", "accepted", "accepted_count", "accepted_prefix", "next_cache_len",
-              "status"):
+    for k in ("n_drafts", "draft_pos", "out_tok", "accepted", "accepted_count", "accepted_prefix",
+              "next_cache_len", "status"):
         assert np.array_equal(r[k], r2[k]), k
     assert np.array_equal(r["ratio"].view(np.uint32), r2["ratio"].view(np.uint32))
