@@ -176,9 +176,10 @@ class ClockSampler:
 # is the one that was captured: (source file, sha256 prefix, bytes, rows the
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
-    ("accept", 2): ("accept.cu", "5ccfccad7a2ff8ae", 152415232 + 3548416, 1128),
-    ("attention", 2): ("attention_tc.cu", "90f7f3d45983421a", 102310144 + 2746368, None),
-    ("attention", 3): ("attention_tc.cu", "90f7f3d45983421a", 53837312 + 197632, None),
+    # acceptance part of a step: accept_kernel (one pass) + resolve_kernel (committed draws)
+    ("accept", 2): ("accept.cu", "beaf1223a65ae37b", 147920768 + 167168 + 3185408, None),
+    ("attention", 2): ("attention_tc.cu", "6836c8344e2b7782", 102307840 + 65024, None),
+    ("attention", 3): ("attention_tc.cu", "6836c8344e2b7782", 53834624 + 78976, None),
     ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
 }
 
