@@ -738,7 +738,10 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
     const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
     if (lane == 0) a.out_tok[r] = pick;
   }
-  pdl_wait();  // under a programmatic launch: exit only after the kernel before it
+  // Under a programmatic launch after the attention (the step's schedule; the
+  // acceptance pass completed before the attention started): exit only after
+  // the attention, so that stream order holds.
+  pdl_wait();
 }
 
 }  // namespace

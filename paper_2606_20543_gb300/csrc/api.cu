@@ -607,14 +607,16 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     // cache_len (a2), so the two need no frontier launch before them.
     a.raster = 1;
     if (lazy_draws(x) && x->B * x->D_max >= 2 * device_sm_count()) {
-      // A lazy pass that fills the GPU, on `stream` alone: acceptance, then
-      // attention, then a7 (counts and the committed draws) as a programmatic
-      // dependent of the attention: it needs only the acceptance's results,
-      // starts once every attention CTA is resident and runs in the registers
-      // they leave free, beside them.
+      // A lazy pass that fills the GPU, on `stream` alone: the acceptance;
+      // the attention, which reads none of its results, as a programmatic
+      // dependent (the tcgen05 kernel starts as the acceptance's CTAs retire
+      // and lets the next kernel be scheduled only once the acceptance has
+      // completed); then a7 (counts and the committed draws) as a
+      // programmatic dependent of the attention: its small CTAs run beside
+      // the attention, in the registers it leaves free.
       e = launch_accept_phase(x, y, ws + attn_ws, stream);
       if (e != cudaSuccess) return SSD_ERR_CUDA;
-      e = launch_attention(a, ws, attn_ws, stream, /*defer_combine=*/true);
+      e = launch_attention(a, ws, attn_ws, stream, /*defer_combine=*/true, /*pdl=*/true);
       if (e != cudaSuccess) return SSD_ERR_CUDA;
       e = launch_finish_phase(x, y, ws + attn_ws, /*pdl=*/true, stream);
       if (e != cudaSuccess) return SSD_ERR_CUDA;

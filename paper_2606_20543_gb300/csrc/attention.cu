@@ -170,6 +170,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   if (!seq_valid || !has_work) {
     // never leave with copies in flight into this CTA's shared memory
     for (int t = 0; t < n_pre; ++t) mbar_wait(&full[t % kStages], 0, a.status);
+    pdl_wait();
     return;
   }
 
@@ -312,7 +313,10 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     // stage s is free for the producer; a timed-out wait anywhere stops every thread
     if (!__syncthreads_and(ok)) { ok = false; break; }
   }
-  if (!ok || !warp_active) return;
+  if (!ok || !warp_active) {
+    pdl_wait();
+    return;
+  }
 
   // ---- epilogue: normalise, write O (bf16) or the split partial (fp32)
   const bool direct = (n_active == 1);
@@ -345,6 +349,9 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
       if ((lane & 3) == 0) L.part_lse[prow] = lse;
     }
   }
+  // launched as a programmatic dependent (the step's schedule): exit only after
+  // the kernel before it, so that stream order holds
+  pdl_wait();
 }
 
 // One warp per (b, j, h) row: merge the active splits by log-sum-exp.
@@ -532,7 +539,7 @@ cudaError_t launch_attention_combine(const AttnArgs& a, void* ws, cudaStream_t s
 }
 
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream,
-                             bool defer_combine) {
+                             bool defer_combine, bool pdl) {
   if (a.B == 0) return cudaSuccess;
   const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
                            attention_rows_hint(a.grid, a.D_max));
@@ -540,7 +547,7 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
   cudaError_t e;
   if (p.tc) {
     e = launch_attention_tc(a, TcPlan{p.splits, p.kps, p.mtiles}, L.seq_ok, L.part_o, L.part_lse,
-                            stream);
+                            stream, pdl);
     if (e != cudaSuccess) return e;
     return (p.splits == 1 || defer_combine) ? cudaSuccess : launch_combine(a, L, stream);
   }
@@ -555,13 +562,15 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
     e = cudaFuncSetAttribute(frontier_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
     if (e != cudaSuccess) return e;
-    frontier_attn_kernel<128><<<grid, block, smem, stream>>>(tmK, tmV, a, L);
+    e = launch_kernel(frontier_attn_kernel<128>, grid, block, smem, stream, false, tmK, tmV, a, L);
+    if (e != cudaSuccess) return e;
   } else {
     const size_t smem = 1024 + kStages * 2 * (KT * 64 * 2) + kStages * 8 + 129 * 4;
     e = cudaFuncSetAttribute(frontier_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
     if (e != cudaSuccess) return e;
-    frontier_attn_kernel<64><<<grid, block, smem, stream>>>(tmK, tmV, a, L);
+    e = launch_kernel(frontier_attn_kernel<64>, grid, block, smem, stream, false, tmK, tmV, a, L);
+    if (e != cudaSuccess) return e;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess || p.splits == 1 || defer_combine) return e;

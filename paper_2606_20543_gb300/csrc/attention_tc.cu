@@ -155,6 +155,82 @@ __device__ __forceinline__ float ex2a(float x) {
   return y;
 }
 
+// 16-lane TMEM accesses of the M = 64 products, whose row m sits in lane
+// 32 (m / 16) + m % 16.  .16x256b: thread t holds rows t/4 and t/4 + 8 of the
+// 16 lanes, columns 8u + 2 (t % 4) + {0, 1} of unit u, as registers 4u + {0, 1}
+// (row t/4) and 4u + {2, 3} (row t/4 + 8).  .16x128b: column 4u + t % 4 of
+// unit u, register 2u (row t/4) and 2u + 1 (row t/4 + 8).
+__device__ __forceinline__ void tld16x256_x8(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tld16x256_x4(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x4.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tst16x256_x8(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x256b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tst16x256_x4(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x256b.x4.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tst16x128_x8(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x128b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // tcgen05 shared-memory descriptor: 128-byte swizzle, version 1.
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
   uint64_t d = 0;
@@ -173,10 +249,10 @@ __device__ __forceinline__ uint64_t sdesc_at(uint64_t d, uint32_t off) {
   return d + (uint64_t)(off >> 4);
 }
 
-// kind::f16 instruction descriptor: fp32 D, bf16 A and B, A K-major, M = 128.
-__host__ __device__ constexpr uint32_t idesc_f16(int n, bool b_mn_major) {
+// kind::f16 instruction descriptor: fp32 D, bf16 A and B, A K-major, M = m (64 or 128).
+__host__ __device__ constexpr uint32_t idesc_f16(int n, bool b_mn_major, int m = kBM) {
   return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
-         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
 struct TcLaunch {
@@ -195,9 +271,9 @@ struct TcItem {
   int32_t kflat[128];  // raster position of each draft of b
 };
 
-template <int D>
+template <int D, int BM>
 constexpr size_t tc_smem_bytes() {
-  return 1024 + (size_t)2 * kBM * D * 2 + (size_t)2 * kNB * KTC * D * 2 + 320 +
+  return 1024 + (size_t)2 * BM * D * 2 + (size_t)2 * kNB * KTC * D * 2 + 320 +
          2 * sizeof(TcItem) + (size_t)6 * kBM * 4;
 }
 
@@ -213,20 +289,22 @@ __device__ __forceinline__ void load_kv_tile(void* dst, const CUtensorMap* map, 
     tma_load_2d(dst, map, 0, row, bar, pol);
 }
 
-template <int D>
+// BM = 128: query tiles of 128 rows, row m in TMEM lane m.  BM = 64 (items of
+// at most 64 query rows): M = 64 products, row m in lane 32 (m / 16) + m % 16,
+// so the rows spread over the four lane quarters and their softmax over all
+// four SM sub-partitions.
+template <int D, int BM>
 __global__ void __launch_bounds__(kThreadsTC, 1)
 frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, AttnArgs a, TcLaunch L) {
+  static_assert(BM == 64 || BM == 128, "query tile");
   constexpr int NSUB = D / 64;
-  constexpr int Q_BYTES = kBM * D * 2;
+  constexpr int Q_BYTES = BM * D * 2;
   constexpr int KV_BYTES = KTC * D * 2;      // one K (or V) tile
-  constexpr uint32_t kIdescS = idesc_f16(KTC, false);
-  constexpr uint32_t kIdescO = idesc_f16(D, true);
+  constexpr uint32_t kIdescS = idesc_f16(KTC, false, BM);
+  constexpr uint32_t kIdescO = idesc_f16(D, true, BM);
   constexpr int HC = KTC / 2;                // S columns per softmax thread (P: HC / 2)
   constexpr int HD = D / 2;                  // O columns per softmax thread
-  // a kernel queued after this one as a programmatic dependent (the step's
-  // counts and draws, which need none of its results) may start beside it
-  pdl_launch_dependents();
 
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ int32_t s_order[kLptMax];
@@ -366,7 +444,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       }
       const int32_t Lk = valid ? cache + nd : 0;
       const int32_t rows_total = valid ? nd * G : 0;
-      const int32_t row0 = mtile * kBM;
+      const int32_t row0 = mtile * BM;
       const int32_t k_lo = split * L.kps;
       const int32_t k_hi = min(Lk, k_lo + L.kps);
       if (!valid || nd == 0 || row0 >= rows_total || k_lo >= Lk) continue;
@@ -401,11 +479,11 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         if (ok) {
           mbar_arrive_expect_tx(&q_full[s], Q_BYTES);
           for (int c = 0; c < NSUB; ++c) {
-            // 3D Q view {d, Hq, B * D_max}: box {64, G, 128 / G} -> rows (j, hg)
+            // 3D Q view {d, Hq, B * D_max}: box {64, G, BM / G} -> rows (j, hg)
             asm volatile(
                 "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
                 " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(
-                    smem_u32(sQ + s * Q_BYTES + c * (kBM * 128))),
+                    smem_u32(sQ + s * Q_BYTES + c * (BM * 128))),
                 "l"(reinterpret_cast<uint64_t>(&tmQ)), "r"(c * 64), "r"(g * G),
                 "r"(b * a.D_max + row0 / G), "r"(smem_u32(&q_full[s])), "l"(polq)
                 : "memory");
@@ -441,6 +519,16 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     // ---------------------------------------------------------- V producer
     // Follows the item slots like the MMA warp; a slot is not rewritten before
     // the softmax has finished its item, which needs every V tile of it.
+    // Launch ordering (programmatic dependent launch): launched as a dependent
+    // of the step's acceptance pass, whose results it does not read, the
+    // kernel starts as the acceptance's CTAs retire; lane 1 waits for the
+    // acceptance to complete and only then lets the kernel queued after this
+    // one (the counts and draws, which read them) be scheduled beside it.
+    // Under a plain launch the wait returns at once.
+    if (lane == 1) {
+      pdl_wait();
+      pdl_launch_dependents();
+    }
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       uint32_t T = 0;
@@ -486,7 +574,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll
           for (int ks = 0; ks < D / 16; ++ks) {
             const int sub = ks >> 2, kin = (ks & 3) * 32;
-            umma(tS + sb * KTC, sdesc_at(dq, sub * (kBM * 128) + kin),
+            umma(tS + sb * KTC, sdesc_at(dq, sub * (BM * 128) + kin),
                  sdesc_at(dk, sub * (KTC * 128) + kin), kIdescS, ks > 0 ? 1u : 0u);
           }
           umma_commit(&s_full[sb]);
@@ -529,6 +617,275 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       }
     }
     __syncwarp();
+  } else if constexpr (BM == 64) {
+    // ------------------------------------------------ softmax, M = 64 items
+    // Item row m sits in TMEM lane 32 (m / 16) + m % 16, so lane quarter q
+    // holds item rows 16q .. 16q + 15.  Warp w takes quarter w % 4 and half
+    // w / 4 of every row's columns; with 16-lane accesses each thread holds two
+    // rows (t / 4 and t / 4 + 8 of the quarter) x 16 columns of its half, and
+    // the four threads t % 4 of a row finish its maxima and sums by shuffles.
+    const int quarter = warp & 3, half = warp >> 2;
+    const int cq = lane & 3;
+    const int32_t rlA = quarter * 16 + (lane >> 2), rlB = rlA + 8;  // item rows of this thread
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    auto xs = [&](int slot, int hf, int32_t rl) -> float& {
+      return xch[(slot * 2 + hf) * kBM + rl];
+    };
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory"); };
+    auto low = [](int32_t n) -> uint64_t {
+      return n <= 0 ? 0ull : (n >= 64 ? ~0ull : ((1ull << n) - 1ull));
+    };
+    bool ok = true;
+    uint32_t T = 0;
+    for (int32_t k = 0; ok; ++k) {
+      const int s = k & 1;
+      if (!mbar_wait(&it_full[s], (k >> 1) & 1, a.status)) { ok = false; break; }
+      const TcItem& it = items[s];
+      const int32_t ntiles = it.ntiles;
+      if (ntiles < 0) break;
+      const int32_t b = it.b, g = it.g, split = it.split, row0 = it.row0;
+      const int32_t rows_total = it.rows_total, cache = it.cache, Lk = it.Lk;
+      const int32_t k_lo = it.k_lo, k_hi = it.k_hi;
+      const bool direct = it.direct != 0;
+      const int32_t* kflat = it.kflat;
+      const uint32_t tO = tO0 + s * 128;
+      const int32_t rA = row0 + rlA, rB = row0 + rlB;
+      const bool liveA = rA < rows_total, liveB = rB < rows_total;
+      const bool warp_live = row0 + quarter * 16 < rows_total;  // same for both warps of a pair
+      const int32_t jqA = liveA ? rA / G : 0, hA = g * G + (liveA ? rA - jqA * G : 0);
+      const int32_t jqB = liveB ? rB / G : 0, hB = g * G + (liveB ? rB - jqB * G : 0);
+      const int32_t qposA = liveA ? kflat[jqA] : 0x7fffffff;
+      const int32_t qposB = liveB ? kflat[jqB] : 0x7fffffff;
+      const bool increasing = it.increasing != 0;
+      int32_t minq = 0x7fffffff;
+      const int32_t j_lo = row0 / G;
+      if (increasing) {
+        minq = kflat[j_lo];
+      } else {
+        const int32_t j_end = (min(rows_total, row0 + BM) + G - 1) / G;
+        for (int32_t j = j_lo + lane; j < j_end; j += 32) minq = min(minq, kflat[j]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) minq = min(minq, __shfl_xor_sync(0xffffffffu, minq, o));
+      }
+      const int32_t mask_from = min(cache, minq + 1);
+      // visibility of the item's drafts to rows A and B (bit j: draft j visible)
+      uint64_t vAlo = 0, vAhi = 0, vBlo = 0, vBhi = 0;
+      if (warp_live && increasing) {
+        const int32_t nA = jqA + 1, nB = jqB + 1;  // 1 .. 128
+        vAlo = nA >= 64 ? ~0ull : ((1ull << nA) - 1ull);
+        vAhi = nA <= 64 ? 0ull : (nA >= 128 ? ~0ull : ((1ull << (nA - 64)) - 1ull));
+        vBlo = nB >= 64 ? ~0ull : ((1ull << nB) - 1ull);
+        vBhi = nB <= 64 ? 0ull : (nB >= 128 ? ~0ull : ((1ull << (nB - 64)) - 1ull));
+      } else if (warp_live) {
+        const int32_t nd = Lk - cache;
+#pragma unroll 1
+        for (int j = 0; j < nd; j += 4) {
+          const int4 kf = *reinterpret_cast<const int4*>(kflat + j);
+          const uint64_t bA = (uint64_t)((uint32_t)(kf.x <= qposA) | ((uint32_t)(kf.y <= qposA) << 1) |
+                                         ((uint32_t)(kf.z <= qposA) << 2) |
+                                         ((uint32_t)(kf.w <= qposA) << 3));
+          const uint64_t bB = (uint64_t)((uint32_t)(kf.x <= qposB) | ((uint32_t)(kf.y <= qposB) << 1) |
+                                         ((uint32_t)(kf.z <= qposB) << 2) |
+                                         ((uint32_t)(kf.w <= qposB) << 3));
+          if (j < 64) {
+            vAlo |= bA << j;
+            vBlo |= bB << j;
+          } else {
+            vAhi |= bA << (j - 64);
+            vBhi |= bB << (j - 64);
+          }
+        }
+      }
+      // keep mask of one row over keys c0 .. c0 + 63 (as in the M = 128 path)
+      auto keep_of = [&](int32_t c0, int32_t qpos, uint64_t vlo, uint64_t vhi) -> uint64_t {
+        const int32_t base = c0 - cache;  // draft index of column 0
+        uint64_t win;
+        if (base >= 128 || base <= -64) win = 0;
+        else if (base >= 64) win = vhi >> (base - 64);
+        else if (base > 0) win = (vlo >> base) | (vhi << (64 - base));
+        else if (base == 0) win = vlo;
+        else win = vlo << (-base);
+        const int32_t seen_end = qpos < cache ? qpos + 1 : cache;
+        return (low(seen_end - c0) | (win & ~low(cache - c0))) & low(k_hi - c0);
+      };
+      float m_runA = -INFINITY, m_runB = -INFINITY, l_runA = 0.f, l_runB = 0.f;
+      for (int t = 0; t < ntiles; ++t, ++T) {
+        const int bb = T & 1, sb = T % kNB;
+        if (!mbar_wait(&s_full[sb], (T / kNB) & 1, a.status)) ok = false;
+        tc_after();
+        float sv[32];
+        if (warp_live) tld16x256_x8(tS + lane_off + sb * KTC + half * HC, sv);
+        bool movedA = false, movedB = false;
+        float alphaA = 1.f, alphaB = 1.f;
+        uint32_t pk[16];
+        if (warp_live) {
+          const int32_t c0 = k_lo + t * KTC + half * HC;
+          if (c0 + HC > k_hi || c0 + HC > mask_from) {
+            const uint64_t keepA = keep_of(c0, qposA, vAlo, vAhi);
+            const uint64_t keepB = keep_of(c0, qposB, vBlo, vBhi);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+#pragma unroll
+              for (int e = 0; e < 2; ++e) {
+                const int jj = 8 * u + 2 * cq + e;
+                if (!((keepA >> jj) & 1ull)) sv[4 * u + e] = -INFINITY;
+                if (!((keepB >> jj) & 1ull)) sv[4 * u + 2 + e] = -INFINITY;
+              }
+          }
+          float a4[4], b4[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            a4[i] = fmaxf(fmaxf(sv[8 * i], sv[8 * i + 1]), fmaxf(sv[8 * i + 4], sv[8 * i + 5]));
+            b4[i] = fmaxf(fmaxf(sv[8 * i + 2], sv[8 * i + 3]), fmaxf(sv[8 * i + 6], sv[8 * i + 7]));
+          }
+          float mxA = fmaxf(fmaxf(a4[0], a4[1]), fmaxf(a4[2], a4[3]));
+          float mxB = fmaxf(fmaxf(b4[0], b4[1]), fmaxf(b4[2], b4[3]));
+          mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
+          mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 1));
+          mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 2));
+          mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 2));
+          // (the pair barrier also orders the partner's tcgen05.ld of S before
+          // this warp overwrites the buffer with P)
+          if (cq == 0) {
+            xs(bb, half, rlA) = mxA;
+            xs(bb, half, rlB) = mxB;
+          }
+          pair_sync();
+          mxA = fmaxf(mxA, xs(bb, half ^ 1, rlA));
+          mxB = fmaxf(mxB, xs(bb, half ^ 1, rlB));
+          // move a running max only when it grows by more than 2^kRescale
+          if (mxA != -INFINITY && (m_runA == -INFINITY || (mxA - m_runA) * c2 > kRescale)) {
+            alphaA = (m_runA == -INFINITY) ? 0.f : ex2a((m_runA - mxA) * c2);
+            m_runA = mxA;
+            movedA = true;
+          }
+          if (mxB != -INFINITY && (m_runB == -INFINITY || (mxB - m_runB) * c2 > kRescale)) {
+            alphaB = (m_runB == -INFINITY) ? 0.f : ex2a((m_runB - mxB) * c2);
+            m_runB = mxB;
+            movedB = true;
+          }
+          const float moffA = (m_runA == -INFINITY) ? 0.f : m_runA * c2;
+          const float moffB = (m_runB == -INFINITY) ? 0.f : m_runB * c2;
+          float sA[4] = {0.f, 0.f, 0.f, 0.f}, sB[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const float eA0 = ex2a(fmaf(sv[4 * u], c2, -moffA));
+            const float eA1 = ex2a(fmaf(sv[4 * u + 1], c2, -moffA));
+            const float eB0 = ex2a(fmaf(sv[4 * u + 2], c2, -moffB));
+            const float eB1 = ex2a(fmaf(sv[4 * u + 3], c2, -moffB));
+            sA[u & 3] += eA0 + eA1;
+            sB[u & 3] += eB0 + eB1;
+            pk[2 * u] = pack_bf16x2(eA0, eA1);
+            pk[2 * u + 1] = pack_bf16x2(eB0, eB1);
+          }
+          l_runA = l_runA * alphaA + ((sA[0] + sA[1]) + (sA[2] + sA[3]));
+          l_runB = l_runB * alphaB + ((sB[0] + sB[1]) + (sB[2] + sB[3]));
+        }
+        if (warp_live) {
+          // O may be rescaled once PV_{T-1} is done
+          if (__any_sync(0xffffffffu, (movedA || movedB) && t > 0)) {
+            if (!mbar_wait(&pv_done[(T - 1) % kNB], ((T - 1) / kNB) & 1, a.status)) ok = false;
+            tc_after();
+            float ov[HD / 2];
+            const uint32_t ta = tO + lane_off + half * HD;
+            if constexpr (HD == 64) tld16x256_x8(ta, ov);
+            else tld16x256_x4(ta, ov);
+#pragma unroll
+            for (int u = 0; u < HD / 8; ++u) {
+              ov[4 * u] *= alphaA;
+              ov[4 * u + 1] *= alphaA;
+              ov[4 * u + 2] *= alphaB;
+              ov[4 * u + 3] *= alphaB;
+            }
+            if constexpr (HD == 64) tst16x256_x8(ta, ov);
+            else tst16x256_x4(ta, ov);
+          }
+          // P_T as bf16 pairs over the first half of its S buffer: this half's
+          // keys are word columns [half * HC / 2, (half + 1) * HC / 2)
+          tst16x128_x8(tS + lane_off + sb * KTC + half * (HC / 2), pk);
+        }
+        tc_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&v_ready[sb]);
+      }
+      // ---- epilogue: wait for the item's last PV product, normalise, write this half
+      const uint32_t Tl = T - 1;
+      if (!mbar_wait(&pv_done[Tl % kNB], (Tl / kNB) & 1, a.status)) ok = false;
+      tc_after();
+      if (warp_live) {
+        float lA = l_runA, lB = l_runB;
+        lA += __shfl_xor_sync(0xffffffffu, lA, 1);
+        lB += __shfl_xor_sync(0xffffffffu, lB, 1);
+        lA += __shfl_xor_sync(0xffffffffu, lA, 2);
+        lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+        if (cq == 0) {
+          xs(2, half, rlA) = lA;
+          xs(2, half, rlB) = lB;
+        }
+        pair_sync();
+        const float ltA = lA + xs(2, half ^ 1, rlA), ltB = lB + xs(2, half ^ 1, rlB);
+        const float invA = ltA > 0.f ? __fdividef(1.0f, ltA) : 0.f;
+        const float invB = ltB > 0.f ? __fdividef(1.0f, ltB) : 0.f;
+        float ov[HD / 2];
+        const uint32_t ta = tO + lane_off + half * HD;
+        if constexpr (HD == 64) tld16x256_x8(ta, ov);
+        else tld16x256_x4(ta, ov);
+        if (ok) {
+          const int colb = half * HD + 2 * cq;
+          if (direct) {
+            __nv_bfloat16* oA = reinterpret_cast<__nv_bfloat16*>(a.o) +
+                                (((int64_t)b * a.D_max + jqA) * a.Hq + hA) * D + colb;
+            __nv_bfloat16* oB = reinterpret_cast<__nv_bfloat16*>(a.o) +
+                                (((int64_t)b * a.D_max + jqB) * a.Hq + hB) * D + colb;
+#pragma unroll
+            for (int u = 0; u < HD / 8; ++u) {
+              if (liveA)
+                *reinterpret_cast<uint32_t*>(oA + 8 * u) =
+                    pack_bf16x2(ov[4 * u] * invA, ov[4 * u + 1] * invA);
+              if (liveB)
+                *reinterpret_cast<uint32_t*>(oB + 8 * u) =
+                    pack_bf16x2(ov[4 * u + 2] * invB, ov[4 * u + 3] * invB);
+            }
+          } else {
+            float* pA = L.part_o +
+                        ((((int64_t)b * a.Hq + hA) * a.D_max + jqA) * L.splits + split) * D + colb;
+            float* pB = L.part_o +
+                        ((((int64_t)b * a.Hq + hB) * a.D_max + jqB) * L.splits + split) * D + colb;
+#pragma unroll
+            for (int u = 0; u < HD / 8; ++u) {
+              if (liveA)
+                *reinterpret_cast<float2*>(pA + 8 * u) =
+                    make_float2(ov[4 * u] * invA, ov[4 * u + 1] * invA);
+              if (liveB)
+                *reinterpret_cast<float2*>(pB + 8 * u) =
+                    make_float2(ov[4 * u + 2] * invB, ov[4 * u + 3] * invB);
+            }
+          }
+          if (half == 0 && cq == 0) {
+            const float lseA =
+                ltA > 0.f ? (m_runA * (c2 / kLog2eTC) + __logf(ltA)) : -INFINITY;
+            const float lseB =
+                ltB > 0.f ? (m_runB * (c2 / kLog2eTC) + __logf(ltB)) : -INFINITY;
+            if (direct) {
+              if (a.lse != nullptr && liveA) a.lse[((int64_t)b * a.Hq + hA) * a.D_max + jqA] = lseA;
+              if (a.lse != nullptr && liveB) a.lse[((int64_t)b * a.Hq + hB) * a.D_max + jqB] = lseB;
+            } else {
+              if (liveA)
+                L.part_lse[(((int64_t)b * a.Hq + hA) * a.D_max + jqA) * L.splits + split] = lseA;
+              if (liveB)
+                L.part_lse[(((int64_t)b * a.Hq + hB) * a.D_max + jqB) * L.splits + split] = lseB;
+            }
+          }
+        }
+      }
+      // O[s] and the item slot are free for item k + 2
+      tc_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&o_empty[s]);
+        mbar_arrive(&it_empty[s]);
+      }
+    }
   } else {
     // ------------------------------------------------------------- softmax
     const int quarter = warp & 3, half = warp >> 2;
@@ -785,10 +1142,17 @@ bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max) {
          D_max * G > SSD_ATTN_TC_MIN_ROWS;
 }
 
+namespace {
+// Query rows per tile: 64 when a KV group's rows fit (M = 64 products, their
+// softmax spread over the four lane quarters), else 128.
+int32_t tc_tile_rows(int32_t D_max, int32_t G) { return D_max * G <= 64 ? 64 : kBM; }
+}  // namespace
+
 TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max) {
   TcPlan p;
   const int32_t G = Hq / Hkv;
-  p.mtiles = (D_max * G + kBM - 1) / kBM;
+  const int32_t bm = tc_tile_rows(D_max, G);
+  p.mtiles = (D_max * G + bm - 1) / bm;
   const int64_t base = (int64_t)B * Hkv * p.mtiles;
   const int32_t target = device_sm_count();  // one CTA per SM
   const int32_t max_splits = max(1, (L_max + 2 * KTC - 1) / (2 * KTC));  // >= 2 tiles each
@@ -802,15 +1166,16 @@ TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int3
 }
 
 cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
-                                float* part_lse, cudaStream_t stream) {
+                                float* part_lse, cudaStream_t stream, bool pdl) {
   EncodeTiledFnTc fn = encode_tc();
   if (fn == nullptr) return cudaErrorInvalidValue;
   const int32_t G = a.Hq / a.Hkv;
+  const int32_t bm = tc_tile_rows(a.D_max, G);
   CUtensorMap tq, tk, tv;
   {
     cuuint64_t dims[3] = {(cuuint64_t)a.d, (cuuint64_t)a.Hq, (cuuint64_t)a.B * a.D_max};
     cuuint64_t strides[2] = {(cuuint64_t)a.d * 2, (cuuint64_t)a.Hq * a.d * 2};
-    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(kBM / G)};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(bm / G)};
     cuuint32_t estr[3] = {1, 1, 1};
     if (fn(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), dims, strides, box,
            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -843,21 +1208,17 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq
   const int64_t n_items = (int64_t)a.B * a.Hkv * p.mtiles * p.splits;
   const dim3 grid((unsigned)std::min<int64_t>(n_items, device_sm_count()));
   const dim3 block(kThreadsTC);
-  cudaError_t e;
-  if (a.d == 128) {
-    const size_t smem = tc_smem_bytes<128>();
-    e = cudaFuncSetAttribute(frontier_attn_tc_kernel<128>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto launch = [&](auto kernel, size_t smem) {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
     if (e != cudaSuccess) return e;
-    frontier_attn_tc_kernel<128><<<grid, block, smem, stream>>>(tq, tk, tv, a, L);
-  } else {
-    const size_t smem = tc_smem_bytes<64>();
-    e = cudaFuncSetAttribute(frontier_attn_tc_kernel<64>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    frontier_attn_tc_kernel<64><<<grid, block, smem, stream>>>(tq, tk, tv, a, L);
-  }
-  return cudaGetLastError();
+    return launch_kernel(kernel, grid, block, smem, stream, pdl, tq, tk, tv, a, L);
+  };
+  if (a.d == 128)
+    return bm == 64 ? launch(frontier_attn_tc_kernel<128, 64>, tc_smem_bytes<128, 64>())
+                    : launch(frontier_attn_tc_kernel<128, 128>, tc_smem_bytes<128, 128>());
+  return bm == 64 ? launch(frontier_attn_tc_kernel<64, 64>, tc_smem_bytes<64, 64>())
+                  : launch(frontier_attn_tc_kernel<64, 128>, tc_smem_bytes<64, 128>());
 }
 
 }  // namespace ssd

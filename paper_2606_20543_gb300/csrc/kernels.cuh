@@ -245,8 +245,12 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
                            int32_t L_max);
 // defer_combine: leave the split-KV combine (if the plan has splits) to
 // launch_attention_combine, so that another kernel can be queued between.
+// pdl: the tcgen05 kernel is launched as a programmatic dependent of the kernel
+// before it (it reads none of that kernel's results, starts as its CTAs retire,
+// and lets the kernel after it be scheduled only once that kernel completed);
+// the mma.sync kernel is always launched plainly.
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream,
-                             bool defer_combine = false);
+                             bool defer_combine = false, bool pdl = false);
 cudaError_t launch_attention_combine(const AttnArgs& a, void* ws, cudaStream_t stream);
 int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
                        int32_t D_max, int32_t L_max);
@@ -263,7 +267,7 @@ struct TcPlan {
 bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max);
 TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
 cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
-                                float* part_lse, cudaStream_t stream);
+                                float* part_lse, cudaStream_t stream, bool pdl = false);
 // Same as launch_attention with the library's static device scratch as the
 // workspace (ssd_verify_attention_noalloc); cudaErrorMemoryAllocation if the
 // problem needs more than SSD_NOALLOC_SCRATCH_BYTES.
