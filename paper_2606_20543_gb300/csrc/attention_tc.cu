@@ -355,6 +355,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     // every S/P buffer starts free: the PV arrivals of the first round
     for (int s = 0; s < kNB; ++s) mbar_arrive(&k_ready[s]);
   }
+  if (warp == kSoftWarps && lane < 3)  // the first copies need the descriptors
+    prefetch_tensormap(lane == 0 ? &tmQ : (lane == 1 ? &tmK : &tmV));
   if (warp == 0) {
     tmem_alloc_tc(tmem_slot, kTmemCols);
     tmem_relinquish_tc();
