@@ -10,11 +10,13 @@
 //
 // Design (GB300): a persistent grid of four CTAs per SM, each walking rows
 // blockIdx.x, blockIdx.x + gridDim.x, ...  A dedicated producer warp streams
-// every row twice with bulk TMA copies, 256 entries per consumer warp of both
-// logit rows per stage, through a shared-memory ring: once from HBM for the
-// statistics, and once more (from L2, microseconds later) for the residual
-// draw; it runs ahead into the next row while the consumers finish the
-// current one.  The consumers are latency-bound, so the arithmetic is kept
+// every row with bulk TMA copies, 256 entries per consumer warp of both logit
+// rows per stage, through a shared-memory ring: once from HBM for the
+// statistics, and, when the kernel draws the residual tokens itself, once
+// more (from L2, microseconds later) for the draw; it runs ahead into the next
+// row while the consumers finish the current one.  Under (A), and in a
+// one-round prefix-commit step (lazy: only the committed tokens are drawn, by
+// resolve_kernel below), every row is streamed once.  The consumers are latency-bound, so the arithmetic is kept
 // short: per first-pass chunk each thread folds its 8 entries of both rows
 // into online (max, sum of 2^x) statistics with a branch-free rescale,
 // three-input maxima and packed fp32 pairs (fma/add .f32x2) for the exponent

@@ -7,7 +7,8 @@
 //
 // Design (GB300, tcgen05 + TMEM): a persistent kernel, one CTA per SM, that
 // walks work items (KV split, sequence, KV head, tile of 128 query rows =
-// drafts x the Hq/Hkv heads sharing the KV head).  Sequences are taken
+// drafts x the Hq/Hkv heads sharing the KV head; 64-row tiles with M = 64
+// products when a KV head's query rows fit in 64).  Sequences are taken
 // longest first and the items are dealt to the CTAs in snake order, so the
 // long items start early and every CTA gets a similar share.
 //  * warp 8 (producer): decodes the next item, checks and converts its draft
