@@ -177,9 +177,9 @@ class ClockSampler:
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
     # acceptance part of a step: accept_kernel (one pass) + resolve_kernel (committed draws)
-    ("accept", 2): ("accept.cu", "beaf1223a65ae37b", 147920768 + 167168 + 3185408, None),
-    ("attention", 2): ("attention_tc.cu", "6836c8344e2b7782", 102307840 + 65024, None),
-    ("attention", 3): ("attention_tc.cu", "6836c8344e2b7782", 53834624 + 78976, None),
+    ("accept", 2): ("accept.cu", "594e516457d01897", 147920896 + 431872 + 3185152, None),
+    ("attention", 2): ("attention_tc.cu", "f04b60df37aa4d9c", 102185472 + 67072, None),
+    ("attention", 3): ("attention_tc.cu", "f04b60df37aa4d9c", 53835776 + 3584, None),
     ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
 }
 
