@@ -646,7 +646,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
 // global memory; the last part to finish (a ticket per sequence) scans the
 // masses in vocabulary order and re-walks the chosen block exactly as the
 // eager kernel does for that row.
-constexpr int kRBlocks = 4;  // blocks per part
+constexpr int kRBlocks = 2;  // blocks per part: one batch of loads
 
 __device__ __forceinline__ void resolve_part_masses(const float4* tp, const float4* dp, int32_t bk0,
                                                     int32_t bk1, int32_t nv, float2 cc, float2 ncp,
@@ -680,6 +680,26 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   extern __shared__ __align__(16) float rmass[];  // [nblocks], last part only
   const int32_t part = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
   const int32_t nblocks = ((a.V + kChunk - 1) / kChunk) * kBlocksPerChunk;  // resolve_blocks(V)
+  const int32_t nv = a.V >> 2;
+  const int32_t bk0 = part * kRBlocks, bk1 = min(nblocks, bk0 + kRBlocks);
+  // The first draft is the most likely committed rejection: its statistics and
+  // this part's blocks of both rows are loaded before the counts are known.
+  const int64_t r0 = (int64_t)b * a.D_max;
+  const float2 st0 = a.stats[r0];
+  float4 xp[kRBlocks][2], xq[kRBlocks][2];
+  auto load_part = [&](const float4* tp, const float4* dp, bool from_p) {
+#pragma unroll
+    for (int k = 0; k < kRBlocks; ++k)
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int32_t i = (bk0 + k) * 64 + half * 32 + lane;
+        const bool in = bk0 + k < bk1 && i < nv;
+        xp[k][half] = in ? tp[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+        xq[k][half] = (in && !from_p) ? dp[i] : xp[k][half];
+      }
+  };
+  load_part(reinterpret_cast<const float4*>(a.tgt + r0 * a.ld),
+            reinterpret_cast<const float4*>(a.drf + r0 * a.ld), false);
   int32_t n = a.n_drafts[b];
   const bool bad_n = n < 0 || n > a.D_max;  // a caller's frontier (ssd_verify_accept)
   n = bad_n ? (n < 0 ? 0 : a.D_max) : n;
@@ -690,8 +710,8 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   int32_t j = -1;
   if (n > 0 && prefix < n) j = prefix;                             // first rejected draft
   else if (a.bonus && n > 0 && prefix == n && n < a.D_max) j = n;  // the bonus row
-  const int64_t r = (int64_t)b * a.D_max + (j < 0 ? 0 : j);
-  const float2 st = j < 0 ? make_float2(NAN, NAN) : a.stats[r];
+  const int64_t r = r0 + (j < 0 ? 0 : j);
+  const float2 st = j < 0 ? make_float2(NAN, NAN) : (j == 0 ? st0 : a.stats[r]);
   if (!(st.x == st.x)) {  // nothing to draw, or an invalid row the acceptance pass reported
     pdl_wait();
     return;
@@ -700,12 +720,21 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   const float c = kLog2e / a.temperature;
   const float2 cc = make_float2(c, c);
   const float2 ncp = make_float2(-st.x, -st.x), ncq = make_float2(-st.y, -st.y);
-  const int32_t nv = a.V >> 2;
   const float4* tp = reinterpret_cast<const float4*>(a.tgt + r * a.ld);
   const float4* dp = reinterpret_cast<const float4*>(a.drf + r * a.ld);
   float* gmass = a.mass + (int64_t)b * nblocks;
-  const int32_t bk0 = part * kRBlocks, bk1 = min(nblocks, bk0 + kRBlocks);
-  resolve_part_masses(tp, dp, bk0, bk1, nv, cc, ncp, ncq, is_bonus, gmass, lane);
+  if (j != 0) load_part(tp, dp, is_bonus);  // the speculative rows were not the committed one
+  // this part's block masses, with the arithmetic of resolve_part_masses
+#pragma unroll
+  for (int k = 0; k < kRBlocks; ++k) {
+    const int32_t bk = bk0 + k;
+    if (bk >= bk1) break;  // warp-uniform
+    float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
+    if (bk * 64 + lane < nv) w0 = weights4(xp[k][0], xq[k][0], cc, ncp, ncq, is_bonus);
+    if (bk * 64 + 32 + lane < nv) w1 = weights4(xp[k][1], xq[k][1], cc, ncp, ncq, is_bonus);
+    const float m = warp_sum(((w0.x + w0.y) + (w0.z + w0.w)) + ((w1.x + w1.y) + (w1.z + w1.w)));
+    if (lane == 0) gmass[bk] = m;
+  }
   // last part to finish: its fence orders every part's masses before its ticket
   __threadfence();
   int32_t last = 0;
