@@ -177,7 +177,7 @@ class ClockSampler:
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
     # acceptance part of a step: accept_kernel (one pass) + resolve_kernel (committed draws)
-    ("accept", 2): ("accept.cu", "594e516457d01897", 147920896 + 431872 + 3185152, None),
+    ("accept", 2): ("accept.cu", "3419b86a0a387073", 147920128 + 249728 + 3382272, None),
     ("attention", 2): ("attention_tc.cu", "f04b60df37aa4d9c", 102185472 + 67072, None),
     ("attention", 3): ("attention_tc.cu", "f04b60df37aa4d9c", 53835776 + 3584, None),
     ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
