@@ -333,9 +333,10 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * rules, ref_rows, strategies (A) and (B) and the fused path draw every row.
  * Streams: logits path — the acceptance pass computes the frontier itself
  * (and writes n_drafts and draft_pos) and the attention computes the same
- * frontier from cache_len.  With committed draws only and at least
- * 2 x (SM count) rows, everything runs on `stream`: acceptance, attention,
- * then the counts and committed draws as a programmatic dependent of the
+ * frontier from cache_len.  With at least 2 x (SM count) rows and either
+ * committed draws only, or strategy (A) with at most (SM count) rows that can
+ * hold a draft, everything runs on `stream`: acceptance, attention,
+ * then the counts (and committed draws) as a programmatic dependent of the
  * attention (they need only the acceptance's results, start once every
  * attention CTA is resident and wait for the attention before they exit, so
  * stream order holds).  Otherwise, and on the fused path (frontier first,

@@ -3,6 +3,8 @@
 // caller's stream.  No allocation, no synchronisation.
 #include <math.h>
 
+#include <algorithm>
+
 #include "kernels.cuh"
 
 using namespace ssd;
@@ -606,7 +608,17 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
     // out (a1 + a3-a5); the attention computes the same frontier from
     // cache_len (a2), so the two need no frontier launch before them.
     a.raster = 1;
-    if (lazy_draws(x) && x->B * x->D_max >= 2 * device_sm_count()) {
+    // Rows that can hold a draft: the frontier bound per sequence (+ the bonus row).
+    const int64_t live_rows =
+        (int64_t)x->B * std::min<int32_t>(x->D_max, attention_rows_hint(x->grid, x->D_max) +
+                                                        (x->commit == SSD_COMMIT_PREFIX_BONUS));
+    // Measured on GB300: lazy (C) gains from hiding its draws under the attention; greedy,
+    // which has nothing to hide, gains from this order only when its pass is short (few
+    // live rows, e.g. the horizontal stage: 33.4 -> 31.5 us), and loses on the sweep.
+    const bool serial =
+        x->B * x->D_max >= 2 * device_sm_count() &&
+        (lazy_draws(x) || (x->strategy == SSD_STRATEGY_GREEDY && live_rows <= device_sm_count()));
+    if (serial) {
       // A lazy pass that fills the GPU, on `stream` alone: the acceptance;
       // the attention, which reads none of its results, as a programmatic
       // dependent (the tcgen05 kernel starts as the acceptance's CTAs retire

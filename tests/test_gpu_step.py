@@ -319,3 +319,54 @@ def test_verify_accept_matches_the_step(ssd):
               "next_cache_len", "status"):
         assert np.array_equal(r[k], r2[k]), k
     assert np.array_equal(r["ratio"].view(np.uint32), r2["ratio"].view(np.uint32))
+
+
+@pytest.mark.parametrize("strategy", ["accept_reject", "greedy", "sample"])
+def test_horizontal_stage_large_batch(ssd, strategy):
+    """The horizontal stage on a batch of 2 x (SM count) padded rows or more, so
+    that (C) and (A) take the single-stream schedule (acceptance, attention,
+    counts as a dependent beside it) and (B) the two-stream one, against the
+    oracle: decisions, committed tokens, bonus tokens and next cache lengths."""
+    from paper_2606_20543_gb300.step import VerifyStep
+    H = W = 16
+    P = 32
+    rng = np.random.default_rng(5)
+    cls = [int(P + x) for x in rng.choice(H * W - 1, size=20, replace=False)]
+    c = synth.make_case("horizontal", grid_h=H, grid_w=W, prefix_len=P, cache_len=cls, Hq=4,
+                        Hkv=4, d=64, V=4096, seed=71, k_v=0)
+    assert c.B * c.D_max >= 2 * torch.cuda.get_device_properties(0).multi_processor_count
+    s = VerifyStep(H, W, P, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V, k_v=0, k_h=5,
+                   strategy=strategy, commit="prefix_bonus")
+    s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=c.tgt_logits,
+             drf_logits=c.drf_logits, uniforms=c.uniforms)
+    s.run()
+    torch.cuda.synchronize()
+    res = s.results()
+    assert res["status"][0] == 0
+    ref = ostep.accept_step(H, W, P, 0, c.cache_len, c.D_max, c.tgt_logits, c.drf_logits,
+                            c.uniforms, strategy=strategy, k_h=5, bonus=True)
+    assert np.array_equal(res["n_drafts"], ref["n_drafts"])
+    rows = ref["decisions"]["rows"]
+    lazy = strategy == "accept_reject"
+    dec = committed_draws(ref["decisions"], res["accepted"][rows], c.D_max) if lazy \
+        else ref["decisions"]
+    ties = compare_decisions(dec, res["out_tok"][rows], res["accepted"][rows],
+                             what=f"horizontal large {strategy}")
+    for b in range(c.B):
+        br = ref["bonus_row"][b]
+        if br < 0:
+            continue
+        if lazy and res["accepted_prefix"][b] != res["n_drafts"][b]:
+            assert res["out_tok"][br] == -1
+        elif not ref["bonus_tie"][b]:
+            assert res["out_tok"][br] == ref["bonus_tok"][b]
+    if ties == 0:
+        assert np.array_equal(res["accepted_count"], ref["accepted_count"])
+        assert np.array_equal(res["next_cache_len"], ref["next_cache_len"])
+    att = ostep.attention_step(H, W, P, c.row_stride, 0, c.cache_len, bf16_to_f64(c.q),
+                               bf16_to_f64(c.k), bf16_to_f64(c.v), c.Hq, c.Hkv, k_h=5)
+    for b, (o_ref, _) in att.items():
+        n = o_ref.shape[0]
+        for h in range(c.Hq):
+            if n:
+                assert attention_error(res["o"][b, :n, h], o_ref[:, h]) < ATTN_TOL
