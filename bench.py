@@ -31,6 +31,22 @@ METRIC = "verify steps/s & accepted tokens/s per GB300; attention+accept HBM GB/
 UNIT = "sequence verify steps/s"  # one unit = one sequence's whole verification pass
 
 
+def max_over_ranks(ms, world, torch, device=None):
+    """The job's time: the slowest rank's (an all-reduce MAX over the process
+    group: NCCL tensors on `device`, gloo tensors on the host); `ms` itself on
+    one rank."""
+    if world <= 1:
+        return ms
+    t = torch.tensor([ms], device=device) if device is not None else torch.tensor([ms])
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, units_per_rank, ms):
+    """Whole-job throughput: the units every rank processed over the job's time."""
+    return world * units_per_rank / (ms / 1000.0)
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -331,10 +347,7 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
     clk = clocks.stop()
     ms = e0.elapsed_time(e1)
     done = int(s.cache_len.sum().item()) == c.B * (c.prefix_len + HW)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, world, torch, dev)
     seq_steps = int(active.sum())
     # dominant kernel at the first step (cache = prefix), per-kernel graphs
     s.cache_len.copy_(init)
@@ -378,7 +391,7 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
     if rank != 0:
         return 0
     line = {
-        "metric": METRIC, "value": world * seq_steps / (ms / 1000.0), "unit": UNIT,
+        "metric": METRIC, "value": job_rate(world, seq_steps, ms), "unit": UNIT,
         "n_gpus": world, "steps": T, "warmup": 2, "ms_per_step": ms / T,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16 attention / f32 acceptance", "data": "synthetic",
@@ -490,10 +503,7 @@ def run_predictor(a, world, rank, dev, torch, ssd):
     clk = clocks.stop()
     ms = e0.elapsed_time(e1)
     calls = reps * chunk
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, world, torch, dev)
     # end to end: the source states in from pinned host memory, the tokens back
     z_host = torch.from_numpy(np.ascontiguousarray(w["z"]).view(np.int16)).view(
         torch.bfloat16).pin_memory()
@@ -518,7 +528,7 @@ def run_predictor(a, world, rank, dev, torch, ssd):
     cpu = None if a.no_cpu_baseline else predictor_oracle_rate(rows, min(a.cpu_seconds, 20.0))
     line = {
         "metric": "draft predictor calls/s (Eq. 2 + argmax GenHead, one row)",
-        "value": world * calls / (ms / 1000.0), "unit": "draft predictor calls/s",
+        "value": job_rate(world, calls, ms), "unit": "draft predictor calls/s",
         "n_gpus": world, "steps": calls, "warmup": max(a.warmup, 3), "ms_per_step": ms / calls,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16 GEMM inputs / f32 accumulation", "data": "synthetic weights",
@@ -695,12 +705,9 @@ def main():
     clk = clocks.stop()
     ms = e0.elapsed_time(e1)
     steps_done = reps * chunk
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, torch, dev)
     ms_per_step = ms / steps_done
-    value = world * steps_done * c.B / (ms / 1000.0)
+    value = job_rate(world, steps_done * c.B, ms)
 
     accepted_tok = []
     for st in steps_obj:
