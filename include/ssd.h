@@ -224,10 +224,10 @@ ssd_status ssd_accept_strategy(int32_t strategy, int32_t rows, int32_t V, const 
                                ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
- * One verify-and-correct round (Sec. 3.3: "We repeat this verify-and-correct
- * procedure for a fixed number of rounds r ... For a rejected position, the
- * previous-round backbone distribution becomes its reference distribution in
- * the next round, while accepted positions retain their current reference").
+ * One verify-and-correct round (Sec. 3.3: the verify-and-correct procedure
+ * runs for a fixed number r of rounds; a position rejected in one round takes
+ * that round's backbone distribution as its reference in the next, and an
+ * accepted position keeps the reference it has).
  * For every row r the rule of ssd_accept_strategy() is applied with
  *     q = softmax(ref_rows[r][0 .. V) / T)   (the row's current reference)
  *     t = tok[r]                             (the position's current token;
