@@ -115,3 +115,65 @@ def test_host_side_validation(lib):
     # workspace too small
     assert so.ssd_verify_attention(ctypes.byref(g), 1, 8, 8, 64, fake, fake, fake, 32, 288, fake,
                                    fake, fake, 0.0, fake, None, None, 0, fake, None) == 7
+
+
+def test_verify_accept_and_step_host_validation(lib):
+    """ssd_verify_accept / ssd_verify_step reject bad arguments on the host
+    (no device memory is touched: every pointer below is a fake)."""
+    so = lib.load()
+    fake = 0x1000
+
+    def args(**kw):
+        a = lib.VerifyArgs()
+        a.grid = lib.grid(16, 16, 32)
+        a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max, a.V = 2, 8, 8, 64, 32, 288, 4096
+        a.cache_len = a.q = a.k = a.v = fake
+        a.tgt_logits = a.drf_logits = fake
+        a.ld = 4096
+        a.temperature = 1.0
+        a.rng = lib.rng(0, 0)
+        for k, v in kw.items():
+            setattr(a, k, v)
+        return a
+
+    def out(**kw):
+        y = lib.VerifyOut()
+        for name in ("n_drafts", "draft_pos", "o", "out_tok", "accepted", "ratio",
+                     "accepted_count", "accepted_prefix", "next_cache_len", "status"):
+            setattr(y, name, fake)
+        for k, v in kw.items():
+            setattr(y, k, v)
+        return y
+
+    def acc(a, y, ws=fake, nbytes=1 << 30):
+        return so.ssd_verify_accept(ctypes.byref(a), ctypes.byref(y), ctypes.c_void_p(ws), nbytes,
+                                    None)
+
+    assert so.ssd_verify_accept(None, None, None, 0, None) == 1
+    assert acc(args(B=0), out()) == 0                                # empty batch: no work
+    g17 = lib.grid(16, 16, 32, row_stride=17)
+    assert acc(args(grid=g17), out()) == 3                           # end-of-line slots
+    assert acc(args(D_max=16), out()) == 2                           # (k_v + 1) W > D_max
+    assert acc(args(cache_len=None), out()) == 1
+    assert acc(args(), out(draft_pos=None)) == 1                     # the frontier is written
+    assert acc(args(commit=99), out()) == 1
+    assert acc(args(strategy=7), out()) == 1
+    assert acc(args(V=4098, ld=4100), out()) == 2                    # V a multiple of 4
+    need = so.ssd_verify_step_workspace(ctypes.byref(args()))
+    assert need > 0
+    assert acc(args(), out(), nbytes=0) == 7
+    # the whole step: the attention's arguments too
+    step = so.ssd_verify_step
+    assert step(ctypes.byref(args(q=None)), ctypes.byref(out()), ctypes.c_void_p(fake), need,
+                None) == 1
+    assert step(ctypes.byref(args(d=96)), ctypes.byref(out()), ctypes.c_void_p(fake), need,
+                None) == 3
+    assert step(ctypes.byref(args()), ctypes.byref(out()), ctypes.c_void_p(fake), need - 1,
+                None) == 7
+    # launch counts: acceptance + attention (+ combine) + counts on the logits path,
+    # and one more (the frontier) on the fused path
+    n_logits = so.ssd_verify_step_launches(ctypes.byref(args()))
+    assert n_logits in (3, 4)
+    fused = args(tgt_logits=None, drf_logits=None, h_tgt=fake, h_drf=fake, w_tgt=fake,
+                 w_drf=fake, hidden=4096)
+    assert so.ssd_verify_step_launches(ctypes.byref(fused)) == n_logits + 1
