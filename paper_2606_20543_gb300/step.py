@@ -32,7 +32,13 @@ class VerifyStep:
 
     Shapes follow include/ssd.h: q [B, D_max, Hq, d], k/v [B, Hkv, L_max, d]
     (bf16), logits [B*D_max, V] (float32) or hidden [B*D_max, hidden] with
-    lm_head weights [hidden, V] (bf16)."""
+    lm_head weights [hidden, V] (bf16).
+
+    Under strategy (C) with commit "prefix" or "prefix_bonus" a step draws only
+    the tokens it commits: out_tok holds the draft token of each accepted row,
+    the residual token of each sequence's first rejection and the bonus token
+    when every draft is accepted; the other rejected rows (discarded by the
+    prefix rule) hold -1.  accepted and ratio are written for every row."""
 
     def __init__(self, grid_h, grid_w, prefix_len, B, Hq, Hkv, d, D_max, L_max, V,
                  hidden=0, k_v=1, row_stride=None, device="cuda", scale=0.0, temperature=1.0,
