@@ -619,12 +619,12 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
         x->B * x->D_max >= 2 * device_sm_count() &&
         (lazy_draws(x) || (x->strategy == SSD_STRATEGY_GREEDY && live_rows <= device_sm_count()));
     if (serial) {
-      // A lazy pass that fills the GPU, on `stream` alone: the acceptance;
-      // the attention, which reads none of its results, as a programmatic
-      // dependent (the tcgen05 kernel starts as the acceptance's CTAs retire
-      // and lets the next kernel be scheduled only once the acceptance has
-      // completed); then a7 (counts and the committed draws) as a
-      // programmatic dependent of the attention: its small CTAs run beside
+      // On `stream` alone: the acceptance; the attention, which reads none of
+      // its results, as a programmatic dependent (the tcgen05 kernel starts
+      // as the acceptance's CTAs retire and lets the next kernel be scheduled
+      // only once the acceptance has completed; the mma.sync kernel starts
+      // after it); then a7 (the counts, with the committed draws when lazy) as
+      // a programmatic dependent of the attention: its small CTAs run beside
       // the attention, in the registers it leaves free.
       e = launch_accept_phase(x, y, ws + attn_ws, stream);
       if (e != cudaSuccess) return SSD_ERR_CUDA;
