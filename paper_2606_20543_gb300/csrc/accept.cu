@@ -61,13 +61,6 @@ constexpr int kMaxV = 1 << 20;                // block-mass table: V / 128 float
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-// 2^x on the MUFU unit (results below 2^-126 flush to zero).
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
 // Barrier among the consumer warps only (the producer warp never joins it).
 __device__ __forceinline__ void consumers_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory");
@@ -81,7 +74,7 @@ __device__ __forceinline__ bool better_arg(float v, int32_t i, float bv, int32_t
 __device__ __forceinline__ void merge(float& m, float& s, float m2, float s2, float c) {
   const float mn = fmaxf(m, m2);
   if (mn == -INFINITY) return;
-  s = s * ex2((m - mn) * c) + s2 * ex2((m2 - mn) * c);
+  s = s * ex2_approx((m - mn) * c) + s2 * ex2_approx((m2 - mn) * c);
   m = mn;
 }
 
@@ -93,17 +86,17 @@ __device__ __forceinline__ float4 weights4(const float4& xp, const float4& xq, f
   const float2 a1 = ffma2(make_float2(xp.z, xp.w), cc, ncp);
   float4 w;
   if (from_p) {
-    w.x = ex2(a0.x);
-    w.y = ex2(a0.y);
-    w.z = ex2(a1.x);
-    w.w = ex2(a1.y);
+    w.x = ex2_approx(a0.x);
+    w.y = ex2_approx(a0.y);
+    w.z = ex2_approx(a1.x);
+    w.w = ex2_approx(a1.y);
   } else {
     const float2 b0 = ffma2(make_float2(xq.x, xq.y), cc, ncq);
     const float2 b1 = ffma2(make_float2(xq.z, xq.w), cc, ncq);
-    w.x = fmaxf(ex2(a0.x) - ex2(b0.x), 0.f);
-    w.y = fmaxf(ex2(a0.y) - ex2(b0.y), 0.f);
-    w.z = fmaxf(ex2(a1.x) - ex2(b1.x), 0.f);
-    w.w = fmaxf(ex2(a1.y) - ex2(b1.y), 0.f);
+    w.x = fmaxf(ex2_approx(a0.x) - ex2_approx(b0.x), 0.f);
+    w.y = fmaxf(ex2_approx(a0.y) - ex2_approx(b0.y), 0.f);
+    w.z = fmaxf(ex2_approx(a1.x) - ex2_approx(b1.x), 0.f);
+    w.w = fmaxf(ex2_approx(a1.y) - ex2_approx(b1.y), 0.f);
   }
   return w;
 }
@@ -115,8 +108,8 @@ __device__ __forceinline__ float2 exp_sum8(const float4& x0, const float4& x1, f
   const float2 a1 = ffma2(make_float2(x0.z, x0.w), cc, nmc);
   const float2 a2 = ffma2(make_float2(x1.x, x1.y), cc, nmc);
   const float2 a3 = ffma2(make_float2(x1.z, x1.w), cc, nmc);
-  const float2 e0 = make_float2(ex2(a0.x), ex2(a0.y)), e1 = make_float2(ex2(a1.x), ex2(a1.y));
-  const float2 e2 = make_float2(ex2(a2.x), ex2(a2.y)), e3 = make_float2(ex2(a3.x), ex2(a3.y));
+  const float2 e0 = make_float2(ex2_approx(a0.x), ex2_approx(a0.y)), e1 = make_float2(ex2_approx(a1.x), ex2_approx(a1.y));
+  const float2 e2 = make_float2(ex2_approx(a2.x), ex2_approx(a2.y)), e3 = make_float2(ex2_approx(a3.x), ex2_approx(a3.y));
   return fadd2(fadd2(e0, e1), fadd2(e2, e3));
 }
 
@@ -406,7 +399,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
       const float nmq = fmaxf(mq, cmq);
       // rescale of the running sums (exactly 1 when the maximum did not move;
       // the initial kLowest is finite, so no -inf - -inf)
-      const float rp = ex2((mp - nmp) * c), rq = ex2((mq - nmq) * c);
+      const float rp = ex2_approx((mp - nmp) * c), rq = ex2_approx((mq - nmq) * c);
       mp = nmp;
       mq = nmq;
       const float2 ep = exp_sum8(p0, p1, cc, make_float2(-mp * c, -mp * c));

@@ -63,99 +63,6 @@ constexpr int kThreadsTC = (kSoftWarps + 4) * 32;  // + K/Q producer, S, V produ
 constexpr float kLog2eTC = 1.4426950408889634f;
 constexpr float kRescale = 8.0f;  // log2 growth of the running max that forces a rescale
 
-__device__ __forceinline__ void tmem_alloc_tc(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(dst)),
-               "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish_tc() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc_tc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tc_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                     uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// D (TMEM) (+)= A (TMEM, 128 lanes x 16 bf16 in 8 columns) * B (shared memory).
-__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                        uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   smem_u32(bar))
-               : "memory");
-}
-__device__ __forceinline__ void tld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-__device__ __forceinline__ void tst32u(uint32_t taddr, const uint32_t* v) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
-      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
-      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
-      "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]),
-      "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]),
-      "r"(v[30]), "r"(v[31])
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tst32(uint32_t taddr, const float* v) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
-      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
-      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
-      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
-      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
-      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
-      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
-      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
-      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
-      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
-      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
-      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ float ex2a(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
 // 16-lane TMEM accesses of the M = 64 products, whose row m sits in lane
 // 32 (m / 16) + m % 16.  .16x256b: thread t holds rows t/4 and t/4 + 8 of the
 // 16 lanes, columns 8u + 2 (t % 4) + {0, 1} of unit u, as registers 4u + {0, 1}
@@ -232,28 +139,9 @@ __device__ __forceinline__ void tst16x128_x8(uint32_t taddr, const uint32_t* v) 
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// tcgen05 shared-memory descriptor: 128-byte swizzle, version 1.
-__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-// The descriptor of base + off: the start address field is (address >> 4) in
-// the low 14 bits, so a 16-byte-multiple offset that keeps the address below
-// 256 KB (all of shared memory) is a plain add.
-__device__ __forceinline__ uint64_t sdesc_at(uint64_t d, uint32_t off) {
-  return d + (uint64_t)(off >> 4);
-}
-
 // kind::f16 instruction descriptor: fp32 D, bf16 A and B, A K-major, M = m (64 or 128).
 __host__ __device__ constexpr uint32_t idesc_f16(int n, bool b_mn_major, int m = kBM) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
-         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+  return idesc_bf16(m, n, false, b_mn_major);
 }
 
 struct TcLaunch {
@@ -359,8 +247,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   if (warp == kSoftWarps && lane < 3)  // the first copies need the descriptors
     prefetch_tensormap(lane == 0 ? &tmQ : (lane == 1 ? &tmK : &tmV));
   if (warp == 0) {
-    tmem_alloc_tc(tmem_slot, kTmemCols);
-    tmem_relinquish_tc();
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
   }
   if (a.B <= kLptMax) {
     // s_order[rank] = the sequence with the rank-th most keys (ties by index)
@@ -379,9 +267,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       s_order[r] = i;
     }
   }
-  tc_before();
+  tc_fence_before();
   __syncthreads();
-  tc_after();
+  tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tS = tmem;            // [kNB] x KTC columns: S_t in fp32, then P_t in bf16
   const uint32_t tO0 = tmem + 256;     // [2] x 128 columns
@@ -566,22 +454,22 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         const int32_t ntiles = items[s].ntiles;
         if (ntiles < 0) break;
         if (!mbar_wait(&q_full[s], (k >> 1) & 1, a.status)) break;
-        tc_after();
-        const uint64_t dq = sdesc(smem_u32(sQ + s * Q_BYTES), 16, 1024);
+        tc_fence_after();
+        const uint64_t dq = smem_desc(smem_u32(sQ + s * Q_BYTES), 16, 1024);
         bool ok = true;
         for (int t = 0; t < ntiles; ++t, ++T) {
           const int sb = T % kNB;
           if (!mbar_wait(&k_ready[sb], (T / kNB) & 1, a.status)) { ok = false; break; }
-          tc_after();
-          const uint64_t dk = sdesc(smem_u32(sK + sb * KV_BYTES), 16, 1024);
+          tc_fence_after();
+          const uint64_t dk = smem_desc(smem_u32(sK + sb * KV_BYTES), 16, 1024);
 #pragma unroll
           for (int ks = 0; ks < D / 16; ++ks) {
             const int sub = ks >> 2, kin = (ks & 3) * 32;
-            umma(tS + sb * KTC, sdesc_at(dq, sub * (BM * 128) + kin),
-                 sdesc_at(dk, sub * (KTC * 128) + kin), kIdescS, ks > 0 ? 1u : 0u);
+            mma_ss(tS + sb * KTC, smem_desc_at(dq, sub * (BM * 128) + kin),
+                 smem_desc_at(dk, sub * (KTC * 128) + kin), kIdescS, ks > 0 ? 1u : 0u);
           }
-          umma_commit(&s_full[sb]);
-          if (t == ntiles - 1) umma_commit(&q_empty[s]);
+          mma_commit(&s_full[sb]);
+          if (t == ntiles - 1) mma_commit(&q_empty[s]);
         }
         if (!ok) break;
       }
@@ -605,16 +493,16 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         for (int t = 0; t < ntiles; ++t, ++T) {
           const int sb = T % kNB;
           if (!mbar_wait(&v_ready[sb], (T / kNB) & 1, a.status)) { ok = false; break; }
-          tc_after();
+          tc_fence_after();
           // A = P in TMEM (16 keys = 8 columns per step), B = V (MN-major: d
           // atoms KTC*128 bytes apart, 8-key groups 1 KB apart; 16 keys = 2 KB)
-          const uint64_t dv = sdesc(smem_u32(sV + sb * KV_BYTES), KTC * 128, 1024);
+          const uint64_t dv = smem_desc(smem_u32(sV + sb * KV_BYTES), KTC * 128, 1024);
 #pragma unroll
           for (int kk = 0; kk < KTC / 16; ++kk)
-            umma_ts(tO0 + s * 128, tS + sb * KTC + kk * 8, sdesc_at(dv, kk * 2048), kIdescO,
+            mma_ts(tO0 + s * 128, tS + sb * KTC + kk * 8, smem_desc_at(dv, kk * 2048), kIdescO,
                     (t == 0 && kk == 0) ? 0u : 1u);
-          umma_commit(&pv_done[sb]);
-          umma_commit(&k_ready[sb]);  // S_{T+kNB} may start: the S/P buffer is free again
+          mma_commit(&pv_done[sb]);
+          mma_commit(&k_ready[sb]);  // S_{T+kNB} may start: the S/P buffer is free again
         }
         if (!ok) break;
       }
@@ -715,7 +603,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       for (int t = 0; t < ntiles; ++t, ++T) {
         const int bb = T & 1, sb = T % kNB;
         if (!mbar_wait(&s_full[sb], (T / kNB) & 1, a.status)) ok = false;
-        tc_after();
+        tc_fence_after();
         float sv[32];
         if (warp_live) tld16x256_x8(tS + lane_off + sb * KTC + half * HC, sv);
         bool movedA = false, movedB = false;
@@ -758,12 +646,12 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           mxB = fmaxf(mxB, xs(bb, half ^ 1, rlB));
           // move a running max only when it grows by more than 2^kRescale
           if (mxA != -INFINITY && (m_runA == -INFINITY || (mxA - m_runA) * c2 > kRescale)) {
-            alphaA = (m_runA == -INFINITY) ? 0.f : ex2a((m_runA - mxA) * c2);
+            alphaA = (m_runA == -INFINITY) ? 0.f : ex2_approx((m_runA - mxA) * c2);
             m_runA = mxA;
             movedA = true;
           }
           if (mxB != -INFINITY && (m_runB == -INFINITY || (mxB - m_runB) * c2 > kRescale)) {
-            alphaB = (m_runB == -INFINITY) ? 0.f : ex2a((m_runB - mxB) * c2);
+            alphaB = (m_runB == -INFINITY) ? 0.f : ex2_approx((m_runB - mxB) * c2);
             m_runB = mxB;
             movedB = true;
           }
@@ -772,10 +660,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           float sA[4] = {0.f, 0.f, 0.f, 0.f}, sB[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int u = 0; u < 8; ++u) {
-            const float eA0 = ex2a(fmaf(sv[4 * u], c2, -moffA));
-            const float eA1 = ex2a(fmaf(sv[4 * u + 1], c2, -moffA));
-            const float eB0 = ex2a(fmaf(sv[4 * u + 2], c2, -moffB));
-            const float eB1 = ex2a(fmaf(sv[4 * u + 3], c2, -moffB));
+            const float eA0 = ex2_approx(fmaf(sv[4 * u], c2, -moffA));
+            const float eA1 = ex2_approx(fmaf(sv[4 * u + 1], c2, -moffA));
+            const float eB0 = ex2_approx(fmaf(sv[4 * u + 2], c2, -moffB));
+            const float eB1 = ex2_approx(fmaf(sv[4 * u + 3], c2, -moffB));
             sA[u & 3] += eA0 + eA1;
             sB[u & 3] += eB0 + eB1;
             pk[2 * u] = pack_bf16x2(eA0, eA1);
@@ -788,7 +676,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           // O may be rescaled once PV_{T-1} is done
           if (__any_sync(0xffffffffu, (movedA || movedB) && t > 0)) {
             if (!mbar_wait(&pv_done[(T - 1) % kNB], ((T - 1) / kNB) & 1, a.status)) ok = false;
-            tc_after();
+            tc_fence_after();
             float ov[HD / 2];
             const uint32_t ta = tO + lane_off + half * HD;
             if constexpr (HD == 64) tld16x256_x8(ta, ov);
@@ -807,14 +695,14 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           // keys are word columns [half * HC / 2, (half + 1) * HC / 2)
           tst16x128_x8(tS + lane_off + sb * KTC + half * (HC / 2), pk);
         }
-        tc_before();
+        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&v_ready[sb]);
       }
       // ---- epilogue: wait for the item's last PV product, normalise, write this half
       const uint32_t Tl = T - 1;
       if (!mbar_wait(&pv_done[Tl % kNB], (Tl / kNB) & 1, a.status)) ok = false;
-      tc_after();
+      tc_fence_after();
       if (warp_live) {
         float lA = l_runA, lB = l_runB;
         lA += __shfl_xor_sync(0xffffffffu, lA, 1);
@@ -882,7 +770,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
       }
       // O[s] and the item slot are free for item k + 2
-      tc_before();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&o_empty[s]);
@@ -955,11 +843,11 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       for (int t = 0; t < ntiles; ++t, ++T) {
         const int bb = T & 1, sb = T % kNB;
         if (!mbar_wait(&s_full[sb], (T / kNB) & 1, a.status)) ok = false;
-        tc_after();
+        tc_fence_after();
         float sv[HC];
         if (warp_live) {
-          tld32(tS + lane_off + sb * KTC + half * HC, sv);
-          tld32(tS + lane_off + sb * KTC + half * HC + 32, sv + 32);
+          tmem_ld32(tS + lane_off + sb * KTC + half * HC, sv);
+          tmem_ld32(tS + lane_off + sb * KTC + half * HC + 32, sv + 32);
         }
         bool moved = false;
         float alpha = 1.f;
@@ -1005,7 +893,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           mx = fmaxf(mx, xslot(bb, half ^ 1));
           // move the running max only when it grows by more than 2^kRescale
           if (mx != -INFINITY && (m_run == -INFINITY || (mx - m_run) * c2 > kRescale)) {
-            alpha = (m_run == -INFINITY) ? 0.f : ex2a((m_run - mx) * c2);
+            alpha = (m_run == -INFINITY) ? 0.f : ex2_approx((m_run - mx) * c2);
             m_run = mx;
             moved = true;
           }
@@ -1013,10 +901,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           float r8[HC / 4];
 #pragma unroll
           for (int i = 0; i < HC / 4; ++i) {
-            const float e0 = ex2a(fmaf(sv[4 * i], c2, -moff));
-            const float e1 = ex2a(fmaf(sv[4 * i + 1], c2, -moff));
-            const float e2 = ex2a(fmaf(sv[4 * i + 2], c2, -moff));
-            const float e3 = ex2a(fmaf(sv[4 * i + 3], c2, -moff));
+            const float e0 = ex2_approx(fmaf(sv[4 * i], c2, -moff));
+            const float e1 = ex2_approx(fmaf(sv[4 * i + 1], c2, -moff));
+            const float e2 = ex2_approx(fmaf(sv[4 * i + 2], c2, -moff));
+            const float e3 = ex2_approx(fmaf(sv[4 * i + 3], c2, -moff));
             r8[i] = (e0 + e1) + (e2 + e3);
             pk[2 * i] = pack_bf16x2(e0, e1);
             pk[2 * i + 1] = pack_bf16x2(e2, e3);
@@ -1031,29 +919,29 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         if (warp_live) {
           if (__any_sync(0xffffffffu, moved && t > 0)) {
             if (!mbar_wait(&pv_done[(T - 1) % kNB], ((T - 1) / kNB) & 1, a.status)) ok = false;
-            tc_after();
+            tc_fence_after();
             float ov[32];
 #pragma unroll 1
             for (int cc = 0; cc < HD / 32; ++cc) {
               const uint32_t ta = tO + lane_off + half * HD + cc * 32;
-              tld32(ta, ov);
+              tmem_ld32(ta, ov);
 #pragma unroll
               for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-              tst32(ta, ov);
+              tmem_st32(ta, ov);
             }
           }
           // P_T as bf16 pairs over the first half of its S buffer: this half's keys
           // are columns [half * HC / 2, (half + 1) * HC / 2)
-          tst32u(tS + lane_off + sb * KTC + half * (HC / 2), pk);
+          tmem_st32(tS + lane_off + sb * KTC + half * (HC / 2), pk);
         }
-        tc_before();
+        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&v_ready[sb]);
       }
       // ---- epilogue: wait for the item's last PV product, normalise, write this half
       const uint32_t Tl = T - 1;
       if (!mbar_wait(&pv_done[Tl % kNB], (Tl / kNB) & 1, a.status)) ok = false;
-      tc_after();
+      tc_fence_after();
       if (warp_live) {
         xslot(2, half) = l_run;
         pair_sync();
@@ -1065,7 +953,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll 1
         for (int cc = 0; cc < HD / 32; ++cc) {
           float ov[32];
-          tld32(tO + lane_off + half * HD + cc * 32, ov);
+          tmem_ld32(tO + lane_off + half * HD + cc * 32, ov);
           if (!live || !ok) continue;
           const int col = half * HD + cc * 32;
           if (direct) {
@@ -1098,7 +986,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
       }
       // O[s] and the item slot are free for item k + 2
-      tc_before();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&o_empty[s]);
@@ -1107,11 +995,11 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     }
   }
   // ---- teardown
-  tc_before();
+  tc_fence_before();
   __syncthreads();
   if (warp == 0) {
-    tc_after();
-    tmem_dealloc_tc(tmem, kTmemCols);
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 

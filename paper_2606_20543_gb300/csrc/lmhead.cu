@@ -51,81 +51,9 @@ struct LmPartial {  // one row, one vocabulary tile (32 bytes)
   float pad;
 };
 
-// ---------------------------------------------------------------- tcgen05
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(dst)),
-               "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-// D[tmem] (+)= A[smem] * B[smem], bf16 inputs, fp32 accumulation.
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// Arrive on `bar` once every MMA this thread issued so far has completed.
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   smem_u32(bar))
-               : "memory");
-}
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// Shared-memory matrix descriptor (tcgen05): start address, leading and
-// stride byte offsets (16-byte units), descriptor version 1, 128-byte swizzle.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
 // Instruction descriptor, kind::f16: fp32 D, bf16 A and B, A K-major,
 // B MN-major, N = 128, M = 128.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
-                            ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-
-__device__ __forceinline__ float ex2f(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
+constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN, false, true);
 
 __device__ __forceinline__ bool better(float v, int32_t i, float bv, int32_t bi) {
   return v > bv || (v == bv && (uint32_t)i < (uint32_t)bi);
@@ -134,7 +62,7 @@ __device__ __forceinline__ bool better(float v, int32_t i, float bv, int32_t bi)
 __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c) {
   const float mn = fmaxf(m, m2);
   if (mn == -INFINITY) return;
-  s = s * ex2f((m - mn) * c) + s2 * ex2f((m2 - mn) * c);
+  s = s * ex2_approx((m - mn) * c) + s2 * ex2_approx((m2 - mn) * c);
   m = mn;
 }
 
@@ -282,8 +210,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
           const uint64_t da_t = smem_desc(st + m * kTileA + kk * 32, 16, 1024);
           const uint64_t da_d = smem_desc(st + (mt + m) * kTileA + kk * 32, 16, 1024);
           const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
-          mma_bf16(tmem + m * 2 * kBN, da_t, db_t, kIdesc, acc);
-          mma_bf16(tmem + m * 2 * kBN + kBN, da_d, db_d, kIdesc, acc);
+          mma_ss(tmem + m * 2 * kBN, da_t, db_t, kIdesc, acc);
+          mma_ss(tmem + m * 2 * kBN + kBN, da_d, db_d, kIdesc, acc);
         }
       }
       mma_commit(&empty[s]);
@@ -337,8 +265,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       const float cmpc = cmp * c, cmqc = cmq * c;
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        lp += ex2f(fmaf(v[i], c, -cmpc));
-        lq += ex2f(fmaf(w[i], c, -cmqc));
+        lp += ex2_approx(fmaf(v[i], c, -cmpc));
+        lq += ex2_approx(fmaf(w[i], c, -cmqc));
       }
       merge_ms(mp, sp, cmp, lp, c);
       merge_ms(mq, sq, cmq, lq, c);
@@ -472,7 +400,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       if (draw) {
 #pragma unroll
         for (int i = 0; i < 32; ++i)
-          mass += fmaxf(ex2f(fmaf(v[i], c, -ri.Cp)) - ex2f(fmaf(w[i], c, -ri.Cq)), 0.f);
+          mass += fmaxf(ex2_approx(fmaf(v[i], c, -ri.Cp)) - ex2_approx(fmaf(w[i], c, -ri.Cq)), 0.f);
       }
     }
     if (draw) L.mass[(int64_t)row * L.ncta + cta] = mass;
@@ -499,7 +427,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
               mk[q] = L.mass[(int64_t)row * L.ncta + k];
             } else {  // masses of p itself, from the tile partials
               const float4 p0 = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta + k)[0];
-              mk[q] = p0.y * ex2f(p0.x * c - ri.Cp);
+              mk[q] = p0.y * ex2_approx(p0.x * c - ri.Cp);
             }
           }
         }
@@ -568,8 +496,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       if (mine && pick < 0) {
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float pv = ex2f(fmaf(v[i], c, -ri.Cp));
-          const float wt = from_p ? pv : fmaxf(pv - ex2f(fmaf(w[i], c, -ri.Cq)), 0.f);
+          const float pv = ex2_approx(fmaf(v[i], c, -ri.Cp));
+          const float wt = from_p ? pv : fmaxf(pv - ex2_approx(fmaf(w[i], c, -ri.Cq)), 0.f);
           cum += wt;
           if (wt > 0.f) {
             lastpos = v0 + ch * 32 + i;
