@@ -85,11 +85,28 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 6
+#define SSD_ABI_VERSION 7
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
 const char* ssd_status_string(ssd_status s);
+
+/* ---------------------------------------------------------------------------
+ * Failure detection (no counterpart in the paper).  Every wait of a kernel on
+ * another CTA, a copy or a product is bounded; a wait that runs out records
+ * SSD_ERR_TIMEOUT in *status, and the kernel skips the rest of its work,
+ * releases its tensor memory and returns, so the context stays usable.  Both
+ * controls are process-wide and apply to launches enqueued after the call.
+ *  ssd_set_wait_limit(polls): the polls after which each bounded wait of the
+ *    kernels with grid-wide waits (the fused lm_head) gives up; 0 restores the
+ *    default, well above a second of waiting.
+ *  ssd_set_barrier_shortfall(n): makes the fused lm_head's grid barriers wait
+ *    for n arrivals more than its CTAs make, so that they cannot complete and
+ *    run out after the wait limit: a way to exercise the timeout path without
+ *    faulting anything.  0 (the default) turns it off.
+ * ------------------------------------------------------------------------- */
+void ssd_set_wait_limit(uint32_t max_polls);
+void ssd_set_barrier_shortfall(uint32_t arrivals);
 
 /* ---------------------------------------------------------------------------
  * a1. Frontier (Sec. 3.3: horizontal heads complete the current row, the
@@ -158,10 +175,12 @@ ssd_status ssd_verify_attention(const ssd_grid* grid, int32_t B, int32_t Hq, int
  *  - Limit: problems whose workspace (ssd_verify_attention_workspace()) is
  *    larger than SSD_NOALLOC_SCRATCH_BYTES are rejected with
  *    SSD_ERR_WORKSPACE before anything is enqueued.
- *  - Set-up: the first call on each device looks up the device address of the
- *    scratch array (cudaGetSymbolAddress, with that device current), which
- *    may load the library's device code; make that first call before any
- *    stream capture.  A failed look-up returns SSD_ERR_CUDA.
+ *  - Set-up: every call looks up the device address of the scratch array on
+ *    the current device (cudaGetSymbolAddress).  The first call on a device
+ *    is its set-up: it may load the library's device code there, so make it
+ *    before any stream capture (and, after a device reset, make the next call
+ *    outside a capture too).  Later look-ups are host-side only.  A failed
+ *    look-up returns SSD_ERR_CUDA.
  *  - Sharing: every call on a device uses the same scratch array and leaves
  *    its contents behind.  Nothing in it needs to start at zero: each call
  *    writes every scratch word it later reads.  Calls that overlap on the

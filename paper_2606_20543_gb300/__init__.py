@@ -21,7 +21,8 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
                 4: "SSD_ERR_CUDA", 5: "SSD_ERR_TIMEOUT", 6: "SSD_ERR_DEVICE_BOUNDS",
                 7: "SSD_ERR_WORKSPACE"}
 
-EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_frontier", "ssd_verify_attention_workspace",
+EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_set_wait_limit",
+            "ssd_set_barrier_shortfall", "ssd_frontier", "ssd_verify_attention_workspace",
             "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
             "ssd_accept_round", "ssd_stage_shift", "ssd_draft_predict_workspace",
             "ssd_draft_predict",
@@ -97,6 +98,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     sig = {
         "ssd_abi_version": (I32, []),
         "ssd_status_string": (ctypes.c_char_p, [I32]),
+        "ssd_set_wait_limit": (None, [ctypes.c_uint32]),
+        "ssd_set_barrier_shortfall": (None, [ctypes.c_uint32]),
         "ssd_frontier": (I32, [ctypes.POINTER(Grid), I32, P, I32, P, P, P, P]),
         "ssd_verify_attention_workspace": (SZ, [I32, I32, I32, I32, I32, I32]),
         "ssd_verify_attention": (I32, [ctypes.POINTER(Grid), I32, I32, I32, I32, P, P, P, I32, I32,
@@ -160,6 +163,16 @@ def rng(seed: int = 0, offset: int = 0, uniforms=None) -> Rng:
 
 def ssd_abi_version() -> int:
     return load().ssd_abi_version()
+
+
+def ssd_set_wait_limit(max_polls: int) -> None:
+    """Poll limit of the bounded device waits of later launches (0: default)."""
+    load().ssd_set_wait_limit(int(max_polls))
+
+
+def ssd_set_barrier_shortfall(arrivals: int) -> None:
+    """Extra arrivals the fused lm_head's grid barriers wait for (0: off)."""
+    load().ssd_set_barrier_shortfall(int(arrivals))
 
 
 def ssd_status_string(code: int) -> str:

@@ -4,10 +4,26 @@
 #include <math.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "kernels.cuh"
 
 using namespace ssd;
+
+namespace ssd {
+
+namespace {
+std::atomic<uint32_t> g_wait_polls{0};
+std::atomic<uint32_t> g_barrier_shortfall{0};
+}  // namespace
+
+uint32_t wait_poll_limit() {
+  const uint32_t p = g_wait_polls.load(std::memory_order_relaxed);
+  return p == 0 ? kMaxPolls : p;
+}
+uint32_t barrier_shortfall() { return g_barrier_shortfall.load(std::memory_order_relaxed); }
+
+}  // namespace ssd
 
 namespace {
 
@@ -96,6 +112,14 @@ ssd_status check_logits(int32_t rows, int32_t V, const float* tgt, const float* 
 extern "C" {
 
 int32_t ssd_abi_version(void) { return SSD_ABI_VERSION; }
+
+void ssd_set_wait_limit(uint32_t max_polls) {
+  g_wait_polls.store(max_polls, std::memory_order_relaxed);
+}
+
+void ssd_set_barrier_shortfall(uint32_t arrivals) {
+  g_barrier_shortfall.store(arrivals, std::memory_order_relaxed);
+}
 
 const char* ssd_status_string(ssd_status s) {
   switch (s) {

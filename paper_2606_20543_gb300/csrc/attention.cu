@@ -19,7 +19,6 @@
 // softmax is the online (running max / running sum) form with quad shuffles.
 // Long caches are split over CTAs; a combine kernel merges the splits by
 // their log-sum-exp.
-#include <mutex>
 
 #include "kernels.cuh"
 
@@ -592,28 +591,21 @@ static cudaError_t launch_combine(const AttnArgs& a, const AttnLaunch& L, cudaSt
 // Scratch of ssd_verify_attention_noalloc(): it stands in for the caller's
 // workspace (per-sequence flags and split-KV partials).  Host code must not
 // pass `g_noalloc_scratch` itself to a kernel: on the host that name is a
-// stand-in, not a device address.  The device address is looked up once per
-// device below.
+// stand-in, not a device address.  Every call looks the device address up
+// below, with the caller's device current.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[SSD_NOALLOC_SCRATCH_BYTES];
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device (set-up on the
-// first call per device, with that device current).  nullptr on failure.
+// Device address of the scratch array on the current device, or nullptr.  The
+// first look-up on a device is its set-up (it may load the library's device
+// code there); later ones are a host-side table look-up.  Looking it up on
+// every call, rather than caching it, means a device reset (which reloads the
+// module, possibly elsewhere) can never leave a stale address behind.
 void* noalloc_scratch() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
-    g_scratch_ptr[dev] = p;
-  }
-  return g_scratch_ptr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+  return p;
 }
 
 }  // namespace

@@ -88,9 +88,10 @@ __device__ __forceinline__ bool give_up(uint32_t poll, const int32_t* status) {
 }
 
 // Bounded wait on an mbarrier phase.  Returns false (and records
-// SSD_ERR_TIMEOUT) if the phase did not complete within kMaxPolls polls.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status) {
-  for (uint32_t i = 0; i < kMaxPolls; ++i) {
+// SSD_ERR_TIMEOUT) if the phase did not complete within max_polls polls.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status,
+                                          uint32_t max_polls = kMaxPolls) {
+  for (uint32_t i = 0; i < max_polls; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if (i > 4096) {
       __nanosleep(128);

@@ -316,4 +316,11 @@ cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
 
 int device_sm_count();
 
+// Failure-detection controls (ssd_set_wait_limit, ssd_set_barrier_shortfall),
+// read by the host at every launch of a kernel with grid-wide waits: the poll
+// limit of its bounded waits (kMaxPolls when unset) and the extra arrivals its
+// grid barriers wait for (0 when unset; > 0 makes them run out).
+uint32_t wait_poll_limit();
+uint32_t barrier_shortfall();
+
 }  // namespace ssd

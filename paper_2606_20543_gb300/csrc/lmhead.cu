@@ -73,19 +73,29 @@ __device__ __forceinline__ uint32_t ld_acquire(const unsigned int* p) {
 }
 
 // Bounded grid barrier over `ncta` co-resident CTAs (cooperative launch).
-// Returns false in every thread if this CTA gave up waiting.
+// ctr[0] counts arrivals over the kernel's barriers (cumulative targets);
+// ctr[1] is an abort flag: a CTA that gives up waiting (after max_polls polls,
+// SSD_ERR_TIMEOUT recorded) raises it before it arrives anywhere else, so a
+// slower CTA that later sees the count reached through that CTA's next
+// arrival fails too instead of going on with missing partials.  Returns false
+// in every thread if this CTA gave up or the kernel was aborted.
 __device__ bool grid_barrier(unsigned int* ctr, unsigned int target, int32_t* status,
-                             int32_t* flag) {
+                             int32_t* flag, uint32_t max_polls) {
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
     atomicAdd(ctr, 1u);
     bool ok = false;
-    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+    for (uint32_t i = 0; i < max_polls; ++i) {
       if (ld_acquire(ctr) >= target) { ok = true; break; }
       if (i > 256) __nanosleep(64);
     }
-    if (!ok) record_status(status, SSD_ERR_TIMEOUT);
+    if (ok) {
+      ok = ld_acquire(ctr + 1) == 0u;
+    } else {
+      atomicExch(ctr + 1, 1u);
+      record_status(status, SSD_ERR_TIMEOUT);
+    }
     __threadfence();
     *flag = ok ? 1 : 0;
   }
@@ -108,6 +118,8 @@ struct LmLaunch {
   LmPartial* part;      // [rows][ncta]
   float* mass;          // [rows][ncta]
   unsigned int* barrier;
+  uint32_t max_polls;   // limit of every bounded wait of the kernel
+  uint32_t shortfall;   // extra arrivals each grid barrier waits for (0; > 0 in tests)
 };
 
 __global__ void __launch_bounds__(kThreadsL, 1)
@@ -168,7 +180,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
       const int s = kb % S;
       int stop = 0;
       if (lane == 0) {
-        if (kb >= S && !mbar_wait(&empty[s], ((kb / S) - 1) & 1, a.status)) {
+        if (kb >= S && !mbar_wait(&empty[s], ((kb / S) - 1) & 1, a.status, L.max_polls)) {
           *fail = 1;
           stop = 1;
         } else {
@@ -195,7 +207,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     if (lane == 0) {
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % S;
-      if (!mbar_wait(&full[s], (kb / S) & 1, a.status)) { *fail = 1; break; }
+      if (!mbar_wait(&full[s], (kb / S) & 1, a.status, L.max_polls)) { *fail = 1; break; }
       tc_fence_after();
       const uint32_t st = smem_u32(smem + s * stage_bytes);
       const uint32_t bt = st + 2 * mt * kTileA, bd = bt + kTileB;
@@ -221,7 +233,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     __syncwarp();
   }
   // every thread waits for the accumulators
-  const bool mma_ok = mbar_wait(done, 0, a.status);
+  const bool mma_ok = mbar_wait(done, 0, a.status, L.max_polls);
   tc_fence_after();
   bool ok = __syncthreads_and(mma_ok) != 0;
   ok = ok && (*fail == 0);
@@ -287,7 +299,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
           make_float4(P.xq_c, P.xp_c, __int_as_float(P.cand), 0.f);
     }
   }
-  ok = grid_barrier(L.barrier, (unsigned)L.ncta, a.status, flag) && ok;
+  ok = grid_barrier(L.barrier, (unsigned)L.ncta + L.shortfall, a.status, flag, L.max_polls) && ok;
 
   // ---- epilogue 2: combine the partials of each row (warp per row, lane l
   // merging tiles l, l + 32, ... in order, then a xor tree: the same arithmetic
@@ -405,7 +417,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     }
     if (draw) L.mass[(int64_t)row * L.ncta + cta] = mass;
   }
-  ok = grid_barrier(L.barrier, 2u * (unsigned)L.ncta, a.status, flag) && ok;
+  ok = grid_barrier(L.barrier, 2u * ((unsigned)L.ncta + L.shortfall), a.status, flag,
+                    L.max_polls) && ok;
 
   // ---- epilogue 4: locate the tile holding u_res * Z (warp per row; lane l
   // owns tiles [l*per, (l+1)*per) and keeps their masses in registers; the
@@ -580,7 +593,7 @@ int stages_for(int mt) { return mt == 1 ? 3 : 2; }
 
 size_t lmhead_workspace(int32_t rows, int32_t V) {
   const size_t ncta = (size_t)(V + kBN - 1) / kBN;
-  return al256(sizeof(unsigned int)) + al256((size_t)rows * ncta * sizeof(LmPartial)) +
+  return al256(2 * sizeof(unsigned int)) + al256((size_t)rows * ncta * sizeof(LmPartial)) +
          al256((size_t)rows * ncta * sizeof(float));
 }
 
@@ -610,9 +623,11 @@ cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaSt
   L.ncta = a.V / kBN;
   L.mt = mt;
   L.stages = stages_for(mt);
+  L.max_polls = wait_poll_limit();
+  L.shortfall = barrier_shortfall();
   unsigned char* w = static_cast<unsigned char*>(ws);
-  L.barrier = reinterpret_cast<unsigned int*>(w);
-  w += al256(sizeof(unsigned int));
+  L.barrier = reinterpret_cast<unsigned int*>(w);  // [0] arrivals, [1] abort flag
+  w += al256(2 * sizeof(unsigned int));
   L.part = reinterpret_cast<LmPartial*>(w);
   w += al256((size_t)a.rows * L.ncta * sizeof(LmPartial));
   L.mass = reinterpret_cast<float*>(w);
@@ -624,7 +639,7 @@ cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaSt
       !make_weight_map(&wt, a.w_tgt, (uint64_t)a.V, (uint64_t)a.K) ||
       !make_weight_map(&wd, a.w_drf, (uint64_t)a.V, (uint64_t)a.K))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaMemsetAsync(L.barrier, 0, sizeof(unsigned int), stream);
+  cudaError_t e = cudaMemsetAsync(L.barrier, 0, 2 * sizeof(unsigned int), stream);
   if (e != cudaSuccess) return e;
   const size_t smem = smem_bytes(mt, L.stages);
   e = cudaFuncSetAttribute(lmhead_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -6,7 +6,8 @@ import numpy as np
 
 import synth
 
-ATTN_TOL = 2e-2     # normwise max relative error per (b, h), bf16 inputs
+ATTN_TOL = 2e-2     # max relative error per (b, h), normwise and elementwise, bf16 inputs
+ATTN_FLOOR = 0.5   # elementwise floor: this fraction of the query row's RMS
 PROB_TOL = 1e-5     # relative error of ratio / log-sum-exp, fp32 logits path
 # Fused lm_head: the logits themselves come from a bf16 x bf16 contraction over
 # K = 4096 accumulated in fp32 on the tensor cores; a logit error of ~1e-5
@@ -21,9 +22,27 @@ def bf16_to_f64(bits):
 
 
 def attention_error(o_gpu, o_ref):
-    """max |gpu - ref| / max |ref| over one (b, h) block."""
-    den = np.abs(o_ref).max()
-    return np.abs(o_gpu - o_ref).max() / max(den, 1e-6)
+    """Relative error of one (b, h) block [rows, d]: the larger of
+      * the normwise error max |gpu - ref| / max |ref|, and
+      * the elementwise error max |gpu - ref| / max(|ref|, ATTN_FLOOR * rms_row(ref)),
+        rms_row being the RMS of that query row's reference output.
+    The elementwise term catches an error in a row or an entry of small
+    magnitude, which the normwise term hides under the block's largest value.
+    Its floor comes from the bf16 arithmetic of the path: P is rounded to bf16
+    (relative 2^-9) before the PV product, so an output entry near zero carries
+    an absolute error of about 2^-9 times the row's RMS whatever its own size;
+    a float64 simulation of that rounding (bf16 Q/K/V, bf16 P and O, 30 to
+    4000 keys, d = 128) gives at most 1.3e-2 with the floor at half the row
+    RMS, inside the 2e-2 bar."""
+    o_gpu = np.asarray(o_gpu, dtype=np.float64)
+    o_ref = np.asarray(o_ref, dtype=np.float64)
+    d = np.abs(o_gpu - o_ref)
+    den = np.abs(o_ref).max(initial=0.0)
+    normwise = d.max(initial=0.0) / max(den, 1e-6)
+    rms = np.sqrt(np.mean(o_ref * o_ref, axis=-1, keepdims=True))
+    floor = np.maximum(ATTN_FLOOR * rms, 1e-6)
+    elementwise = (d / np.maximum(np.abs(o_ref), floor)).max(initial=0.0)
+    return max(normwise, elementwise)
 
 
 def committed_draws(dec, accepted, D_max):
@@ -46,19 +65,55 @@ def committed_draws(dec, accepted, D_max):
     return out
 
 
-def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what="", tol=PROB_TOL):
+# Near-ties seen by every decision comparison of the session, reported at the
+# end of the run (tests/conftest.py): (case, rows, rows in the accept band,
+# rows in the resample band, rows excused because they differ inside a band).
+NEAR_TIES = []
+# Rows that may differ from the oracle inside a near-tie band, per compared
+# case: 2 plus 1% of the rows.  A row differs inside the resample band when the
+# GPU's fp32 CDF (block sums of 256 entries, then a scan of the block masses)
+# and the oracle's fp64 cumulative sum fall on opposite sides of u_res * Z; on
+# GB300 about one row in 17 of the band did (1420 rows, V = 4096 to 100000),
+# i.e. an error near 1e-7 * Z, so a row differs with probability about
+# 2e-7 times its number of positive residual entries: up to ~0.5% at V = 65536.
+MAX_EXCUSED_BASE = 2
+
+
+def max_excused_rows(rows):
+    return MAX_EXCUSED_BASE + rows // 100
+
+
+def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what="", tol=PROB_TOL,
+                      max_excused=None):
     """Bit-exact comparison of accept flags and tokens, except near-tie rows.
 
     dec: oracle accept_rows() dict for the compared rows; out_tok/accepted:
-    the GPU's values for the same rows.  Returns the number of excused rows."""
-    tie = dec["tie_accept"] | dec["tie_resample"]
+    the GPU's values for the same rows.  A row may differ only inside a
+    near-tie band:
+      * |alpha - u_acc| < 1e-4 (the accept decision itself), or
+      * u_res * Z within 1e-6 * Z of a boundary of the chosen CDF bin (the
+        residual draw; the fp32 normalisers and block sums of the GPU's CDF
+        carry a relative error of order 1e-7 at these vocabularies),
+    and at most max_excused rows per case (default: max_excused_rows) may do
+    so.  Every case's near-tie counts are recorded in NEAR_TIES and printed at
+    the end of the session.
+    Returns the number of rows excused (rows that differ inside a band)."""
+    if max_excused is None:
+        max_excused = max_excused_rows(int(np.size(out_tok)))
+    tie_acc = np.asarray(dec["tie_accept"], dtype=bool)
+    tie_res = np.asarray(dec["tie_resample"], dtype=bool) & ~tie_acc
     acc_g = accepted.astype(bool)
-    ok_acc = (acc_g == dec["accepted"]) | tie
-    ok_tok = (out_tok == dec["out_tok"]) | tie
-    bad = np.nonzero(~(ok_acc & ok_tok))[0]
+    differ = (acc_g != dec["accepted"]) | (out_tok != dec["out_tok"])
+    excused = differ & (tie_acc | tie_res)
+    bad = np.nonzero(differ & ~(tie_acc | tie_res))[0]
+    NEAR_TIES.append((what, int(differ.size), int(tie_acc.sum()), int(tie_res.sum()),
+                      int(excused.sum())))
     assert bad.size == 0, (f"{what}: {bad.size} rows differ, first {bad[:5]}: gpu tok "
                            f"{out_tok[bad[:5]]} acc {acc_g[bad[:5]]}, oracle tok "
                            f"{dec['out_tok'][bad[:5]]} acc {dec['accepted'][bad[:5]]}")
+    assert excused.sum() <= max_excused, (
+        f"{what}: {int(excused.sum())} near-tie rows differ (allowed {max_excused}): "
+        f"{np.nonzero(excused)[0][:8]}")
     if ratio is not None:
         ref = dec["ratio"]
         fin = np.isfinite(ref) & (ref < 1e30)
@@ -68,4 +123,4 @@ def compare_decisions(dec, out_tok, accepted, ratio=None, lse=None, what="", tol
         for k, key in enumerate(("lse_p", "lse_q")):
             rel = np.abs(lse[:, k] - dec[key]) / np.abs(dec[key])
             assert rel.max(initial=0) < tol, f"{what}: {key} rel err {rel.max()}"
-    return int(tie.sum())
+    return int(excused.sum())

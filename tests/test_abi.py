@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 6
+    assert lib.ssd_abi_version() == 7
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 

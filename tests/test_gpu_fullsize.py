@@ -126,9 +126,17 @@ def test_config5_first_steps_match_oracle_replay(ssd):
         else:
             break
         if t == 0:
-            # attention of the first step on sampled sequences and heads
+            # the first step row by row: accept flags, committed tokens and
+            # ratios of every draft, and attention on every head of two sequences
             r = s.results()
-            check_attention(c, r, seqs=[0, 5], heads=[0, 13, 31])
+            tg, dr, u = inputs(0)
+            ref = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, oh["cache_len"],
+                                    c.D_max, tg, dr, u)
+            rows = ref["decisions"]["rows"]
+            dec = committed_draws(ref["decisions"], r["accepted"][rows], c.D_max)
+            compare_decisions(dec, r["out_tok"][rows], r["accepted"][rows], r["ratio"][rows],
+                              what="cfg5 step 0")
+            check_attention(c, r, seqs=[0, 5])
         s.cache_len.copy_(s.next_cache_len)
     assert s.status.item() == 0
 
@@ -159,3 +167,20 @@ def test_config5_replay_to_completion_invariants(ssd):
     assert (prev == c.prefix_len + HW).all() and (total == HW).all()
     assert s.status.item() == 0
     assert steps >= HW // (2 * c.grid_w)  # at most two rows per step
+
+
+@pytest.mark.parametrize("B", [8, 2])
+def test_config5_late_step_every_row(ssd, B):
+    """A teacher-forced late step of the 64x64 replay at full size (V = 65536,
+    up to 128 drafts per sequence, caches of about 4100 to 4350 keys): every
+    row's accept flag, committed token and ratio against the oracle, and the
+    attention of every head of two sequences.  B = 8 is the bench's launch;
+    with B = 2 the attention splits every KV cache over several CTAs and
+    merges the partials (the split-KV path)."""
+    rng = np.random.default_rng(50 + B)
+    cl = 256 + 64 * rng.integers(59, 63, size=B) + rng.integers(0, 64, size=B)
+    cl[0] = 256 + 64 * 62  # a frontier of two whole rows: 128 drafts
+    c = synth.config5(B=B, cache_len=cl.astype(np.int32), seed=51 + B)
+    _, r = run_case(c)
+    check_decisions(c, r)
+    check_attention(c, r, seqs=[0, B - 1])
