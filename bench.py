@@ -1,14 +1,19 @@
 """Throughput of the SSD verification pass on GB300.
 
-One bench step = one whole verification pass (frontier, frontier attention,
-acceptance with residual resampling, counts) over one batch of synthetic
-input, through the C ABI of libssd.  The default workload is the 24x24
-(LlamaGen-XL-like) sweep: 25 cache lengths 120 -> 696 (one grid row apart),
-each an independent batch-1 verification problem with its own seed, issued
-together as one ragged batch of 25 sequences per ssd_verify_step call.
+One verification pass (frontier, frontier attention, acceptance with
+residual resampling, counts) runs through the C ABI of libssd.  The default
+workload is the largest single-GPU configuration: the seeded replay of the
+2D frontier schedule on 8 sequences of 64x64 grids (256-token prefixes,
+32x128 MHA, V = 65536) to grid completion, every step's accepted counts
+setting the next cache lengths and frontier on the device.  One bench step
+is one whole replay (about 4000 verification passes of 8 sequences); the
+value is sequence verify steps per second at the median replay time.
+`--config 1..4` select the other workloads, where one bench step is one
+verification pass over the workload's batch.
 
 Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle
-(the float64 restatement of the method) on the same workload instead.
+(the float64 restatement of the method) on bounded samples of the same
+workload instead, and reports the samples it ran.
 """
 from __future__ import annotations
 
@@ -50,10 +55,15 @@ def job_rate(world, units_per_rank, ms):
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed bench steps (default: 20 replays for config 5, 2000 passes "
+                         "otherwise)")
+    ap.add_argument("--warmup", type=int, default=None,
+                    help="untimed bench steps first (default: 3 replays / 20 passes)")
     ap.add_argument("--impl", default="ssd", choices=["ssd", "reference"])
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--e2e-steps", type=int, default=48,
+                    help="verification passes of the end-to-end leg of the config-5 replay")
     ap.add_argument("--fused-batch", type=int, default=1,
                     help="sequences of the fused-head workload (config 4): 1, or up to 5 "
                          "(240 draft rows) for the batched variant")
@@ -77,6 +87,10 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="approximate budget of the CPU-oracle sample")
     a = ap.parse_args()
+    if a.steps is None:
+        a.steps = 20 if a.config == 5 and not a.predictor else 2000
+    if a.warmup is None:
+        a.warmup = 3 if a.config == 5 and not a.predictor else 20
     if a.strategy != "accept_reject" and a.config in (4, 5):
         ap.error("--strategy other than accept_reject needs a logits workload (configs 1-3)")
     if (a.rounds != 1 or a.staged) and a.config in (4, 5):
@@ -122,11 +136,11 @@ WORKLOAD_NAMES = {
 
 def algorithmic_bytes(c, n_drafts, bonus=False):
     """Bytes one verification pass must move: every K/V row of the visible
-    keys once per KV head, Q and O of each draft, both logit rows of each
+    keys once per KV head (for sequences with drafts), Q and O of each draft, both logit rows of each
     draft (and of each sequence's bonus row in the horizontal stage), and the
     per-row / per-sequence outputs."""
     n = np.asarray(n_drafts, dtype=np.int64)
-    L = c.cache_len.astype(np.int64) + n
+    L = np.where(n > 0, c.cache_len.astype(np.int64) + n, 0)  # an empty frontier reads nothing
     kv = int((L * c.Hkv * c.d * 2 * 2).sum())
     qo = int((n * c.Hq * c.d * 2 * 2).sum())
     attn = kv + qo + int(n.sum()) * c.Hq * 4  # + lse
@@ -258,31 +272,137 @@ def sub_case(c, seqs):
     return s
 
 
-def cpu_oracle_rate(c, budget_s, strategy="accept_reject"):
+def oracle_threads():
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
+    return int(threads) if threads else (os.cpu_count() or 1)
+
+
+class NearTies:
+    """Rows of GPU decisions compared with the oracle's on the same inputs:
+    rows inside the accept band (|alpha - u_acc| < 1e-4), inside the resample
+    band (u_res * Z within 1e-6 * Z of a CDF boundary), and rows whose flag or
+    token differs (inside a band, and outside any band)."""
+
+    def __init__(self):
+        self.rows = self.accept_band = self.resample_band = 0
+        self.differ_in_band = self.differ_outside = 0
+
+    def add(self, dec, gpu_acc, gpu_tok, committed_only=True):
+        """dec: the oracle's decisions of one sequence's drafts (in order);
+        gpu_acc / gpu_tok: the GPU's for the same rows.  committed_only: the
+        GPU draws only the first rejected draft's token (prefix rule)."""
+        acc = np.asarray(gpu_acc).astype(bool)
+        tok = np.asarray(gpu_tok)
+        want = np.array(dec["out_tok"], copy=True)
+        if committed_only:
+            rej = np.nonzero(~acc)[0]
+            want[rej[1:]] = -1
+        ta = np.asarray(dec["tie_accept"], bool)
+        tr = np.asarray(dec["tie_resample"], bool) & ~ta
+        differ = (acc != dec["accepted"]) | (tok != want)
+        self.rows += int(acc.size)
+        self.accept_band += int(ta.sum())
+        self.resample_band += int(tr.sum())
+        self.differ_in_band += int((differ & (ta | tr)).sum())
+        self.differ_outside += int((differ & ~(ta | tr)).sum())
+
+    def report(self, sample):
+        return {"rows": self.rows, "accept_band": self.accept_band,
+                "resample_band": self.resample_band, "differing_in_band": self.differ_in_band,
+                "differing_outside_bands": self.differ_outside, "sample": sample}
+
+
+def cpu_oracle_rate(c, budget_s, strategy="accept_reject", gpu=None, min_passes=1):
     """Sequence verify steps/s of the oracle on a bounded sample of the
     workload: whole sequences of the batch, one after another (cycling over
-    the batch), until about budget_s seconds of CPU work are done."""
-    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
+    the batch), until about budget_s seconds of CPU work are done.  With
+    `gpu` (the GPU's out_tok / accepted of one pass over the same inputs) the
+    sampled sequences' decisions are also compared: returns (rate dict,
+    NearTies)."""
     t0 = time.perf_counter()
     done = 0
+    ties = NearTies()
     while True:
-        oracle_pass(sub_case(c, [done % c.B]), strategy)
+        b = done % c.B
+        r = oracle_pass(sub_case(c, [b]), strategy)
+        if gpu is not None and done < c.B:
+            n = int(r["n_drafts"][0])
+            rows = b * c.D_max + np.arange(n)
+            dec = {k: np.asarray(v)[:n] for k, v in r["decisions"].items() if k != "rows"}
+            ties.add(dec, gpu["accepted"][rows], gpu["out_tok"][rows],
+                     committed_only=strategy == "accept_reject")
+        done += 1
+        if time.perf_counter() - t0 > budget_s and done >= min_passes:
+            break
+    el = time.perf_counter() - t0
+    rate = done / el  # sequence verification passes per second
+    cores = oracle_threads()
+    return ({"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+             "sample": f"{done} sequence passes over the batch's sequences in turn ({el:.1f} s); "
+                       f"float64 NumPy, BLAS threads up to {cores}"}, ties)
+
+
+# ------------------------------------------------------------ config-5 replay
+def frontier_sizes(grid_h, grid_w, prefix_len, k_v, cache_len):
+    """Drafts per sequence after cache_len (the rest of the current row plus
+    the k_v rows below it, clipped at the last row): the host's copy of the
+    frontier rule, used only to size the copies of the end-to-end leg."""
+    n_c = np.asarray(cache_len, dtype=np.int64) - prefix_len
+    y0, col = n_c // grid_w, n_c % grid_w
+    below = np.clip(grid_h - 1 - y0, 0, k_v)
+    n = (grid_w - col) + below * grid_w
+    return np.where(y0 >= grid_h, 0, n)
+
+
+def replay_state_case(c, pool, seed, t, cache_len):
+    """The config-5 case at replay step t in state cache_len: that step's
+    logit set and Philox uniforms (views; no copies of the logits)."""
+    import copy
+    s = copy.copy(c)
+    s.cache_len = np.asarray(cache_len, dtype=np.int32)
+    s.tgt_logits, s.drf_logits = pool[t % len(pool)]
+    s.uniforms = synth.philox_uniforms(seed, t, c.B * c.D_max)
+    return s
+
+
+def replay_oracle_sample(c, pool, seed, states, budget_s):
+    """The oracle, teacher-forced from the GPU's replay: one sequence pass per
+    sampled state (step t, the GPU's cache lengths before it, its accept flags
+    and tokens), cycling over the states and their active sequences until
+    about budget_s seconds of CPU work are done.  Returns (rate dict,
+    NearTies of the compared rows)."""
+    jobs = [(st, b) for st in states for b in range(c.B) if st["n_drafts"][b] > 0]
+    ties = NearTies()
+    t0 = time.perf_counter()
+    done = 0
+    while jobs:
+        st, b = jobs[done % len(jobs)]
+        cs = replay_state_case(c, pool, seed, st["t"], st["cache_len"])
+        r = oracle_pass(sub_case(cs, [b]))
+        if done < len(jobs):
+            n = int(r["n_drafts"][0])
+            assert n == int(st["n_drafts"][b])
+            rows = b * c.D_max + np.arange(n)
+            dec = {k: np.asarray(v)[:n] for k, v in r["decisions"].items() if k != "rows"}
+            ties.add(dec, st["accepted"][rows], st["out_tok"][rows])
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
     el = time.perf_counter() - t0
-    rate = done / el  # sequence verification passes per second
-    cores = int(threads) if threads else (os.cpu_count() or 1)
-    return {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{done} sequence passes over the batch's first sequences ({el:.1f} s); "
-                      f"float64 NumPy, BLAS threads up to {cores}"}
+    cores = oracle_threads()
+    steps = sorted({st["t"] for st, _ in jobs[:done]})
+    return ({"value": done / el, "unit": UNIT, "cores": cores, "kind": "oracle",
+             "sample": f"{done} sequence passes teacher-forced from the GPU replay's states at "
+                       f"steps {steps[:12]}{'...' if len(steps) > 12 else ''} ({el:.1f} s); "
+                       f"float64 NumPy, BLAS threads up to {cores}"}, ties)
 
 
-# ------------------------------------------------------------ config-5 replay
-def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
+def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
     """The 8 x 64x64 replay to grid completion: every step's accepted counts set
-    the next cache lengths and frontier on the device.  Timed end to end from
-    empty grids to completion; steps are issued as CUDA graphs of 64."""
+    the next cache lengths and frontier on the device.  One bench step is one
+    whole replay from empty grids to completion (steps issued as CUDA graphs
+    of 64); each replay is timed on its own and the median is reported."""
+    import copy
     c = synth.config5(seed=5 + 1000 * rank, with_logits=False)
     pool = synth.replay_pool(c.B, c.D_max, c.V, seed=c.seed)
     s = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V,
@@ -291,6 +411,7 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
     init = s.cache_len.clone()
     dpool = [(torch.from_numpy(t).to(dev), torch.from_numpy(d).to(dev)) for t, d in pool]
     seed = c.seed
+    HW = c.grid_h * c.grid_w
 
     def step(t):
         tg, dr = dpool[t % len(dpool)]
@@ -299,19 +420,30 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
         s.run()
         s.cache_len.copy_(s.next_cache_len)
 
-    # eager pass: trajectory length, per-sequence active steps, accepted drafts
+    # eager pass: trajectory length, per-sequence active steps, accepted
+    # drafts, and the GPU's state and decisions every 64th step
     s.cache_len.copy_(init)
-    HW = c.grid_h * c.grid_w
     active, accepted, T = np.zeros(c.B, np.int64), 0, 0
+    states, attn_bytes_total, acc_bytes_total = [], 0, 0
     while True:
+        cl = s.cache_len.cpu().numpy().copy()
         step(T)
         nd = s.n_drafts.cpu().numpy()
         if nd.sum() == 0:
             break
+        cc = copy.copy(c)
+        cc.cache_len = cl
+        ab, cb = algorithmic_bytes(cc, nd)
+        attn_bytes_total += ab
+        acc_bytes_total += cb
+        if T % 64 == 0:
+            states.append({"t": T, "cache_len": cl, "n_drafts": nd.copy(),
+                           "accepted": s.accepted.cpu().numpy(), "out_tok": s.out_tok.cpu().numpy()})
         active += nd > 0
         accepted += int(s.accepted_count.sum().item())
         T += 1
     assert int(s.cache_len.sum().item()) == c.B * (c.prefix_len + HW)
+    seq_steps = int(active.sum())
     chunk = 64
     graphs = []
     s.cache_len.copy_(init)
@@ -323,38 +455,45 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
                 step(t)
         graphs.append(g)
     launches = ssd.ssd_verify_step_launches(s.args) * T
-    for _ in range(2):  # warm-up replays
+    stream = torch.cuda.current_stream(dev)
+
+    def replay():
         s.cache_len.copy_(init)
         for g in graphs:
             g.replay()
+
+    for _ in range(a.warmup):
+        replay()
     torch.cuda.synchronize(dev)
-    s.cache_len.copy_(init)
-    torch.cuda.synchronize(dev)
+
+    # ---------------- timed region: K whole replays, each between its own events
     clocks = ClockSampler(dev.index or 0)
     clocks.start()
     time.sleep(0.2)
     if world > 1:
         torch.distributed.barrier()
-    stream = torch.cuda.current_stream(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for g in graphs:
-        g.replay()
-    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(a.steps)]
+    for e0, e1 in ev:
+        s.cache_len.copy_(init)
+        e0.record(stream)
+        for g in graphs:
+            g.replay()
+        e1.record(stream)
     torch.cuda.synchronize(dev)
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
-    ms = e0.elapsed_time(e1)
+    per = [e0.elapsed_time(e1) for e0, e1 in ev]
     done = int(s.cache_len.sum().item()) == c.B * (c.prefix_len + HW)
-    ms = max_over_ranks(ms, world, torch, dev)
-    seq_steps = int(active.sum())
-    # dominant kernel at the first step (cache = prefix), per-kernel graphs
-    s.cache_len.copy_(init)
-    step(0)
-    s.cache_len.copy_(init)
-    torch.cuda.synchronize(dev)
-    kk = 50
+    ms = max_over_ranks(statistics.median(per), world, torch, dev)
+    total_ms = max_over_ranks(sum(per), world, torch, dev)
+
+    # ---------------- per-kernel durations at three replay states (the first
+    # step, the middle and near the end): each entry point captured as a graph
+    # of back-to-back launches, timed with events on the launching stream
+    kk = 20
     wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
     ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
 
@@ -373,50 +512,184 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu):
         torch.cuda.synchronize(dev)
         return k0.elapsed_time(k1) / kk
 
-    attn_ms = timed(lambda i, cs: ssd.ssd_verify_attention(
-        s.g, c.B, c.Hq, c.Hkv, c.d, s.cache_len, s.n_drafts, s.draft_pos, c.D_max, c.L_max, s.q,
-        s.k, s.v, 0.0, s.o, None, ws, wsb, s.status, cs))
     def acc_call(i, cs):  # the step's acceptance part (decisions, committed draws, counts)
         s.args.tgt_logits, s.args.drf_logits = dpool[i % 2][0].data_ptr(), dpool[i % 2][1].data_ptr()
         s.set_rng(seed, i)
         ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes, cs)
 
-    acc_ms = timed(acc_call)
-    nd0 = s.n_drafts.cpu().numpy()
-    attn_bytes, acc_bytes = algorithmic_bytes(c, nd0)
-    kern = {"attention": (attn_bytes, attn_ms), "accept": (acc_bytes, acc_ms)}
+    def attn_call(i, cs):
+        ssd.ssd_verify_attention(s.g, c.B, c.Hq, c.Hkv, c.d, s.cache_len, s.n_drafts, s.draft_pos,
+                                 c.D_max, c.L_max, s.q, s.k, s.v, 0.0, s.o, None, ws, wsb,
+                                 s.status, cs)
+
+    probe = [states[0], states[len(states) // 2], states[-1]]
+    kern = {"attention": [0, 0.0], "accept": [0, 0.0]}
+    per_state = []
+    for st in probe:
+        s.cache_len.copy_(torch.from_numpy(st["cache_len"].astype(np.int32)).to(dev))
+        acc_ms = timed(acc_call)   # also writes the state's frontier (n_drafts, draft_pos)
+        attn_ms = timed(attn_call)
+        cc = copy.copy(c)
+        cc.cache_len = st["cache_len"]
+        ab, cb = algorithmic_bytes(cc, st["n_drafts"])
+        kern["attention"][0] += ab
+        kern["attention"][1] += attn_ms
+        kern["accept"][0] += cb
+        kern["accept"][1] += acc_ms
+        per_state.append({"step": st["t"], "max_cache_len": int(st["cache_len"].max()),
+                          "drafts": int(st["n_drafts"].sum()),
+                          "attention": {"bytes": ab, "ms": attn_ms,
+                                        "gbs": ab / (attn_ms / 1000.0) / 1e9},
+                          "accept": {"bytes": cb, "ms": acc_ms,
+                                     "gbs": cb / (acc_ms / 1000.0) / 1e9}})
     dom = max(kern, key=lambda k: kern[k][1])
     hbm_peak, peak_kind = measured_peaks()
     achieved = kern[dom][0] / (kern[dom][1] / 1000.0) / 1e9
+
+    # ---------------- end to end through ssd_verify_step with host inputs: every
+    # pass copies its frontier's logit rows (both sets), the drafts' Q and their
+    # K/V slots from pinned host memory, and reads back the counts and
+    # decisions, which set the next pass's copies; the KV cache itself stays on
+    # the device (it only grows by the appended draft slots)
+    E = max(1, min(a.e2e_steps, T))
+    pinned = lambda x: torch.from_numpy(x).pin_memory()  # noqa: E731
+    host_logits = [(pinned(t), pinned(d)) for t, d in pool]
+    host_q = pinned(np.ascontiguousarray(c.q).view(np.int16)).view(torch.bfloat16)
+    k16, v16 = c.k.view(np.int16), c.v.view(np.int16)
+    stage = [torch.empty((c.B, c.D_max, c.Hkv, c.d), dtype=torch.int16, pin_memory=True)
+             for _ in range(2)]
+    dstage = [torch.empty((c.B, c.D_max, c.Hkv, c.d), dtype=torch.bfloat16, device=dev)
+              for _ in range(2)]
+    e_tg, e_dr = dpool[0]  # device logit buffers of the leg (the timed replays are done)
+    s.args.tgt_logits, s.args.drf_logits = e_tg.data_ptr(), e_dr.data_ptr()
+    outs = {n: torch.empty(getattr(s, n).shape, dtype=getattr(s, n).dtype, pin_memory=True)
+            for n in ("next_cache_len", "accepted_count", "n_drafts", "out_tok", "accepted")}
+    d2h = sum(t.numel() * t.element_size() for t in outs.values())
+    h2d_total, e2e_seq_steps = 0, 0
+    host_cl = c.cache_len.astype(np.int64).copy()
+    s.cache_len.copy_(init)
+    torch.cuda.synchronize(dev)
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for t in range(E):
+        nd = frontier_sizes(c.grid_h, c.grid_w, c.prefix_len, c.k_v, host_cl)
+        ht, hd = host_logits[t % len(host_logits)]
+        for b in range(c.B):
+            n, cl = int(nd[b]), int(host_cl[b])
+            if n == 0:
+                continue
+            r0 = b * c.D_max
+            e_tg[r0:r0 + n].copy_(ht[r0:r0 + n], non_blocking=True)
+            e_dr[r0:r0 + n].copy_(hd[r0:r0 + n], non_blocking=True)
+            s.q[b, :n].copy_(host_q[b, :n], non_blocking=True)
+            for src, st_h, st_d, dst in ((k16, stage[0], dstage[0], s.k),
+                                         (v16, stage[1], dstage[1], s.v)):
+                st_h[b, :n].numpy()[...] = src[b, :, cl:cl + n].transpose(1, 0, 2)
+                st_d[b, :n].copy_(st_h[b, :n].view(torch.bfloat16), non_blocking=True)
+                dst[b, :, cl:cl + n].copy_(st_d[b, :n].transpose(0, 1))
+            h2d_total += n * (2 * c.V * 4 + c.Hq * c.d * 2 + 2 * c.Hkv * c.d * 2)
+        s.set_rng(seed, t)
+        s.run(stream)
+        for name, hb in outs.items():
+            hb.copy_(getattr(s, name), non_blocking=True)
+        stream.synchronize()
+        e2e_seq_steps += int((nd > 0).sum())
+        host_cl = outs["next_cache_len"].numpy().astype(np.int64)
+        s.cache_len.copy_(s.next_cache_len)
+    f1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = f0.elapsed_time(f1)
+    e2e_value = world * e2e_seq_steps / (e2e_ms / 1000.0)
+    status = int(s.status.item())
     if rank != 0:
         return 0
+
+    cpu, ties = None, None
+    if not a.no_cpu_baseline:
+        cpu, ties = replay_oracle_sample(c, pool, seed, states, a.cpu_seconds)
     line = {
         "metric": METRIC, "value": job_rate(world, seq_steps, ms), "unit": UNIT,
-        "n_gpus": world, "steps": T, "warmup": 2, "ms_per_step": ms / T,
+        "n_gpus": world, "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16 attention / f32 acceptance", "data": "synthetic",
-        "config": {"workload": "replay to grid completion: 8 x 64x64 grids, prefix 256, "
-                               "32x128 MHA, V=65536, Zipf draft vs N(0,2^2)-perturbed target",
+        "config": {"workload": WORKLOAD_NAMES[5],
+                   "bench_step": f"one whole replay to grid completion ({T} verification passes "
+                                 f"of {c.B} sequences, {seq_steps} sequence verify steps)",
                    "replay_steps": T, "sequence_steps": seq_steps,
-                   "logits": "2 device-resident sets of 537 MB alternate by step; Philox offset = step",
-                   "issue": "CUDA graphs of 64 steps; device cache lengths drive the next step",
+                   "logits": "2 device-resident sets of 537 MB alternate by pass; Philox "
+                             "offset = pass index",
+                   "l2": "every pass streams its frontier's logit rows (up to 537 MB) and the "
+                         "visible K/V: inputs larger than the 129 MB L2",
+                   "issue": "CUDA graphs of 64 passes; device cache lengths drive the next pass",
                    "completed": done, "parallelism": f"replicas x{world}"},
+        "median_replay_ms": ms, "replay_ms": per, "timed_region_ms": total_ms,
+        "verify_pass_us": 1000.0 * ms / T,
         "committed_tokens_per_s": world * c.B * HW / (ms / 1000.0),
         "accepted_drafts_per_s": world * accepted / (ms / 1000.0),
-        "replay_ms": ms,
+        "accepted_tokens_per_s": world * accepted / (ms / 1000.0),
+        "hbm_gbs_per_step": (attn_bytes_total + acc_bytes_total) / (ms / 1000.0) / 1e9,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": achieved / hbm_peak,
-                     "traffic": measured_traffic(dom, a.config, c.B * c.D_max),
-                     "peak_kind": peak_kind, "state": "first replay step (cache = prefix)",
+                     "traffic": measured_traffic(dom, 5, None),
+                     "peak_kind": peak_kind,
+                     "state": "bytes and launch times summed over three replay states "
+                              f"(steps {[st['t'] for st in probe]})",
                      "kernels": {k: {"bytes": b, "ms": m, "gbs": b / (m / 1000.0) / 1e9}
-                                 for k, (b, m) in kern.items()}},
+                                 for k, (b, m) in kern.items()},
+                     "states": per_state},
         "clocks": clk,
-        "gpu_launches": launches,
-        "device_status": int(s.status.item()),
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d_total / E),
+                "d2h_bytes_per_step": d2h, "steps": E,
+                "what": f"the first {E} verification passes of the replay through "
+                        "ssd_verify_step, inputs copied from pinned host memory and results "
+                        "read back every pass; per-pass bytes averaged"},
+        "near_ties": None if ties is None else ties.report(
+            "the oracle's teacher-forced passes of the CPU baseline vs the GPU's decisions in "
+            "the same states"),
+        "gpu_launches": launches * a.steps,
+        "device_status": status,
         "cpu_baseline": cpu,
     }
     print(json.dumps(line))
     return 0
+
+
+def batch1_latency(a, dev, torch, VerifyStep, points=(120, 408, 672), sets=12):
+    """Step latency at batch 1 (the paper's setting: one image) on three
+    cache lengths of the 24x24 sweep: a graph of back-to-back single-sequence
+    steps over `sets` rotating input sets (together larger than L2), timed
+    with events.  Returns {cache_len: microseconds per step}."""
+    out = {}
+    n = 200
+    for cl in points:
+        objs = []
+        for k in range(sets):
+            c = synth.config2(points=[cl], seed0=500 + k)
+            st = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max,
+                            c.L_max, c.V, device=dev)
+            st.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, tgt_logits=c.tgt_logits,
+                      drf_logits=c.drf_logits)
+            objs.append(st)
+        for i in range(2 * sets):
+            objs[i % sets].set_rng(9, i)
+            objs[i % sets].run()
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(n):
+                objs[i % sets].set_rng(9, i)
+                objs[i % sets].run()
+        g.replay()
+        torch.cuda.synchronize(dev)
+        stream = torch.cuda.current_stream(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        out[str(cl)] = 1000.0 * e0.elapsed_time(e1) / n
+        del objs, g
+    return out
 
 
 # ------------------------------------------------------- the draft predictor
@@ -549,6 +822,59 @@ def run_predictor(a, world, rank, dev, torch, ssd):
     return 0
 
 
+# ----------------------------------------------------- the reference arm
+def reference_arm(a, rank):
+    """`--impl reference`: the oracle, as it stands, on the host cores.  Each
+    bench step is one sequence's verification pass of the workload (configs
+    1-4: the batch's sequences in turn; config 5: states spread evenly over
+    the replay, from the empty grid to its last row, each with its step's
+    logit set and uniforms); W untimed passes, then K timed ones.  Only rank 0
+    runs; the other ranks exit without work."""
+    if rank != 0:
+        return 0
+    if a.config == 5:
+        c = synth.config5(seed=5, with_logits=False)
+        pool = synth.replay_pool(c.B, c.D_max, c.V, seed=c.seed)
+        HW, N = c.grid_h * c.grid_w, a.warmup + a.steps
+
+        def case(i):
+            n_c = min(HW - 1, int(HW * (i + 0.5) / max(N, 1)))
+            cl = np.full(c.B, c.prefix_len + n_c, dtype=np.int32)
+            return sub_case(replay_state_case(c, pool, c.seed, i, cl), [i % c.B])
+        what = (f"one sequence pass per step at replay states spread evenly over the 64x64 "
+                f"grid ({N} states)")
+    else:
+        c = workload(a.config, 0)
+
+        def case(i):
+            return sub_case(c, [i % c.B])
+        what = "one sequence pass per step, the batch's sequences in turn"
+    for i in range(a.warmup):
+        oracle_pass(case(i), a.strategy)
+    el = 0.0
+    for i in range(a.warmup, a.warmup + a.steps):
+        ci = case(i)
+        t0 = time.perf_counter()
+        oracle_pass(ci, a.strategy)
+        el += time.perf_counter() - t0
+    value = a.steps / el if el > 0 else 0.0
+    cores = oracle_threads()
+    cpu = {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+           "sample": f"{a.steps} timed sequence passes after {a.warmup} untimed ({el:.1f} s): "
+                     f"{what}; float64 NumPy, BLAS threads up to {cores}"}
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
+            "ms_per_step": 1000.0 * el / max(a.steps, 1), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAMES[a.config],
+                       "bench_step": "one sequence verification pass of the oracle"},
+            "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
 # -------------------------------------------------------------------- main
 def main():
     a = parse()
@@ -569,20 +895,7 @@ def main():
                                                       "d2h_bytes_per_step": 0}}))
         return 0
     if a.impl == "reference":
-        if rank != 0:
-            return 0
-        c = workload(a.config, 0)
-        cpu = cpu_oracle_rate(c, a.cpu_seconds, a.strategy)
-        line = {"impl": "reference", "metric": METRIC, "value": cpu["value"], "unit": UNIT,
-                "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
-                "ms_per_step": 1000.0 * c.B / cpu["value"], "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": WORKLOAD_NAMES[a.config]},
-                "cpu_baseline": cpu,
-                "e2e": {"value": cpu["value"], "unit": UNIT, "h2d_bytes_per_step": 0,
-                        "d2h_bytes_per_step": 0}}
-        print(json.dumps(line))
-        return 0
+        return reference_arm(a, rank)
 
     import torch
     if not torch.cuda.is_available():
@@ -607,10 +920,7 @@ def main():
         return rc
 
     if a.config == 5:
-        cpu = None
-        if rank == 0 and not a.no_cpu_baseline:
-            cpu = cpu_oracle_rate(synth.config5(seed=5, B=1), a.cpu_seconds)
-        rc = run_replay(a, world, rank, dev, torch, ssd, VerifyStep, cpu)
+        rc = run_replay(a, world, rank, dev, torch, ssd, VerifyStep)
         if world > 1:
             torch.distributed.destroy_process_group()
         return rc
@@ -822,9 +1132,24 @@ def main():
             torch.distributed.destroy_process_group()
         return 0
 
-    cpu = None
-    if not a.no_cpu_baseline:
-        cpu = cpu_oracle_rate(cases[0], a.cpu_seconds, a.strategy)
+    cpu, ties = None, None
+    if not a.no_cpu_baseline and not a.staged and R == 1:
+        # the oracle on the first input set with the uniforms of pass 0, and
+        # the near-ties of the GPU's decisions for the same pass
+        import copy
+        st0 = steps_obj[0]
+        st0.set_rng(seed, 0)
+        st0.run(stream)
+        torch.cuda.synchronize(dev)
+        gpu = {"out_tok": st0.out_tok.cpu().numpy(), "accepted": st0.accepted.cpu().numpy()}
+        c0 = copy.copy(cases[0])
+        c0.uniforms = synth.philox_uniforms(seed, 0, c.B * c.D_max)
+        cpu, ties = (cpu_oracle_rate(c0, a.cpu_seconds, a.strategy, gpu=gpu) if not a.horizontal
+                     else (cpu_oracle_rate(c0, a.cpu_seconds, a.strategy)[0], None))
+    elif not a.no_cpu_baseline:
+        cpu = cpu_oracle_rate(cases[0], a.cpu_seconds, a.strategy)[0]
+    batch1 = batch1_latency(a, dev, torch, VerifyStep) if a.config == 2 and R == 1 and \
+        not a.horizontal else None
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps_done,
@@ -859,6 +1184,9 @@ def main():
                 "d2h_bytes_per_step": d2h, "steps": ke},
         "gpu_launches": launches * steps_done,
         "device_status": status,
+        "near_ties": None if ties is None else ties.report(
+            "the CPU baseline's oracle passes vs the GPU's decisions of the same pass"),
+        "batch1_step_us": batch1,
         "cpu_baseline": cpu,
     }
     print(json.dumps(line))
