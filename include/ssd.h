@@ -98,12 +98,13 @@ const char* ssd_status_string(ssd_status s);
  * releases its tensor memory and returns, so the context stays usable.  Both
  * controls are process-wide and apply to launches enqueued after the call.
  *  ssd_set_wait_limit(polls): the polls after which each bounded wait of the
- *    kernels with grid-wide waits (the fused lm_head) gives up; 0 restores the
- *    default, well above a second of waiting.
- *  ssd_set_barrier_shortfall(n): makes the fused lm_head's grid barriers wait
- *    for n arrivals more than its CTAs make, so that they cannot complete and
- *    run out after the wait limit: a way to exercise the timeout path without
- *    faulting anything.  0 (the default) turns it off.
+ *    kernels with grid-wide waits (the fused lm_head, the draft predictor)
+ *    gives up; 0 restores the default, well above a second of waiting.
+ *  ssd_set_barrier_shortfall(n): makes those kernels' grid-wide waits (the
+ *    lm_head's grid barriers, the predictor's wait for the previous product)
+ *    expect n arrivals more than their CTAs make, so that they cannot
+ *    complete and run out after the wait limit: a way to exercise the timeout
+ *    path without faulting anything.  0 (the default) turns it off.
  * ------------------------------------------------------------------------- */
 void ssd_set_wait_limit(uint32_t max_polls);
 void ssd_set_barrier_shortfall(uint32_t arrivals);
@@ -437,12 +438,14 @@ ssd_status ssd_verify_accept(const ssd_verify_args* args, const ssd_verify_out* 
  *   out_tok  dev int32 [rows] (out); out_hidden dev float32 [rows][d] or NULL
  *            (out: h_hat, the predicted pre-norm hidden state)
  *   workspace dev, >= ssd_draft_predict_workspace(rows, d, m, V) bytes
- * Every GEMM input is bf16 with fp32 accumulation (the four projections run
- * as cuBLAS GEMMs: the library creates one cuBLAS handle per device and host
- * thread on the first call, which must be outside any stream capture; the
- * handle works in `workspace` and allocates nothing afterwards).
- * Supported: rows >= 1, d, m multiples of 8, V a multiple of 4, every
- * pointer 16-byte aligned.  A cuBLAS failure returns SSD_ERR_CUDA.
+ * Every product input is bf16 with fp32 accumulation on the tensor cores
+ * (one cooperative kernel, one CTA per SM, streams every weight matrix once;
+ * more than 128 rows run as one launch per 128 rows).  The workspace size
+ * depends on the current device's SM count.  The kernel's CTAs wait on each
+ * other between the products with bounded waits: one that runs out records
+ * SSD_ERR_TIMEOUT and the call writes no tokens.
+ * Supported: rows >= 1; d, m and V multiples of 128 (other multiples of 8 /
+ * 4 return SSD_ERR_UNSUPPORTED); every pointer 16-byte aligned.
  * ------------------------------------------------------------------------- */
 size_t ssd_draft_predict_workspace(int32_t rows, int32_t d, int32_t m, int32_t V);
 ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, const void* z,

@@ -315,7 +315,8 @@ ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, cons
                              size_t workspace_bytes, int32_t* status, ssd_stream_t stream) {
   if (rows <= 0 || d <= 0 || m <= 0 || V <= 0) return SSD_ERR_SHAPE;
   if (d % 8 != 0 || m % 8 != 0 || V % 4 != 0) return SSD_ERR_SHAPE;
-  if ((int64_t)rows * 2 * m >= (int64_t)1 << 31 || (int64_t)rows * V >= (int64_t)1 << 31)
+  if (!predictor_supported(d, m, V)) return SSD_ERR_UNSUPPORTED;
+  if ((int64_t)rows * 2 * d >= (int64_t)1 << 31 || (int64_t)rows * m >= (int64_t)1 << 31)
     return SSD_ERR_UNSUPPORTED;
   const void* ptrs[] = {z, w0, w1, w3, w2, gamma1, gamma2, w_head, out_tok, status};
   for (const void* q : ptrs)
@@ -343,7 +344,7 @@ ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, cons
   p.eps = eps;
   p.out_tok = out_tok;
   p.out_hidden = out_hidden;
-  return from_cuda(launch_predictor(p, workspace, workspace_bytes, (cudaStream_t)stream));
+  return from_cuda(launch_predictor(p, workspace, workspace_bytes, status, (cudaStream_t)stream));
 }
 
 ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,

@@ -1003,24 +1003,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   }
 }
 
-typedef CUresult (*EncodeTiledFnTc)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                    const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                    const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFnTc encode_tc() {
-  static EncodeTiledFnTc fn = nullptr;
-  if (fn == nullptr) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFnTc>(p);
-  }
-  return fn;
-}
-
 }  // namespace
 
 #ifndef SSD_ATTN_TC_MIN_ROWS
@@ -1058,7 +1040,7 @@ TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int3
 
 cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
                                 float* part_lse, cudaStream_t stream, bool pdl) {
-  EncodeTiledFnTc fn = encode_tc();
+  EncodeTiledFn fn = tensor_map_encoder();
   if (fn == nullptr) return cudaErrorInvalidValue;
   const int32_t G = a.Hq / a.Hkv;
   const int32_t bm = tc_tile_rows(a.D_max, G);

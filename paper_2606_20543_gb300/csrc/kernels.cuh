@@ -310,11 +310,27 @@ struct PredictorArgs {
   int32_t* out_tok;     // [rows]
   float* out_hidden;    // fp32 [rows][d] or nullptr (then in the workspace)
 };
+// Workspace of launch_predictor (for the current device's SM count); 0 if
+// the shape is unsupported.  More than 128 rows run as several launches, one
+// per 128 rows, over the same workspace.
 size_t predictor_workspace(int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden);
-cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
+bool predictor_supported(int32_t d, int32_t m, int32_t V);  // multiples of 128
+cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes, int32_t* status,
                              cudaStream_t stream);
 
 int device_sm_count();
+
+// cuTensorMapEncodeTiled, reached through the runtime's driver entry point
+// (so the library loads without linking the driver); nullptr if unavailable.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
+// A bf16 tensor map with the 128-byte swizzle: `rank` dimensions (innermost
+// first), byte strides of dimensions 1.. and the box; false on failure.
+bool bf16_tensor_map(CUtensorMap* map, const void* base, uint32_t rank, const uint64_t* dims,
+                     const uint64_t* strides, const uint32_t* box);
 
 // Failure-detection controls (ssd_set_wait_limit, ssd_set_barrier_shortfall),
 // read by the host at every launch of a kernel with grid-wide waits: the poll

@@ -531,28 +531,10 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   }
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn_l() {
-  static EncodeTiledFn fn = nullptr;
-  if (fn == nullptr) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
-  }
-  return fn;
-}
-
 // bf16 [outer][inner] matrix, box [box_outer x 64 inner], 128-byte swizzle.
 bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
               uint32_t box_outer) {
-  EncodeTiledFn fn = encode_fn_l();
+  EncodeTiledFn fn = tensor_map_encoder();
   if (fn == nullptr) return false;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {inner * 2};
@@ -567,7 +549,7 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer
 // column blocks} (the last dimension steps 128 B along a row); a box
 // {64, kBK, 2} is one CTA's [2 blocks][kBK rows][128 B] weight tile in one copy.
 bool make_weight_map(CUtensorMap* map, const void* base, uint64_t V, uint64_t K) {
-  EncodeTiledFn fn = encode_fn_l();
+  EncodeTiledFn fn = tensor_map_encoder();
   if (fn == nullptr) return false;
   cuuint64_t dims[3] = {64, K, V / 64};
   cuuint64_t strides[2] = {V * 2, 128};

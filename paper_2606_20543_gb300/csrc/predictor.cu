@@ -4,25 +4,46 @@
 //   h_hat = W0 z + SwiGLU(RMSNorm(W0 z)),  z = [h ; e],
 //   SwiGLU(x) = W2 (silu(W1 x) * W3 x),    t_hat = argmax GenHead(RMSNorm(h_hat)).
 //
-// Design (GB300): for one row of W grid columns the predictor is a chain of
-// skinny products (rows <= a few hundred) that stream 268 MB of weights per
-// head plus the 4096 x V GenHead, so it is bound by HBM, not by the tensor
-// cores.  The four projections and the GenHead are plain GEMMs and run as
-// cuBLAS bf16 GEMMs (fp32 accumulation on the tensor cores, fp32 outputs);
-// everything between them is a kernel of this file (float4 accesses, several
-// loads in flight per thread: these kernels are latency-bound at a few dozen
-// rows), and the data flow needs no copies:
-//   H  = W0 z                 GEMM into the caller's hidden-state buffer (fp32)
-//   At = RMSNorm(H) * gamma1  rmsnorm_kernel (bf16, the next GEMM's input)
-//   UV = At [W1 | W3]^T       two GEMMs into the halves of one fp32 buffer
-//   G  = silu(U) * V          swiglu_kernel (bf16)
-//   H  = H + G W2^T           GEMM with beta = 1: the residual in place
-//   Hn = RMSNorm(H) * gamma2  rmsnorm_kernel (bf16)
-//   L  = Hn W_head            GEMM (fp32 logits, rows x V)
-//   t  = argmax L             argmax_kernel (lowest index on ties)
-#include <cublas_v2.h>
-#include <cuda_bf16.h>
-
+// Design (GB300): for one grid row of positions the predictor is a chain of
+// skinny products — at most 128 rows against four weight matrices of 64 MB
+// and the 128 MB GenHead at the paper's head size — so it is bound by reading
+// the weights once from HBM.  One persistent cooperative kernel (one CTA per
+// SM) runs the whole chain in four phases.  RMSNorm(x) g = s(x) (x * g) with
+// the row scale s(x) = 1 / sqrt(mean(x^2) + eps), and s commutes with the
+// products that follow, so every product input is an elementwise bf16 array
+// that the previous phase writes tile by tile, and the row scale is applied
+// to the product's output:
+//   P0  A  = W0 z                        (features d, K = 2d);  Ag = bf16(A * g1)
+//   P1  U  = s(A) W1 Ag, Vg = s(A) W3 Ag (features m, K = d);   G = bf16(silu(U) * Vg)
+//   P2  h  = A + W2 G                    (features d, K = m);   Hg = bf16(h * g2)
+//   P3  l  = W_head^T Hg                 (features V, K = d);   t = argmax l
+// (the GenHead's row scale s(h) > 0 leaves the argmax unchanged; the lowest
+// index wins ties).  Every product is D[128 features x N rows] += W[128 x 16]
+// X[16 x N] on the tensor cores (tcgen05.mma kind::f16, fp32 accumulation in
+// tensor memory): weights on M, the rows (padded to N, a multiple of 16) on N.
+// A phase's work is a list of units (128 features x 128 K, or 128 features x
+// 64 K of both W1 and W3), 32 KB of weights each; CTA c takes one contiguous
+// range of every phase's units, so a feature tile is split over at most a few
+// CTAs along K (split-K partials summed in a fixed order).
+//   * warps 0, 1: weight producers (alternate units, one or two TMA copies per
+//     unit) running ahead through all four phases: the weights do not depend
+//     on the activations, so the weight stream keeps going while a phase
+//     waits for the previous one to finish;
+//   * warp 3, lane 0: activation producer — once every tile of the previous
+//     phase is final (a bounded wait on a counter), one TMA copy of each
+//     unit's activation tile X (K-major, 128-byte swizzle) from z, Ag, G or
+//     Hg; warp 3 also allocates and frees the tensor memory;
+//   * warp 2: issues the MMAs of each unit into one of two TMEM accumulators
+//     (the next tile's products overlap the previous tile's epilogue);
+//   * warps 4-7: the epilogue.  Each TMEM lane is one feature; the CTA's
+//     partial of a tile goes to the workspace, then a ticket per tile: the
+//     last contributor sums the tile's partials in slot order and finishes it
+//     (A, Ag and A's squares per row; G; h and Hg; the tile's argmax per row),
+//     then counts the tile done.  The last tile of P3 reduces the tiles'
+//     argmaxes to the tokens.
+// Numerics: every product input is bf16 (z, the weights, Ag, G, Hg); A, U,
+// Vg, h and the logits are fp32; every sum runs in a fixed order, so results
+// do not depend on timing.
 #include <algorithm>
 
 #include "kernels.cuh"
@@ -31,183 +52,781 @@ namespace ssd {
 
 namespace {
 
-constexpr int kNormThreads = 256;
+constexpr int kPThreads = 256;       // 8 warps
+constexpr int kWarpMma = 2;
+constexpr int kWarpX = 3;            // activation producer; allocates / frees tensor memory
+constexpr int kEpiWarp0 = 4;         // warps 4-7: TMEM lane quarters 0-3
+constexpr int kEpiThreads = 128;
+constexpr int kUnitBytes = 32768;    // weights per unit
+constexpr int kMaxRows = 128;
+constexpr int kPhases = 4;
+constexpr int kBarEpi = 1;           // named barrier of the epilogue warps
+constexpr int kMaxSlots = 8;         // most CTAs sharing one feature tile
 
-__device__ __forceinline__ float block_sum(float v, float* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  v = warp_sum(v);
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  float t = 0.f;
-  if (warp == 0) {
-    t = lane < (int)(blockDim.x >> 5) ? red[lane] : 0.f;
-    t = warp_sum(t);
-    if (lane == 0) red[0] = t;
-  }
-  __syncthreads();
-  return red[0];
+struct PredPhase {
+  int32_t units;    // units of the phase
+  int32_t upt;      // units per feature tile
+  int32_t tiles;    // feature tiles of 128
+  int32_t kw;       // K per unit: 128, or 64 (P1: W1 and W3 tiles of 64)
+  int32_t slots;    // most CTAs contributing to one tile
+};
+
+struct PredLaunch {
+  PredPhase ph[kPhases];
+  int32_t ncta, rows, nn, nc;  // rows, MMA N (rows padded to 16), TMEM columns per accumulator
+  int32_t stages;              // ring slots (weights + activations of one unit each)
+  int32_t d, m, V;
+  uint32_t max_polls, shortfall;
+  float eps;
+  const float* gamma1;
+  const float* gamma2;
+  float* hid;                  // fp32 [rows][d]: A, then h_hat
+  __nv_bfloat16* ag;           // bf16 [rows][d]: A * g1, then h_hat * g2
+  __nv_bfloat16* g;            // bf16 [rows][m]: silu(U) * Vg
+  float* ss;                   // fp32 [d/128][128]: per-tile sums of squares of A's rows
+  float2* amax;                // [V/128][128]: (max logit, index) per tile and row
+  float* part;                 // split-K partials
+  unsigned int* ctr;           // tickets [4][max tiles], done [4], abort
+  int32_t max_tiles;
+  int32_t* out_tok;
+  int32_t* status;
+};
+
+__device__ __forceinline__ int64_t unit_start(int32_t c, int32_t units, int32_t ncta) {
+  return (int64_t)c * units / ncta;
+}
+// The CTA whose range holds unit u.
+__device__ __forceinline__ int32_t unit_cta(int64_t u, int32_t units, int32_t ncta) {
+  return (int32_t)(((u + 1) * ncta + units - 1) / units) - 1;
 }
 
-// One CTA per row: y = x / sqrt(mean(x^2) + eps) * gamma, rounded to bf16.
-// float4 accesses, unrolled so that several loads are in flight (d % 4 == 0).
-__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __restrict__ x,
-                                                               const float* __restrict__ gamma,
-                                                               float eps, int32_t d,
-                                                               __nv_bfloat16* __restrict__ y) {
-  __shared__ float red[32];
-  const float4* xr = reinterpret_cast<const float4*>(x + (int64_t)blockIdx.x * d);
-  const float4* g4 = reinterpret_cast<const float4*>(gamma);
-  uint2* yr = reinterpret_cast<uint2*>(y + (int64_t)blockIdx.x * d);
-  const int32_t n4 = d >> 2;
-  float ss = 0.f;
-#pragma unroll 4
-  for (int32_t i = threadIdx.x; i < n4; i += blockDim.x) {
-    const float4 v = xr[i];
-    ss += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
-  }
-  const float inv = 1.0f / sqrtf(block_sum(ss, red) / (float)d + eps);
-#pragma unroll 4
-  for (int32_t i = threadIdx.x; i < n4; i += blockDim.x) {
-    const float4 v = xr[i], gm = g4[i];
-    uint2 o;
-    o.x = pack_bf16x2(v.x * inv * gm.x, v.y * inv * gm.y);
-    o.y = pack_bf16x2(v.z * inv * gm.z, v.w * inv * gm.w);
-    yr[i] = o;
-  }
+__device__ __forceinline__ void bar_named(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
-// g = silu(u) * v over rows x m; uv holds [u | v] per row (2m floats).
-__global__ void swiglu_kernel(const float* __restrict__ uv, int32_t rows, int32_t m,
-                              __nv_bfloat16* __restrict__ g) {
-  const int64_t n = (int64_t)rows * m;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / m, j = i - r * m;
-    const float u = uv[r * 2 * m + j], v = uv[r * 2 * m + m + j];
-    g[i] = __float2bfloat16_rn(u / (1.0f + expf(-u)) * v);
-  }
+// Named barrier that also ORs a predicate over its `count` threads: every
+// thread of the group leaves with the same answer from the same barrier.
+__device__ __forceinline__ bool bar_or(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
+      " bar.red.or.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"(pred ? 1u : 0u), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
 }
 
-// One CTA per row: the first index of the maximum logit (V % 4 == 0; float4
-// loads, unrolled so that several are in flight).
-__global__ void __launch_bounds__(kNormThreads) argmax_kernel(const float* __restrict__ logits,
-                                                              int32_t V,
-                                                              int32_t* __restrict__ out_tok) {
-  __shared__ float sv[32];
-  __shared__ int32_t si[32];
-  const float4* lr = reinterpret_cast<const float4*>(logits + (int64_t)blockIdx.x * V);
-  float bv = -INFINITY;
-  int32_t bi = 0x7fffffff;
-#pragma unroll 4
-  for (int32_t i = threadIdx.x; i < (V >> 2); i += blockDim.x) {
-    const float4 v = lr[i];  // ascending index per thread: the first maximum is kept
-    if (v.x > bv) { bv = v.x; bi = 4 * i; }
-    if (v.y > bv) { bv = v.y; bi = 4 * i + 1; }
-    if (v.z > bv) { bv = v.z; bi = 4 * i + 2; }
-    if (v.w > bv) { bv = v.w; bi = 4 * i + 3; }
+__device__ __forceinline__ uint32_t ld_acquire_u32(const unsigned int* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Order this thread's generic-proxy global accesses with async-proxy (TMA)
+// accesses: after writing an array that other CTAs will load by TMA, and
+// after learning that such an array is complete, before loading it.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Release / acquire at GPU scope (lighter than a sequentially consistent
+// fence): orders this thread's earlier writes before, and its later reads
+// after, the ticket and counter atomics that publish and claim them.
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+
+// Counters, one per 128-byte line so that CTAs counting different tiles do
+// not contend for one line: tickets [4][max tiles], done [4], abort.
+constexpr int kCtrStride = 32;
+__device__ __forceinline__ unsigned int* ticket(const PredLaunch& L, int p, int f) {
+  return L.ctr + (p * L.max_tiles + f) * kCtrStride;
+}
+__device__ __forceinline__ unsigned int* done_ctr(const PredLaunch& L, int p) {
+  return L.ctr + (kPhases * L.max_tiles + p) * kCtrStride;
+}
+__device__ __forceinline__ unsigned int* abort_flag(const PredLaunch& L) {
+  return L.ctr + (kPhases * L.max_tiles + kPhases) * kCtrStride;
+}
+
+// Bounded wait until *ctr >= target; false (SSD_ERR_TIMEOUT recorded, abort
+// raised) if it gave up, or if another CTA aborted the kernel.
+__device__ bool wait_count(const PredLaunch& L, const unsigned int* ctr, uint32_t target) {
+  for (uint32_t i = 0; i < L.max_polls; ++i) {
+    if (ld_acquire_u32(ctr) >= target) return ld_acquire_u32(abort_flag(L)) == 0u;
+    if ((i & 1023u) == 1023u && ld_acquire_u32(abort_flag(L)) != 0u) return false;
+    if (i > 64) __nanosleep(128);
   }
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  atomicExch(abort_flag(L), 1u);
+  record_status(L.status, SSD_ERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ void warp_argmax(float& v, int32_t& i) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-    const int32_t oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-  }
-  if (lane == 0) { sv[warp] = bv; si[warp] = bi; }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
-      if (sv[w] > bv || (sv[w] == bv && si[w] < bi)) { bv = sv[w]; bi = si[w]; }
-    out_tok[blockIdx.x] = bi;
+    const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+    const int32_t oi = __shfl_xor_sync(0xffffffffu, i, o);
+    if (ov > v || (ov == v && oi < i)) {
+      v = ov;
+      i = oi;
+    }
   }
 }
 
-// cuBLAS handle per device and host thread, created on first use.
-constexpr int kMaxDevices = 64;
-cublasStatus_t blas_handle(cublasHandle_t* out) {
-  thread_local cublasHandle_t handles[kMaxDevices] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-    return CUBLAS_STATUS_NOT_INITIALIZED;
-  if (handles[dev] == nullptr) {
-    const cublasStatus_t s = cublasCreate(&handles[dev]);
-    if (s != CUBLAS_STATUS_SUCCESS) return s;
+}  // namespace
+
+namespace {
+
+// Epilogue of the last contributor of tile f of phase p: the tile's partials
+// summed in slot order, then the phase's finishing step.  Thread et (0..127)
+// takes features f * 128 + 4 q .. + 3 (q = et % 32, 16-byte loads) of rows
+// et / 32 + 4 i; the 32 lanes of a warp hold one row's 128 features, so row
+// reductions are warp reductions.  Each batch issues RB rows x NACC
+// accumulators x SMAX slots (32 float4, slots beyond cnt predicated off)
+// before summing any, so a tile costs a few round trips to L2.
+// srow: [128] (the row scales of A, P1).
+template <int SMAX, int NACC>
+__device__ void finish_tile(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
+                            float* srow) {
+  constexpr int RB = 32 / (SMAX * NACC) > 0 ? 32 / (SMAX * NACC) : 1;
+  const PredPhase& ph = L.ph[p];
+  const int w = et >> 5, q = et & 31;
+  const int32_t feat = f * 128 + 4 * q;
+  const int64_t tile_stride = (int64_t)NACC * L.nn * 128;
+  const float* base = L.part + (int64_t)f * ph.slots * tile_stride + 4 * q;
+  if (p == 1) {  // the row scales s(A) from the per-tile sums of squares (fixed order)
+    for (int32_t r = et; r < L.rows; r += kEpiThreads) {
+      float s = 0.f;
+      for (int32_t t = 0; t < L.d / 128; ++t) s += __ldcg(L.ss + (int64_t)t * 128 + r);
+      srow[r] = 1.0f / sqrtf(s / (float)L.d + L.eps);
+    }
+    bar_named(kBarEpi, kEpiThreads);
   }
-  *out = handles[dev];
-  return CUBLAS_STATUS_SUCCESS;
+  float4 ga = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (p == 0) ga = __ldg(reinterpret_cast<const float4*>(L.gamma1 + feat));
+  if (p == 2) ga = __ldg(reinterpret_cast<const float4*>(L.gamma2 + feat));
+  const int32_t my_rows = (L.rows - w + 3) / 4;  // rows w, w + 4, ... below L.rows
+  for (int32_t i0 = 0; i0 < my_rows; i0 += RB) {
+    float4 v[RB][NACC][SMAX];
+#pragma unroll
+    for (int b = 0; b < RB; ++b)
+#pragma unroll
+      for (int a = 0; a < NACC; ++a)
+#pragma unroll
+        for (int sl = 0; sl < SMAX; ++sl) {
+          v[b][a][sl] = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (sl < cnt && i0 + b < my_rows) {
+            const int32_t r = w + 4 * (i0 + b);
+            v[b][a][sl] = __ldcg(reinterpret_cast<const float4*>(
+                base + sl * tile_stride + ((int64_t)a * L.nn + r) * 128));
+          }
+        }
+#pragma unroll
+    for (int b = 0; b < RB; ++b) {
+      if (i0 + b >= my_rows) continue;  // the same in every lane of the warp
+      const int32_t r = w + 4 * (i0 + b);
+      float4 x[NACC];
+#pragma unroll
+      for (int a = 0; a < NACC; ++a) {
+        x[a] = v[b][a][0];
+#pragma unroll
+        for (int sl = 1; sl < SMAX; ++sl) {  // slot order; the predicated-off slots add zero
+          x[a].x += v[b][a][sl].x;
+          x[a].y += v[b][a][sl].y;
+          x[a].z += v[b][a][sl].z;
+          x[a].w += v[b][a][sl].w;
+        }
+      }
+      if (NACC == 2) {  // P1: G = silu(U) * Vg with U, Vg scaled by the row's s(A)
+        const float sr = srow[r];
+        const float4 uu = x[0], vv = x[NACC - 1];
+        const float u0 = uu.x * sr, u1 = uu.y * sr, u2 = uu.z * sr, u3 = uu.w * sr;
+        uint2 o;
+        o.x = pack_bf16x2(u0 / (1.0f + expf(-u0)) * (vv.x * sr), u1 / (1.0f + expf(-u1)) * (vv.y * sr));
+        o.y = pack_bf16x2(u2 / (1.0f + expf(-u2)) * (vv.z * sr), u3 / (1.0f + expf(-u3)) * (vv.w * sr));
+        *reinterpret_cast<uint2*>(L.g + (int64_t)r * L.m + feat) = o;
+      } else if (p == 3) {  // the tile's argmax for row r (lowest index on ties)
+        float bv = x[0].x;
+        int32_t bi = feat;
+        if (x[0].y > bv) { bv = x[0].y; bi = feat + 1; }
+        if (x[0].z > bv) { bv = x[0].z; bi = feat + 2; }
+        if (x[0].w > bv) { bv = x[0].w; bi = feat + 3; }
+        warp_argmax(bv, bi);
+        if (q == 0) L.amax[(int64_t)f * 128 + r] = make_float2(bv, __int_as_float(bi));
+      } else {  // P0: A, Ag = bf16(A * g1), A's squares; P2: h = A + sum, Hg = bf16(h * g2)
+        float* hp = L.hid + (int64_t)r * L.d + feat;
+        float4 y = x[0];
+        if (p == 2) {
+          const float4 a0 = __ldcg(reinterpret_cast<const float4*>(hp));
+          y = make_float4(a0.x + y.x, a0.y + y.y, a0.z + y.z, a0.w + y.w);
+        }
+        *reinterpret_cast<float4*>(hp) = y;
+        uint2 o;
+        o.x = pack_bf16x2(y.x * ga.x, y.y * ga.y);
+        o.y = pack_bf16x2(y.z * ga.z, y.w * ga.w);
+        *reinterpret_cast<uint2*>(L.ag + (int64_t)r * L.d + feat) = o;
+        if (p == 0) {
+          const float sq = warp_sum((y.x * y.x + y.y * y.y) + (y.z * y.z + y.w * y.w));
+          if (q == 0) L.ss[(int64_t)f * 128 + r] = sq;
+        }
+      }
+    }
+  }
 }
+
+template <int NACC>
+__device__ void finish_tile_n(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
+                              float* srow) {
+  switch (cnt) {  // the slot count fixes the batch shape (one batch for 24 rows up to 5 slots)
+    case 1: finish_tile<1, NACC>(L, p, f, cnt, et, srow); break;
+    case 2: finish_tile<2, NACC>(L, p, f, cnt, et, srow); break;
+    case 3: finish_tile<3, NACC>(L, p, f, cnt, et, srow); break;
+    case 4: finish_tile<4, NACC>(L, p, f, cnt, et, srow); break;
+    case 5: finish_tile<5, NACC>(L, p, f, cnt, et, srow); break;
+    case 6: finish_tile<6, NACC>(L, p, f, cnt, et, srow); break;
+    default: finish_tile<8, NACC>(L, p, f, cnt, et, srow); break;
+  }
+}
+
+__device__ void finish_tile_any(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
+                                float* srow) {
+  if (p == 1)
+    finish_tile_n<2>(L, p, f, cnt, et, srow);
+  else
+    finish_tile_n<1>(L, p, f, cnt, et, srow);
+}
+
+__device__ __forceinline__ void issue_weights(const PredLaunch& L, int p, int32_t u,
+                                              unsigned char* dst, uint64_t* bar, uint64_t pol,
+                                              const CUtensorMap* tmW0, const CUtensorMap* tmW1,
+                                              const CUtensorMap* tmW3, const CUtensorMap* tmW2,
+                                              const CUtensorMap* tmWH) {
+  const PredPhase& ph = L.ph[p];
+  const int32_t f = u / ph.upt, j = u - f * ph.upt;
+  if (p == 0) {
+    tma_load_3d(dst, tmW0, 0, f * 128, 2 * j, bar, pol);
+  } else if (p == 1) {
+    tma_load_2d(dst, tmW1, j * 64, f * 128, bar, pol);
+    tma_load_2d(dst + 16384, tmW3, j * 64, f * 128, bar, pol);
+  } else if (p == 2) {
+    tma_load_3d(dst, tmW2, 0, f * 128, 2 * j, bar, pol);
+  } else {
+    tma_load_3d(dst, tmWH, 0, j * 128, 2 * f, bar, pol);
+  }
+}
+
+// The activation tile of unit u: rows x kw entries of the phase's input from
+// column j * kw, as [kw / 64][nn rows][128 B] (rows past `rows` read as zero).
+__device__ __forceinline__ void issue_x(const PredLaunch& L, int p, int32_t u, unsigned char* dst,
+                                        uint64_t* bar, uint64_t pol, const CUtensorMap* tmZ,
+                                        const CUtensorMap* tmAg, const CUtensorMap* tmG,
+                                        const CUtensorMap* tmHg) {
+  const PredPhase& ph = L.ph[p];
+  const int32_t j = u % ph.upt;
+  if (p == 0)
+    tma_load_3d(dst, tmZ, 0, 0, 2 * j, bar, pol);
+  else if (p == 1)
+    tma_load_2d(dst, tmAg, j * 64, 0, bar, pol);  // box {64, nn}
+  else if (p == 2)
+    tma_load_3d(dst, tmG, 0, 0, 2 * j, bar, pol);
+  else
+    tma_load_3d(dst, tmHg, 0, 0, 2 * j, bar, pol);  // the 3D view of the same array
+}
+
+}  // namespace
+
+namespace {
+
+__global__ void __launch_bounds__(kPThreads, 1)
+predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant__ CUtensorMap tmW1,
+                 const __grid_constant__ CUtensorMap tmW3, const __grid_constant__ CUtensorMap tmW2,
+                 const __grid_constant__ CUtensorMap tmWH, const __grid_constant__ CUtensorMap tmZ,
+                 const __grid_constant__ CUtensorMap tmAg, const __grid_constant__ CUtensorMap tmG,
+                 const __grid_constant__ CUtensorMap tmHg, PredLaunch L) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // ring slot: the unit's weights (32 KB), then its activation tile (two
+  // 64-wide K atoms of nn rows); one barrier per slot for both
+  const int S = L.stages;
+  const uint32_t xslot = (uint32_t)L.nn * 256u;
+  const uint32_t slot_bytes = kUnitBytes + xslot;
+  unsigned char* ring = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + S * slot_bytes);
+  uint64_t* empty = full + S;
+  uint64_t* acc_full = empty + S;      // [2]
+  uint64_t* acc_empty = acc_full + 2;  // [2]
+  uint64_t* mma_done = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  // a role that gives up raises `fail`; the epilogue warps decide to stop only
+  // through a reducing named barrier (bar_or), so they leave their loop together
+  volatile int32_t* fail = reinterpret_cast<volatile int32_t*>(tmem_slot + 1);
+  uint32_t* bcast = reinterpret_cast<uint32_t*>(tmem_slot + 2);  // [2]
+  float* srow = reinterpret_cast<float*>(tmem_slot + 8);          // [128]
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int32_t cta = blockIdx.x;
+  uint32_t ncols = 32;
+  while (ncols < (uint32_t)(4 * L.nc)) ncols <<= 1;
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 2);  // the weight producer's and the activation producer's arrivals
+      mbar_init(&empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&acc_full[s], 1);
+      mbar_init(&acc_empty[s], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(mma_done, 1);
+    *fail = 0;
+    fence_barrier_init();
+  }
+  if (warp == kWarpX) {
+    tmem_alloc(tmem_slot, ncols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp <= 1) {
+    // ---- weight producers: unit gu (counted over all phases) is issued by
+    // warp gu % 2 into ring slot gu % S
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      uint32_t gu = 0;
+      bool ok = true;
+      for (int p = 0; p < kPhases && ok; ++p) {
+        const PredPhase& ph = L.ph[p];
+        const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
+        for (int64_t u = lo; u < hi; ++u, ++gu) {
+          if ((int)(gu & 1u) != warp) continue;
+          const uint32_t s = gu % S;
+          if (*fail || (gu >= (uint32_t)S &&
+                        !mbar_wait(&empty[s], ((gu / S) - 1) & 1, L.status, L.max_polls))) {
+            *fail = 1;
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], kUnitBytes);
+          issue_weights(L, p, (int32_t)u, ring + s * slot_bytes, &full[s], pol, &tmW0, &tmW1,
+                        &tmW3, &tmW2, &tmWH);
+        }
+      }
+      // copies still in flight can only be among the last S units issued:
+      // wait for those before the CTA may exit
+      for (uint32_t x = gu > (uint32_t)S ? gu - S : 0; x < gu; ++x)
+        if ((int)(x & 1u) == warp) mbar_wait(&full[x % S], (x / S) & 1, nullptr, L.max_polls);
+    }
+    __syncwarp();
+  } else if (warp == kWarpX) {
+    // ---- activation producer
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_last();  // read again by the CTAs sharing a K range
+      uint32_t gu = 0;
+      bool ok = true;
+      for (int p = 0; p < kPhases && ok; ++p) {
+        const PredPhase& ph = L.ph[p];
+        if (p >= 1) {  // every tile of the previous phase final
+          if (*fail ||
+              !wait_count(L, done_ctr(L, p - 1), (uint32_t)L.ph[p - 1].tiles + L.shortfall)) {
+            *fail = 1;
+            break;
+          }
+          fence_proxy_async_global();
+        }
+        const uint32_t bytes = (uint32_t)L.nn * ph.kw * 2;
+        const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
+        for (int64_t u = lo; u < hi; ++u, ++gu) {
+          const uint32_t s = gu % S;
+          if (*fail || (gu >= (uint32_t)S &&
+                        !mbar_wait(&empty[s], ((gu / S) - 1) & 1, L.status, L.max_polls))) {
+            *fail = 1;
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], bytes);
+          issue_x(L, p, (int32_t)u, ring + s * slot_bytes + kUnitBytes, &full[s], pol, &tmZ,
+                  &tmAg, &tmG, &tmHg);
+        }
+      }
+      for (uint32_t x = gu > (uint32_t)S ? gu - S : 0; x < gu; ++x)
+        mbar_wait(&full[x % S], (x / S) & 1, nullptr, L.max_polls);
+    }
+    __syncwarp();
+  } else if (warp == kWarpMma) {
+    // ---- MMA issue: one thread
+    if (lane == 0) {
+      const uint32_t idk = idesc_bf16(128, L.nn, false, false);
+      const uint32_t idmn = idesc_bf16(128, L.nn, true, false);
+      const uint32_t xatom = (uint32_t)L.nn * 128u;  // one 64-wide K atom of the activations
+      uint32_t gu = 0, tc = 0;
+      bool ok = true;
+      for (int p = 0; p < kPhases && ok; ++p) {
+        const PredPhase& ph = L.ph[p];
+        const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
+        uint32_t buf = 0;
+        int32_t j = (int32_t)(lo % ph.upt);  // K step of unit u inside its tile
+        for (int64_t u = lo; u < hi; ++u, ++gu, j = (j + 1 == ph.upt) ? 0 : j + 1) {
+          const bool first = (u == lo) || j == 0;
+          const bool last = (u == hi - 1) || j == ph.upt - 1;
+          if (first) {
+            buf = tc & 1u;
+            if (tc >= 2 && !mbar_wait(&acc_empty[buf], ((tc >> 1) - 1) & 1, L.status, L.max_polls)) {
+              ok = false;
+              break;
+            }
+          }
+          if (!mbar_wait(&full[gu % S], (gu / S) & 1, L.status, L.max_polls)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t wb = smem_u32(ring + (gu % S) * slot_bytes);
+          const uint64_t dx = smem_desc(wb + kUnitBytes, 16, 1024);
+          const uint32_t dacc = tmem + buf * 2u * (uint32_t)L.nc;
+          const uint32_t a0 = first ? 0u : 1u;
+          if (p == 1) {  // W1 and W3 tiles of 64 K against one activation atom
+            const uint64_t dw = smem_desc(wb, 16, 1024);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint32_t acc = kk > 0 ? 1u : a0;
+              mma_ss(dacc, smem_desc_at(dw, kk * 32), smem_desc_at(dx, kk * 32), idk, acc);
+              mma_ss(dacc + L.nc, smem_desc_at(dw, 16384 + kk * 32), smem_desc_at(dx, kk * 32), idk,
+                     acc);
+            }
+          } else if (p == 3) {  // GenHead: vocabulary contiguous (MN-major), halves 16 KB apart
+            const uint64_t dw = smem_desc(wb, 16384, 1024);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_ss(dacc, smem_desc_at(dw, kk * 2048),
+                     smem_desc_at(dx, (kk >> 2) * xatom + (kk & 3) * 32), idmn, kk > 0 ? 1u : a0);
+          } else {  // K-major: two 64-wide K atoms of 16 KB
+            const uint64_t dw = smem_desc(wb, 16, 1024);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_ss(dacc, smem_desc_at(dw, (kk >> 2) * 16384 + (kk & 3) * 32),
+                     smem_desc_at(dx, (kk >> 2) * xatom + (kk & 3) * 32), idk, kk > 0 ? 1u : a0);
+          }
+          mma_commit(&empty[gu % S]);
+          if (last) {
+            mma_commit(&acc_full[buf]);
+            ++tc;
+          }
+        }
+      }
+      if (!ok) *fail = 1;
+      mma_commit(mma_done);  // arrives once every MMA issued above has completed
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue (warps 4-7): TMEM lane = feature et of the tile
+    const int et = tid - kEpiWarp0 * 32;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    uint32_t tc = 0;
+    bool ok = true;
+    for (int p = 0; p < kPhases && ok; ++p) {
+      const PredPhase& ph = L.ph[p];
+      const int nacc = p == 1 ? 2 : 1;
+      const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
+      const int32_t f0 = (int32_t)(lo / ph.upt), f1 = (int32_t)((hi - 1) / ph.upt);
+      for (int32_t f = f0; f <= f1; ++f, ++tc) {
+        const uint32_t buf = tc & 1u;
+        bool stop = false;
+        if (lane == 0) {
+          stop = *fail != 0 || !mbar_wait(&acc_full[buf], (tc >> 1) & 1, L.status, L.max_polls);
+          if (stop) *fail = 1;
+        }
+        if (bar_or(kBarEpi, kEpiThreads, stop)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int32_t first = unit_cta((int64_t)f * ph.upt, ph.units, L.ncta);
+        const int32_t lastc = unit_cta((int64_t)(f + 1) * ph.upt - 1, ph.units, L.ncta);
+        float* dst = L.part + ((int64_t)f * ph.slots + (cta - first)) * nacc * L.nn * 128 + et;
+        for (int a = 0; a < nacc; ++a) {
+          for (int32_t ch = 0; ch < L.nc / 32; ++ch) {
+            float v[32];
+            tmem_ld32(tmem + lane_base + buf * 2u * (uint32_t)L.nc + a * L.nc + ch * 32, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int32_t r = ch * 32 + i;
+              if (r < L.rows) __stcg(dst + ((int64_t)a * L.nn + r) * 128, v[i]);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        fence_acq_rel_gpu();  // the partial before the ticket
+        bar_named(kBarEpi, kEpiThreads);
+        if (et == 0) bcast[0] = atomicAdd(ticket(L, p, f), 1u);
+        bar_named(kBarEpi, kEpiThreads);
+        if (bcast[0] != (uint32_t)(lastc - first)) continue;  // not the last contributor
+        fence_acq_rel_gpu();  // every contributor's partial after the ticket
+        finish_tile_any(L, p, f, lastc - first + 1, et, srow);
+        fence_proxy_async_global();  // Ag, G, Hg are loaded by TMA in the next phase
+        fence_acq_rel_gpu();
+        bar_named(kBarEpi, kEpiThreads);
+        if (et == 0) bcast[1] = atomicAdd(done_ctr(L, p), 1u);
+        bar_named(kBarEpi, kEpiThreads);
+        if (p == 3 && bcast[1] == (uint32_t)(ph.tiles - 1)) {
+          // the last tile of the vocabulary: reduce the tiles' argmaxes (warp w
+          // takes rows w, w + 4, ...; lane l tiles l, l + 32, ...; the lower
+          // index wins between equal maxima, so the first maximum is kept)
+          fence_acq_rel_gpu();
+          const int q = et & 31;
+          for (int32_t r = et >> 5; r < L.rows; r += 4) {
+            float bv = -INFINITY;
+            int32_t bi = 0x7fffffff;
+            for (int32_t t = q; t < ph.tiles; t += 32) {
+              const float2 e = __ldcg(L.amax + (int64_t)t * 128 + r);
+              const int32_t ei = __float_as_int(e.y);
+              if (e.x > bv || (e.x == bv && ei < bi)) {
+                bv = e.x;
+                bi = ei;
+              }
+            }
+            warp_argmax(bv, bi);
+            if (q == 0) L.out_tok[r] = bi;
+          }
+        }
+      }
+    }
+  }
+
+  // ---- teardown: every MMA complete before tensor memory is freed
+  if (warp == kWarpX && lane == 0) mbar_wait(mma_done, 0, nullptr, L.max_polls);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpX) {
+    tc_fence_after();
+    tmem_dealloc(tmem, ncols);
+  }
+}
+
+}  // namespace
+
+namespace {
 
 size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
-constexpr size_t kBlasWorkspace = (size_t)32 << 20;
+
+struct PredPlan {
+  PredPhase ph[kPhases];
+  int32_t ncta, nn, nc, stages, max_tiles;
+  size_t part_floats, smem;
+};
+
+int32_t tile_slots(const PredPhase& ph, int32_t ncta) {
+  int32_t most = 1;
+  for (int32_t f = 0; f < ph.tiles; ++f) {
+    const int64_t u0 = (int64_t)f * ph.upt, u1 = (int64_t)(f + 1) * ph.upt - 1;
+    const int32_t c0 = (int32_t)(((u0 + 1) * ncta + ph.units - 1) / ph.units) - 1;
+    const int32_t c1 = (int32_t)(((u1 + 1) * ncta + ph.units - 1) / ph.units) - 1;
+    most = std::max(most, c1 - c0 + 1);
+  }
+  return most;
+}
+
+PredPlan make_plan(int32_t rows, int32_t d, int32_t m, int32_t V, int32_t sm_count) {
+  PredPlan P;
+  // P0: W0 [d][2d]; P1: W1, W3 [m][d] in 64-wide K steps; P2: W2 [d][m];
+  // P3: W_head [d][V] (vocabulary on M)
+  const int32_t tiles[kPhases] = {d / 128, m / 128, d / 128, V / 128};
+  const int32_t K[kPhases] = {2 * d, d, m, d};
+  const int32_t kw[kPhases] = {128, 64, 128, 128};
+  int32_t min_units = INT32_MAX;
+  for (int p = 0; p < kPhases; ++p) {
+    P.ph[p].tiles = tiles[p];
+    P.ph[p].kw = kw[p];
+    P.ph[p].upt = K[p] / kw[p];
+    P.ph[p].units = tiles[p] * P.ph[p].upt;
+    min_units = std::min(min_units, P.ph[p].units);
+  }
+  // every CTA takes at least one unit of every phase, and no tile is split over
+  // more than kMaxSlots CTAs (the finisher sums at most that many partials)
+  P.ncta = std::max(1, std::min(sm_count, min_units));
+  for (;;) {
+    int32_t most = 1;
+    for (int p = 0; p < kPhases; ++p) most = std::max(most, tile_slots(P.ph[p], P.ncta));
+    if (most <= kMaxSlots || P.ncta == 1) break;
+    --P.ncta;
+  }
+  P.max_tiles = 0;
+  P.part_floats = 0;
+  P.nn = (rows + 15) / 16 * 16;
+  P.nc = (P.nn + 31) / 32 * 32;
+  for (int p = 0; p < kPhases; ++p) {
+    P.ph[p].slots = tile_slots(P.ph[p], P.ncta);
+    P.max_tiles = std::max(P.max_tiles, P.ph[p].tiles);
+    const size_t nacc = p == 1 ? 2 : 1;
+    P.part_floats = std::max(P.part_floats,
+                             (size_t)P.ph[p].tiles * P.ph[p].slots * nacc * P.nn * 128);
+  }
+  const size_t slot = (size_t)kUnitBytes + (size_t)P.nn * 256;
+  const size_t budget = 232448;  // 227 KB of dynamic shared memory per CTA
+  P.stages = (int32_t)std::min<size_t>(8, (budget - 1024 - 2048) / slot);
+  P.smem = 1024 + (size_t)P.stages * slot + (2 * P.stages + 5) * 8 + 32 + kMaxRows * 4;
+  return P;
+}
+
+struct PredWs {
+  unsigned int* ctr;
+  float* part;
+  float* ss;
+  __nv_bfloat16* ag;
+  __nv_bfloat16* g;
+  float2* amax;
+  float* hid;
+  size_t bytes;
+};
+
+PredWs carve(const PredPlan& P, int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden,
+             void* base) {
+  PredWs w;
+  unsigned char* b = static_cast<unsigned char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    unsigned char* p = b + off;
+    off += al256(n);
+    return p;
+  };
+  w.ctr = reinterpret_cast<unsigned int*>(
+      take((size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4));
+  w.part = reinterpret_cast<float*>(take(P.part_floats * 4));
+  w.ss = reinterpret_cast<float*>(take((size_t)(d / 128) * 128 * 4));
+  w.ag = reinterpret_cast<__nv_bfloat16*>(take((size_t)rows * d * 2));
+  w.g = reinterpret_cast<__nv_bfloat16*>(take((size_t)rows * m * 2));
+  w.amax = reinterpret_cast<float2*>(take((size_t)(V / 128) * 128 * 8));
+  w.hid = own_hidden ? reinterpret_cast<float*>(take((size_t)rows * d * 4)) : nullptr;
+  w.bytes = off;
+  return w;
+}
+
+bool shapes_ok(int32_t rows, int32_t d, int32_t m, int32_t V) {
+  return rows >= 1 && rows <= kMaxRows && d >= 128 && m >= 128 && V >= 128 && d % 128 == 0 &&
+         m % 128 == 0 && V % 128 == 0;
+}
+
+// One launch over at most kMaxRows rows.
+cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32_t* status,
+                        cudaStream_t stream) {
+  if (!shapes_ok(a.rows, a.d, a.m, a.V)) return cudaErrorInvalidValue;
+  const PredPlan P = make_plan(a.rows, a.d, a.m, a.V, device_sm_count());
+  const PredWs w = carve(P, a.rows, a.d, a.m, a.V, a.out_hidden == nullptr, ws);
+  if (ws == nullptr || ws_bytes < w.bytes) return cudaErrorInvalidValue;
+
+  PredLaunch L;
+  for (int p = 0; p < kPhases; ++p) L.ph[p] = P.ph[p];
+  L.ncta = P.ncta;
+  L.rows = a.rows;
+  L.nn = P.nn;
+  L.nc = P.nc;
+  L.stages = P.stages;
+  L.d = a.d;
+  L.m = a.m;
+  L.V = a.V;
+  L.max_polls = wait_poll_limit();
+  L.shortfall = barrier_shortfall();
+  L.eps = a.eps;
+  L.gamma1 = a.gamma1;
+  L.gamma2 = a.gamma2;
+  L.hid = a.out_hidden != nullptr ? a.out_hidden : w.hid;
+  L.ag = w.ag;
+  L.g = w.g;
+  L.ss = w.ss;
+  L.amax = w.amax;
+  L.part = w.part;
+  L.ctr = w.ctr;
+  L.max_tiles = P.max_tiles;
+  L.out_tok = a.out_tok;
+  L.status = status;
+
+  const uint64_t d = (uint64_t)a.d, m = (uint64_t)a.m, V = (uint64_t)a.V, R = (uint64_t)a.rows;
+  const uint32_t nn = (uint32_t)P.nn;
+  CUtensorMap t0, t1, t3, t2, th, tz, tag, tg, thg;
+  bool ok = true;
+  {  // W0 [d][2d]: {64, d rows, 2d / 64 column blocks}, box {64, 128, 2}
+    const uint64_t dims[3] = {64, d, 2 * d / 64}, str[2] = {2 * d * 2, 128};
+    const uint32_t box[3] = {64, 128, 2};
+    ok = ok && bf16_tensor_map(&t0, a.w0, 3, dims, str, box);
+  }
+  {  // W1, W3 [m][d]: {d, m}, box {64, 128}
+    const uint64_t dims[2] = {d, m}, str[1] = {d * 2};
+    const uint32_t box[2] = {64, 128};
+    ok = ok && bf16_tensor_map(&t1, a.w1, 2, dims, str, box) &&
+         bf16_tensor_map(&t3, a.w3, 2, dims, str, box);
+  }
+  {  // W2 [d][m]: {64, d rows, m / 64}, box {64, 128, 2}
+    const uint64_t dims[3] = {64, d, m / 64}, str[2] = {m * 2, 128};
+    const uint32_t box[3] = {64, 128, 2};
+    ok = ok && bf16_tensor_map(&t2, a.w2, 3, dims, str, box);
+  }
+  {  // W_head [d][V]: {64 vocabulary entries, d rows, V / 64}, box {64, 128 K, 2}
+    const uint64_t dims[3] = {64, d, V / 64}, str[2] = {V * 2, 128};
+    const uint32_t box[3] = {64, 128, 2};
+    ok = ok && bf16_tensor_map(&th, a.w_head, 3, dims, str, box);
+  }
+  {  // activations [rows][K] as {64, rows, K / 64}, box {64, nn, 2}: [2][nn][128 B]
+    const uint32_t box[3] = {64, nn, 2};
+    const uint64_t dz[3] = {64, R, 2 * d / 64}, sz[2] = {2 * d * 2, 128};
+    const uint64_t dg[3] = {64, R, m / 64}, sg[2] = {m * 2, 128};
+    const uint64_t dh[3] = {64, R, d / 64}, sh[2] = {d * 2, 128};
+    ok = ok && bf16_tensor_map(&tz, a.z, 3, dz, sz, box) &&
+         bf16_tensor_map(&tg, w.g, 3, dg, sg, box) && bf16_tensor_map(&thg, w.ag, 3, dh, sh, box);
+    // Ag in 64-wide K steps (P1): {d, rows}, box {64, nn}
+    const uint64_t da[2] = {d, R}, sa[1] = {d * 2};
+    const uint32_t ba[2] = {64, nn};
+    ok = ok && bf16_tensor_map(&tag, w.ag, 2, da, sa, ba);
+  }
+  if (!ok) return cudaErrorInvalidValue;
+  cudaError_t e = cudaMemsetAsync(
+      w.ctr, 0, (size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4, stream);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(predictor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)P.smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)P.ncta, 1, 1);
+  cfg.blockDim = dim3(kPThreads, 1, 1);
+  cfg.dynamicSmemBytes = P.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, predictor_kernel, t0, t1, t3, t2, th, tz, tag, tg, thg, L);
+}
 
 }  // namespace
 
 size_t predictor_workspace(int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden) {
-  size_t b = al256(kBlasWorkspace);
-  b += al256((size_t)rows * d * 2);       // At / Hn (bf16)
-  b += al256((size_t)rows * 2 * m * 4);   // [U | V] (fp32)
-  b += al256((size_t)rows * m * 2);       // G (bf16)
-  b += al256((size_t)rows * V * 4);       // logits (fp32)
-  if (own_hidden) b += al256((size_t)rows * d * 4);
-  return b;
+  rows = std::min(rows, kMaxRows);  // more rows run as several launches over one workspace
+  if (!shapes_ok(rows, d, m, V)) return 0;
+  const PredPlan P = make_plan(rows, d, m, V, device_sm_count());
+  return carve(P, rows, d, m, V, own_hidden, nullptr).bytes;
 }
 
-cudaError_t launch_predictor(const PredictorArgs& p, void* ws, size_t ws_bytes,
-                             cudaStream_t stream) {
-  if (ws_bytes < predictor_workspace(p.rows, p.d, p.m, p.V, p.out_hidden == nullptr))
-    return cudaErrorInvalidValue;
-  unsigned char* w = static_cast<unsigned char*>(ws);
-  void* blas_ws = w;
-  w += al256(kBlasWorkspace);
-  __nv_bfloat16* nrm = reinterpret_cast<__nv_bfloat16*>(w);
-  w += al256((size_t)p.rows * p.d * 2);
-  float* uv = reinterpret_cast<float*>(w);
-  w += al256((size_t)p.rows * 2 * p.m * 4);
-  __nv_bfloat16* g = reinterpret_cast<__nv_bfloat16*>(w);
-  w += al256((size_t)p.rows * p.m * 2);
-  float* logits = reinterpret_cast<float*>(w);
-  w += al256((size_t)p.rows * p.V * 4);
-  float* H = p.out_hidden;
-  if (H == nullptr) H = reinterpret_cast<float*>(w);
+bool predictor_supported(int32_t d, int32_t m, int32_t V) { return shapes_ok(1, d, m, V); }
 
-  const int32_t rows = p.rows, d = p.d, m = p.m;
-  const int swg_blocks = (int)std::min<int64_t>(((int64_t)rows * m + 255) / 256,
-                                                4 * (int64_t)device_sm_count());
-  cublasHandle_t h;
-  if (blas_handle(&h) != CUBLAS_STATUS_SUCCESS) return cudaErrorUnknown;
-  if (cublasSetStream(h, stream) != CUBLAS_STATUS_SUCCESS ||
-      cublasSetWorkspace(h, blas_ws, kBlasWorkspace) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
-  // Y[rows][N] (ld ldy) = (accumulate ? Y : 0) + X[rows][K] op(W); W [N][K]
-  // (a linear layer's [out][in], as the column-major product Y^T = W X^T), or
-  // [K][N] when w_kn
-  auto product = [&](int32_t N, int32_t K, const void* x, const void* w, bool w_kn, float* y,
-                     int32_t ldy, bool accumulate) -> cudaError_t {
-    const float alpha = 1.0f, beta = accumulate ? 1.0f : 0.0f;
-    const cublasStatus_t st =
-        w_kn ? cublasGemmEx(h, CUBLAS_OP_N, CUBLAS_OP_N, N, rows, K, &alpha, w, CUDA_R_16BF, N, x,
-                            CUDA_R_16BF, K, &beta, y, CUDA_R_32F, ldy, CUBLAS_COMPUTE_32F,
-                            CUBLAS_GEMM_DEFAULT)
-             : cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, N, rows, K, &alpha, w, CUDA_R_16BF, K, x,
-                            CUDA_R_16BF, K, &beta, y, CUDA_R_32F, ldy, CUBLAS_COMPUTE_32F,
-                            CUBLAS_GEMM_DEFAULT);
-    return st == CUBLAS_STATUS_SUCCESS ? cudaSuccess : cudaErrorUnknown;
-  };
-  cudaError_t e;
-  // H = W0 z
-  if ((e = product(d, 2 * d, p.z, p.w0, false, H, d, false)) != cudaSuccess) return e;
-  rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma1, p.eps, d, nrm);
-  // [U | V] = At [W1 | W3]^T: two products into the halves of each row of uv
-  if ((e = product(m, d, nrm, p.w1, false, uv, 2 * m, false)) != cudaSuccess) return e;
-  if ((e = product(m, d, nrm, p.w3, false, uv + m, 2 * m, false)) != cudaSuccess) return e;
-  swiglu_kernel<<<swg_blocks, 256, 0, stream>>>(uv, rows, m, g);
-  // H = H + G W2^T (the residual)
-  if ((e = product(d, m, g, p.w2, false, H, d, true)) != cudaSuccess) return e;
-  rmsnorm_kernel<<<rows, kNormThreads, 0, stream>>>(H, p.gamma2, p.eps, d, nrm);
-  // logits[rows][V] = Hn[rows][d] W_head[d][V]
-  if ((e = product(p.V, d, nrm, p.w_head, true, logits, p.V, false)) != cudaSuccess) return e;
-  argmax_kernel<<<rows, kNormThreads, 0, stream>>>(logits, p.V, p.out_tok);
-  return cudaGetLastError();
+cudaError_t launch_predictor(const PredictorArgs& a, void* ws, size_t ws_bytes, int32_t* status,
+                             cudaStream_t stream) {
+  for (int32_t r0 = 0; r0 < a.rows; r0 += kMaxRows) {
+    PredictorArgs c = a;
+    c.rows = std::min(kMaxRows, a.rows - r0);
+    c.z = static_cast<const __nv_bfloat16*>(a.z) + (int64_t)r0 * 2 * a.d;
+    c.out_tok = a.out_tok + r0;
+    c.out_hidden = a.out_hidden != nullptr ? a.out_hidden + (int64_t)r0 * a.d : nullptr;
+    const cudaError_t e = launch_rows(c, ws, ws_bytes, status, stream);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace ssd

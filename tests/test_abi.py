@@ -95,13 +95,16 @@ def test_host_side_validation(lib):
              fake, 1 << 30, fake, None) == 2
     assert W(4, 60, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
              fake, 1 << 30, fake, None) == 2
-    assert W(4, 64, 128, 256, None, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
-             fake, 1 << 30, fake, None) == 1
-    assert W(4, 64, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, -1.0, fake, None,
-             fake, 1 << 30, fake, None) == 1
-    need = so.ssd_draft_predict_workspace(4, 64, 128, 256)
-    assert need > 0
     assert W(4, 64, 128, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, 1 << 30, fake, None) == 3  # d not a multiple of 128
+    assert so.ssd_draft_predict_workspace(4, 64, 128, 256) == 0
+    assert W(4, 128, 256, 256, None, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
+             fake, 1 << 30, fake, None) == 1
+    assert W(4, 128, 256, 256, fake, fake, fake, fake, fake, fake, fake, fake, -1.0, fake, None,
+             fake, 1 << 30, fake, None) == 1
+    need = so.ssd_draft_predict_workspace(4, 128, 256, 256)
+    assert need > 0
+    assert W(4, 128, 256, 256, fake, fake, fake, fake, fake, fake, fake, fake, 1e-6, fake, None,
              fake, need - 1, fake, None) == 7
     for good in (lib.STRATEGY_ACCEPT_REJECT, lib.STRATEGY_GREEDY, lib.STRATEGY_SAMPLE):
         assert so.ssd_accept_strategy(good, 0, 4096, None, None, 4096, None, 1.0,

@@ -65,6 +65,7 @@ def test_against_a_torch_restatement(seed):
     logits = F.rms_norm(h, (h.shape[-1],), t["g2"], eps=1e-6) @ t["Wh"]
     h_o, l_o, tok = pr.predict(z, W0, W1, W2, W3, g1, g2, Wh, round_like_gpu=False)
     assert np.allclose(h_o, h.numpy(), rtol=1e-10, atol=1e-12)
+    assert np.allclose(l_o, logits.numpy(), rtol=1e-10, atol=1e-12)  # the row scales included
     assert np.array_equal(tok, torch.argmax(logits, 1).numpy())
     # with the GPU's bf16 rounding points the result moves by bf16-level error only
     h_b, l_b, _ = pr.predict(z, W0, W1, W2, W3, g1, g2, Wh)
