@@ -85,7 +85,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 7
+#define SSD_ABI_VERSION 8
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -290,6 +290,22 @@ typedef enum {
   SSD_COMMIT_FIRST_ROW = 3,
   SSD_COMMIT_PREFIX_BONUS = 4
 } ssd_commit;
+
+/* Commit pass (Sec. 3.3: after the final round one more forward pass commits
+ * the corrected block and updates the KV cache).  For every sequence b, with
+ * the frontier of cache_len[b] under `grid` (as ssd_frontier):
+ *   SSD_COMMIT_BLOCK      next_cache_len[b] = cache_len[b] + n_drafts
+ *   SSD_COMMIT_FIRST_ROW  next_cache_len[b] = cache_len[b] + min(n_drafts, W - c)
+ *   SSD_COMMIT_NONE       next_cache_len[b] = cache_len[b]
+ * The pass's attention over the committed block is ssd_verify_attention; the
+ * committed tokens are the ones the last round left (the pass changes none).
+ * The prefix rules need accept decisions (ssd_verify_step): they return
+ * SSD_ERR_INVALID_ARG.  Device errors: cache_len outside the grid ->
+ * DEVICE_BOUNDS (next_cache_len = cache_len).
+ *   cache_len, next_cache_len  dev int32 [B] (may alias) */
+ssd_status ssd_commit_pass(const ssd_grid* grid, int32_t B, const int32_t* cache_len,
+                           int32_t D_max, int32_t commit, int32_t* next_cache_len,
+                           int32_t* status, ssd_stream_t stream);
 
 /* Staged schedule (App. multi-row, "commit the first row, then refine the
  * trailing row"): for every sequence b and j < W, slot b * D_max + j of tok

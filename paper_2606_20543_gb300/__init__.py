@@ -24,7 +24,8 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_set_wait_limit",
             "ssd_set_barrier_shortfall", "ssd_frontier", "ssd_verify_attention_workspace",
             "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
-            "ssd_accept_round", "ssd_stage_shift", "ssd_draft_predict_workspace",
+            "ssd_accept_round", "ssd_stage_shift", "ssd_commit_pass",
+            "ssd_draft_predict_workspace",
             "ssd_draft_predict",
             "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
             "ssd_verify_step_workspace", "ssd_verify_step_launches", "ssd_verify_step",
@@ -112,6 +113,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_accept_round": (I32, [I32, I32, I32, P, I64, P, P, F, ctypes.POINTER(Rng), P, P, P, P,
                                    P, P]),
         "ssd_stage_shift": (I32, [I32, I32, I32, P, P, P]),
+        "ssd_commit_pass": (I32, [ctypes.POINTER(Grid), I32, P, I32, I32, P, P, P]),
         "ssd_draft_predict_workspace": (SZ, [I32, I32, I32, I32]),
         "ssd_draft_predict": (I32, [I32, I32, I32, I32, P, P, P, P, P, P, P, P, F, P, P, P, SZ,
                                     P, P]),
@@ -239,6 +241,14 @@ def ssd_accept_round(strategy, rows, V, tgt_logits, ld, ref_rows, tok, temperatu
         strategy, rows, V, _ptr(tgt_logits), ld, _ptr(ref_rows), _ptr(tok), temperature,
         ctypes.byref(r), _ptr(out_tok), _ptr(accepted), _ptr(ratio), _ptr(lse), _ptr(status),
         _stream(stream)))
+
+
+def ssd_commit_pass(g: Grid, B, cache_len, D_max, commit, next_cache_len, status,
+                    stream=None) -> None:
+    c = COMMITS.get(commit, commit)
+    _check("ssd_commit_pass", load().ssd_commit_pass(ctypes.byref(g), B, _ptr(cache_len), D_max,
+                                                     c, _ptr(next_cache_len), _ptr(status),
+                                                     _stream(stream)))
 
 
 def ssd_stage_shift(B, D_max, W, tok, ref_rows, stream=None) -> None:

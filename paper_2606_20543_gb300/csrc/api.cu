@@ -347,6 +347,23 @@ ssd_status ssd_draft_predict(int32_t rows, int32_t d, int32_t m, int32_t V, cons
   return from_cuda(launch_predictor(p, workspace, workspace_bytes, status, (cudaStream_t)stream));
 }
 
+ssd_status ssd_commit_pass(const ssd_grid* grid, int32_t B, const int32_t* cache_len,
+                           int32_t D_max, int32_t commit, int32_t* next_cache_len,
+                           int32_t* status, ssd_stream_t stream) {
+  ssd_status s = check_grid(grid);
+  if (s != SSD_OK) return s;
+  if (grid->row_stride != grid->grid_w) return SSD_ERR_UNSUPPORTED;
+  if (commit != SSD_COMMIT_NONE && commit != SSD_COMMIT_BLOCK && commit != SSD_COMMIT_FIRST_ROW)
+    return SSD_ERR_INVALID_ARG;
+  if (B < 0 || D_max <= 0) return SSD_ERR_SHAPE;
+  if ((int64_t)(grid->k_v + 1) * grid->grid_w > D_max) return SSD_ERR_SHAPE;
+  if (B == 0) return SSD_OK;
+  if (cache_len == nullptr || next_cache_len == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  return from_cuda(launch_commit(*grid, commit, B, D_max, cache_len, next_cache_len, status,
+                                 (cudaStream_t)stream));
+}
+
 ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
                            const float** ref_rows, ssd_stream_t stream) {
   if (B < 0 || D_max <= 0 || W < 0 || 2 * (int64_t)W > D_max) return SSD_ERR_SHAPE;

@@ -74,6 +74,40 @@ __global__ void stage_shift_kernel(int32_t B, int32_t D_max, int32_t W, int32_t*
   }
 }
 
+// Commit pass (Sec. 3.3: after the final round one more forward pass commits
+// the corrected block): the next cache length of every sequence under a
+// commit rule that needs no accept decisions.
+__global__ void commit_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_max,
+                              const int32_t* __restrict__ cache_len,
+                              int32_t* __restrict__ next_cache_len, int32_t* status) {
+  const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int32_t cl = cache_len[b];
+  const int32_t n = frontier_drafts(g, cl, D_max);
+  if (n < 0) {
+    record_status(status, SSD_ERR_DEVICE_BOUNDS);
+    next_cache_len[b] = cl;
+    return;
+  }
+  int32_t advance = 0;
+  if (commit == SSD_COMMIT_BLOCK) {
+    advance = n;
+  } else if (commit == SSD_COMMIT_FIRST_ROW) {
+    const int32_t n_c = cl - g.prefix_len;
+    advance = min(n, g.grid_w - n_c % g.grid_w);
+  }
+  next_cache_len[b] = cl + advance;
+}
+
+cudaError_t launch_commit(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
+                          const int32_t* cache_len, int32_t* next_cache_len, int32_t* status,
+                          cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  commit_kernel<<<(B + 127) / 128, 128, 0, stream>>>(g, commit, B, D_max, cache_len,
+                                                     next_cache_len, status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
                             cudaStream_t stream) {

@@ -60,6 +60,11 @@ cudaError_t launch_counts(const ssd_grid& g, int32_t commit, int32_t B, int32_t 
                           const uint8_t* accepted, int32_t* accepted_count,
                           int32_t* accepted_prefix, int32_t* next_cache_len, int32_t* status,
                           bool pdl, cudaStream_t stream);
+// Commit pass: next cache length per sequence under SSD_COMMIT_NONE / BLOCK /
+// FIRST_ROW of the frontier of cache_len under `g`.
+cudaError_t launch_commit(const ssd_grid& g, int32_t commit, int32_t B, int32_t D_max,
+                          const int32_t* cache_len, int32_t* next_cache_len, int32_t* status,
+                          cudaStream_t stream);
 // Staged schedule: slot j of every sequence takes slot W + j (j < W) of the
 // per-row tokens and reference pointers.
 cudaError_t launch_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,

@@ -11,7 +11,9 @@ import numpy as np
 import torch
 
 from . import (COMMITS, STRATEGIES, Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid,
-               row_addresses, ssd_stage_shift, ssd_verify_step, ssd_verify_step_workspace)
+               row_addresses, ssd_commit_pass, ssd_frontier, ssd_stage_shift,
+               ssd_verify_attention, ssd_verify_attention_workspace, ssd_verify_step,
+               ssd_verify_step_workspace)
 
 
 def _dev(shape, dtype, device):
@@ -251,3 +253,127 @@ class VerifyRounds:
                      False, stream)
         finally:
             s.args.grid.k_v = 1
+
+
+class VerifySchedule:
+    """The whole decoding schedule of one image (batch 1) over the buffers of
+    a VerifyStep: Sec. 3.3 (horizontal heads until the first row is complete,
+    then k_v rows drafted below at a time, verified and corrected), Sec. 4
+    "SSD Configuration" (5 horizontal drafts with one round; r rounds for one
+    vertical row, or staged b / i rounds for two) and App. "Multi-Row
+    Anticipation Ablations" (b base rounds on both rows, commit the first row,
+    i rounds on the trailing row, commit it).
+
+    Every verification round is one ssd_verify_step; every commit pass is the
+    frontier, its attention (ssd_verify_attention) and ssd_commit_pass.  Each
+    is one step, a backbone forward pass in the paper's count.  The horizontal
+    stage runs on the first row alone (a one-row grid, so that its bonus
+    token stays in that row); the device cache length drives every frontier,
+    and the host reads it after each step to know where the schedule is.
+
+    step_inputs(t) gives step t's target and draft logits (device float32
+    [>= D_max + 1, V]); the uniforms of step t are Philox(seed, t).  They
+    must stay alive and unchanged for the whole run: later rounds read earlier
+    rounds' rows as references."""
+
+    def __init__(self, step: VerifyStep, k_h=5, k_v=1, b=2, i=0):
+        if step.B != 1:
+            raise ValueError("the schedule replays one image (batch 1)")
+        if k_v not in (1, 2) or b < 1 or i < 0 or k_h < 1:
+            raise ValueError("k_v in {1, 2}, b >= 1, i >= 0, k_h >= 1")
+        W = step.g.grid_w
+        if step.D_max < k_v * W or step.D_max < k_h + 1:
+            raise ValueError("D_max must hold k_v rows and the horizontal bonus row")
+        self.s, self.k_h, self.k_v, self.b, self.i = step, k_h, k_v, b, i
+        self.rounds = VerifyRounds(step)
+        self.att_ws_bytes = ssd_verify_attention_workspace(step.B, step.Hq, step.Hkv, step.d,
+                                                           step.D_max, step.L_max)
+        self.att_ws = _dev((max(self.att_ws_bytes, 256),), torch.uint8, step.device)
+
+    def _grid(self, grid_h, k_h, k_v) -> Grid:
+        g0 = self.s.g
+        return make_grid(grid_h, g0.grid_w, g0.prefix_len, g0.row_stride, k_v, k_h)
+
+    def _cache(self) -> int:
+        return int(self.s.cache_len[0].item())
+
+    def _commit_pass(self, g: Grid, mode: str, stream=None) -> None:
+        s = self.s
+        ssd_frontier(g, s.B, s.cache_len, s.D_max, s.n_drafts, s.draft_pos, s.status, stream)
+        ssd_verify_attention(g, s.B, s.Hq, s.Hkv, s.d, s.cache_len, s.n_drafts, s.draft_pos,
+                             s.D_max, s.L_max, s.q, s.k, s.v, s.scale, s.o, None, self.att_ws,
+                             self.att_ws_bytes, s.status, stream)
+        ssd_commit_pass(g, s.B, s.cache_len, s.D_max, mode, s.next_cache_len, s.status, stream)
+        s.cache_len.copy_(s.next_cache_len)
+
+    def run(self, step_inputs, seed=0, on_step=None, stream=None) -> int:
+        """Replay to grid completion; returns the number of steps.
+        on_step(t, kind, info) is called after each step (kind 'horizontal',
+        'round' or 'commit'); info holds the host-side cache length before the
+        step and, for rounds and horizontal steps, the device tensors of the
+        decisions (valid until the next step)."""
+        s = self.s
+        a = s.args
+        g0 = s.g
+        H, W, prefix = g0.grid_h, g0.grid_w, g0.prefix_len
+        saved = (a.grid, a.commit, a.strategy, a.ref_rows, a.ref_init, a.draft_tok,
+                 a.tgt_logits, a.drf_logits)
+        t = 0
+        try:
+            # ---- horizontal stage on the first row
+            a.grid = self._grid(1, self.k_h, 0)
+            a.commit = COMMITS["prefix_bonus"]
+            a.ref_rows, a.ref_init, a.draft_tok = None, 0, None
+            cache = self._cache()
+            while cache - prefix < W:
+                tg, dr = step_inputs(t)
+                a.tgt_logits, a.drf_logits = tg.data_ptr(), dr.data_ptr()
+                s.set_rng(seed, t)
+                ssd_verify_step(a, s.out, s.workspace, s.ws_bytes, stream)
+                if on_step is not None:
+                    on_step(t, "horizontal", dict(cache_len=cache))
+                s.cache_len.copy_(s.next_cache_len)
+                cache = self._cache()
+                t += 1
+            # ---- vertical stage
+            while cache - prefix < H * W:
+                y0 = (cache - prefix) // W
+                k = min(self.k_v, H - y0)
+                g = self._grid(H, 0, k - 1)
+                a.grid = g
+                tg0, dr0 = step_inputs(t)
+                a.drf_logits = dr0.data_ptr()
+                self.rounds.reset()
+                tgts = [step_inputs(t + r)[0] for r in range(self.b)]
+                self._rounds(tgts, t, seed, True, on_step, cache, stream)
+                t += self.b
+                self._commit_pass(g, "first_row" if k > 1 else "block", stream)
+                if on_step is not None:
+                    on_step(t, "commit", dict(cache_len=cache))
+                cache = self._cache()
+                t += 1
+                if k > 1:  # the trailing row: its slots move to the front
+                    ssd_stage_shift(s.B, s.D_max, W, self.rounds.tokens, self.rounds.ref_rows,
+                                    stream)
+                    g1 = self._grid(H, 0, 0)
+                    a.grid = g1
+                    tgts = [step_inputs(t + r)[0] for r in range(self.i)]
+                    self._rounds(tgts, t, seed, False, on_step, cache, stream)
+                    t += self.i
+                    self._commit_pass(g1, "block", stream)
+                    if on_step is not None:
+                        on_step(t, "commit", dict(cache_len=cache))
+                    cache = self._cache()
+                    t += 1
+        finally:
+            (a.grid, a.commit, a.strategy, a.ref_rows, a.ref_init, a.draft_tok, a.tgt_logits,
+             a.drf_logits) = saved
+        return t
+
+    def _rounds(self, tgts, t0, seed, first_round, on_step, cache, stream):
+        """Rounds t0, t0 + 1, ... of the current frontier, one at a time so
+        that on_step sees each; nothing is committed."""
+        for r, tg in enumerate(tgts):
+            self.rounds.run([tg], "none", None, seed, t0 + r, first_round and r == 0, stream)
+            if on_step is not None:
+                on_step(t0 + r, "round", dict(cache_len=cache, tokens=self.rounds.tokens))

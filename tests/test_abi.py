@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 7
+    assert lib.ssd_abi_version() == 8
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 
@@ -88,6 +88,10 @@ def test_host_side_validation(lib):
     assert so.ssd_accept_round(5, 4, 4096, fake, 4096, fake, None, 1.0, ctypes.byref(r), fake,
                                fake, None, None, fake, None) == 1
     assert so.ssd_stage_shift(2, 48, 25, fake, None, None) == 2
+    # commit pass: only the rules that need no decisions
+    assert so.ssd_commit_pass(ctypes.byref(g), 1, fake, 32, lib.COMMIT_PREFIX, fake, fake, None) == 1
+    assert so.ssd_commit_pass(ctypes.byref(g), 1, fake, 15, lib.COMMIT_BLOCK, fake, fake, None) == 2
+    assert so.ssd_commit_pass(ctypes.byref(g), 0, None, 32, lib.COMMIT_BLOCK, None, None, None) == 0
     assert so.ssd_stage_shift(0, 48, 24, None, None, None) == 0
     # draft predictor: shapes, null pointers, workspace
     W = so.ssd_draft_predict
