@@ -211,6 +211,9 @@ MEASURED_TRAFFIC = {
     ("attention", 2): ("attention_tc.cu", "f04b60df37aa4d9c", 102185472 + 67072, None),
     ("attention", 3): ("attention_tc.cu", "f04b60df37aa4d9c", 53835776 + 3584, None),
     ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
+    # 8 x 64x64 replay, first step (1024 draft rows): accept_kernel alone; the
+    # bench scales it to the rows of the replay states it sums
+    ("accept", 5): ("accept.cu", "5476c5787745e93a", 536944896 + 3043328, 1024),
 }
 
 
@@ -630,7 +633,11 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
         "hbm_gbs_per_step": (attn_bytes_total + acc_bytes_total) / (ms / 1000.0) / 1e9,
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": achieved / hbm_peak,
-                     "traffic": measured_traffic(dom, 5, None),
+                     "traffic": measured_traffic(dom, 5, sum(int(st["n_drafts"].sum())
+                                                             for st in probe)),
+                     "traffic_note": "ncu DRAM bytes of accept_kernel at the first step, scaled "
+                                     "by the rows of the summed states (the committed draws' "
+                                     "resolve kernel not included)",
                      "peak_kind": peak_kind,
                      "state": "bytes and launch times summed over three replay states "
                               f"(steps {[st['t'] for st in probe]})",

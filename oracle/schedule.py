@@ -82,7 +82,9 @@ def replay(H, W, prefix, k_h, k_v, b, i, D_max, step_inputs, temperature=1.0,
     row).  Returns (steps, grid_tok, hist): hist has one entry per step with
     its kind ('horizontal', 'round', 'commit'), the cache length before it,
     its draft count, and for rounds and horizontal steps the accept flags,
-    the tokens after it and the count of near-tie rows."""
+    the tokens after it, the near-tie rows (tie_rows: accept or draw within
+    the bands of ``oracle.accept``; bonus_tie for the bonus draw) and their
+    count."""
     HW = H * W
     cache = prefix
     grid = np.full(HW, -1, np.int64)
@@ -109,9 +111,10 @@ def replay(H, W, prefix, k_h, k_v, b, i, D_max, step_inputs, temperature=1.0,
         if adv > n_d:
             committed.append(bonus)
         grid[n_c:n_c + adv] = committed
+        tie = dec["tie_accept"] | dec["tie_resample"]
         record("horizontal", n_d, accepted=dec["accepted"].copy(), tokens=np.array(committed),
-               ties=int(dec["tie_accept"].sum() + dec["tie_resample"].sum()
-                        + (margin < acc.NEAR_TIE_CDF)))
+               tie_rows=tie.copy(), bonus_tie=bool(margin < acc.NEAR_TIE_CDF),
+               ties=int(tie.sum() + (margin < acc.NEAR_TIE_CDF)))
         cache = nxt
         t += 1
 
@@ -141,8 +144,9 @@ def replay(H, W, prefix, k_h, k_v, b, i, D_max, step_inputs, temperature=1.0,
                 for j in np.nonzero(rej)[0]:
                     ref[offset + j] = ("tgt", t, j)
                 tok[offset:] = d["out_tok"]
+                tie = d["tie_accept"] | d["tie_resample"]
                 record("round", m, accepted=d["accepted"].copy(), tokens=tok[offset:].copy(),
-                       ties=int(d["tie_accept"].sum() + d["tie_resample"].sum()))
+                       tie_rows=tie.copy(), ties=int(tie.sum()))
                 t += 1
             # the commit pass: the frontier's first row, or what is left
             first = W - (cache - prefix) % W
