@@ -251,10 +251,11 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     tmem_relinquish();
   }
   if (a.B <= kLptMax) {
-    // s_order[rank] = the sequence with the rank-th most keys (ties by index)
+    // s_order[rank] = the sequence with the rank-th most keys (ties by index);
+    // a sequence with no drafts ranks last (its items are empty)
     for (int32_t i = tid; i < a.B; i += blockDim.x) {
       const int32_t c = a.cache_len[i], n = attn_drafts(a, i);
-      s_key[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
+      s_key[i] = (c >= 0 && n > 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
     }
     __syncthreads();
     for (int32_t i = tid; i < a.B; i += blockDim.x) {

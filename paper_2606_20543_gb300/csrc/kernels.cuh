@@ -224,14 +224,16 @@ __device__ __forceinline__ int32_t attn_draft_pos(const AttnArgs& a, int32_t b, 
 // Longest-first work order for the attention grids: CTA row `rank` (of B)
 // takes the sequence with the rank-th most keys (cache_len + n_drafts, ties by
 // index), so the longest sequences start in the first wave instead of being
-// left for the last one.  Batches above kLptMax keep their order.  Every
+// left for the last one.  A sequence with no drafts (a finished grid) has
+// nothing to attend and ranks last, so its empty items do not take the first
+// rounds of the dealing.  Batches above kLptMax keep their order.  Every
 // thread of the block must call it; `skey` is shared memory of kLptMax + 1 ints.
 constexpr int kLptMax = 256;
 __device__ __forceinline__ int32_t longest_first(const AttnArgs& a, int32_t rank, int32_t* skey) {
   if (a.B > kLptMax) return rank;
   for (int32_t i = threadIdx.x; i < a.B; i += blockDim.x) {
     const int32_t c = a.cache_len[i], n = attn_drafts(a, i);
-    skey[i] = (c >= 0 && n >= 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
+    skey[i] = (c >= 0 && n > 0 && c <= a.L_max && n <= a.D_max) ? c + n : 0;
   }
   __syncthreads();
   for (int32_t i = threadIdx.x; i < a.B; i += blockDim.x) {
