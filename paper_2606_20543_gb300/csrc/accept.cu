@@ -271,7 +271,21 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
   __shared__ Shared sh;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int32_t nch = (a.V + kChunk - 1) / kChunk;
-
+  __shared__ int32_t s_early;
+  if (warp == 0) {
+    // mode 1: always; mode 2: when the step's frontiers leave at most half of
+    // the CTAs a row (most SMs idle while the busy CTAs stream their rows)
+    bool early = a.early_dependents == 1;
+    if (a.early_dependents == 2 && a.cache_len != nullptr) {
+      int32_t live = 0;
+      for (int32_t b = lane; b < a.rows / a.D_max; b += 32)
+        live += frontier_drafts(a.grid, a.cache_len[b], a.D_max);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) live += __shfl_xor_sync(0xffffffffu, live, o);
+      early = 2 * live <= (int32_t)gridDim.x;
+    }
+    if (lane == 0) s_early = early ? 1 : 0;
+  }
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sh.full[s], 1);
@@ -280,6 +294,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
     fence_barrier_init();
   }
   __syncthreads();
+  if (s_early) pdl_launch_dependents();
 
   // (A) never draws and lazy (C) leaves its draws to launch_resolve: one pass
   const int32_t passes = (STRATEGY == SSD_STRATEGY_GREEDY || a.lazy) ? 1 : 2;

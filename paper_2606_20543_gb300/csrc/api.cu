@@ -491,8 +491,12 @@ ssd_status check_accept_part(const ssd_verify_args* x, const ssd_verify_out* y) 
 
 // Logits path, a1 + a3-a5: the acceptance pass, which computes the frontier
 // itself and writes it out (n_drafts, draft_pos).
+#ifndef SSD_ACCEPT_EARLY_PDL
+#define SSD_ACCEPT_EARLY_PDL 1
+#endif
+
 cudaError_t launch_accept_phase(const ssd_verify_args* x, const ssd_verify_out* y, void* ws,
-                                cudaStream_t stream) {
+                                cudaStream_t stream, int early_dependents = 0) {
   const bool lazy = lazy_draws(x);
   const AcceptWs w = carve_accept(x, ws);
   AcceptArgs c;
@@ -522,6 +526,7 @@ cudaError_t launch_accept_phase(const ssd_verify_args* x, const ssd_verify_out* 
   c.n_drafts_out = y->n_drafts;
   c.draft_pos = y->draft_pos;
   c.tickets = w.tickets;
+  c.early_dependents = early_dependents;
   return launch_accept(c, stream);
 }
 
@@ -668,7 +673,7 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
       // after it); then a7 (the counts, with the committed draws when lazy) as
       // a programmatic dependent of the attention: its small CTAs run beside
       // the attention, in the registers it leaves free.
-      e = launch_accept_phase(x, y, ws + attn_ws, stream);
+      e = launch_accept_phase(x, y, ws + attn_ws, stream, /*early_dependents=*/SSD_ACCEPT_EARLY_PDL);
       if (e != cudaSuccess) return SSD_ERR_CUDA;
       e = launch_attention(a, ws, attn_ws, stream, /*defer_combine=*/true, /*pdl=*/true);
       if (e != cudaSuccess) return SSD_ERR_CUDA;

@@ -25,7 +25,7 @@ def _bf(x):
     return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).cuda()
 
 
-def run_attention(ssd, c, scale=0.0, edit_pos=None):
+def run_attention(ssd, c, scale=0.0, edit_pos=None, ws=None):
     dev = "cuda"
     g = ssd.grid(c.grid_h, c.grid_w, c.prefix_len, c.row_stride, c.k_v)
     cl = torch.from_numpy(c.cache_len.astype(np.int32)).to(dev)
@@ -39,7 +39,8 @@ def run_attention(ssd, c, scale=0.0, edit_pos=None):
     o = torch.zeros((c.B, c.D_max, c.Hq, c.d), dtype=torch.bfloat16, device=dev)
     lse = torch.zeros((c.B, c.Hq, c.D_max), dtype=torch.float32, device=dev)
     wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
-    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    if ws is None:
+        ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
     ssd.ssd_verify_attention(g, c.B, c.Hq, c.Hkv, c.d, cl, nd, pos, c.D_max, c.L_max, q, k, v,
                              scale, o, lse, ws, wsb, status)
     torch.cuda.synchronize()
@@ -100,6 +101,32 @@ def test_long_cache_many_splits(ssd):
     # a long cache on one sequence: the key range is split over CTAs and merged
     c = synth.make_case("long", grid_h=64, grid_w=64, prefix_len=256, cache_len=[256 + 64 * 40 + 9],
                         Hq=4, Hkv=4, d=128, V=64, seed=7, with_logits=False)
+    check_case(ssd, c)
+
+
+def test_split_merge_ignores_workspace_contents(ssd):
+    """The tcgen05 kernel merges its KV splits itself: the CTA whose
+    partials complete a tile merges them, counted by per-launch tickets in
+    the workspace.  Whatever the workspace held before (all ones, zeros, the
+    tickets and partials of earlier launches of this and of another case),
+    the result is the same, bit for bit."""
+    c = synth.make_case("long", grid_h=64, grid_w=64, prefix_len=256, cache_len=[256 + 64 * 40 + 9],
+                        Hq=4, Hkv=4, d=128, V=64, seed=7, with_logits=False)
+    other = synth.make_case("long2", grid_h=64, grid_w=64, prefix_len=256,
+                            cache_len=[256 + 64 * 21 + 3], Hq=4, Hkv=4, d=128, V=64, seed=8,
+                            with_logits=False)
+    wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device="cuda")
+    outs = []
+    for fill in (0xFF, 0x00, None, "other", None):
+        if fill == "other":
+            run_attention(ssd, other, ws=ws)
+        elif fill is not None:
+            ws.fill_(fill)
+        outs.append(run_attention(ssd, c, ws=ws))
+    for o, lse, nd, st in outs:
+        assert st == 0
+        assert np.array_equal(o, outs[0][0]) and np.array_equal(lse, outs[0][1])
     check_case(ssd, c)
 
 

@@ -184,3 +184,22 @@ def test_config5_late_step_every_row(ssd, B):
     _, r = run_case(c)
     check_decisions(c, r)
     check_attention(c, r, seqs=[0, B - 1])
+
+
+@pytest.mark.parametrize("active", [1, 2])
+def test_config5_tail_step_every_row(ssd, active):
+    """The end of the 8-sequence replay: `active` sequences still have drafts
+    (caches of about 4100 to 4350 keys), the other grids are complete (cache
+    = prefix + 4096, empty frontier: no rows, no attention items, ranked last
+    in the attention's dealing).  Every row's decisions and the attention of
+    every head of the active sequences against the oracle."""
+    B = 8
+    rng = np.random.default_rng(70 + active)
+    cl = np.full(B, 256 + 64 * 64)
+    act = np.sort(rng.choice(B, size=active, replace=False))
+    cl[act] = 256 + 64 * rng.integers(59, 63, size=active) + rng.integers(0, 64, size=active)
+    c = synth.config5(B=B, cache_len=cl.astype(np.int32), seed=71 + active)
+    _, r = run_case(c)
+    assert (r["n_drafts"][np.setdiff1d(np.arange(B), act)] == 0).all()
+    check_decisions(c, r)
+    check_attention(c, r, seqs=[int(b) for b in act])
