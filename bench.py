@@ -1049,18 +1049,12 @@ def main():
                                  c.D_max, c.L_max, s.q, s.k, s.v, 0.0, s.o, None, ws, wsb,
                                  s.status, cs)
 
-    lm_wsb = ssd.ssd_lmhead_accept_workspace(c.B * c.D_max, c.V) if c.hidden else 0
-    lm_ws = torch.empty(max(lm_wsb, 256), dtype=torch.uint8, device=dev)
-
     def acc_call(i, cs):
+        # the step's acceptance part as the step launches it (decisions, the
+        # committed draws, counts; the fused path: frontier, lm_head, counts)
         s = steps_obj[i & 1]
         s.set_rng(seed, i)
-        if c.hidden:
-            ssd.ssd_lmhead_accept(c.B * c.D_max, c.V, c.hidden, s.h_tgt, s.h_drf, s.w_tgt,
-                                  s.w_drf, None, 1.0, s.rng, s.out_tok, s.accepted, s.ratio, None,
-                                  lm_ws, lm_wsb, s.status, cs)
-        else:  # the step's acceptance part as the step launches it (decisions, draws, counts)
-            ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes, cs)
+        ssd.ssd_verify_accept(s.args, s.out, s.workspace, s.ws_bytes, cs)
 
     def kernel_ms(call):
         gr = torch.cuda.CUDAGraph()
@@ -1081,8 +1075,8 @@ def main():
     attn_ms = kernel_ms(attn_call)
     acc_ms = kernel_ms(acc_call)
     hbm_peak, peak_kind = measured_peaks()
-    # the standalone fused call processes every row of the padded batch; the
-    # logits path's acceptance part reads the frontier's rows (and bonus rows)
+    # the fused lm_head processes every row of the padded batch; the logits
+    # path's acceptance part reads the frontier's rows (and bonus rows)
     if c.hidden:
         acc_bytes_all = 2 * c.hidden * c.V * 2 + c.B * c.D_max * (2 * c.hidden * 2 + 9)
     else:

@@ -325,9 +325,10 @@ ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
  *   other arguments as ssd_accept(); lse may be NULL.
  *   workspace     dev, >= ssd_lmhead_accept_workspace(rows, V) bytes
  * Supported: 1 <= rows <= 256, K % 64 == 0, V % 128 == 0, V / 128 no more
- * than the co-resident CTAs of the device.  The kernel's CTAs meet at two
+ * than the co-resident CTAs of the device.  The kernel's CTAs meet at three
  * bounded grid barriers; a barrier that waits too long records
- * SSD_ERR_TIMEOUT and the kernel returns without writing its outputs.
+ * SSD_ERR_TIMEOUT and the kernel returns without writing its outputs (the
+ * first barrier; a later one leaves the decisions written before it).
  * ------------------------------------------------------------------------- */
 size_t ssd_lmhead_accept_workspace(int32_t rows, int32_t V);
 ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_tgt,
@@ -365,8 +366,10 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * rejected rows (never committed: the drafts after the first rejection are
  * discarded) and of an uncommitted bonus row is -1; accepted and ratio are
  * written for every row.  The committed token is the one the full draw
- * (ssd_accept_strategy) gives for that row, bit for bit.  The other commit
- * rules, ref_rows, strategies (A) and (B) and the fused path draw every row.
+ * (ssd_accept_strategy) gives for that row, bit for bit.  The fused path
+ * with SSD_COMMIT_PREFIX draws likewise only each sequence's first rejected
+ * draft.  The other commit rules, ref_rows and strategies (A) and (B) draw
+ * every row.
  * Streams: logits path — the acceptance pass computes the frontier itself
  * (and writes n_drafts and draft_pos) and the attention computes the same
  * frontier from cache_len.  With at least 2 x (SM count) rows and either

@@ -585,6 +585,9 @@ cudaError_t launch_fused_accept(const ssd_verify_args* x, const ssd_verify_out* 
   h.status = y->status;
   h.n_drafts = y->n_drafts;
   h.D_max = x->D_max;
+  // a one-round prefix commit keeps one drawn token per sequence: draw only it
+  h.lazy = x->commit == SSD_COMMIT_PREFIX ? 1 : 0;
+  h.counters_zeroed = 1;  // by the frontier kernel before it
   cudaError_t e = launch_lmhead(h, ws, ws_bytes, stream);
   if (e != cudaSuccess) return e;
   return launch_counts(x->grid, x->commit, x->B, x->D_max, x->cache_len, y->n_drafts, y->accepted,
@@ -704,7 +707,7 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   // acceptance and the counts on a side stream, joined back into `stream`.
   if (side_stream(&side) != cudaSuccess) return SSD_ERR_CUDA;
   e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts, y->draft_pos, y->status,
-                      stream);
+                      stream, lmhead_counters(ws + attn_ws), kLmheadCounters);
   if (e != cudaSuccess) return SSD_ERR_CUDA;
   if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
       cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
@@ -735,7 +738,8 @@ ssd_status ssd_verify_accept(const ssd_verify_args* x, const ssd_verify_out* y, 
   cudaStream_t st = (cudaStream_t)stream;
   if (x->tgt_logits == nullptr) {
     cudaError_t e = launch_frontier(x->grid, x->B, x->cache_len, x->D_max, y->n_drafts,
-                                    y->draft_pos, y->status, st);
+                                    y->draft_pos, y->status, st, lmhead_counters(workspace),
+                                    kLmheadCounters);
     if (e != cudaSuccess) return SSD_ERR_CUDA;
     return from_cuda(launch_fused_accept(x, y, workspace, workspace_bytes, st));
   }

@@ -21,11 +21,15 @@
 
 namespace ssd {
 
-// One block per sequence.  Writes n_drafts[b] and draft_pos[b][0..D_max).
+// One block per sequence.  Writes n_drafts[b] and draft_pos[b][0..D_max);
+// block 0 also clears `zero` [n_zero] (the grid-barrier words of the kernel
+// that follows, which then needs no memset of its own).
 __global__ void frontier_kernel(ssd_grid g, const int32_t* __restrict__ cache_len, int32_t D_max,
                                 int32_t* __restrict__ n_drafts, int32_t* __restrict__ draft_pos,
-                                int32_t* status) {
+                                int32_t* status, unsigned int* zero, int32_t n_zero) {
   const int32_t b = blockIdx.x;
+  if (b == 0)
+    for (int32_t i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0u;
   const int32_t n_c = cache_len[b] - g.prefix_len;
   const int32_t n = frontier_drafts(g, cache_len[b], D_max);
   if (threadIdx.x == 0) {
@@ -110,9 +114,10 @@ cudaError_t launch_commit(const ssd_grid& g, int32_t commit, int32_t B, int32_t 
 
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
-                            cudaStream_t stream) {
+                            cudaStream_t stream, unsigned int* zero, int32_t n_zero) {
   if (B == 0) return cudaSuccess;
-  frontier_kernel<<<B, 128, 0, stream>>>(g, cache_len, D_max, n_drafts, draft_pos, status);
+  frontier_kernel<<<B, 128, 0, stream>>>(g, cache_len, D_max, n_drafts, draft_pos, status, zero,
+                                         zero != nullptr ? n_zero : 0);
   return cudaGetLastError();
 }
 

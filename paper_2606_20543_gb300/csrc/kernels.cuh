@@ -49,9 +49,12 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
 }
 
 // ---- frontier.cu
+// zero (nullable) [n_zero]: words cleared on the way (the fused lm_head's
+// grid-barrier counters, lmhead_counters(), for a launch after this one).
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
-                            cudaStream_t stream);
+                            cudaStream_t stream, unsigned int* zero = nullptr,
+                            int32_t n_zero = 0);
 // pdl: launched as a programmatic dependent of the kernel before it on the
 // stream (it may start while that kernel runs, needs none of its results and
 // waits for it before exiting, so stream order is kept).
@@ -309,8 +312,17 @@ struct LmHeadArgs {
   int32_t* status;
   const int32_t* n_drafts;  // nullable, as AcceptArgs
   int32_t D_max;
+  // With n_drafts: draw only the first rejected row of each sequence (the
+  // token a one-round prefix commit keeps); other rejected rows get -1.
+  int32_t lazy = 0;
+  // The barrier words at the start of the workspace were cleared by a kernel
+  // earlier on the stream (launch_frontier's `zero`): no memset.
+  int32_t counters_zeroed = 0;
 };
 size_t lmhead_workspace(int32_t rows, int32_t V);
+// The grid-barrier words at the start of a workspace and their count.
+inline unsigned int* lmhead_counters(void* ws) { return static_cast<unsigned int*>(ws); }
+constexpr int32_t kLmheadCounters = 2;
 ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K);
 cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream);
 

@@ -19,10 +19,14 @@
 //    (target, draft), tcgen05.commit releasing each stage;
 //  * epilogue: tcgen05.ld of each row's tile, per-tile softmax partials to a
 //    small workspace, a bounded grid barrier (the launch is cooperative, so
-//    every CTA is resident), a warp-parallel combine of the partials in a
-//    fixed order (identical in every CTA), the decision, per-tile residual
-//    masses, a second barrier, and the CTA holding the CDF crossing scans
-//    its row tile sequentially.  Logits stay in TMEM throughout.
+//    every CTA is resident), a warp-parallel combine of each row's partials
+//    in a fixed order by one CTA (row r by CTA r mod the grid), which takes
+//    the decision and publishes the row's normalisers; a second barrier; the
+//    rows to draw (every rejected row, or, inside a one-round prefix-commit
+//    step, only each sequence's first rejection: the one token the commit
+//    keeps), their per-tile residual masses, a third barrier, and the CTA
+//    holding the CDF crossing scans its row tile sequentially.  Logits stay
+//    in TMEM throughout.
 #include "kernels.cuh"
 
 namespace ssd {
@@ -113,10 +117,16 @@ struct LmSmemRow {  // per-row results of the decision, broadcast inside the CTA
   int32_t pad;
 };
 
+struct LmRowRec {   // one row's combine, for every CTA after the second barrier
+  float Cp, Cq, u_res;
+  int32_t state;    // 1: valid and rejected (a draw candidate), else 0
+};
+
 struct LmLaunch {
   int32_t ncta, mt, stages;
   LmPartial* part;      // [rows][ncta]
   float* mass;          // [rows][ncta]
+  LmRowRec* rec;        // [rows] each row's decision, written by the CTA that combined it
   unsigned int* barrier;
   uint32_t max_polls;   // limit of every bounded wait of the kernel
   uint32_t shortfall;   // extra arrivals each grid barrier waits for (0; > 0 in tests)
@@ -301,100 +311,123 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
   }
   ok = grid_barrier(L.barrier, (unsigned)L.ncta + L.shortfall, a.status, flag, L.max_polls) && ok;
 
-  // ---- epilogue 2: combine the partials of each row (warp per row, lane l
-  // merging tiles l, l + 32, ... in order, then a xor tree: the same arithmetic
-  // in every CTA), decide, and on rejection prepare the draw.  All loads of a
-  // row are issued before any merge.
-  for (int m = 0; m < mt && ok; ++m) {
-    for (int rl = warp; rl < kBM; rl += kCombWarps) {
-      const int32_t row = m * kBM + rl;
-      LmSmemRow& ri = rowinfo[m * kBM + rl];
-      if (row >= rows) {
-        if (lane == 0) ri.state = 0;
-        continue;
-      }
-      bool pad = false;
-      if (a.n_drafts != nullptr) {
-        const int32_t b = row / a.D_max, j = row - b * a.D_max;
-        pad = j >= a.n_drafts[b];
-      }
-      if (pad) {
-        if (lane == 0) {
-          ri.state = 0;
-          if (cta == 0) {
-            a.out_tok[row] = -1;
-            a.accepted[row] = 0;
-            if (a.ratio) a.ratio[row] = 0.f;
-            if (a.lse) { a.lse[2 * row] = 0.f; a.lse[2 * row + 1] = 0.f; }
-          }
-        }
-        continue;
-      }
-      const float4* prow = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta);
-      float4 q0[kMaxTilesPerLane], q1[kMaxTilesPerLane];
-#pragma unroll
-      for (int j = 0; j < kMaxTilesPerLane; ++j) {
-        const int k = lane + 32 * j;
-        if (k < L.ncta) {
-          q0[j] = prow[2 * k];
-          q1[j] = prow[2 * k + 1];
-        }
-      }
-      float Mp = -INFINITY, Sp = 0.f, Mq = -INFINITY, Sq = 0.f, xq = -INFINITY, xp = 0.f;
-      int32_t t = 0x7fffffff;
-#pragma unroll
-      for (int j = 0; j < kMaxTilesPerLane; ++j) {
-        if (lane + 32 * j < L.ncta) {
-          merge_ms(Mp, Sp, q0[j].x, q0[j].y, c);
-          merge_ms(Mq, Sq, q0[j].z, q0[j].w, c);
-          const int32_t ck = __float_as_int(q1[j].z);
-          if (ck >= 0 && better(q1[j].x, ck, xq, t)) { xq = q1[j].x; xp = q1[j].y; t = ck; }
-        }
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        merge_ms(Mp, Sp, __shfl_xor_sync(0xffffffffu, Mp, o), __shfl_xor_sync(0xffffffffu, Sp, o), c);
-        merge_ms(Mq, Sq, __shfl_xor_sync(0xffffffffu, Mq, o), __shfl_xor_sync(0xffffffffu, Sq, o), c);
-        const float oq = __shfl_xor_sync(0xffffffffu, xq, o);
-        const float op = __shfl_xor_sync(0xffffffffu, xp, o);
-        const int32_t ot = __shfl_xor_sync(0xffffffffu, t, o);
-        if (better(oq, ot, xq, t)) { xq = oq; xp = op; t = ot; }
-      }
+  // ---- epilogue 2: combine the partials of each row and decide.  Row r is
+  // combined by CTA r % ncta alone (one warp per row; lane l merges tiles l,
+  // l + 32, ... in order, then a xor tree), which writes its outputs and its
+  // record for the other CTAs.  All loads of a row are issued before any merge.
+  for (int32_t row = cta + L.ncta * warp; row < rows && ok; row += L.ncta * kCombWarps) {
+    bool pad = false;
+    if (a.n_drafts != nullptr) {
+      const int32_t b = row / a.D_max, j = row - b * a.D_max;
+      pad = j >= a.n_drafts[b];
+    }
+    if (pad) {
       if (lane == 0) {
-        const int32_t given = a.draft_tok != nullptr ? a.draft_tok[row] : -1;
-        const bool valid_t = (t >= 0 && t < a.V) && (given < 0 || t == given);
-        float ratio = 0.f;
-        bool acc = false;
-        const float2 u = row_uniforms(a.rng, row);
-        if (valid_t) {
-          const float l2p = (xp - Mp) * c - log2f(Sp);
-          const float l2q = (xq - Mq) * c - log2f(Sq);
-          ratio = exp2f(l2p - l2q);
-          acc = u.x < fminf(ratio, 1.0f);
-        }
-        ri.Cp = Mp * c + log2f(Sp);
-        ri.Cq = Mq * c + log2f(Sq);
-        ri.u_res = u.y;
-        ri.state = (valid_t && !acc) ? 1 : 0;
-        ri.from_p = 0;
-        ri.cstar = -1;
-        if (cta == 0) {
-          if (!valid_t) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
-          a.accepted[row] = acc ? 1 : 0;
-          if (acc) a.out_tok[row] = t;
-          else if (!valid_t) a.out_tok[row] = -1;
-          if (a.ratio) a.ratio[row] = ratio;
-          if (a.lse) {
-            a.lse[2 * row] = Mp / a.temperature + log2f(Sp) * kLn2L;
-            a.lse[2 * row + 1] = Mq / a.temperature + log2f(Sq) * kLn2L;
-          }
-        }
+        L.rec[row].state = 0;
+        a.out_tok[row] = -1;
+        a.accepted[row] = 0;
+        if (a.ratio) a.ratio[row] = 0.f;
+        if (a.lse) { a.lse[2 * row] = 0.f; a.lse[2 * row + 1] = 0.f; }
+      }
+      continue;
+    }
+    const float4* prow = reinterpret_cast<const float4*>(L.part + (int64_t)row * L.ncta);
+    float4 q0[kMaxTilesPerLane], q1[kMaxTilesPerLane];
+#pragma unroll
+    for (int j = 0; j < kMaxTilesPerLane; ++j) {
+      const int k = lane + 32 * j;
+      if (k < L.ncta) {
+        q0[j] = __ldcg(prow + 2 * k);
+        q1[j] = __ldcg(prow + 2 * k + 1);
+      }
+    }
+    float Mp = -INFINITY, Sp = 0.f, Mq = -INFINITY, Sq = 0.f, xq = -INFINITY, xp = 0.f;
+    int32_t t = 0x7fffffff;
+#pragma unroll
+    for (int j = 0; j < kMaxTilesPerLane; ++j) {
+      if (lane + 32 * j < L.ncta) {
+        merge_ms(Mp, Sp, q0[j].x, q0[j].y, c);
+        merge_ms(Mq, Sq, q0[j].z, q0[j].w, c);
+        const int32_t ck = __float_as_int(q1[j].z);
+        if (ck >= 0 && better(q1[j].x, ck, xq, t)) { xq = q1[j].x; xp = q1[j].y; t = ck; }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      merge_ms(Mp, Sp, __shfl_xor_sync(0xffffffffu, Mp, o), __shfl_xor_sync(0xffffffffu, Sp, o), c);
+      merge_ms(Mq, Sq, __shfl_xor_sync(0xffffffffu, Mq, o), __shfl_xor_sync(0xffffffffu, Sq, o), c);
+      const float oq = __shfl_xor_sync(0xffffffffu, xq, o);
+      const float op = __shfl_xor_sync(0xffffffffu, xp, o);
+      const int32_t ot = __shfl_xor_sync(0xffffffffu, t, o);
+      if (better(oq, ot, xq, t)) { xq = oq; xp = op; t = ot; }
+    }
+    if (lane == 0) {
+      const int32_t given = a.draft_tok != nullptr ? a.draft_tok[row] : -1;
+      const bool valid_t = (t >= 0 && t < a.V) && (given < 0 || t == given);
+      float ratio = 0.f;
+      bool acc = false;
+      const float2 u = row_uniforms(a.rng, row);
+      if (valid_t) {
+        const float l2p = (xp - Mp) * c - log2f(Sp);
+        const float l2q = (xq - Mq) * c - log2f(Sq);
+        ratio = exp2f(l2p - l2q);
+        acc = u.x < fminf(ratio, 1.0f);
+      }
+      LmRowRec rr;
+      rr.Cp = Mp * c + log2f(Sp);
+      rr.Cq = Mq * c + log2f(Sq);
+      rr.u_res = u.y;
+      rr.state = (valid_t && !acc) ? 1 : 0;
+      L.rec[row] = rr;
+      if (!valid_t) record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
+      a.accepted[row] = acc ? 1 : 0;
+      if (acc) a.out_tok[row] = t;
+      else a.out_tok[row] = -1;  // a drawn row's token is written in epilogue 5
+      if (a.ratio) a.ratio[row] = ratio;
+      if (a.lse) {
+        a.lse[2 * row] = Mp / a.temperature + log2f(Sp) * kLn2L;
+        a.lse[2 * row + 1] = Mq / a.temperature + log2f(Sq) * kLn2L;
+      }
+    }
+  }
+  ok = grid_barrier(L.barrier, 2u * ((unsigned)L.ncta + L.shortfall), a.status, flag,
+                    L.max_polls) && ok;
+
+  // ---- the rows to draw, in every CTA: every valid rejected row, or (lazy)
+  // the first rejected row of each sequence among its drafts
+  int32_t* first = reinterpret_cast<int32_t*>(rowinfo + mt * kBM);  // [rows / D_max]
+  const bool lazy = a.lazy != 0 && a.n_drafts != nullptr;
+  const int32_t ngroups = lazy ? rows / a.D_max : 0;
+  for (int32_t g = tid; g < ngroups; g += kThreadsL) first[g] = 0x7fffffff;
+  __syncthreads();
+  if (lazy && ok) {
+    for (int32_t row = tid; row < rows; row += kThreadsL) {
+      const int32_t b = row / a.D_max, j = row - b * a.D_max;
+      if (j < a.n_drafts[b] && __ldcg(a.accepted + row) == 0) atomicMin(&first[b], j);
+    }
+  }
+  __syncthreads();
+  for (int32_t r = tid; r < mt * kBM; r += kThreadsL) {
+    LmSmemRow& ri = rowinfo[r];
+    ri.state = 0;
+    ri.from_p = 0;
+    ri.cstar = -1;
+    if (r < rows && ok) {
+      // the record of another CTA, read from L2
+      const float4 rv = __ldcg(reinterpret_cast<const float4*>(L.rec + r));
+      const bool pick = __float_as_int(rv.w) == 1 &&
+                        (!lazy || r - (r / a.D_max) * a.D_max == first[r / a.D_max]);
+      if (pick) {
+        ri.Cp = rv.x;
+        ri.Cq = rv.y;
+        ri.u_res = rv.z;
+        ri.state = 1;
       }
     }
   }
   __syncthreads();
 
-  // ---- epilogue 3: residual mass of this tile for every rejected row
+  // ---- epilogue 3: residual mass of this tile for every row to draw
   // (sequential over the tile in vocabulary order; TMEM warps)
   for (int m = 0; m < mt && ok && warp < kTmemWarps; ++m) {
     const int32_t row = m * kBM + tid;
@@ -405,6 +438,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     // every lane of the warp takes part in tcgen05.ld; rows that do not draw
     // simply discard the values
     const bool draw = row < rows && ri.state == 1;
+    if (!__any_sync(0xffffffffu, draw)) continue;  // warp-uniform: no row of this warp draws
 #pragma unroll 1
     for (int ch = 0; ch < kBN / 32; ++ch) {
       tmem_ld32(tp + ch * 32, v);
@@ -417,7 +451,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     }
     if (draw) L.mass[(int64_t)row * L.ncta + cta] = mass;
   }
-  ok = grid_barrier(L.barrier, 2u * ((unsigned)L.ncta + L.shortfall), a.status, flag,
+  ok = grid_barrier(L.barrier, 3u * ((unsigned)L.ncta + L.shortfall), a.status, flag,
                     L.max_polls) && ok;
 
   // ---- epilogue 4: locate the tile holding u_res * Z (warp per row; lane l
@@ -497,6 +531,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmHt, const __grid_cons
     const int32_t row = m * kBM + tid;
     const LmSmemRow& ri = rowinfo[m * kBM + tid];
     const bool mine = row < rows && ri.state == 1 && ri.cstar == cta;
+    if (!__any_sync(0xffffffffu, mine)) continue;  // warp-uniform
     const bool from_p = ri.from_p != 0;
     const uint32_t tp = tmem + lane_off + m * 2 * kBN, tq = tp + kBN;
     float v[32], w[32];
@@ -565,18 +600,24 @@ size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 int row_tiles(int32_t rows) { return (rows + kBM - 1) / kBM; }
 
 size_t smem_bytes(int mt, int stages) {
+  // + the first rejected draft of each sequence (at most one per row)
   return 1024 + (size_t)stages * (2 * mt * kTileA + 2 * kTileB) + (2 * stages + 1) * 8 + 16 +
-         (size_t)mt * kBM * sizeof(LmSmemRow);
+         (size_t)mt * kBM * sizeof(LmSmemRow) + (size_t)mt * kBM * sizeof(int32_t);
 }
 
-int stages_for(int mt) { return mt == 1 ? 3 : 2; }
+// As many stages as the shared memory holds, at most 8.
+int stages_for(int mt) {
+  int s = 8;
+  while (s > 2 && smem_bytes(mt, s) > 232448) --s;
+  return s;
+}
 
 }  // namespace
 
 size_t lmhead_workspace(int32_t rows, int32_t V) {
   const size_t ncta = (size_t)(V + kBN - 1) / kBN;
   return al256(2 * sizeof(unsigned int)) + al256((size_t)rows * ncta * sizeof(LmPartial)) +
-         al256((size_t)rows * ncta * sizeof(float));
+         al256((size_t)rows * ncta * sizeof(float)) + al256((size_t)rows * sizeof(LmRowRec));
 }
 
 ssd_status lmhead_check(int32_t rows, int32_t V, int32_t K) {
@@ -613,6 +654,8 @@ cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaSt
   L.part = reinterpret_cast<LmPartial*>(w);
   w += al256((size_t)a.rows * L.ncta * sizeof(LmPartial));
   L.mass = reinterpret_cast<float*>(w);
+  w += al256((size_t)a.rows * L.ncta * sizeof(float));
+  L.rec = reinterpret_cast<LmRowRec*>(w);
   CUtensorMap ht, hd, wt, wd;
   // hidden [rows][K]: boxes of 128 rows (rows past `rows` read as zero);
   // weights [K][V]: boxes of 64 K-rows x 128 vocabulary entries (3D view)
@@ -621,8 +664,11 @@ cudaError_t launch_lmhead(const LmHeadArgs& a, void* ws, size_t ws_bytes, cudaSt
       !make_weight_map(&wt, a.w_tgt, (uint64_t)a.V, (uint64_t)a.K) ||
       !make_weight_map(&wd, a.w_drf, (uint64_t)a.V, (uint64_t)a.K))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaMemsetAsync(L.barrier, 0, 2 * sizeof(unsigned int), stream);
-  if (e != cudaSuccess) return e;
+  cudaError_t e = cudaSuccess;
+  if (!a.counters_zeroed) {
+    e = cudaMemsetAsync(L.barrier, 0, kLmheadCounters * sizeof(unsigned int), stream);
+    if (e != cudaSuccess) return e;
+  }
   const size_t smem = smem_bytes(mt, L.stages);
   e = cudaFuncSetAttribute(lmhead_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem);

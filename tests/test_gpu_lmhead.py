@@ -9,7 +9,8 @@ import torch
 import synth
 from oracle import lmhead as olm
 from oracle import step as ostep
-from tests.helpers import FUSED_PROB_TOL, bf16_to_f64, compare_decisions, max_excused_rows
+from tests.helpers import (FUSED_PROB_TOL, bf16_to_f64, committed_draws, compare_decisions,
+                           max_excused_rows)
 
 pytestmark = pytest.mark.gpu
 
@@ -59,6 +60,7 @@ def make_inputs(rows, K, V, seed, w_std=0.02):
     (48, 512, 2048, 0.05, 1),     # 16 tiles, ragged ring wrap-around (8 K blocks, 3 stages)
     (200, 256, 1024, 0.05, 2),    # two row tiles (rows 128..199 in the second)
     (48, 4096, 16384, 0.02, 3),   # the fused-head workload: 128 tiles, 64 K blocks
+    (256, 4096, 16384, 0.02, 4),  # the most rows: two full row tiles, two rows per CTA's combine
 ])
 def test_fused_lmhead_matches_oracle(ssd, rows, K, V, w_std, seed):
     ht, hd, wt, wd, u = make_inputs(rows, K, V, seed, w_std)
@@ -90,11 +92,14 @@ def test_fused_identical_heads_accept_everything(ssd):
     assert st == 0 and acc.all() and np.all(ratio == 1.0)
 
 
-def test_verify_step_fused_path(ssd):
-    """ssd_verify_step with hidden states + lm_head weights (config-4 shapes,
-    two sequences: a full 48-draft frontier and a 24-draft last row)."""
+@pytest.mark.parametrize("points", [[120, 672], [120, 130, 140, 150, 160]])
+def test_verify_step_fused_path(ssd, points):
+    """ssd_verify_step with hidden states + lm_head weights (config-4 shapes:
+    a full 48-draft frontier and a 24-draft last row; five sequences, 240
+    rows in two row tiles).  The prefix commit draws only each sequence's
+    first rejected draft."""
     from paper_2606_20543_gb300.step import VerifyStep
-    c = synth.config4(points=[120, 672])
+    c = synth.config4(points=points)
     s = VerifyStep(c.grid_h, c.grid_w, c.prefix_len, c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max, c.V,
                    hidden=c.hidden)
     s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v, h_tgt=c.h_tgt, h_drf=c.h_drf,
@@ -107,9 +112,11 @@ def test_verify_step_fused_path(ssd):
     lq = olm.logits(bf16_to_f64(c.h_drf), bf16_to_f64(c.w_drf))
     ref = ostep.accept_step(c.grid_h, c.grid_w, c.prefix_len, c.k_v, c.cache_len, c.D_max, lp, lq,
                             c.uniforms)
-    assert np.array_equal(r["n_drafts"], ref["n_drafts"]) and list(r["n_drafts"]) == [48, 24]
+    assert np.array_equal(r["n_drafts"], ref["n_drafts"])
     rows = ref["decisions"]["rows"]
-    ties = compare_decisions(ref["decisions"], r["out_tok"][rows], r["accepted"][rows],
+    # a prefix-commit step draws only each sequence's first rejected draft
+    dec = committed_draws(ref["decisions"], r["accepted"][rows], c.D_max)
+    ties = compare_decisions(dec, r["out_tok"][rows], r["accepted"][rows],
                              r["ratio"][rows], what="fused step", tol=FUSED_PROB_TOL)
     pad = np.setdiff1d(np.arange(c.B * c.D_max), rows)
     assert np.all(r["out_tok"][pad] == -1) and np.all(r["accepted"][pad] == 0)
