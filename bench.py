@@ -206,14 +206,13 @@ class ClockSampler:
 # is the one that was captured: (source file, sha256 prefix, bytes, rows the
 # captured launch processed or None for a launch of the bench's own shape).
 MEASURED_TRAFFIC = {
-    # acceptance part of a step: accept_kernel (one pass) + resolve_kernel (committed draws)
-    ("accept", 2): ("accept.cu", "3419b86a0a387073", 147920128 + 249728 + 3382272, None),
-    ("attention", 2): ("attention_tc.cu", "f04b60df37aa4d9c", 102185472 + 67072, None),
-    ("attention", 3): ("attention_tc.cu", "f04b60df37aa4d9c", 53835776 + 3584, None),
-    ("lmhead_accept", 4): ("lmhead.cu", "b3d943c2cf5f717f", 269338368 + 2763776, None),
+    # (kernel, config): (source, sha256 prefix of the source the capture ran,
+    # DRAM bytes read + written in one launch, rows of that launch or None)
+    ("attention", 2): ("attention_tc.cu", "cf1328b23a34be8d", 102179584 + 2470656, None),
+    ("lmhead_accept", 4): ("lmhead.cu", "07f252f7b825ad8e", 269314560 + 2795520, None),
     # 8 x 64x64 replay, first step (1024 draft rows): accept_kernel alone; the
     # bench scales it to the rows of the replay states it sums
-    ("accept", 5): ("accept.cu", "5476c5787745e93a", 536944896 + 3043328, 1024),
+    ("accept", 5): ("accept.cu", "f5a51c0947bed819", 536945152 + 3111680, 1024),
 }
 
 
@@ -1094,10 +1093,18 @@ def main():
         peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
             os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
         tpk = peaks.get("bf16_tflops", 1900.0)
+        tpk_s = peaks.get("bf16_tflops_sustained", 1700.0)
         tflops = flops / (acc_ms / 1000.0) / 1e12
+        rows = c.B * c.D_max
         tensor_info = {"kernel": "lmhead_accept", "achieved_tflops": tflops, "peak_tflops": tpk,
-                       "frac": tflops / tpk, "rows": c.B * c.D_max,
-                       "note": "rows padded to 128 per MMA tile; HBM-bound at this row count"}
+                       "frac": tflops / tpk, "peak_tflops_sustained": tpk_s,
+                       "frac_sustained": tflops / tpk_s, "rows": rows,
+                       "peak_kind": "measured" if "bf16_tflops" in peaks else "fallback",
+                       "time": "the step's acceptance part (frontier, fused lm_head, counts)",
+                       "note": ("HBM-bound at this row count (48 flop per weight byte)"
+                                if rows <= 128 else
+                                f"{rows} rows in two 128-row tiles: the most tensor memory holds "
+                                "(2 tiles x 2 heads x 128 columns = 512)")}
 
     # ---------------- end to end: host buffers, copies inside the timed region
     host = {}
@@ -1157,7 +1164,11 @@ def main():
         "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 attention / f32 acceptance",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD_NAMES[a.config], "strategy": a.strategy,
+        "config": {"workload": (WORKLOAD_NAMES[a.config] if not (a.config == 4 and c.B > 1) else
+                                f"fused lm_head, {c.B} sequences x 48 drafts = {c.B * c.D_max} "
+                                "rows per weight pass: 24x24, prefix 120, cache 120, 16x128 MHA, "
+                                "hidden bf16 [rows x 4096], W_t, W_d bf16 [4096 x 16384]"),
+                   "strategy": a.strategy,
                    "verify_rounds": (f"staged b={a.staged[0]}, i={a.staged[1]}" if a.staged
                                      else a.rounds),
                    "stage": (f"horizontal: k_h={a.horizontal} drafts, prefix + bonus token"

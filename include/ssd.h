@@ -85,7 +85,7 @@ typedef struct {
 } ssd_rng;
 
 /* ABI version of this header (increment on any signature change). */
-#define SSD_ABI_VERSION 8
+#define SSD_ABI_VERSION 9
 int32_t ssd_abi_version(void);
 
 /* Human-readable name of a status code (static string). */
@@ -314,6 +314,23 @@ ssd_status ssd_commit_pass(const ssd_grid* grid, int32_t B, const int32_t* cache
  * rounds (k_v = 0).  Requires 2 * W <= D_max. */
 ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
                            const float** ref_rows, ssd_stream_t stream);
+
+/* The tokens one step committed, into each sequence's grid (Sec. 3.3: the
+ * accepted prefix, then the first rejected draft's resampled token, fill the
+ * next raster positions).  For every b, with n_c = cache_len[b] - prefix_len
+ * and adv = next_cache_len[b] - cache_len[b]:
+ *     grid_tok[b][n_c + j] = out_tok[b * D_max + j],  0 <= j < adv.
+ * Call it after a step and before next_cache_len becomes cache_len; with it
+ * the grid, the cache lengths and the step index are the whole state of a
+ * replay (paper_2606_20543_gb300.step.ReplayState dumps and restores them).
+ *   cache_len, next_cache_len  dev int32 [B];  out_tok dev int32 [B * D_max]
+ *   grid_tok   dev int32 [B][hw] (in/out: only the committed slots change)
+ * A sequence whose advance leaves [0, D_max] or the grid records
+ * SSD_ERR_DEVICE_BOUNDS in *status and writes nothing. */
+ssd_status ssd_record_commit(int32_t B, int32_t D_max, int32_t prefix_len, int32_t hw,
+                             const int32_t* cache_len, const int32_t* next_cache_len,
+                             const int32_t* out_tok, int32_t* grid_tok, int32_t* status,
+                             ssd_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * a6. Fused lm_head + acceptance (Sec. 3.3, after Eq. 2: tokens are decoded

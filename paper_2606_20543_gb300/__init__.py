@@ -24,7 +24,7 @@ STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "S
 EXPORTED = ["ssd_abi_version", "ssd_status_string", "ssd_set_wait_limit",
             "ssd_set_barrier_shortfall", "ssd_frontier", "ssd_verify_attention_workspace",
             "ssd_verify_attention", "ssd_verify_attention_noalloc", "ssd_accept", "ssd_accept_strategy",
-            "ssd_accept_round", "ssd_stage_shift", "ssd_commit_pass",
+            "ssd_accept_round", "ssd_stage_shift", "ssd_commit_pass", "ssd_record_commit",
             "ssd_draft_predict_workspace",
             "ssd_draft_predict",
             "ssd_lmhead_accept_workspace", "ssd_lmhead_accept",
@@ -114,6 +114,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                    P, P]),
         "ssd_stage_shift": (I32, [I32, I32, I32, P, P, P]),
         "ssd_commit_pass": (I32, [ctypes.POINTER(Grid), I32, P, I32, I32, P, P, P]),
+        "ssd_record_commit": (I32, [I32, I32, I32, I32, P, P, P, P, P, P]),
         "ssd_draft_predict_workspace": (SZ, [I32, I32, I32, I32]),
         "ssd_draft_predict": (I32, [I32, I32, I32, I32, P, P, P, P, P, P, P, P, F, P, P, P, SZ,
                                     P, P]),
@@ -254,6 +255,14 @@ def ssd_commit_pass(g: Grid, B, cache_len, D_max, commit, next_cache_len, status
 def ssd_stage_shift(B, D_max, W, tok, ref_rows, stream=None) -> None:
     _check("ssd_stage_shift", load().ssd_stage_shift(B, D_max, W, _ptr(tok), _ptr(ref_rows),
                                                      _stream(stream)))
+
+
+def ssd_record_commit(B, D_max, prefix_len, hw, cache_len, next_cache_len, out_tok, grid_tok,
+                      status, stream=None) -> None:
+    _check("ssd_record_commit",
+           load().ssd_record_commit(B, D_max, prefix_len, hw, _ptr(cache_len),
+                                    _ptr(next_cache_len), _ptr(out_tok), _ptr(grid_tok),
+                                    _ptr(status), _stream(stream)))
 
 
 def ssd_draft_predict_workspace(rows, d, m, V) -> int:

@@ -364,6 +364,19 @@ ssd_status ssd_commit_pass(const ssd_grid* grid, int32_t B, const int32_t* cache
                                  (cudaStream_t)stream));
 }
 
+ssd_status ssd_record_commit(int32_t B, int32_t D_max, int32_t prefix_len, int32_t hw,
+                             const int32_t* cache_len, const int32_t* next_cache_len,
+                             const int32_t* out_tok, int32_t* grid_tok, int32_t* status,
+                             ssd_stream_t stream) {
+  if (B < 0 || D_max <= 0 || prefix_len < 0 || hw <= 0) return SSD_ERR_SHAPE;
+  if (B == 0) return SSD_OK;
+  if (cache_len == nullptr || next_cache_len == nullptr || out_tok == nullptr ||
+      grid_tok == nullptr || status == nullptr)
+    return SSD_ERR_INVALID_ARG;
+  return from_cuda(launch_record_commit(B, D_max, prefix_len, hw, cache_len, next_cache_len,
+                                        out_tok, grid_tok, status, (cudaStream_t)stream));
+}
+
 ssd_status ssd_stage_shift(int32_t B, int32_t D_max, int32_t W, int32_t* tok,
                            const float** ref_rows, ssd_stream_t stream) {
   if (B < 0 || D_max <= 0 || W < 0 || 2 * (int64_t)W > D_max) return SSD_ERR_SHAPE;

@@ -112,6 +112,37 @@ cudaError_t launch_commit(const ssd_grid& g, int32_t commit, int32_t B, int32_t 
   return cudaGetLastError();
 }
 
+// The committed tokens of one step into each sequence's grid (Sec. 3.3: the
+// accepted prefix and the first rejected draft's resampled token take the
+// next raster positions).  One block per sequence: the step advanced the cache
+// from cache_len[b] to next_cache_len[b], i.e. tokens out_tok[b][0 .. adv) at
+// grid positions n_c .. n_c + adv.
+__global__ void record_commit_kernel(int32_t D_max, int32_t prefix_len, int32_t hw,
+                                     const int32_t* __restrict__ cache_len,
+                                     const int32_t* __restrict__ next_cache_len,
+                                     const int32_t* __restrict__ out_tok,
+                                     int32_t* __restrict__ grid_tok, int32_t* status) {
+  const int32_t b = blockIdx.x;
+  const int32_t n_c = cache_len[b] - prefix_len;
+  const int32_t adv = next_cache_len[b] - cache_len[b];
+  if (n_c < 0 || adv < 0 || adv > D_max || n_c + adv > hw) {
+    if (threadIdx.x == 0) record_status(status, SSD_ERR_DEVICE_BOUNDS);
+    return;
+  }
+  for (int32_t j = threadIdx.x; j < adv; j += blockDim.x)
+    grid_tok[(int64_t)b * hw + n_c + j] = out_tok[(int64_t)b * D_max + j];
+}
+
+cudaError_t launch_record_commit(int32_t B, int32_t D_max, int32_t prefix_len, int32_t hw,
+                                 const int32_t* cache_len, const int32_t* next_cache_len,
+                                 const int32_t* out_tok, int32_t* grid_tok, int32_t* status,
+                                 cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  record_commit_kernel<<<B, 128, 0, stream>>>(D_max, prefix_len, hw, cache_len, next_cache_len,
+                                              out_tok, grid_tok, status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,
                             int32_t* n_drafts, int32_t* draft_pos, int32_t* status,
                             cudaStream_t stream, unsigned int* zero, int32_t n_zero) {

@@ -49,6 +49,10 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
 }
 
 // ---- frontier.cu
+cudaError_t launch_record_commit(int32_t B, int32_t D_max, int32_t prefix_len, int32_t hw,
+                                 const int32_t* cache_len, const int32_t* next_cache_len,
+                                 const int32_t* out_tok, int32_t* grid_tok, int32_t* status,
+                                 cudaStream_t stream);
 // zero (nullable) [n_zero]: words cleared on the way (the fused lm_head's
 // grid-barrier counters, lmhead_counters(), for a launch after this one).
 cudaError_t launch_frontier(const ssd_grid& g, int32_t B, const int32_t* cache_len, int32_t D_max,

@@ -11,7 +11,7 @@ import numpy as np
 import torch
 
 from . import (COMMITS, STRATEGIES, Grid, Rng, VerifyArgs, VerifyOut, grid as make_grid,
-               row_addresses, ssd_commit_pass, ssd_frontier, ssd_stage_shift,
+               row_addresses, ssd_commit_pass, ssd_frontier, ssd_record_commit, ssd_stage_shift,
                ssd_verify_attention, ssd_verify_attention_workspace, ssd_verify_step,
                ssd_verify_step_workspace)
 
@@ -27,6 +27,28 @@ def _as_torch(x, dtype):
     if dtype == torch.bfloat16:
         return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
     return torch.from_numpy(x)
+
+
+class ReplayState:
+    """The state of a replay of one batch between two steps: the index of the
+    next step (its Philox counter offset), the seed, every sequence's cache
+    length and its committed grid tokens (raster order, -1 where nothing is
+    committed yet).  With the step's inputs a function of the step index, this
+    is all a replay needs to resume.  ``save`` / ``load`` use one .npz file."""
+
+    def __init__(self, step: int, seed: int, cache_len, grid_tok):
+        self.step, self.seed = int(step), int(seed)
+        self.cache_len = np.asarray(cache_len, np.int32)
+        self.grid_tok = np.asarray(grid_tok, np.int32)
+
+    def save(self, path) -> None:
+        np.savez(path, step=self.step, seed=self.seed, cache_len=self.cache_len,
+                 grid_tok=self.grid_tok)
+
+    @classmethod
+    def load(cls, path) -> "ReplayState":
+        z = np.load(path)
+        return cls(int(z["step"]), int(z["seed"]), z["cache_len"], z["grid_tok"])
 
 
 class VerifyStep:
@@ -163,6 +185,35 @@ class VerifyStep:
     # -------------------------------------------------------------------- run
     def run(self, stream=None) -> None:
         ssd_verify_step(self.args, self.out, self.workspace, self.ws_bytes, stream)
+
+    # ------------------------------------------------------- replay bookkeeping
+    def track_grid(self) -> None:
+        """Allocate the committed-token grid [B, H*W] (-1: not committed) that
+        advance() fills, for a replay that is to be dumped or resumed."""
+        hw = self.g.grid_h * self.g.grid_w
+        self.grid_tok = torch.full((self.B, hw), -1, dtype=torch.int32, device=self.device)
+
+    def advance(self, stream=None) -> None:
+        """After run(): write the step's committed tokens into grid_tok (if
+        tracked) and make next_cache_len the next step's cache length."""
+        if getattr(self, "grid_tok", None) is not None:
+            ssd_record_commit(self.B, self.D_max, self.g.prefix_len, self.grid_tok.shape[1],
+                              self.cache_len, self.next_cache_len, self.out_tok, self.grid_tok,
+                              self.status, stream)
+        self.cache_len.copy_(self.next_cache_len)
+
+    def state(self, step: int, seed: int) -> ReplayState:
+        """The replay's state before step `step` (copied to the host)."""
+        return ReplayState(step, seed, self.cache_len.cpu().numpy(),
+                           self.grid_tok.cpu().numpy())
+
+    def restore(self, st: ReplayState) -> int:
+        """Load a dumped state; returns the step to run next."""
+        if getattr(self, "grid_tok", None) is None:
+            self.track_grid()
+        self.cache_len.copy_(torch.from_numpy(st.cache_len.astype(np.int32)))
+        self.grid_tok.copy_(torch.from_numpy(st.grid_tok.astype(np.int32)))
+        return st.step
 
     def results(self) -> dict:
         names = ["n_drafts", "draft_pos", "out_tok", "accepted", "ratio", "accepted_count",

@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.ssd_abi_version() == 8
+    assert lib.ssd_abi_version() == 9
     for code, name in lib.STATUS_NAMES.items():
         assert lib.ssd_status_string(code) == name
 
@@ -184,3 +184,15 @@ def test_verify_accept_and_step_host_validation(lib):
     fused = args(tgt_logits=None, drf_logits=None, h_tgt=fake, h_drf=fake, w_tgt=fake,
                  w_drf=fake, hidden=4096)
     assert so.ssd_verify_step_launches(ctypes.byref(fused)) == n_logits + 1
+
+
+def test_replay_state_file_roundtrip(tmp_path):
+    import numpy as np
+    from paper_2606_20543_gb300.step import ReplayState
+    g = np.full((2, 16), -1, np.int32)
+    g[0, :5] = [3, 1, 4, 1, 5]
+    st = ReplayState(17, 5, np.array([37, 32], np.int32), g)
+    st.save(tmp_path / "s.npz")
+    back = ReplayState.load(tmp_path / "s.npz")
+    assert (back.step, back.seed) == (17, 5)
+    assert np.array_equal(back.cache_len, st.cache_len) and np.array_equal(back.grid_tok, g)

@@ -74,3 +74,57 @@ def test_reduced_replay_trajectory_matches_oracle(ssd):
         assert len(g_hist) == len(o_hist)
         assert np.array_equal(g_final, o_final)
     assert (g_final == P + H * W).all()
+
+
+def test_replay_resumes_from_a_dumped_state(ssd, tmp_path):
+    """Checkpoint / resume: the replay's state (next step, seed, cache
+    lengths, committed grid tokens) dumped halfway to a file and loaded into
+    a fresh VerifyStep gives the same steps and the same grid as the
+    uninterrupted replay; the grid equals the oracle replay's while no
+    accept near-tie occurs."""
+    from paper_2606_20543_gb300.step import ReplayState, VerifyStep
+    H = W = 16
+    P, B, V, seed = 32, 2, 4096, 23
+    D_max = 2 * W
+    inputs = stream(B, D_max, V, seed)
+    c = synth.make_case("replay", grid_h=H, grid_w=W, prefix_len=P, cache_len=[P] * B, Hq=4,
+                        Hkv=4, d=64, V=V, seed=1, with_logits=False)
+
+    def fresh():
+        s = VerifyStep(H, W, P, B, 4, 4, 64, D_max, c.L_max, V)
+        s.upload(cache_len=c.cache_len, q=c.q, k=c.k, v=c.v)
+        s.track_grid()
+        return s
+
+    def advance(s, t0, t_stop=None):
+        t = t0
+        while t_stop is None or t < t_stop:
+            lp, lq, u = inputs(t)
+            s.upload(tgt_logits=lp, drf_logits=lq, uniforms=u)
+            s.run()
+            if s.n_drafts.sum().item() == 0:
+                return t
+            s.advance()
+            t += 1
+        return t
+
+    full = fresh()
+    T = advance(full, 0)
+    grid_full = full.grid_tok.cpu().numpy()
+    assert (full.cache_len.cpu().numpy() == P + H * W).all() and (grid_full >= 0).all()
+
+    half = fresh()
+    advance(half, 0, T // 2)
+    path = tmp_path / "replay_state.npz"
+    half.state(T // 2, seed).save(path)
+    del half
+    resumed = fresh()
+    t0 = resumed.restore(ReplayState.load(path))
+    assert t0 == T // 2
+    assert advance(resumed, t0) == T
+    assert np.array_equal(resumed.grid_tok.cpu().numpy(), grid_full)
+    assert full.status.item() == 0 and resumed.status.item() == 0
+
+    o_hist, o_grid, _ = ostep.replay(H, W, P, 1, B, D_max, inputs)
+    if not any(h["accept_ties"] for h in o_hist):
+        assert np.array_equal(grid_full, o_grid)
