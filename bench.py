@@ -492,9 +492,10 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
     ms = max_over_ranks(statistics.median(per), world, torch, dev)
     total_ms = max_over_ranks(sum(per), world, torch, dev)
 
-    # ---------------- per-kernel durations at three replay states (the first
-    # step, the middle and near the end): each entry point captured as a graph
-    # of back-to-back launches, timed with events on the launching stream
+    # ---------------- per-kernel durations at eight replay states spread evenly
+    # over the passes (the first step to near the end): each entry point
+    # captured as a graph of back-to-back launches, timed with events on the
+    # launching stream
     kk = 20
     wsb = ssd.ssd_verify_attention_workspace(c.B, c.Hq, c.Hkv, c.d, c.D_max, c.L_max)
     ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
@@ -524,7 +525,8 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
                                  c.D_max, c.L_max, s.q, s.k, s.v, 0.0, s.o, None, ws, wsb,
                                  s.status, cs)
 
-    probe = [states[0], states[len(states) // 2], states[-1]]
+    n_probe = min(8, len(states))
+    probe = [states[round(i * (len(states) - 1) / max(1, n_probe - 1))] for i in range(n_probe)]
     kern = {"attention": [0, 0.0], "accept": [0, 0.0]}
     per_state = []
     for st in probe:
@@ -638,8 +640,8 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
                                      "by the rows of the summed states (the committed draws' "
                                      "resolve kernel not included)",
                      "peak_kind": peak_kind,
-                     "state": "bytes and launch times summed over three replay states "
-                              f"(steps {[st['t'] for st in probe]})",
+                     "state": f"bytes and launch times summed over {len(probe)} replay states "
+                              f"spread evenly over the passes (steps {[st['t'] for st in probe]})",
                      "kernels": {k: {"bytes": b, "ms": m, "gbs": b / (m / 1000.0) / 1e9}
                                  for k, (b, m) in kern.items()},
                      "states": per_state},
