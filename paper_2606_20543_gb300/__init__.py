@@ -15,6 +15,7 @@ from typing import Optional
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libssd.so")
+DEBUG_LIB_PATH = os.path.join(HERE, "libssd_debug.so")
 
 SSD_OK = 0
 STATUS_NAMES = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_SHAPE", 3: "SSD_ERR_UNSUPPORTED",
@@ -86,11 +87,15 @@ class VerifyOut(ctypes.Structure):
 _LIB: Optional[ctypes.CDLL] = None
 
 
-def load(path: str = LIB_PATH) -> ctypes.CDLL:
-    """Load libssd.so (built by ``paper_2606_20543_gb300.build``); raise if absent."""
+def load(path: Optional[str] = None) -> ctypes.CDLL:
+    """Load libssd.so (built by ``paper_2606_20543_gb300.build``); raise if
+    absent.  With SSD_LIBRARY=debug in the environment the default is the
+    bounds-checking build libssd_debug.so (``build --debug-bounds``)."""
     global _LIB
     if _LIB is not None:
         return _LIB
+    if path is None:
+        path = DEBUG_LIB_PATH if os.environ.get("SSD_LIBRARY") == "debug" else LIB_PATH
     if not os.path.exists(path):
         raise RuntimeError(f"libssd.so not built ({path} missing): run "
                            "`python -m paper_2606_20543_gb300.build` (needs nvcc)")

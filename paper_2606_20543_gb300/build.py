@@ -1,6 +1,9 @@
 """Build libssd.so in-tree: every .cu under csrc/ compiled for sm_103a in
 parallel with nvcc, linked with the static CUDA runtime (the library then
 needs only the driver at run time).  Usage: python -m paper_2606_20543_gb300.build
+[--force] [-v] [--debug-bounds]; --debug-bounds builds libssd_debug.so with
+SSD_DEBUG_BOUNDS=1 (the kernels' index checks, recorded in the status word),
+which the binding loads when SSD_LIBRARY=debug is set.
 """
 from __future__ import annotations
 
@@ -33,32 +36,41 @@ def sources():
     return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
 
 
-def _digest() -> str:
+DEBUG_BUILD = os.path.join(HERE, "_build_debug")
+DEBUG_LIB = os.path.join(HERE, "libssd_debug.so")
+DEBUG_FLAGS = ["-DSSD_DEBUG_BOUNDS=1"]
+
+
+def _digest(flags=None) -> str:
+    flags = FLAGS if flags is None else flags
     h = hashlib.sha256()
     for p in sorted(os.listdir(CSRC)) + ["../../include/ssd.h"]:
         path = os.path.normpath(os.path.join(CSRC, p))
         if os.path.isfile(path):
             h.update(p.encode())
             h.update(open(path, "rb").read())
-    h.update(" ".join(ARCH + FLAGS).encode())
+    h.update(" ".join(ARCH + flags).encode())
     h.update(os.uname().machine.encode())
     return h.hexdigest()
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile (if sources changed) and return the path of libssd.so."""
-    os.makedirs(BUILD, exist_ok=True)
-    stamp = os.path.join(BUILD, "stamp")
-    dig = _digest()
-    if not force and os.path.exists(LIB) and os.path.exists(stamp) and open(stamp).read() == dig:
-        return LIB
+def build(force: bool = False, verbose: bool = False, debug_bounds: bool = False) -> str:
+    """Compile (if sources changed) and return the path of libssd.so (or,
+    with debug_bounds, of libssd_debug.so)."""
+    build_dir, lib = (DEBUG_BUILD, DEBUG_LIB) if debug_bounds else (BUILD, LIB)
+    flags = FLAGS + (DEBUG_FLAGS if debug_bounds else [])
+    os.makedirs(build_dir, exist_ok=True)
+    stamp = os.path.join(build_dir, "stamp")
+    dig = _digest(flags)
+    if not force and os.path.exists(lib) and os.path.exists(stamp) and open(stamp).read() == dig:
+        return lib
     cc = nvcc()
     procs = []
     objs = []
     for src in sources():
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         objs.append(obj)
-        cmd = [cc] + ARCH + FLAGS + ["-c", src, "-o", obj]
+        cmd = [cc] + ARCH + flags + ["-c", src, "-o", obj]
         if verbose:
             cmd += ["-Xptxas", "-v"]
         procs.append((src, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)))
@@ -71,16 +83,17 @@ def build(force: bool = False, verbose: bool = False) -> str:
             print(out)
     if failed:
         raise RuntimeError("nvcc failed:\n" + "\n".join(failed))
-    tmp = LIB + ".tmp"
+    tmp = lib + ".tmp"
     link = [cc] + ARCH + ["-shared", "-o", tmp] + objs + ["-cudart", "static"]
     r = subprocess.run(link, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n" + r.stdout.decode())
-    os.replace(tmp, LIB)
+    os.replace(tmp, lib)
     with open(stamp, "w") as f:
         f.write(dig)
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv,
+                debug_bounds="--debug-bounds" in sys.argv))

@@ -626,7 +626,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) accept_kernel(AcceptArgs
           if (sample || is_bonus) a.accepted[r] = 0;
           record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
         }
-      } else {
+      } else if (dbg_in(bk, nblocks, a.status)) {
         const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
         if (lane == 0) {
           a.out_tok[r] = pick;
@@ -719,6 +719,11 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   if (n > 0 && prefix < n) j = prefix;                             // first rejected draft
   else if (a.bonus && n > 0 && prefix == n && n < a.D_max) j = n;  // the bonus row
   const int64_t r = r0 + (j < 0 ? 0 : j);
+  // (debug builds: the committed row against the batch's rows)
+  if (!dbg_in(r, (int64_t)a.B * a.D_max, a.status)) {
+    pdl_wait();
+    return;
+  }
   const float2 st = j < 0 ? make_float2(NAN, NAN) : (j == 0 ? st0 : a.stats[r]);
   if (!(st.x == st.x)) {  // nothing to draw, or an invalid row the acceptance pass reported
     pdl_wait();
@@ -773,7 +778,7 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
       if (is_bonus) a.accepted[r] = 0;
       record_status(a.status, SSD_ERR_DEVICE_BOUNDS);
     }
-  } else {
+  } else if (dbg_in(bk, nblocks, a.status)) {
     const int32_t pick = walk_block(tp, dp, bk, nv, cc, ncp, ncq, from_p, tb, lane);
     if (lane == 0) a.out_tok[r] = pick;
   }

@@ -327,6 +327,12 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     const int32_t j = r / G, h = g * G + r % G;
     const float inv_l = l_run[i] > 0.f ? 1.0f / l_run[i] : 0.f;
     const float lse = (l_run[i] > 0.f) ? (m_run[i] * (c2 / kLog2e) + logf(l_run[i])) : -INFINITY;
+    // (debug builds: the row's store index against its buffer)
+    if (direct ? !dbg_in(((int64_t)b * a.D_max + j) * a.Hq + h, (int64_t)a.B * a.D_max * a.Hq,
+                         a.status)
+               : !dbg_in((((int64_t)b * a.Hq + h) * a.D_max + j) * L.splits + split,
+                         (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status))
+      continue;
     if (direct) {
       __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.o) +
                           (((int64_t)b * a.D_max + j) * a.Hq + h) * D;
@@ -372,6 +378,7 @@ __global__ void attn_combine_kernel(AttnArgs a, AttnLaunch L) {
   const int32_t n_active = (Lk + L.kps - 1) / L.kps;
   if (n_active <= 1) return;  // written directly by the attention kernel
   const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + j) * L.splits;
+  if (!dbg_in(prow + n_active - 1, (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status)) return;
   float mx = -INFINITY;
   for (int s = 0; s < n_active; ++s) mx = fmaxf(mx, L.part_lse[prow + s]);
   constexpr int PER = D / 32;

@@ -189,6 +189,10 @@ __device__ __forceinline__ void merge_row(const AttnArgs& a, const TcLaunch& L, 
                                           int32_t h, int32_t jq, int32_t nsplit, int col0,
                                           int step, bool write_lse) {
   const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits;
+  if (!dbg_in(prow, (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status) ||
+      !dbg_in(prow + nsplit - 1, (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status) ||
+      !dbg_in(((int64_t)b * a.D_max + jq) * a.Hq + h, (int64_t)a.B * a.D_max * a.Hq, a.status))
+    return;
   float mx = -INFINITY;
   for (int32_t s = 0; s < nsplit; ++s) mx = fmaxf(mx, __ldcg(L.part_lse + prow + s));
   float acc[NU * W];
@@ -807,6 +811,13 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         const uint32_t ta = tO + lane_off + half * HD;
         if constexpr (HD == 64) tld16x256_x8(ta, ov);
         else tld16x256_x4(ta, ov);
+        // (debug builds: the rows' store indexes against their buffers)
+        const int64_t n_rows_o = (int64_t)a.B * a.D_max * a.Hq;
+        const int64_t n_rows_p = (int64_t)a.B * a.Hq * a.D_max * L.splits;
+        const bool sA = liveA && (direct ? dbg_in(((int64_t)b * a.D_max + jqA) * a.Hq + hA, n_rows_o, a.status)
+                                         : dbg_in((((int64_t)b * a.Hq + hA) * a.D_max + jqA) * L.splits + split, n_rows_p, a.status));
+        const bool sB = liveB && (direct ? dbg_in(((int64_t)b * a.D_max + jqB) * a.Hq + hB, n_rows_o, a.status)
+                                         : dbg_in((((int64_t)b * a.Hq + hB) * a.D_max + jqB) * L.splits + split, n_rows_p, a.status));
         if (ok) {
           const int colb = half * HD + 2 * cq;
           if (direct) {
@@ -816,10 +827,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                                 (((int64_t)b * a.D_max + jqB) * a.Hq + hB) * D + colb;
 #pragma unroll
             for (int u = 0; u < HD / 8; ++u) {
-              if (liveA)
+              if (sA)
                 *reinterpret_cast<uint32_t*>(oA + 8 * u) =
                     pack_bf16x2(ov[4 * u] * invA, ov[4 * u + 1] * invA);
-              if (liveB)
+              if (sB)
                 *reinterpret_cast<uint32_t*>(oB + 8 * u) =
                     pack_bf16x2(ov[4 * u + 2] * invB, ov[4 * u + 3] * invB);
             }
@@ -830,10 +841,10 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                         ((((int64_t)b * a.Hq + hB) * a.D_max + jqB) * L.splits + split) * D + colb;
 #pragma unroll
             for (int u = 0; u < HD / 8; ++u) {
-              if (liveA)
+              if (sA)
                 *reinterpret_cast<float2*>(pA + 8 * u) =
                     make_float2(ov[4 * u] * invA, ov[4 * u + 1] * invA);
-              if (liveB)
+              if (sB)
                 *reinterpret_cast<float2*>(pB + 8 * u) =
                     make_float2(ov[4 * u + 2] * invB, ov[4 * u + 3] * invB);
             }
@@ -844,12 +855,12 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             const float lseB =
                 ltB > 0.f ? (m_runB * (c2 / kLog2eTC) + __logf(ltB)) : -INFINITY;
             if (direct) {
-              if (a.lse != nullptr && liveA) a.lse[((int64_t)b * a.Hq + hA) * a.D_max + jqA] = lseA;
-              if (a.lse != nullptr && liveB) a.lse[((int64_t)b * a.Hq + hB) * a.D_max + jqB] = lseB;
+              if (a.lse != nullptr && sA) a.lse[((int64_t)b * a.Hq + hA) * a.D_max + jqA] = lseA;
+              if (a.lse != nullptr && sB) a.lse[((int64_t)b * a.Hq + hB) * a.D_max + jqB] = lseB;
             } else {
-              if (liveA)
+              if (sA)
                 L.part_lse[(((int64_t)b * a.Hq + hA) * a.D_max + jqA) * L.splits + split] = lseA;
-              if (liveB)
+              if (sB)
                 L.part_lse[(((int64_t)b * a.Hq + hB) * a.D_max + jqB) * L.splits + split] = lseB;
             }
           }
@@ -861,7 +872,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           pair_sync();
           if (half == 0 && lane == 0) {
             const int64_t tix = (((int64_t)b * a.Hkv + g) * L.mtiles + row0 / BM) * 4 + quarter;
-            s_last[quarter] = (ok && ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
+            s_last[quarter] = (ok && dbg_in(tix, (int64_t)a.B * a.Hkv * L.mtiles * 4, a.status) &&
+                               ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
           }
           pair_sync();
           if (s_last[quarter]) {
@@ -1055,11 +1067,16 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         // its instruction count is its cost
         const float inv_l = l_tot > 0.f ? __fdividef(1.0f, l_tot) : 0.f;
         const float lse = (l_tot > 0.f) ? (m_run * (c2 / kLog2eTC) + __logf(l_tot)) : -INFINITY;
+        // (debug builds: the row's store index against its buffer)
+        const bool sL = live && (direct ? dbg_in(((int64_t)b * a.D_max + jq) * a.Hq + h,
+                                                 (int64_t)a.B * a.D_max * a.Hq, a.status)
+                                        : dbg_in((((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split,
+                                                 (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status));
 #pragma unroll 1
         for (int cc = 0; cc < HD / 32; ++cc) {
           float ov[32];
           tmem_ld32(tO + lane_off + half * HD + cc * 32, ov);
-          if (!live || !ok) continue;
+          if (!sL || !ok) continue;
           const int col = half * HD + cc * 32;
           if (direct) {
             __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.o) +
@@ -1082,7 +1099,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                   ov[i] * inv_l, ov[i + 1] * inv_l, ov[i + 2] * inv_l, ov[i + 3] * inv_l);
           }
         }
-        if (live && ok && half == 0) {
+        if (sL && ok && half == 0) {
           if (direct) {
             if (a.lse != nullptr) a.lse[((int64_t)b * a.Hq + h) * a.D_max + jq] = lse;
           } else {
@@ -1096,7 +1113,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           pair_sync();
           if (half == 0 && lane == 0) {
             const int64_t tix = (((int64_t)b * a.Hkv + g) * L.mtiles + row0 / BM) * 4 + quarter;
-            s_last[quarter] = (ok && ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
+            s_last[quarter] = (ok && dbg_in(tix, (int64_t)a.B * a.Hkv * L.mtiles * 4, a.status) &&
+                               ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
           }
           pair_sync();
           if (s_last[quarter] && live) {

@@ -37,6 +37,29 @@ __device__ __forceinline__ void record_status(int32_t* status, int32_t code) {
   if (status != nullptr) atomicCAS(status, (int32_t)SSD_OK, code);
 }
 
+// Debug build (SSD_DEBUG_BOUNDS=1: `python -m paper_2606_20543_gb300.build
+// --debug-bounds` writes libssd_debug.so): the kernels check the indexes of
+// their global stores and of the loads they compute from device data
+// against the extent of the buffer; an index outside records
+// SSD_ERR_DEVICE_BOUNDS in the status word and the access is skipped (no
+// trap, no assert).  Release builds compile every check to `true`.
+#ifndef SSD_DEBUG_BOUNDS
+#define SSD_DEBUG_BOUNDS 0
+#endif
+__device__ __forceinline__ bool dbg_in(int64_t i, int64_t n, int32_t* status) {
+#if SSD_DEBUG_BOUNDS
+  if (i < 0 || i >= n) {
+    record_status(status, SSD_ERR_DEVICE_BOUNDS);
+    return false;
+  }
+#else
+  (void)i;
+  (void)n;
+  (void)status;
+#endif
+  return true;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
