@@ -208,7 +208,6 @@ class ClockSampler:
 MEASURED_TRAFFIC = {
     # (kernel, config): (source, sha256 prefix of the source the capture ran,
     # DRAM bytes read + written in one launch, rows of that launch or None)
-    ("attention", 2): ("attention_tc.cu", "cf1328b23a34be8d", 102179584 + 2470656, None),
     ("lmhead_accept", 4): ("lmhead.cu", "07f252f7b825ad8e", 269314560 + 2795520, None),
     # 8 x 64x64 replay, first step (1024 draft rows): accept_kernel alone; the
     # bench scales it to the rows of the replay states it sums

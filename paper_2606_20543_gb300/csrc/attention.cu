@@ -72,7 +72,6 @@ struct AttnLaunch {
   float* part_o;         // [B][Hq][D_max][splits][d] fp32 (splits > 1)
   float* part_lse;       // [B][Hq][D_max][splits]
   int32_t* seq_ok;       // [B] 1 if the sequence's inputs were in range
-  unsigned long long* tickets;  // tcgen05 split launches: in-kernel merge tickets
 };
 
 // Validity of one sequence's frontier; identical in every CTA of b.
@@ -360,8 +359,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   pdl_wait();
 }
 
-// One warp per (b, j, h) row: merge the active splits of the mma.sync kernel
-// by log-sum-exp (the tcgen05 kernel merges its own).
+// One warp per (b, j, h) row: merge the active splits by log-sum-exp.
 template <int D>
 __global__ void attn_combine_kernel(AttnArgs a, AttnLaunch L) {
   const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -511,13 +509,7 @@ size_t attention_workspace(int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_
                            int32_t L_max) {
   size_t bytes = align256((size_t)B * sizeof(int32_t));
   int32_t splits = 1;
-  size_t tickets = 0;
-  for (int32_t hint : {D_max, 0}) {
-    const Plan p = make_plan(B, Hq, Hkv, d, D_max, L_max, hint);
-    splits = max(splits, p.splits);
-    if (p.tc && p.splits > 1) tickets = max(tickets, tc_ticket_count(B, Hkv, p.mtiles));
-  }
-  bytes += align256(tickets * sizeof(unsigned long long));
+  for (int32_t hint : {D_max, 0}) splits = max(splits, make_plan(B, Hq, Hkv, d, D_max, L_max, hint).splits);
   if (splits > 1) {
     const size_t prow = (size_t)B * Hq * D_max * splits;
     bytes += align256(prow * d * sizeof(float)) + align256(prow * sizeof(float));
@@ -530,9 +522,7 @@ static cudaError_t launch_combine(const AttnArgs& a, const AttnLaunch& L, cudaSt
 int attention_launches(const ssd_grid& g, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
                        int32_t D_max, int32_t L_max) {
   if (B == 0) return 0;
-  // the mma.sync kernel's split launches add the combine kernel
-  const Plan p = make_plan(B, Hq, Hkv, d, D_max, L_max, attention_rows_hint(g, D_max));
-  return (!p.tc && p.splits > 1) ? 2 : 1;
+  return make_plan(B, Hq, Hkv, d, D_max, L_max, attention_rows_hint(g, D_max)).splits > 1 ? 2 : 1;
 }
 
 namespace {
@@ -546,11 +536,6 @@ AttnLaunch carve(const AttnArgs& a, const Plan& p, void* ws) {
   unsigned char* w = static_cast<unsigned char*>(ws);
   L.seq_ok = reinterpret_cast<int32_t*>(w);
   w += align256((size_t)a.B * sizeof(int32_t));
-  L.tickets = nullptr;
-  if (p.tc && p.splits > 1) {
-    L.tickets = reinterpret_cast<unsigned long long*>(w);
-    w += align256(tc_ticket_count(a.B, a.Hkv, p.mtiles) * sizeof(unsigned long long));
-  }
   L.part_o = nullptr;
   L.part_lse = nullptr;
   if (p.splits > 1) {
@@ -568,7 +553,7 @@ cudaError_t launch_attention_combine(const AttnArgs& a, void* ws, cudaStream_t s
   if (a.B == 0) return cudaSuccess;
   const Plan p = make_plan(a.B, a.Hq, a.Hkv, a.d, a.D_max, a.L_max,
                            attention_rows_hint(a.grid, a.D_max));
-  return (p.tc || p.splits == 1) ? cudaSuccess : launch_combine(a, carve(a, p, ws), stream);
+  return p.splits == 1 ? cudaSuccess : launch_combine(a, carve(a, p, ws), stream);
 }
 
 cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaStream_t stream,
@@ -579,9 +564,10 @@ cudaError_t launch_attention(const AttnArgs& a, void* ws, size_t ws_bytes, cudaS
   const AttnLaunch L = carve(a, p, ws);
   cudaError_t e;
   if (p.tc) {
-    // split partials are merged inside the kernel
-    return launch_attention_tc(a, TcPlan{p.splits, p.kps, p.mtiles}, L.seq_ok, L.part_o,
-                               L.part_lse, L.tickets, stream, pdl);
+    e = launch_attention_tc(a, TcPlan{p.splits, p.kps, p.mtiles}, L.seq_ok, L.part_o, L.part_lse,
+                            stream, pdl);
+    if (e != cudaSuccess) return e;
+    return (p.splits == 1 || defer_combine) ? cudaSuccess : launch_combine(a, L, stream);
   }
   CUtensorMap tmK, tmV;
   const int64_t rows = (int64_t)a.B * a.Hkv * a.L_max;

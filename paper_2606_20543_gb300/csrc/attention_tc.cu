@@ -149,100 +149,14 @@ struct TcLaunch {
   float* part_o;
   float* part_lse;
   int32_t* seq_ok;
-  unsigned long long* tickets;  // splits > 1: [B][Hkv][mtiles][4] split tickets (any contents)
 };
-
-// Split-KV merge inside the kernel.  One ticket per (sequence, KV head,
-// query tile, TMEM lane quarter): after writing its partials, the pair of
-// softmax warps of a quarter arrives once per split; the arrival that
-// completes the count merges the splits of the quarter's rows.  A ticket is
-// tagged with the launch's grid id, so a count left by an earlier launch
-// never carries over (the workspace may hold anything), and the completing
-// arrival clears it.  The retry loop is bounded by the contenders (one CAS
-// fails only when another succeeds).
-__device__ __forceinline__ bool ticket_complete(unsigned long long* t, int32_t need,
-                                                int32_t* status) {
-  unsigned long long gid;
-  asm volatile("mov.u64 %0, %%gridid;" : "=l"(gid));
-  const unsigned long long tag = gid << 8;
-  unsigned long long cur = *reinterpret_cast<volatile unsigned long long*>(t);
-  for (int i = 0; i < 512; ++i) {
-    const unsigned long long next = (cur & ~0xffull) == tag ? cur + 1ull : (tag | 1ull);
-    const unsigned long long prev = atomicCAS(t, cur, next);
-    if (prev == cur) {
-      if ((int32_t)(next & 0xffull) < need) return false;
-      atomicExch(t, 0ull);
-      return true;
-    }
-    cur = prev;
-  }
-  record_status(status, SSD_ERR_TIMEOUT);
-  return false;
-}
-
-// Log-sum-exp merge of the nsplit partials of one (b, h, jq) row over the
-// columns col0 + step * u + {0, .., W - 1}, u < NU (W = 2 or 4): weights
-// exp(lse_s - max), O = sum w_s O_s / sum w_s, lse = max + log(sum w_s).
-// Partials are read from L2 (written by other CTAs of this launch).
-template <int D, int NU, int W>
-__device__ __forceinline__ void merge_row(const AttnArgs& a, const TcLaunch& L, int32_t b,
-                                          int32_t h, int32_t jq, int32_t nsplit, int col0,
-                                          int step, bool write_lse) {
-  const int64_t prow = (((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits;
-  if (!dbg_in(prow, (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status) ||
-      !dbg_in(prow + nsplit - 1, (int64_t)a.B * a.Hq * a.D_max * L.splits, a.status) ||
-      !dbg_in(((int64_t)b * a.D_max + jq) * a.Hq + h, (int64_t)a.B * a.D_max * a.Hq, a.status))
-    return;
-  float mx = -INFINITY;
-  for (int32_t s = 0; s < nsplit; ++s) mx = fmaxf(mx, __ldcg(L.part_lse + prow + s));
-  float acc[NU * W];
-#pragma unroll
-  for (int i = 0; i < NU * W; ++i) acc[i] = 0.f;
-  float wsum = 0.f;
-  for (int32_t s = 0; s < nsplit; ++s) {
-    const float ls = __ldcg(L.part_lse + prow + s);
-    const float w = ls == -INFINITY ? 0.f : expf(ls - mx);
-    wsum += w;
-    const float* po = L.part_o + (prow + s) * D + col0;
-#pragma unroll
-    for (int u = 0; u < NU; ++u) {
-      if constexpr (W == 4) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(po + step * u));
-        acc[4 * u] += w * v.x;
-        acc[4 * u + 1] += w * v.y;
-        acc[4 * u + 2] += w * v.z;
-        acc[4 * u + 3] += w * v.w;
-      } else {
-        const float2 v = __ldcg(reinterpret_cast<const float2*>(po + step * u));
-        acc[2 * u] += w * v.x;
-        acc[2 * u + 1] += w * v.y;
-      }
-    }
-  }
-  const float inv = 1.0f / wsum;
-  __nv_bfloat16* ob =
-      reinterpret_cast<__nv_bfloat16*>(a.o) + (((int64_t)b * a.D_max + jq) * a.Hq + h) * D + col0;
-#pragma unroll
-  for (int u = 0; u < NU; ++u) {
-    if constexpr (W == 4) {
-      uint2 w2;
-      w2.x = pack_bf16x2(acc[4 * u] * inv, acc[4 * u + 1] * inv);
-      w2.y = pack_bf16x2(acc[4 * u + 2] * inv, acc[4 * u + 3] * inv);
-      *reinterpret_cast<uint2*>(ob + step * u) = w2;
-    } else {
-      *reinterpret_cast<uint32_t*>(ob + step * u) = pack_bf16x2(acc[2 * u] * inv, acc[2 * u + 1] * inv);
-    }
-  }
-  if (write_lse && a.lse != nullptr) a.lse[((int64_t)b * a.Hq + h) * a.D_max + jq] = mx + logf(wsum);
-}
 
 // One work item (KV split, sequence, KV head, query tile) as the producer
 // hands it to the MMA and softmax warps; ntiles < 0 ends the CTA's work.
 struct TcItem {
   int32_t b, g, split, row0, rows_total, cache, Lk, k_lo, k_hi, ntiles, direct;
   int32_t increasing;  // kflat strictly increasing (the raster frontier): draft j sees draft j' iff j' <= j
-  int32_t nsplit;      // splits of this sequence's keys (1: direct)
-  int32_t pad[3];
+  int32_t pad[4];
   int32_t kflat[128];  // raster position of each draft of b
 };
 
@@ -284,7 +198,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ int32_t s_order[kLptMax];
   __shared__ int32_t s_key[kLptMax];
-  __shared__ int32_t s_last[4];  // per lane quarter: this arrival completed the tile's splits
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sQ = smem;                         // [2][Q_BYTES]
@@ -309,6 +222,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 
   const int32_t G = a.Hq / a.Hkv;
   const int32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int32_t per_b = a.Hkv * L.splits * L.mtiles;
+  const int64_t n_items = (int64_t)a.B * per_b;
 
   // ---- set-up: barriers, TMEM, the longest-first order of the sequences
   if (tid == 0) {
@@ -357,9 +272,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int32_t splits = L.splits, kps = L.kps;
-  const int32_t per_b = a.Hkv * splits * L.mtiles;
-  const int64_t n_items = (int64_t)a.B * per_b;
   const uint32_t tS = tmem;            // [kNB] x KTC columns: S_t in fp32, then P_t in bf16
   const uint32_t tO0 = tmem + 256;     // [2] x 128 columns
 
@@ -384,7 +296,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       int32_t rem = (int32_t)(i - (int64_t)rank_b * per_b);
       const int32_t mtile = rem % L.mtiles;
       rem /= L.mtiles;
-      const int32_t split = rem % splits, g = rem / splits;
+      const int32_t split = rem % L.splits, g = rem / L.splits;
       const int32_t b = (a.B <= kLptMax) ? s_order[rank_b] : rank_b;
       const int32_t cache = a.cache_len[b], nd = attn_drafts(a, b);
       const bool shape_ok = nd >= 0 && nd <= a.D_max && cache >= 0 && cache <= a.L_max - nd;
@@ -425,8 +337,8 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
       const int32_t Lk = valid ? cache + nd : 0;
       const int32_t rows_total = valid ? nd * G : 0;
       const int32_t row0 = mtile * BM;
-      const int32_t k_lo = split * kps;
-      const int32_t k_hi = min(Lk, k_lo + kps);
+      const int32_t k_lo = split * L.kps;
+      const int32_t k_hi = min(Lk, k_lo + L.kps);
       if (!valid || nd == 0 || row0 >= rows_total || k_lo >= Lk) continue;
       const int32_t ntiles = (k_hi - k_lo + KTC - 1) / KTC;
       const int s = k & 1;
@@ -448,8 +360,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         it.k_lo = k_lo;
         it.k_hi = k_hi;
         it.ntiles = ntiles;
-        it.nsplit = (Lk + kps - 1) / kps;
-        it.direct = it.nsplit == 1;
+        it.direct = ((Lk + L.kps - 1) / L.kps) == 1;
         it.increasing = increasing ? 1 : 0;
       }
       __syncwarp();
@@ -505,11 +416,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     // kernel starts as the acceptance's CTAs retire; lane 1 waits for the
     // acceptance to complete and only then lets the kernel queued after this
     // one (the counts and draws, which read them) be scheduled beside it.
-    // Under a plain launch the wait returns at once.
-    if (lane == 1) {
-      pdl_wait();
-      pdl_launch_dependents();
-    }
+    // Under a plain launch the wait returns at once.  The wait sits in the
+    // other branch of the V loop's lane test, so that lane 0 never waits at
+    // the reconvergence point of a block of its own.
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       uint32_t T = 0;
@@ -532,6 +441,9 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
           load_kv_tile<D>(sV + sb * KV_BYTES, &tmV, kvrow0 + t * KTC, &v_ready[sb], pol);
         }
       }
+    } else if (lane == 1) {
+      pdl_wait();
+      pdl_launch_dependents();
     }
     __syncwarp();
   } else if (warp == kSoftWarps + 1) {
@@ -865,26 +777,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             }
           }
         }
-        if (!direct) {
-          // release this pair's partials; the arrival completing the tile's
-          // splits merges the quarter's rows (same columns as written above)
-          __threadfence();
-          pair_sync();
-          if (half == 0 && lane == 0) {
-            const int64_t tix = (((int64_t)b * a.Hkv + g) * L.mtiles + row0 / BM) * 4 + quarter;
-            s_last[quarter] = (ok && dbg_in(tix, (int64_t)a.B * a.Hkv * L.mtiles * 4, a.status) &&
-                               ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
-          }
-          pair_sync();
-          if (s_last[quarter]) {
-            __threadfence();
-            const int colb = half * HD + 2 * cq;
-            if (liveA)
-              merge_row<D, HD / 8, 2>(a, L, b, hA, jqA, it.nsplit, colb, 8, half == 0 && cq == 0);
-            if (liveB)
-              merge_row<D, HD / 8, 2>(a, L, b, hB, jqB, it.nsplit, colb, 8, half == 0 && cq == 0);
-          }
-        }
       }
       // O[s] and the item slot are free for item k + 2
       tc_fence_before();
@@ -1106,25 +998,6 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             L.part_lse[(((int64_t)b * a.Hq + h) * a.D_max + jq) * L.splits + split] = lse;
           }
         }
-        if (!direct) {
-          // release this pair's partials; the arrival completing the tile's
-          // splits merges the quarter's rows (this thread's row and half)
-          __threadfence();
-          pair_sync();
-          if (half == 0 && lane == 0) {
-            const int64_t tix = (((int64_t)b * a.Hkv + g) * L.mtiles + row0 / BM) * 4 + quarter;
-            s_last[quarter] = (ok && dbg_in(tix, (int64_t)a.B * a.Hkv * L.mtiles * 4, a.status) &&
-                               ticket_complete(L.tickets + tix, it.nsplit, a.status)) ? 1 : 0;
-          }
-          pair_sync();
-          if (s_last[quarter] && live) {
-            __threadfence();
-#pragma unroll 1
-            for (int cc = 0; cc < HD / 32; ++cc)
-              merge_row<D, 8, 4>(a, L, b, h, jq, it.nsplit, half * HD + cc * 32, 4,
-                                 half == 0 && cc == 0);
-          }
-        }
       }
       // O[s] and the item slot are free for item k + 2
       tc_fence_before();
@@ -1180,8 +1053,7 @@ TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int3
 }
 
 cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
-                                float* part_lse, unsigned long long* tickets, cudaStream_t stream,
-                                bool pdl) {
+                                float* part_lse, cudaStream_t stream, bool pdl) {
   EncodeTiledFn fn = tensor_map_encoder();
   if (fn == nullptr) return cudaErrorInvalidValue;
   const int32_t G = a.Hq / a.Hkv;
@@ -1219,9 +1091,6 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq
   L.part_o = part_o;
   L.part_lse = part_lse;
   L.seq_ok = seq_ok;
-  L.tickets = tickets;
-  if (L.splits > 1 && (tickets == nullptr || part_o == nullptr || part_lse == nullptr))
-    return cudaErrorInvalidValue;
   // persistent: one CTA per SM (at most one per work item)
   const int64_t n_items = (int64_t)a.B * a.Hkv * p.mtiles * p.splits;
   const dim3 grid((unsigned)std::min<int64_t>(n_items, device_sm_count()));

@@ -286,14 +286,8 @@ struct TcPlan {
 };
 bool attention_tc_supported(int32_t Hq, int32_t Hkv, int32_t d, int32_t D_max);
 TcPlan attention_tc_plan(int32_t B, int32_t Hq, int32_t Hkv, int32_t D_max, int32_t L_max);
-// Split launches merge their partials in the kernel (no combine launch):
-// tickets [B][Hkv][mtiles][4] (tc_ticket_count), any initial contents.
 cudaError_t launch_attention_tc(const AttnArgs& a, const TcPlan& p, int32_t* seq_ok, float* part_o,
-                                float* part_lse, unsigned long long* tickets, cudaStream_t stream,
-                                bool pdl = false);
-inline size_t tc_ticket_count(int32_t B, int32_t Hkv, int32_t mtiles) {
-  return (size_t)B * Hkv * mtiles * 4;
-}
+                                float* part_lse, cudaStream_t stream, bool pdl = false);
 // Same as launch_attention with the library's static device scratch as the
 // workspace (ssd_verify_attention_noalloc); cudaErrorMemoryAllocation if the
 // problem needs more than SSD_NOALLOC_SCRATCH_BYTES.

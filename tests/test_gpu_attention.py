@@ -105,11 +105,10 @@ def test_long_cache_many_splits(ssd):
 
 
 def test_split_merge_ignores_workspace_contents(ssd):
-    """The tcgen05 kernel merges its KV splits itself: the CTA whose
-    partials complete a tile merges them, counted by per-launch tickets in
-    the workspace.  Whatever the workspace held before (all ones, zeros, the
-    tickets and partials of earlier launches of this and of another case),
-    the result is the same, bit for bit."""
+    """A KV cache split over CTAs: partials in the workspace, merged by the
+    combine kernel.  Whatever the workspace held before (all ones, zeros, the
+    partials of earlier launches of this and of another case), the result is
+    the same, bit for bit."""
     c = synth.make_case("long", grid_h=64, grid_w=64, prefix_len=256, cache_len=[256 + 64 * 40 + 9],
                         Hq=4, Hkv=4, d=128, V=64, seed=7, with_logits=False)
     other = synth.make_case("long2", grid_h=64, grid_w=64, prefix_len=256,
