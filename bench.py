@@ -553,14 +553,16 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
     # pass copies its frontier's logit rows (both sets), the drafts' Q and their
     # K/V slots from pinned host memory, and reads back the counts and
     # decisions, which set the next pass's copies; the KV cache itself stays on
-    # the device (it only grows by the appended draft slots)
+    # the device (it only grows by the appended draft slots).  The host holds
+    # the new K/V slot-major ([B][L_max][Hkv][d], as a forward pass emits them
+    # for all heads of a token), so each sequence's slots are one contiguous copy,
+    # spread over the heads by a device copy.
     E = max(1, min(a.e2e_steps, T))
     pinned = lambda x: torch.from_numpy(x).pin_memory()  # noqa: E731
     host_logits = [(pinned(t), pinned(d)) for t, d in pool]
     host_q = pinned(np.ascontiguousarray(c.q).view(np.int16)).view(torch.bfloat16)
-    k16, v16 = c.k.view(np.int16), c.v.view(np.int16)
-    stage = [torch.empty((c.B, c.D_max, c.Hkv, c.d), dtype=torch.int16, pin_memory=True)
-             for _ in range(2)]
+    host_kv = [pinned(np.ascontiguousarray(x.view(np.int16).transpose(0, 2, 1, 3))).view(torch.bfloat16)
+               for x in (c.k, c.v)]
     dstage = [torch.empty((c.B, c.D_max, c.Hkv, c.d), dtype=torch.bfloat16, device=dev)
               for _ in range(2)]
     e_tg, e_dr = dpool[0]  # device logit buffers of the leg (the timed replays are done)
@@ -585,10 +587,8 @@ def run_replay(a, world, rank, dev, torch, ssd, VerifyStep):
             e_tg[r0:r0 + n].copy_(ht[r0:r0 + n], non_blocking=True)
             e_dr[r0:r0 + n].copy_(hd[r0:r0 + n], non_blocking=True)
             s.q[b, :n].copy_(host_q[b, :n], non_blocking=True)
-            for src, st_h, st_d, dst in ((k16, stage[0], dstage[0], s.k),
-                                         (v16, stage[1], dstage[1], s.v)):
-                st_h[b, :n].numpy()[...] = src[b, :, cl:cl + n].transpose(1, 0, 2)
-                st_d[b, :n].copy_(st_h[b, :n].view(torch.bfloat16), non_blocking=True)
+            for src, st_d, dst in ((host_kv[0], dstage[0], s.k), (host_kv[1], dstage[1], s.v)):
+                st_d[b, :n].copy_(src[b, cl:cl + n], non_blocking=True)
                 dst[b, :, cl:cl + n].copy_(st_d[b, :n].transpose(0, 1))
             h2d_total += n * (2 * c.V * 4 + c.Hq * c.d * 2 + 2 * c.Hkv * c.d * 2)
         s.set_rng(seed, t)
