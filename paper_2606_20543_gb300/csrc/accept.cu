@@ -721,12 +721,12 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   const int64_t r = r0 + (j < 0 ? 0 : j);
   // (debug builds: the committed row against the batch's rows)
   if (!dbg_in(r, (int64_t)a.B * a.D_max, a.status)) {
-    pdl_wait();
+    if (pdl_first_block()) pdl_wait();
     return;
   }
   const float2 st = j < 0 ? make_float2(NAN, NAN) : (j == 0 ? st0 : a.stats[r]);
   if (!(st.x == st.x)) {  // nothing to draw, or an invalid row the acceptance pass reported
-    pdl_wait();
+    if (pdl_first_block()) pdl_wait();
     return;
   }
   const bool is_bonus = j == n;
@@ -754,7 +754,7 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
   if (lane == 0) last = atomicAdd(&a.tickets[b], 1) == (int32_t)gridDim.x - 1;
   last = __shfl_sync(0xffffffffu, last, 0);
   if (!last) {
-    pdl_wait();
+    if (pdl_first_block()) pdl_wait();
     return;
   }
   __threadfence();
@@ -783,9 +783,9 @@ __global__ void __launch_bounds__(32, 32) resolve_kernel(ResolveArgs a) {
     if (lane == 0) a.out_tok[r] = pick;
   }
   // Under a programmatic launch after the attention (the step's schedule; the
-  // acceptance pass completed before the attention started): exit only after
-  // the attention, so that stream order holds.
-  pdl_wait();
+  // acceptance pass completed before the attention let this kernel in): block
+  // 0 exits only after the attention, so that stream order holds.
+  if (pdl_first_block()) pdl_wait();
 }
 
 }  // namespace

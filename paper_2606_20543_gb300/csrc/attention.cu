@@ -92,6 +92,16 @@ __device__ __forceinline__ bool load_draft_positions(const AttnArgs& a, int32_t 
   return *bad == 0;
 }
 
+// Launched as a programmatic dependent (the step's schedule): block 0 exits
+// only after the kernel before it, and lets the next kernel be scheduled
+// then, so that stream order holds.
+__device__ __forceinline__ void pdl_exit() {
+  if (pdl_first_block()) {
+    pdl_wait();
+    pdl_launch_dependents();
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kMaxWarps * 32, 1)
 frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -100,7 +110,9 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   constexpr int TILE_BYTES = KT * D * 2;       // one K (or V) tile
   constexpr int KSTEPS = D / 16;               // k16 steps of QK^T
   constexpr int NT_O = D / 8;                  // n8 tiles of O
-  pdl_launch_dependents();  // as in the tcgen05 kernel: a dependent may start beside it
+  // as in the tcgen05 kernel: a dependent may start beside it once block 0
+  // has seen the kernel before this one complete (block 0 triggers on exit)
+  if (!pdl_first_block()) pdl_launch_dependents();
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the swizzle atoms
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -169,7 +181,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
   if (!seq_valid || !has_work) {
     // never leave with copies in flight into this CTA's shared memory
     for (int t = 0; t < n_pre; ++t) mbar_wait(&full[t % kStages], 0, a.status);
-    pdl_wait();
+    pdl_exit();
     return;
   }
 
@@ -313,7 +325,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     if (!__syncthreads_and(ok)) { ok = false; break; }
   }
   if (!ok || !warp_active) {
-    pdl_wait();
+    pdl_exit();
     return;
   }
 
@@ -354,9 +366,7 @@ frontier_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
       if ((lane & 3) == 0) L.part_lse[prow] = lse;
     }
   }
-  // launched as a programmatic dependent (the step's schedule): exit only after
-  // the kernel before it, so that stream order holds
-  pdl_wait();
+  pdl_exit();
 }
 
 // One warp per (b, j, h) row: merge the active splits by log-sum-exp.

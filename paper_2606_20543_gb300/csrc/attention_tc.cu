@@ -413,10 +413,12 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     // the softmax has finished its item, which needs every V tile of it.
     // Launch ordering (programmatic dependent launch): launched as a dependent
     // of the step's acceptance pass, whose results it does not read, the
-    // kernel starts as the acceptance's CTAs retire; lane 1 waits for the
-    // acceptance to complete and only then lets the kernel queued after this
-    // one (the counts and draws, which read them) be scheduled beside it.
-    // Under a plain launch the wait returns at once.  The wait sits in the
+    // kernel starts as the acceptance's CTAs retire; lane 1 of block 0 waits
+    // for the acceptance to complete and only then lets the kernel queued
+    // after this one (the counts and draws, which read them) be scheduled
+    // beside it; lane 1 of the other blocks lets it be scheduled at once (it
+    // is scheduled when every block has).  Under a plain launch the wait
+    // returns at once.  The wait sits in the
     // other branch of the V loop's lane test, so that lane 0 never waits at
     // the reconvergence point of a block of its own.
     if (lane == 0) {
@@ -442,7 +444,7 @@ frontier_attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
       }
     } else if (lane == 1) {
-      pdl_wait();
+      if (pdl_first_block()) pdl_wait();
       pdl_launch_dependents();
     }
     __syncwarp();

@@ -32,6 +32,15 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 // completed with its memory visible (a no-op in a kernel launched without
 // the programmatic attribute).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// In a chain of programmatic launches one block orders the chain: block 0
+// waits for the kernel before it to complete before it lets the kernel after
+// it be scheduled and before it exits, so neither the next kernel nor the
+// grid's completion can overtake the previous kernel.  The other blocks let
+// the next kernel be scheduled at their start and exit freely, so no block
+// but one idles in a wait beside the running kernels.
+__device__ __forceinline__ bool pdl_first_block() {
+  return blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0;
+}
 
 __device__ __forceinline__ void record_status(int32_t* status, int32_t code) {
   if (status != nullptr) atomicCAS(status, (int32_t)SSD_OK, code);

@@ -50,7 +50,7 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
                               int32_t* __restrict__ next_cache_len, int32_t* status) {
   const int32_t b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (b >= B) {
-    pdl_wait();
+    if (pdl_first_block()) pdl_wait();
     return;
   }
   int32_t n = n_drafts[b];
@@ -60,7 +60,8 @@ __global__ void counts_kernel(ssd_grid g, int32_t commit, int32_t B, int32_t D_m
   }
   sequence_counts(g, commit, b, D_max, cache_len, n, accepted, accepted_count, accepted_prefix,
                   next_cache_len, threadIdx.x & 31);
-  pdl_wait();  // under a programmatic launch: exit only after the kernel before it
+  // under a programmatic launch: block 0 exits only after the kernel before it
+  if (pdl_first_block()) pdl_wait();
 }
 
 // Staged schedule: the trailing row (slots W .. 2W-1) becomes the frontier of
