@@ -195,3 +195,28 @@ def test_sampling_with_given_tokens_and_temperature(ssd):
     assert st == 0
     dec = oacc.accept_rows(tgt, drf, u, draft_tok=dt, temperature=0.7, strategy="sample")
     compare_decisions(dec, tok, acc, ratio, what="sample T=0.7")
+
+
+@pytest.mark.parametrize("strategy", ["accept_reject", "greedy"])
+def test_masked_vocabulary_entries(ssd, strategy):
+    """Degenerate distributions: a quarter of the vocabulary is masked (-inf)
+    in the target and another quarter in the draft, and in every other row
+    the draft's token is one the target masks (p(t) = 0: ratio 0, always
+    rejected, the residual token drawn from the target's unmasked entries).
+    Decisions, tokens and ratios against the oracle; no masked token is ever
+    drawn."""
+    rng = np.random.default_rng(9)
+    rows, V = 32, 4096
+    tgt, drf = synth._logits_normal(rng, rows, V)
+    tgt, drf = tgt.astype(np.float32), drf.astype(np.float32)
+    tgt[:, :1024] = -np.inf
+    drf[:, 2048:3072] = -np.inf
+    drf[::2, 5] = 50.0
+    u = synth.philox_uniforms(9, 3, rows)
+    tok, acc, ratio, lse, st = run_accept(ssd, tgt, drf, u, strategy=strategy)
+    assert st == 0
+    dec = oacc.accept_rows(tgt, drf, u, strategy=strategy)
+    compare_decisions(dec, tok, acc, ratio, lse, what=f"masked {strategy}")
+    assert not np.isin(tok, np.arange(1024)).any()
+    if strategy == "accept_reject":
+        assert not acc[::2].any() and np.all(ratio[::2] == 0.0)

@@ -248,3 +248,17 @@ def test_mma_sync_shuffled_draft_order(ssd):
 def test_sweep_shape_shuffled_draft_order(ssd):
     c = synth.config2(points=[120, 144, 408, 672], with_logits=False)
     _check_permuted_frontier(ssd, c)
+
+
+@pytest.mark.parametrize("B", [1, 20])
+def test_empty_cache_and_no_prefix(ssd, B):
+    """The first verification pass of an image with no text prefix: cache
+    length 0, so every draft attends to itself and the drafts before it only
+    (the whole key range is the drafted block).  B = 1 splits nothing; B = 20
+    adds sequences at their last row and finished ones (no drafts)."""
+    cl = [0] + [24 * 23 + (k % 24) for k in range(1, B)]
+    if B > 1:
+        cl[1] = 24 * 24  # finished grid: empty frontier
+    c = synth.make_case("no_prefix", grid_h=24, grid_w=24, prefix_len=0, cache_len=cl, Hq=8,
+                        Hkv=8, d=128, V=64, seed=17, with_logits=False)
+    check_case(ssd, c)

@@ -370,3 +370,24 @@ def test_horizontal_stage_large_batch(ssd, strategy):
         for h in range(c.Hq):
             if n:
                 assert attention_error(res["o"][b, :n, h], o_ref[:, h]) < ATTN_TOL
+
+
+def test_step_with_masked_vocabulary(ssd):
+    """The whole step (one-pass acceptance, committed draws, counts) on logits
+    with masked (-inf) vocabulary entries: a quarter of the target's and
+    another quarter of the draft's, and the draft tokens of every third row
+    masked by the target (always rejected).  Against the oracle; no masked
+    token is committed."""
+    import copy
+    c = copy.copy(synth.config2(points=[120, 312, 480, 672]))
+    tg, dr = c.tgt_logits.copy(), c.drf_logits.copy()
+    tg[:, :4096] = -np.inf
+    dr[:, 8192:12288] = -np.inf
+    dr[::3, 7] = 60.0
+    c.tgt_logits, c.drf_logits = tg, dr
+    s = make_step(c)
+    s.run()
+    torch.cuda.synchronize()
+    res = s.results()
+    check_step(c, res)
+    assert not np.isin(res["out_tok"], np.arange(4096)).any()
