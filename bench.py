@@ -211,7 +211,7 @@ MEASURED_TRAFFIC = {
     ("lmhead_accept", 4): ("lmhead.cu", "07f252f7b825ad8e", 269314560 + 2795520, None),
     # 8 x 64x64 replay, first step (1024 draft rows): accept_kernel alone; the
     # bench scales it to the rows of the replay states it sums
-    ("accept", 5): ("accept.cu", "f5a51c0947bed819", 536945152 + 3111680, 1024),
+    ("accept", 5): ("accept.cu", "db1c6b21e30787b5", 536945152 + 3072000, 1024),
 }
 
 
