@@ -237,7 +237,7 @@ def graph_kernel_ms(call, kk, stream, dev, torch, flush_bytes=256 << 20):
     charge the kernel that follows for evicting it)."""
     buf = torch.ones(flush_bytes // 4, dtype=torch.float32, device=dev)
 
-    def replay_ms(with_calls):
+    def capture(with_calls):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
             cs = torch.cuda.current_stream()
@@ -247,6 +247,9 @@ def graph_kernel_ms(call, kk, stream, dev, torch, flush_bytes=256 << 20):
                     call(i, cs)
         g.replay()
         torch.cuda.synchronize(dev)
+        return g
+
+    def replay_ms(g):
         k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         k0.record(stream)
         g.replay()
@@ -254,7 +257,14 @@ def graph_kernel_ms(call, kk, stream, dev, torch, flush_bytes=256 << 20):
         torch.cuda.synchronize(dev)
         return k0.elapsed_time(k1)
 
-    return max(0.0, replay_ms(True) - replay_ms(False)) / kk
+    # the two graphs timed alternately, three times each (medians), so that a
+    # clock or power transition does not land on one of them only
+    g_with, g_flush = capture(True), capture(False)
+    t_with, t_flush = [], []
+    for _ in range(3):
+        t_with.append(replay_ms(g_with))
+        t_flush.append(replay_ms(g_flush))
+    return max(0.0, statistics.median(t_with) - statistics.median(t_flush)) / kk
 
 
 def measured_peaks():
