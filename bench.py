@@ -1145,8 +1145,11 @@ def main():
                                 "(2 tiles x 2 heads x 128 columns = 512)")}
 
     # ---------------- end to end: host buffers, copies inside the timed region
+    # (every per-step input whole, one copy each: a copy per sequence costs more
+    # in calls than the padding saves; lm_head weights are model parameters,
+    # resident on the device)
     host = {}
-    in_names = ("cache_len", "q", "k", "v") + (("h_tgt", "h_drf", "w_tgt", "w_drf") if c.hidden
+    in_names = ("cache_len", "q", "k", "v") + (("h_tgt", "h_drf") if c.hidden
                                                else ("tgt", "drf"))
     for name in in_names:
         t = getattr(st, name)
@@ -1236,7 +1239,12 @@ def main():
                                  for k, (b, m) in kern.items()}},
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "steps": ke},
+                "d2h_bytes_per_step": d2h, "steps": ke,
+                "what": "each step through ssd_verify_step with every per-step input (cache "
+                        "lengths, Q, K/V, " + ("hidden states; lm_head weights resident"
+                                               if c.hidden else "logits") +
+                        ") copied whole from pinned host memory and the decisions and counts "
+                        "read back"},
         "gpu_launches": launches * steps_done,
         "device_status": status,
         "near_ties": None if ties is None else ties.report(
