@@ -376,6 +376,9 @@ ssd_status ssd_lmhead_accept(int32_t rows, int32_t V, int32_t K, const void* h_t
  * ref_rows is written (the draft row, or the target row when the row is
  * not accepted), so no pass over ref_rows is needed before a block.
  * commit: an ssd_commit; the counts' next_cache_len follows it.
+ * out->next_cache_len must not overlap args->cache_len (SSD_ERR_INVALID_ARG):
+ * the counts run beside the attention, which reads cache_len.
+ * ssd_verify_accept() runs its kernels in stream order and allows it.
  * Draws: under strategy (C) from logits with commit SSD_COMMIT_PREFIX or
  * SSD_COMMIT_PREFIX_BONUS and no ref_rows, the step draws only the token it
  * commits: the residual token of each sequence's first rejected draft, or

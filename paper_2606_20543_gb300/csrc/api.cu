@@ -641,6 +641,13 @@ ssd_status ssd_verify_step(const ssd_verify_args* x, const ssd_verify_out* y, vo
   if (y->draft_pos == nullptr || y->o == nullptr) return SSD_ERR_INVALID_ARG;
   s = check_accept_part(x, y);
   if (s != SSD_OK) return s;
+  // The counts write next_cache_len while the attention (beside them, or as
+  // the kernel they depend on programmatically) may still read cache_len.
+  {
+    const uintptr_t c0 = (uintptr_t)x->cache_len, n0 = (uintptr_t)y->next_cache_len;
+    const uintptr_t len = (uintptr_t)x->B * sizeof(int32_t);
+    if (c0 < n0 + len && n0 < c0 + len) return SSD_ERR_INVALID_ARG;
+  }
   if (!(x->scale >= 0.f) || !isfinite(x->scale)) return SSD_ERR_INVALID_ARG;
   const size_t need = ssd_verify_step_workspace(x);
   if (workspace == nullptr || workspace_bytes < need) return SSD_ERR_WORKSPACE;

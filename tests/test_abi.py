@@ -148,6 +148,7 @@ def test_verify_accept_and_step_host_validation(lib):
         for name in ("n_drafts", "draft_pos", "o", "out_tok", "accepted", "ratio",
                      "accepted_count", "accepted_prefix", "next_cache_len", "status"):
             setattr(y, name, fake)
+        y.next_cache_len = fake + 0x1000  # disjoint from cache_len
         for k, v in kw.items():
             setattr(y, k, v)
         return y
@@ -177,6 +178,10 @@ def test_verify_accept_and_step_host_validation(lib):
                 None) == 3
     assert step(ctypes.byref(args()), ctypes.byref(out()), ctypes.c_void_p(fake), need - 1,
                 None) == 7
+    # next_cache_len overlapping cache_len (the counts advance it beside the attention)
+    for at in (fake, fake + 4, fake - 4):
+        assert step(ctypes.byref(args()), ctypes.byref(out(next_cache_len=at)),
+                    ctypes.c_void_p(fake), need, None) == 1
     # launch counts: acceptance + attention (+ combine) + counts on the logits path,
     # and one more (the frontier) on the fused path
     n_logits = so.ssd_verify_step_launches(ctypes.byref(args()))
