@@ -29,18 +29,27 @@
 //     unit) running ahead through all four phases: the weights do not depend
 //     on the activations, so the weight stream keeps going while a phase
 //     waits for the previous one to finish;
-//   * warp 3, lane 0: activation producer — once every tile of the previous
-//     phase is final (a bounded wait on a counter), one TMA copy of each
+//   * warp 3: activation producer — lane 0 issues one TMA copy of each
 //     unit's activation tile X (K-major, 128-byte swizzle) from z, Ag, G or
-//     Hg; warp 3 also allocates and frees the tensor memory;
+//     Hg once the tile of the previous phase that X is cut from is final.
+//     With at most 64 rows the unit waits for that one tile (the whole warp
+//     polls a window of 32 tiles per round trip, so a CTA starts a phase as
+//     soon as the tiles it reads are final, not the last tile of the grid);
+//     with more rows, where a tile's finish is heavier and competes with the
+//     next phase's stream, for every tile of the previous phase.  Warp 3 also
+//     allocates and frees the tensor memory;
 //   * warp 2: issues the MMAs of each unit into one of two TMEM accumulators
 //     (the next tile's products overlap the previous tile's epilogue);
 //   * warps 4-7: the epilogue.  Each TMEM lane is one feature; the CTA's
-//     partial of a tile goes to the workspace, then a ticket per tile: the
-//     last contributor sums the tile's partials in slot order and finishes it
-//     (A, Ag and A's squares per row; G; h and Hg; the tile's argmax per row),
-//     then counts the tile done.  The last tile of P3 reduces the tiles'
-//     argmaxes to the tokens.
+//     partial of a tile goes to the workspace (even and odd phases in
+//     separate buffers, since a CTA may start a phase while another still sums
+//     the previous phase's partials), then a ticket per tile: the last
+//     contributor sums the tile's partials in slot order and finishes it (A,
+//     Ag and A's squares per row; G; h and Hg; the tile's argmax per row,
+//     raised into one 64-bit key per row with atomicMax), then counts the
+//     tile final on its ticket and on the phase's counter.  The row scales
+//     s(A) are summed once per CTA from the P0 tiles' squares before its first
+//     P1 finish; the last tile of P3 to finish turns the keys into the tokens.
 // Numerics: every product input is bf16 (z, the weights, Ag, G, Hg); A, U,
 // Vg, h and the logits are fp32; every sum runs in a fixed order, so results
 // do not depend on timing.
@@ -77,6 +86,7 @@ struct PredLaunch {
   int32_t stages;              // ring slots (weights + activations of one unit each)
   int32_t d, m, V;
   uint32_t max_polls, shortfall;
+  int32_t tile_waits;          // activation copies wait per tile (else per phase)
   float eps;
   const float* gamma1;
   const float* gamma2;
@@ -84,8 +94,9 @@ struct PredLaunch {
   __nv_bfloat16* ag;           // bf16 [rows][d]: A * g1, then h_hat * g2
   __nv_bfloat16* g;            // bf16 [rows][m]: silu(U) * Vg
   float* ss;                   // fp32 [d/128][128]: per-tile sums of squares of A's rows
-  float2* amax;                // [V/128][128]: (max logit, index) per tile and row
-  float* part;                 // split-K partials
+  unsigned long long* best;    // [rows]: the argmax key of each row (zeroed with the counters)
+  float* part;                 // split-K partials: even phases at part, odd at part + part_odd
+  int64_t part_odd;
   unsigned int* ctr;           // tickets [4][max tiles], done [4], abort
   int32_t max_tiles;
   int32_t* out_tok;
@@ -179,35 +190,78 @@ __device__ __forceinline__ void warp_argmax(float& v, int32_t& i) {
 
 namespace {
 
+// The vocabulary argmax of each row is kept as one 64-bit key per row,
+// raised with atomicMax by every finished GenHead tile: the logit in an
+// order-preserving unsigned form (NaN as the lowest key) above the inverted
+// index, so the largest logit wins and the lower index among equal ones
+// (-0 is taken as +0, which compares equal to it).
+__device__ __forceinline__ unsigned long long argmax_key(float v, int32_t i) {
+  uint32_t u = v == 0.f ? 0u : __float_as_uint(v);
+  u = (v != v) ? 0u : ((u & 0x80000000u) ? ~u : (u | 0x80000000u));
+  return ((unsigned long long)u << 32) | (unsigned long long)(0xffffffffu - (uint32_t)i);
+}
+__device__ __forceinline__ int32_t argmax_index(unsigned long long key) {
+  return (int32_t)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
+}
+
+// The finishing step of one row r of a tile from its summed products x.
+// P0 (p = 0): A = x, Ag = bf16(A * g1) and A's squares; P2: h = A + x,
+// Hg = bf16(h * g2).
+__device__ __forceinline__ void emit_hidden(const PredLaunch& L, int p, int32_t f, int32_t r,
+                                            int32_t feat, int q, float4 x, float4 a0, float4 ga) {
+  float4 y = x;
+  if (p == 2) y = make_float4(a0.x + y.x, a0.y + y.y, a0.z + y.z, a0.w + y.w);
+  *reinterpret_cast<float4*>(L.hid + (int64_t)r * L.d + feat) = y;
+  uint2 o;
+  o.x = pack_bf16x2(y.x * ga.x, y.y * ga.y);
+  o.y = pack_bf16x2(y.z * ga.z, y.w * ga.w);
+  *reinterpret_cast<uint2*>(L.ag + (int64_t)r * L.d + feat) = o;
+  if (p == 0) {
+    const float sq = warp_sum((y.x * y.x + y.y * y.y) + (y.z * y.z + y.w * y.w));
+    if (q == 0) L.ss[(int64_t)f * 128 + r] = sq;
+  }
+}
+// P1: G = bf16(silu(U) * Vg) with U, Vg scaled by the row's s(A).
+__device__ __forceinline__ void emit_gate(const PredLaunch& L, int32_t r, int32_t feat, float4 uu,
+                                          float4 vv, float sr) {
+  const float u0 = uu.x * sr, u1 = uu.y * sr, u2 = uu.z * sr, u3 = uu.w * sr;
+  uint2 o;
+  o.x = pack_bf16x2(u0 / (1.0f + expf(-u0)) * (vv.x * sr), u1 / (1.0f + expf(-u1)) * (vv.y * sr));
+  o.y = pack_bf16x2(u2 / (1.0f + expf(-u2)) * (vv.z * sr), u3 / (1.0f + expf(-u3)) * (vv.w * sr));
+  *reinterpret_cast<uint2*>(L.g + (int64_t)r * L.m + feat) = o;
+}
+// P3: the tile's argmax for row r (lowest index on ties) raised into the row's key.
+__device__ __forceinline__ void emit_argmax(const PredLaunch& L, int32_t r, int32_t feat, int q,
+                                            float4 x) {
+  float bv = x.x;
+  int32_t bi = feat;
+  if (x.y > bv) { bv = x.y; bi = feat + 1; }
+  if (x.z > bv) { bv = x.z; bi = feat + 2; }
+  if (x.w > bv) { bv = x.w; bi = feat + 3; }
+  warp_argmax(bv, bi);
+  if (q == 0) atomicMax(L.best + r, argmax_key(bv, bi));
+}
+
 // Epilogue of the last contributor of tile f of phase p: the tile's partials
 // summed in slot order, then the phase's finishing step.  Thread et (0..127)
 // takes features f * 128 + 4 q .. + 3 (q = et % 32, 16-byte loads) of rows
 // et / 32 + 4 i; the 32 lanes of a warp hold one row's 128 features, so row
 // reductions are warp reductions.  Each batch issues RB rows x NACC
-// accumulators x SMAX slots (32 float4, slots beyond cnt predicated off)
-// before summing any, so a tile costs a few round trips to L2.
-// srow: [128] (the row scales of A, P1).
+// accumulators x SMAX slots (32 float4) before summing any, so a tile costs a
+// few round trips to L2.  srow: [128] the row scales s(A) (P1).
 template <int SMAX, int NACC>
-__device__ void finish_tile(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
-                            float* srow) {
+__device__ void finish_tile_t(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
+                              const float* srow) {
   constexpr int RB = 32 / (SMAX * NACC) > 0 ? 32 / (SMAX * NACC) : 1;
   const PredPhase& ph = L.ph[p];
   const int w = et >> 5, q = et & 31;
   const int32_t feat = f * 128 + 4 * q;
   const int64_t tile_stride = (int64_t)NACC * L.nn * 128;
-  const float* base = L.part + (int64_t)f * ph.slots * tile_stride + 4 * q;
-  if (p == 1) {  // the row scales s(A) from the per-tile sums of squares (fixed order)
-    for (int32_t r = et; r < L.rows; r += kEpiThreads) {
-      float s = 0.f;
-      for (int32_t t = 0; t < L.d / 128; ++t) s += __ldcg(L.ss + (int64_t)t * 128 + r);
-      srow[r] = 1.0f / sqrtf(s / (float)L.d + L.eps);
-    }
-    bar_named(kBarEpi, kEpiThreads);
-  }
+  const float* base = L.part + (p & 1) * L.part_odd + (int64_t)f * ph.slots * tile_stride + 4 * q;
   float4 ga = make_float4(0.f, 0.f, 0.f, 0.f);
   if (p == 0) ga = __ldg(reinterpret_cast<const float4*>(L.gamma1 + feat));
   if (p == 2) ga = __ldg(reinterpret_cast<const float4*>(L.gamma2 + feat));
-  const int32_t my_rows = (L.rows - w + 3) / 4;  // rows w, w + 4, ... below L.rows
+  const int32_t my_rows = (L.rows - w + 3) / 4;
   for (int32_t i0 = 0; i0 < my_rows; i0 += RB) {
     float4 v[RB][NACC][SMAX];
 #pragma unroll
@@ -239,38 +293,14 @@ __device__ void finish_tile(const PredLaunch& L, int p, int32_t f, int32_t cnt, 
           x[a].w += v[b][a][sl].w;
         }
       }
-      if (NACC == 2) {  // P1: G = silu(U) * Vg with U, Vg scaled by the row's s(A)
-        const float sr = srow[r];
-        const float4 uu = x[0], vv = x[NACC - 1];
-        const float u0 = uu.x * sr, u1 = uu.y * sr, u2 = uu.z * sr, u3 = uu.w * sr;
-        uint2 o;
-        o.x = pack_bf16x2(u0 / (1.0f + expf(-u0)) * (vv.x * sr), u1 / (1.0f + expf(-u1)) * (vv.y * sr));
-        o.y = pack_bf16x2(u2 / (1.0f + expf(-u2)) * (vv.z * sr), u3 / (1.0f + expf(-u3)) * (vv.w * sr));
-        *reinterpret_cast<uint2*>(L.g + (int64_t)r * L.m + feat) = o;
-      } else if (p == 3) {  // the tile's argmax for row r (lowest index on ties)
-        float bv = x[0].x;
-        int32_t bi = feat;
-        if (x[0].y > bv) { bv = x[0].y; bi = feat + 1; }
-        if (x[0].z > bv) { bv = x[0].z; bi = feat + 2; }
-        if (x[0].w > bv) { bv = x[0].w; bi = feat + 3; }
-        warp_argmax(bv, bi);
-        if (q == 0) L.amax[(int64_t)f * 128 + r] = make_float2(bv, __int_as_float(bi));
-      } else {  // P0: A, Ag = bf16(A * g1), A's squares; P2: h = A + sum, Hg = bf16(h * g2)
-        float* hp = L.hid + (int64_t)r * L.d + feat;
-        float4 y = x[0];
-        if (p == 2) {
-          const float4 a0 = __ldcg(reinterpret_cast<const float4*>(hp));
-          y = make_float4(a0.x + y.x, a0.y + y.y, a0.z + y.z, a0.w + y.w);
-        }
-        *reinterpret_cast<float4*>(hp) = y;
-        uint2 o;
-        o.x = pack_bf16x2(y.x * ga.x, y.y * ga.y);
-        o.y = pack_bf16x2(y.z * ga.z, y.w * ga.w);
-        *reinterpret_cast<uint2*>(L.ag + (int64_t)r * L.d + feat) = o;
-        if (p == 0) {
-          const float sq = warp_sum((y.x * y.x + y.y * y.y) + (y.z * y.z + y.w * y.w));
-          if (q == 0) L.ss[(int64_t)f * 128 + r] = sq;
-        }
+      if (NACC == 2) {
+        emit_gate(L, r, feat, x[0], x[NACC - 1], srow[r]);
+      } else if (p == 3) {
+        emit_argmax(L, r, feat, q, x[0]);
+      } else {
+        float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (p == 2) a0 = __ldcg(reinterpret_cast<const float4*>(L.hid + (int64_t)r * L.d + feat));
+        emit_hidden(L, p, f, r, feat, q, x[0], a0, ga);
       }
     }
   }
@@ -278,24 +308,42 @@ __device__ void finish_tile(const PredLaunch& L, int p, int32_t f, int32_t cnt, 
 
 template <int NACC>
 __device__ void finish_tile_n(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
-                              float* srow) {
+                              const float* srow) {
   switch (cnt) {  // the slot count fixes the batch shape (one batch for 24 rows up to 5 slots)
-    case 1: finish_tile<1, NACC>(L, p, f, cnt, et, srow); break;
-    case 2: finish_tile<2, NACC>(L, p, f, cnt, et, srow); break;
-    case 3: finish_tile<3, NACC>(L, p, f, cnt, et, srow); break;
-    case 4: finish_tile<4, NACC>(L, p, f, cnt, et, srow); break;
-    case 5: finish_tile<5, NACC>(L, p, f, cnt, et, srow); break;
-    case 6: finish_tile<6, NACC>(L, p, f, cnt, et, srow); break;
-    default: finish_tile<8, NACC>(L, p, f, cnt, et, srow); break;
+    case 1: finish_tile_t<1, NACC>(L, p, f, cnt, et, srow); break;
+    case 2: finish_tile_t<2, NACC>(L, p, f, cnt, et, srow); break;
+    case 3: finish_tile_t<3, NACC>(L, p, f, cnt, et, srow); break;
+    case 4: finish_tile_t<4, NACC>(L, p, f, cnt, et, srow); break;
+    case 5: finish_tile_t<5, NACC>(L, p, f, cnt, et, srow); break;
+    case 6: finish_tile_t<6, NACC>(L, p, f, cnt, et, srow); break;
+    default: finish_tile_t<8, NACC>(L, p, f, cnt, et, srow); break;
   }
 }
 
 __device__ void finish_tile_any(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
-                                float* srow) {
+                                const float* srow) {
   if (p == 1)
     finish_tile_n<2>(L, p, f, cnt, et, srow);
   else
     finish_tile_n<1>(L, p, f, cnt, et, srow);
+}
+
+// The row scales s(A) = 1 / sqrt(mean(A^2) + eps) of every row from the P0
+// tiles' sums of squares, into srow (shared): four threads per row, each
+// summing every fourth tile, then combined in a fixed order.
+__device__ void row_scales(const PredLaunch& L, int et, float* srow) {
+  const int k = et & 3;
+  const int32_t nt = L.d / 128;
+  for (int32_t r0 = 0; r0 < L.rows; r0 += kEpiThreads / 4) {
+    const int32_t r = r0 + (et >> 2);
+    float s = 0.f;
+    if (r < L.rows)
+#pragma unroll 8
+      for (int32_t t = k; t < nt; t += 4) s += __ldcg(L.ss + (int64_t)t * 128 + r);
+    s += __shfl_xor_sync(0xffffffffu, s, 1);
+    s += __shfl_xor_sync(0xffffffffu, s, 2);
+    if (r < L.rows && k == 0) srow[r] = 1.0f / sqrtf(s / (float)L.d + L.eps);
+  }
 }
 
 __device__ __forceinline__ void issue_weights(const PredLaunch& L, int p, int32_t u,
@@ -384,6 +432,12 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
     *fail = 0;
     fence_barrier_init();
   }
+  if (warp == kWarpMma && lane < 9) {  // the descriptors of the first copies of every phase
+    const CUtensorMap* map = lane == 0 ? &tmW0 : lane == 1 ? &tmW1 : lane == 2 ? &tmW3
+                           : lane == 3 ? &tmW2 : lane == 4 ? &tmWH : lane == 5 ? &tmZ
+                           : lane == 6 ? &tmAg : lane == 7 ? &tmG : &tmHg;
+    prefetch_tensormap(map);
+  }
   if (warp == kWarpX) {
     tmem_alloc(tmem_slot, ncols);
     tmem_relinquish();
@@ -424,39 +478,99 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
     }
     __syncwarp();
   } else if (warp == kWarpX) {
-    // ---- activation producer
-    if (lane == 0) {
-      const uint64_t pol = policy_evict_last();  // read again by the CTAs sharing a K range
-      uint32_t gu = 0;
-      bool ok = true;
-      for (int p = 0; p < kPhases && ok; ++p) {
-        const PredPhase& ph = L.ph[p];
-        if (p >= 1) {  // every tile of the previous phase final
-          if (*fail ||
-              !wait_count(L, done_ctr(L, p - 1), (uint32_t)L.ph[p - 1].tiles + L.shortfall)) {
-            *fail = 1;
-            break;
-          }
+    // ---- activation producer: lane 0 issues the copies.  Per-tile waits:
+    // to learn which tiles of the previous phase are final, every lane polls
+    // one tile of a window of 32 starting at the one the next unit reads, so
+    // one round trip answers for the units that follow.
+    const uint64_t pol = policy_evict_last();  // read again by the CTAs sharing a K range
+    uint32_t gu = 0;
+    bool ok = true;
+    for (int p = 0; p < kPhases && ok; ++p) {
+      const PredPhase& ph = L.ph[p];
+      int32_t wbase = -1;  // tiles wbase + k of the previous phase are final for the bits k of wmask
+      uint32_t wmask = 0;
+      bool all_final = p == 0;  // P0 reads z
+      if (p >= 1 && !L.tile_waits) {  // every tile of the previous phase final first
+        bool got = true;
+        if (lane == 0) {
+          got = *fail == 0 &&
+                wait_count(L, done_ctr(L, p - 1), (uint32_t)L.ph[p - 1].tiles + L.shortfall);
+          if (!got) *fail = 1;
           fence_proxy_async_global();
         }
-        const uint32_t bytes = (uint32_t)L.nn * ph.kw * 2;
-        const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
-        for (int64_t u = lo; u < hi; ++u, ++gu) {
-          const uint32_t s = gu % S;
+        if (!__shfl_sync(0xffffffffu, got, 0)) {
+          ok = false;
+          break;
+        }
+        all_final = true;
+      }
+      const uint32_t bytes = (uint32_t)L.nn * ph.kw * 2;
+      const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
+      for (int64_t u = lo; u < hi; ++u, ++gu) {
+        const uint32_t s = gu % S;
+        if (!all_final) {
+          const int32_t need = (int32_t)((u % ph.upt) * ph.kw / 128);
+          if (!(need >= wbase && need < wbase + 32 && ((wmask >> (need - wbase)) & 1u))) {
+            const PredPhase& pp = L.ph[p - 1];
+            const int32_t t = need + lane;
+            uint32_t target = 0xffffffffu;  // a tile past the end is never final
+            if (t < pp.tiles) {
+              const int32_t c0 = unit_cta((int64_t)t * pp.upt, pp.units, L.ncta);
+              const int32_t c1 = unit_cta((int64_t)(t + 1) * pp.upt - 1, pp.units, L.ncta);
+              target = (uint32_t)(c1 - c0 + 2) + L.shortfall;  // every contributor, then the finisher
+            }
+            wbase = need;
+            wmask = 0;
+            bool got = false, stop = *fail != 0;
+            for (uint32_t i = 0; i < L.max_polls && !stop; ++i) {
+              const bool f = target != 0xffffffffu && !((wmask >> lane) & 1u) &&
+                             ld_acquire_u32(ticket(L, p - 1, t)) >= target;
+              wmask |= __ballot_sync(0xffffffffu, f);
+              if (wmask & 1u) {
+                got = true;
+                break;
+              }
+              if ((i & 1023u) == 1023u)
+                stop = __shfl_sync(0xffffffffu, lane == 0 && ld_acquire_u32(abort_flag(L)) != 0u, 0);
+              if (i > 64) __nanosleep(128);
+            }
+            __syncwarp();
+            if (lane == 0) {
+              if (got) {
+                got = ld_acquire_u32(abort_flag(L)) == 0u;
+              } else if (!stop) {  // the poll limit ran out
+                atomicExch(abort_flag(L), 1u);
+                record_status(L.status, SSD_ERR_TIMEOUT);
+              }
+              if (!got) *fail = 1;
+              // the acquiring lanes' loads before the copies of this lane
+              fence_acq_rel_gpu();
+              fence_proxy_async_global();
+            }
+            if (!__shfl_sync(0xffffffffu, got, 0)) {
+              ok = false;
+              break;
+            }
+          }
+        }
+        if (lane == 0) {
           if (*fail || (gu >= (uint32_t)S &&
                         !mbar_wait(&empty[s], ((gu / S) - 1) & 1, L.status, L.max_polls))) {
             *fail = 1;
             ok = false;
-            break;
+          } else {
+            mbar_arrive_expect_tx(&full[s], bytes);
+            issue_x(L, p, (int32_t)u, ring + s * slot_bytes + kUnitBytes, &full[s], pol, &tmZ,
+                    &tmAg, &tmG, &tmHg);
           }
-          mbar_arrive_expect_tx(&full[s], bytes);
-          issue_x(L, p, (int32_t)u, ring + s * slot_bytes + kUnitBytes, &full[s], pol, &tmZ,
-                  &tmAg, &tmG, &tmHg);
         }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
       }
+    }
+    if (lane == 0)
       for (uint32_t x = gu > (uint32_t)S ? gu - S : 0; x < gu; ++x)
         mbar_wait(&full[x % S], (x / S) & 1, nullptr, L.max_polls);
-    }
     __syncwarp();
   } else if (warp == kWarpMma) {
     // ---- MMA issue: one thread
@@ -528,7 +642,7 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
     const int et = tid - kEpiWarp0 * 32;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t tc = 0;
-    bool ok = true;
+    bool ok = true, have_scales = false;
     for (int p = 0; p < kPhases && ok; ++p) {
       const PredPhase& ph = L.ph[p];
       const int nacc = p == 1 ? 2 : 1;
@@ -548,7 +662,8 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
         tc_fence_after();
         const int32_t first = unit_cta((int64_t)f * ph.upt, ph.units, L.ncta);
         const int32_t lastc = unit_cta((int64_t)(f + 1) * ph.upt - 1, ph.units, L.ncta);
-        float* dst = L.part + ((int64_t)f * ph.slots + (cta - first)) * nacc * L.nn * 128 + et;
+        float* dst = L.part + (p & 1) * L.part_odd +
+                     ((int64_t)f * ph.slots + (cta - first)) * nacc * L.nn * 128 + et;
         for (int a = 0; a < nacc; ++a) {
           for (int32_t ch = 0; ch < L.nc / 32; ++ch) {
             float v[32];
@@ -569,32 +684,36 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
         bar_named(kBarEpi, kEpiThreads);
         if (bcast[0] != (uint32_t)(lastc - first)) continue;  // not the last contributor
         fence_acq_rel_gpu();  // every contributor's partial after the ticket
+        if (p == 1 && !have_scales) {
+          // the row scales s(A), once every P0 tile is final
+          bool stop2 = false;
+          if (et == 0) {
+            stop2 = *fail != 0 ||
+                    !wait_count(L, done_ctr(L, 0), (uint32_t)L.ph[0].tiles + L.shortfall);
+            if (stop2) *fail = 1;
+          }
+          if (bar_or(kBarEpi, kEpiThreads, stop2)) {
+            ok = false;
+            break;
+          }
+          fence_acq_rel_gpu();
+          row_scales(L, et, srow);
+          bar_named(kBarEpi, kEpiThreads);
+          have_scales = true;
+        }
         finish_tile_any(L, p, f, lastc - first + 1, et, srow);
         fence_proxy_async_global();  // Ag, G, Hg are loaded by TMA in the next phase
         fence_acq_rel_gpu();
         bar_named(kBarEpi, kEpiThreads);
-        if (et == 0) bcast[1] = atomicAdd(done_ctr(L, p), 1u);
+        if (et == 0) {
+          atomicAdd(ticket(L, p, f), 1u);  // the tile is final
+          bcast[1] = atomicAdd(done_ctr(L, p), 1u);
+        }
         bar_named(kBarEpi, kEpiThreads);
         if (p == 3 && bcast[1] == (uint32_t)(ph.tiles - 1)) {
-          // the last tile of the vocabulary: reduce the tiles' argmaxes (warp w
-          // takes rows w, w + 4, ...; lane l tiles l, l + 32, ...; the lower
-          // index wins between equal maxima, so the first maximum is kept)
+          // the last tile of the vocabulary: every tile's key is in
           fence_acq_rel_gpu();
-          const int q = et & 31;
-          for (int32_t r = et >> 5; r < L.rows; r += 4) {
-            float bv = -INFINITY;
-            int32_t bi = 0x7fffffff;
-            for (int32_t t = q; t < ph.tiles; t += 32) {
-              const float2 e = __ldcg(L.amax + (int64_t)t * 128 + r);
-              const int32_t ei = __float_as_int(e.y);
-              if (e.x > bv || (e.x == bv && ei < bi)) {
-                bv = e.x;
-                bi = ei;
-              }
-            }
-            warp_argmax(bv, bi);
-            if (q == 0) L.out_tok[r] = bi;
-          }
+          for (int32_t r = et; r < L.rows; r += kEpiThreads) L.out_tok[r] = argmax_index(__ldcg(L.best + r));
         }
       }
     }
@@ -619,7 +738,7 @@ size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 struct PredPlan {
   PredPhase ph[kPhases];
   int32_t ncta, nn, nc, stages, max_tiles;
-  size_t part_floats, smem;
+  size_t part_floats, part_odd, smem;
 };
 
 int32_t tile_slots(const PredPhase& ph, int32_t ncta) {
@@ -658,16 +777,18 @@ PredPlan make_plan(int32_t rows, int32_t d, int32_t m, int32_t V, int32_t sm_cou
     --P.ncta;
   }
   P.max_tiles = 0;
-  P.part_floats = 0;
+  size_t part_max[2] = {0, 0};
   P.nn = (rows + 15) / 16 * 16;
   P.nc = (P.nn + 31) / 32 * 32;
   for (int p = 0; p < kPhases; ++p) {
     P.ph[p].slots = tile_slots(P.ph[p], P.ncta);
     P.max_tiles = std::max(P.max_tiles, P.ph[p].tiles);
     const size_t nacc = p == 1 ? 2 : 1;
-    P.part_floats = std::max(P.part_floats,
-                             (size_t)P.ph[p].tiles * P.ph[p].slots * nacc * P.nn * 128);
+    part_max[p & 1] = std::max(part_max[p & 1],
+                               (size_t)P.ph[p].tiles * P.ph[p].slots * nacc * P.nn * 128);
   }
+  P.part_odd = (part_max[0] + 63) / 64 * 64;
+  P.part_floats = P.part_odd + part_max[1];
   const size_t slot = (size_t)kUnitBytes + (size_t)P.nn * 256;
   const size_t budget = 232448;  // 227 KB of dynamic shared memory per CTA
   P.stages = (int32_t)std::min<size_t>(8, (budget - 1024 - 2048) / slot);
@@ -677,11 +798,12 @@ PredPlan make_plan(int32_t rows, int32_t d, int32_t m, int32_t V, int32_t sm_cou
 
 struct PredWs {
   unsigned int* ctr;
+  unsigned long long* best;  // after the counters: zeroed with them
+  size_t zero_bytes;         // counters and keys
   float* part;
   float* ss;
   __nv_bfloat16* ag;
   __nv_bfloat16* g;
-  float2* amax;
   float* hid;
   size_t bytes;
 };
@@ -696,13 +818,14 @@ PredWs carve(const PredPlan& P, int32_t rows, int32_t d, int32_t m, int32_t V, b
     off += al256(n);
     return p;
   };
-  w.ctr = reinterpret_cast<unsigned int*>(
-      take((size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4));
+  const size_t ctr_bytes = al256((size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4);
+  w.zero_bytes = ctr_bytes + (size_t)kMaxRows * 8;
+  w.ctr = reinterpret_cast<unsigned int*>(take(w.zero_bytes));
+  w.best = reinterpret_cast<unsigned long long*>(reinterpret_cast<unsigned char*>(w.ctr) + ctr_bytes);
   w.part = reinterpret_cast<float*>(take(P.part_floats * 4));
   w.ss = reinterpret_cast<float*>(take((size_t)(d / 128) * 128 * 4));
   w.ag = reinterpret_cast<__nv_bfloat16*>(take((size_t)rows * d * 2));
   w.g = reinterpret_cast<__nv_bfloat16*>(take((size_t)rows * m * 2));
-  w.amax = reinterpret_cast<float2*>(take((size_t)(V / 128) * 128 * 8));
   w.hid = own_hidden ? reinterpret_cast<float*>(take((size_t)rows * d * 4)) : nullptr;
   w.bytes = off;
   return w;
@@ -733,6 +856,7 @@ cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32
   L.V = a.V;
   L.max_polls = wait_poll_limit();
   L.shortfall = barrier_shortfall();
+  L.tile_waits = a.rows <= 64;  // measured: faster up to 48 rows, slower at 128
   L.eps = a.eps;
   L.gamma1 = a.gamma1;
   L.gamma2 = a.gamma2;
@@ -740,8 +864,9 @@ cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32
   L.ag = w.ag;
   L.g = w.g;
   L.ss = w.ss;
-  L.amax = w.amax;
+  L.best = w.best;
   L.part = w.part;
+  L.part_odd = (int64_t)P.part_odd;
   L.ctr = w.ctr;
   L.max_tiles = P.max_tiles;
   L.out_tok = a.out_tok;
@@ -785,8 +910,7 @@ cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32
     ok = ok && bf16_tensor_map(&tag, w.ag, 2, da, sa, ba);
   }
   if (!ok) return cudaErrorInvalidValue;
-  cudaError_t e = cudaMemsetAsync(
-      w.ctr, 0, (size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4, stream);
+  cudaError_t e = cudaMemsetAsync(w.ctr, 0, w.zero_bytes, stream);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(predictor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)P.smem);
