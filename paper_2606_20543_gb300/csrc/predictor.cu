@@ -346,6 +346,23 @@ __device__ void row_scales(const PredLaunch& L, int et, float* srow) {
   }
 }
 
+// The epilogue warps' row scales: once every P0 tile is final (a bounded wait
+// by one thread), s(A) of every row into srow.  False if the wait gave up or
+// another role failed (every epilogue thread gets the same answer).
+__device__ bool ensure_row_scales(const PredLaunch& L, int et, float* srow,
+                                  volatile int32_t* fail) {
+  bool stop = false;
+  if (et == 0) {
+    stop = *fail != 0 || !wait_count(L, done_ctr(L, 0), (uint32_t)L.ph[0].tiles + L.shortfall);
+    if (stop) *fail = 1;
+  }
+  if (bar_or(kBarEpi, kEpiThreads, stop)) return false;
+  fence_acq_rel_gpu();
+  row_scales(L, et, srow);
+  bar_named(kBarEpi, kEpiThreads);
+  return true;
+}
+
 __device__ __forceinline__ void issue_weights(const PredLaunch& L, int p, int32_t u,
                                               unsigned char* dst, uint64_t* bar, uint64_t pol,
                                               const CUtensorMap* tmW0, const CUtensorMap* tmW1,
@@ -646,6 +663,15 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
     for (int p = 0; p < kPhases && ok; ++p) {
       const PredPhase& ph = L.ph[p];
       const int nacc = p == 1 ? 2 : 1;
+      if (p == 1 && !L.tile_waits) {
+        // per-phase waits: the P1 products start once every P0 tile is final,
+        // so the row scales are summed then, beside the first products
+        if (!ensure_row_scales(L, et, srow, fail)) {
+          ok = false;
+          break;
+        }
+        have_scales = true;
+      }
       const int64_t lo = unit_start(cta, ph.units, L.ncta), hi = unit_start(cta + 1, ph.units, L.ncta);
       const int32_t f0 = (int32_t)(lo / ph.upt), f1 = (int32_t)((hi - 1) / ph.upt);
       for (int32_t f = f0; f <= f1; ++f, ++tc) {
@@ -684,21 +710,11 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
         bar_named(kBarEpi, kEpiThreads);
         if (bcast[0] != (uint32_t)(lastc - first)) continue;  // not the last contributor
         fence_acq_rel_gpu();  // every contributor's partial after the ticket
-        if (p == 1 && !have_scales) {
-          // the row scales s(A), once every P0 tile is final
-          bool stop2 = false;
-          if (et == 0) {
-            stop2 = *fail != 0 ||
-                    !wait_count(L, done_ctr(L, 0), (uint32_t)L.ph[0].tiles + L.shortfall);
-            if (stop2) *fail = 1;
-          }
-          if (bar_or(kBarEpi, kEpiThreads, stop2)) {
+        if (p == 1 && !have_scales) {  // per-tile waits: before the CTA's first P1 finish
+          if (!ensure_row_scales(L, et, srow, fail)) {
             ok = false;
             break;
           }
-          fence_acq_rel_gpu();
-          row_scales(L, et, srow);
-          bar_named(kBarEpi, kEpiThreads);
           have_scales = true;
         }
         finish_tile_any(L, p, f, lastc - first + 1, et, srow);
