@@ -186,6 +186,17 @@ class VerifyStep:
     def run(self, stream=None) -> None:
         ssd_verify_step(self.args, self.out, self.workspace, self.ws_bytes, stream)
 
+    def use_cache_buffers(self, cache_len, next_cache_len) -> None:
+        """Read the step's cache lengths from `cache_len` and write the next
+        ones to `next_cache_len` (two distinct device int32 [B] tensors).
+        Alternating two buffers chains steps with no copy of next_cache_len
+        back into cache_len between them (step t reads buffer t % 2)."""
+        if cache_len.data_ptr() == next_cache_len.data_ptr():
+            raise ValueError("cache_len and next_cache_len must be distinct buffers")
+        self.cache_len, self.next_cache_len = cache_len, next_cache_len
+        self.args.cache_len = cache_len.data_ptr()
+        self.out.next_cache_len = next_cache_len.data_ptr()
+
     # ------------------------------------------------------- replay bookkeeping
     def track_grid(self) -> None:
         """Allocate the committed-token grid [B, H*W] (-1: not committed) that
