@@ -71,6 +71,10 @@ constexpr int kMaxRows = 128;
 constexpr int kPhases = 4;
 constexpr int kBarEpi = 1;           // named barrier of the epilogue warps
 constexpr int kMaxSlots = 8;         // most CTAs sharing one feature tile
+// One 128-byte line per row's argmax key: every GenHead tile raises every
+// row's key at the end of the kernel, and keys packed 16 to a line serialised
+// those atomics on a few lines of L2.
+constexpr int kKeyStride = 16;
 
 struct PredPhase {
   int32_t units;    // units of the phase
@@ -94,7 +98,7 @@ struct PredLaunch {
   __nv_bfloat16* ag;           // bf16 [rows][d]: A * g1, then h_hat * g2
   __nv_bfloat16* g;            // bf16 [rows][m]: silu(U) * Vg
   float* ss;                   // fp32 [d/128][128]: per-tile sums of squares of A's rows
-  unsigned long long* best;    // [rows]: the argmax key of each row (zeroed with the counters)
+  unsigned long long* best;    // [rows][kKeyStride]: the argmax key of row r at best[r * kKeyStride]
   float* part;                 // split-K partials: even phases at part, odd at part + part_odd
   int64_t part_odd;
   unsigned int* ctr;           // tickets [4][max tiles], done [4], abort
@@ -239,7 +243,12 @@ __device__ __forceinline__ void emit_argmax(const PredLaunch& L, int32_t r, int3
   if (x.z > bv) { bv = x.z; bi = feat + 2; }
   if (x.w > bv) { bv = x.w; bi = feat + 3; }
   warp_argmax(bv, bi);
-  if (q == 0) atomicMax(L.best + r, argmax_key(bv, bi));
+  if (q == 0) {  // a reduction without a result: the warp goes on at once (measured:
+                 // atomicMax here held each row's finish for a round trip)
+    const unsigned long long key = argmax_key(bv, bi);
+    asm volatile("red.relaxed.gpu.global.max.u64 [%0], %1;"
+                 ::"l"(L.best + (int64_t)r * kKeyStride), "l"(key) : "memory");
+  }
 }
 
 // Epilogue of the last contributor of tile f of phase p: the tile's partials
@@ -247,12 +256,15 @@ __device__ __forceinline__ void emit_argmax(const PredLaunch& L, int32_t r, int3
 // takes features f * 128 + 4 q .. + 3 (q = et % 32, 16-byte loads) of rows
 // et / 32 + 4 i; the 32 lanes of a warp hold one row's 128 features, so row
 // reductions are warp reductions.  Each batch issues RB rows x NACC
-// accumulators x SMAX slots (32 float4) before summing any, so a tile costs a
-// few round trips to L2.  srow: [128] the row scales s(A) (P1).
+// accumulators x SMAX slots (at most 32 float4) before summing any, so a tile
+// costs a few round trips to L2.  srow: [128] the row scales s(A) (P1).
 template <int SMAX, int NACC>
 __device__ void finish_tile_t(const PredLaunch& L, int p, int32_t f, int32_t cnt, int et,
                               const float* srow) {
-  constexpr int RB = 32 / (SMAX * NACC) > 0 ? 32 / (SMAX * NACC) : 1;
+  // rows per batch: up to 32 loads in flight, at most 8 rows (a longer unrolled
+  // body only lengthens code that runs once per phase; 8 rows cover 24-row
+  // calls in one batch)
+  constexpr int RB = 32 / (SMAX * NACC) > 8 ? 8 : (32 / (SMAX * NACC) > 0 ? 32 / (SMAX * NACC) : 1);
   const PredPhase& ph = L.ph[p];
   const int w = et >> 5, q = et & 31;
   const int32_t feat = f * 128 + 4 * q;
@@ -729,7 +741,7 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
         if (p == 3 && bcast[1] == (uint32_t)(ph.tiles - 1)) {
           // the last tile of the vocabulary: every tile's key is in
           fence_acq_rel_gpu();
-          for (int32_t r = et; r < L.rows; r += kEpiThreads) L.out_tok[r] = argmax_index(__ldcg(L.best + r));
+          for (int32_t r = et; r < L.rows; r += kEpiThreads) L.out_tok[r] = argmax_index(__ldcg(L.best + (int64_t)r * kKeyStride));
         }
       }
     }
@@ -835,7 +847,7 @@ PredWs carve(const PredPlan& P, int32_t rows, int32_t d, int32_t m, int32_t V, b
     return p;
   };
   const size_t ctr_bytes = al256((size_t)(kPhases * P.max_tiles + kPhases + 1) * kCtrStride * 4);
-  w.zero_bytes = ctr_bytes + (size_t)kMaxRows * 8;
+  w.zero_bytes = ctr_bytes + (size_t)kMaxRows * kKeyStride * 8;
   w.ctr = reinterpret_cast<unsigned int*>(take(w.zero_bytes));
   w.best = reinterpret_cast<unsigned long long*>(reinterpret_cast<unsigned char*>(w.ctr) + ctr_bytes);
   w.part = reinterpret_cast<float*>(take(P.part_floats * 4));
