@@ -734,7 +734,8 @@ predictor_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant
         fence_acq_rel_gpu();
         bar_named(kBarEpi, kEpiThreads);
         if (et == 0) {
-          atomicAdd(ticket(L, p, f), 1u);  // the tile is final
+          // the tile is final (a reduction: nothing waits for its result)
+          asm volatile("red.relaxed.gpu.global.add.u32 [%0], 1;" ::"l"(ticket(L, p, f)) : "memory");
           bcast[1] = atomicAdd(done_ctr(L, p), 1u);
         }
         bar_named(kBarEpi, kEpiThreads);
