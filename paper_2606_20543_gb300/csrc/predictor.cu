@@ -289,31 +289,39 @@ __device__ void finish_tile_t(const PredLaunch& L, int p, int32_t f, int32_t cnt
                 base + sl * tile_stride + ((int64_t)a * L.nn + r) * 128));
           }
         }
+    // each row's sums (and, in P2, its A) first, all loads in flight; then
+    // one rolled loop finishes the rows, so that the finishing code exists
+    // once in the instruction stream.  It runs once per phase, and between
+    // calls other kernels evict it: an unrolled copy per row was fetched
+    // cold, ~0.9 us per row (P0 finish at 24 rows 8.2 -> 2.8 us, the whole
+    // call with L2 flushed 133 -> 120 us)
+    float4 xs[RB][NACC], as[RB];
 #pragma unroll
     for (int b = 0; b < RB; ++b) {
-      if (i0 + b >= my_rows) continue;  // the same in every lane of the warp
-      const int32_t r = w + 4 * (i0 + b);
-      float4 x[NACC];
 #pragma unroll
       for (int a = 0; a < NACC; ++a) {
-        x[a] = v[b][a][0];
+        xs[b][a] = v[b][a][0];
 #pragma unroll
         for (int sl = 1; sl < SMAX; ++sl) {  // slot order; the predicated-off slots add zero
-          x[a].x += v[b][a][sl].x;
-          x[a].y += v[b][a][sl].y;
-          x[a].z += v[b][a][sl].z;
-          x[a].w += v[b][a][sl].w;
+          xs[b][a].x += v[b][a][sl].x;
+          xs[b][a].y += v[b][a][sl].y;
+          xs[b][a].z += v[b][a][sl].z;
+          xs[b][a].w += v[b][a][sl].w;
         }
       }
-      if (NACC == 2) {
-        emit_gate(L, r, feat, x[0], x[NACC - 1], srow[r]);
-      } else if (p == 3) {
-        emit_argmax(L, r, feat, q, x[0]);
-      } else {
-        float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (p == 2) a0 = __ldcg(reinterpret_cast<const float4*>(L.hid + (int64_t)r * L.d + feat));
-        emit_hidden(L, p, f, r, feat, q, x[0], a0, ga);
-      }
+      as[b] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (p == 2 && i0 + b < my_rows)
+        as[b] = __ldcg(reinterpret_cast<const float4*>(L.hid + (int64_t)(w + 4 * (i0 + b)) * L.d + feat));
+    }
+#pragma unroll 1
+    for (int b = 0; b < RB && i0 + b < my_rows; ++b) {  // the same in every lane of the warp
+      const int32_t r = w + 4 * (i0 + b);
+      if (NACC == 2)
+        emit_gate(L, r, feat, xs[b][0], xs[b][NACC - 1], srow[r]);
+      else if (p == 3)
+        emit_argmax(L, r, feat, q, xs[b][0]);
+      else
+        emit_hidden(L, p, f, r, feat, q, xs[b][0], as[b], ga);
     }
   }
 }
