@@ -46,7 +46,7 @@
 //     the previous phase's partials), then a ticket per tile: the last
 //     contributor sums the tile's partials in slot order and finishes it (A,
 //     Ag and A's squares per row; G; h and Hg; the tile's argmax per row,
-//     raised into one 64-bit key per row with atomicMax), then counts the
+//     raised into one 64-bit key per row by a max reduction), then counts the
 //     tile final on its ticket and on the phase's counter.  The row scales
 //     s(A) are summed once per CTA from the P0 tiles' squares before its first
 //     P1 finish; the last tile of P3 to finish turns the keys into the tokens.
@@ -72,8 +72,8 @@ constexpr int kPhases = 4;
 constexpr int kBarEpi = 1;           // named barrier of the epilogue warps
 constexpr int kMaxSlots = 8;         // most CTAs sharing one feature tile
 // One 128-byte line per row's argmax key: every GenHead tile raises every
-// row's key at the end of the kernel, and keys packed 16 to a line serialised
-// those atomics on a few lines of L2.
+// row's key near the end of the kernel, and the rows' reductions go to
+// separate lines.
 constexpr int kKeyStride = 16;
 
 struct PredPhase {
@@ -195,7 +195,7 @@ __device__ __forceinline__ void warp_argmax(float& v, int32_t& i) {
 namespace {
 
 // The vocabulary argmax of each row is kept as one 64-bit key per row,
-// raised with atomicMax by every finished GenHead tile: the logit in an
+// raised by a max reduction from every finished GenHead tile: the logit in an
 // order-preserving unsigned form (NaN as the lowest key) above the inverted
 // index, so the largest logit wins and the lower index among equal ones
 // (-0 is taken as +0, which compares equal to it).
