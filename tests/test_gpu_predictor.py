@@ -66,8 +66,8 @@ def _check(w, g1, g2, eps, tok, hid):
 
 @pytest.mark.parametrize("rows,d,m,V", [(24, 256, 512, 4096), (5, 128, 256, 1152),
                                         # either side of the switch from per-tile to
-                                        # per-phase activation waits (64 rows)
-                                        (64, 512, 1024, 4096), (65, 512, 1024, 4096)])
+                                        # per-phase activation waits (80 rows)
+                                        (80, 512, 1024, 4096), (81, 512, 1024, 4096)])
 def test_predictor_small(ssd, rows, d, m, V):
     w, g1, g2 = _case(70 + rows, rows, d, m, V)
     tok, hid = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6)
