@@ -71,6 +71,7 @@ constexpr int kMaxRows = 128;
 constexpr int kPhases = 4;
 constexpr int kBarEpi = 1;           // named barrier of the epilogue warps
 constexpr int kMaxSlots = 8;         // most CTAs sharing one feature tile
+constexpr int kTileWaitRows = 80;    // up to this many rows: per-tile activation waits
 // One 128-byte line per row's argmax key: every GenHead tile raises every
 // row's key near the end of the kernel, and the rows' reductions go to
 // separate lines.
@@ -807,6 +808,21 @@ PredPlan make_plan(int32_t rows, int32_t d, int32_t m, int32_t V, int32_t sm_cou
   // every CTA takes at least one unit of every phase, and no tile is split over
   // more than kMaxSlots CTAs (the finisher sums at most that many partials)
   P.ncta = std::max(1, std::min(sm_count, min_units));
+  if (rows > kTileWaitRows) {
+    // many rows: the tiles' finishes, not the stream, set the phase
+    // boundaries, so take the largest CTA count (down to 3/4 of the SMs) that
+    // divides every phase's units: every CTA's range then starts and ends on
+    // a tile boundary, so a tile's contributors end together and fewer of them
+    // share it (at the paper's sizes 128 CTAs: 4, 2, 4 and 1 per tile)
+    for (int32_t c = P.ncta; c >= (P.ncta * 3) / 4 && c >= 1; --c) {
+      bool all = true;
+      for (int p = 0; p < kPhases; ++p) all = all && (P.ph[p].units % c == 0);
+      if (all) {
+        P.ncta = c;
+        break;
+      }
+    }
+  }
   for (;;) {
     int32_t most = 1;
     for (int p = 0; p < kPhases; ++p) most = std::max(most, tile_slots(P.ph[p], P.ncta));
@@ -895,7 +911,7 @@ cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32
   L.shortfall = barrier_shortfall();
   // measured (graphs of back-to-back calls): per-tile waits 136 vs 144 us at 72
   // rows, 147 vs 145 at 90, 150 vs 148 at 128
-  L.tile_waits = a.rows <= 80;
+  L.tile_waits = a.rows <= kTileWaitRows;
   L.eps = a.eps;
   L.gamma1 = a.gamma1;
   L.gamma2 = a.gamma2;
@@ -970,10 +986,16 @@ cudaError_t launch_rows(const PredictorArgs& a, void* ws, size_t ws_bytes, int32
 }  // namespace
 
 size_t predictor_workspace(int32_t rows, int32_t d, int32_t m, int32_t V, bool own_hidden) {
-  rows = std::min(rows, kMaxRows);  // more rows run as several launches over one workspace
-  if (!shapes_ok(rows, d, m, V)) return 0;
-  const PredPlan P = make_plan(rows, d, m, V, device_sm_count());
-  return carve(P, rows, d, m, V, own_hidden, nullptr).bytes;
+  // more rows run as several launches over one workspace: launches of
+  // kMaxRows rows and a last one of the rest, whose plan may differ
+  const int32_t full = std::min(rows, kMaxRows), rest = rows > kMaxRows ? rows % kMaxRows : 0;
+  if (!shapes_ok(full, d, m, V)) return 0;
+  const int sm = device_sm_count();
+  size_t bytes = carve(make_plan(full, d, m, V, sm), full, d, m, V, own_hidden, nullptr).bytes;
+  if (rest > 0)
+    bytes = std::max(bytes,
+                     carve(make_plan(rest, d, m, V, sm), rest, d, m, V, own_hidden, nullptr).bytes);
+  return bytes;
 }
 
 bool predictor_supported(int32_t d, int32_t m, int32_t V) { return shapes_ok(1, d, m, V); }

@@ -92,10 +92,10 @@ def test_predictor_without_hidden_output(ssd):
 
 
 @pytest.mark.parametrize("rows,d,m,V", [(128, 256, 512, 2048), (130, 256, 512, 2048),
-                                        (1, 128, 256, 256)])
+                                        (200, 256, 512, 2048), (1, 128, 256, 256)])
 def test_predictor_row_limits(ssd, rows, d, m, V):
-    """128 rows (one launch's largest row tile), 130 (two launches over one
-    workspace) and a single row."""
+    """128 rows (one launch's largest row tile), 130 and 200 (two launches over
+    one workspace, the second with a plan of its own) and a single row."""
     w, g1, g2 = _case(90 + rows, rows, d, m, V)
     tok, hid = _run(ssd, rows, d, m, V, w, g1, g2, 1e-6)
     ties = _check(w, g1, g2, 1e-6, tok, hid)
